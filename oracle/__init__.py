@@ -1,0 +1,35 @@
+"""Plain fp64 CPU oracle for one LTD draft-and-verify cycle.
+
+TEST INFRASTRUCTURE ONLY.  Nothing in the product path (the CUDA library and
+its Python binding) may import, call or link anything in this package; only
+the tests, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
+``bench.py`` use it.  It shares no code with the CUDA path: the two meet only
+through the seeded inputs of ``paper_2603_01639_gb300.workload``.
+
+Every function follows the paper (Zhang et al., "Learning To Draft: Adaptive
+Speculative Decoding with Reinforcement Learning", §3.2 "Draft-and-Verify
+Cycle") or, where the paper is silent, the reading stated in its docstring.
+All pins are in ``tests/test_oracle_pins.py``; no function here is left
+"parity unpinned".
+"""
+
+from .ltd_oracle import (  # noqa: F401
+    GAMMA,
+    OracleTree,
+    accept_greedy,
+    accept_stochastic,
+    compact_kv,
+    cycle,
+    expand_level,
+    grow_tree,
+    log_softmax,
+    mask_words,
+    mix64,
+    rank_by_logit,
+    select_verify,
+    splitmix64_stream,
+    tree_attention,
+    uniform_gumbel,
+    uniform_ratio,
+    v_all,
+)

@@ -1,0 +1,526 @@
+"""Pins of the fp64 oracle against facts that do not come from the oracle:
+a hand-worked example, closed forms, library routines (scipy log_softmax,
+torch scaled_dot_product_attention), brute force on tiny inputs, invariants,
+the published splitmix64 test vector and a Monte-Carlo test of the
+lossless-sampling theorem.  A final group plants plausible mistakes in the
+oracle and checks that these pins catch them."""
+
+import json
+import math
+import os
+from fractions import Fraction
+
+import numpy as np
+import pytest
+import scipy.special
+import scipy.stats
+import torch
+
+import oracle
+from oracle import ltd_oracle as O
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _worked():
+    with open(os.path.join(GOLDEN, "worked_cycle.json")) as f:
+        return json.load(f)
+
+
+def _rows_from_weights(weights):
+    return np.log(np.asarray(weights, dtype=np.float64))
+
+
+# ------------------------------------------------------------ worked example
+def test_worked_example_tree():
+    g = _worked()
+    rows = _rows_from_weights(g["draft_row_weights"])
+    tree = oracle.grow_tree(g["root_token"], rows, g["W"], g["L"])
+    assert tree.n_nodes == len(g["expected_nodes"]) == oracle.v_all(g["W"], g["L"])
+    for node in g["expected_nodes"]:
+        i = node["id"]
+        assert tree.token[i] == node["token"]
+        assert tree.parent[i] == node["parent"]
+        assert tree.depth[i] == node["depth"]
+        assert tree.cum[i] == pytest.approx(math.log(Fraction(node["cum"])), abs=1e-12)
+    assert tree.frontier == g["expected_frontier_after_level"][str(g["L"])]
+
+
+def test_worked_example_frontiers_per_level():
+    g = _worked()
+    rows = _rows_from_weights(g["draft_row_weights"])
+    for L in (1, 2, 3):
+        tree = oracle.grow_tree(g["root_token"], rows, g["W"], L)
+        assert tree.frontier == g["expected_frontier_after_level"][str(L)]
+
+
+def test_worked_example_select_and_accept():
+    g = _worked()
+    rows = _rows_from_weights(g["draft_row_weights"])
+    tree = oracle.grow_tree(g["root_token"], rows, g["W"], g["L"])
+    ids, pos, mask, _ = oracle.select_verify(tree, g["N"], g["ctx"])
+    assert list(ids) == g["expected_slots"]
+    assert list(pos) == g["expected_pos"]
+    words = oracle.mask_words(mask)
+    assert [int(w[0]) for w in words] == g["expected_mask_words"]
+    target = np.asarray(g["target_rows"], dtype=np.float64)
+    path, a, bonus = oracle.accept_greedy(tree, ids, target)
+    assert path == g["expected_path"]
+    assert a == g["expected_accept_len"]
+    assert bonus == g["expected_bonus"]
+    res = oracle.cycle(g["root_token"], rows, g["W"], g["L"], g["N"], g["ctx"], target)
+    assert res["new_ctx"] == g["expected_new_ctx"]
+
+
+# ------------------------------------------------------------- expansion pins
+def _random_tree(seed, W, L, vocab, ties=False):
+    rng = np.random.default_rng(seed)
+    R = 1 + (L - 1) * W
+    rows = rng.standard_normal((R, vocab))
+    if ties:
+        rows = np.round(rows * 2) / 2  # many exact ties
+    root = int(rng.integers(vocab))
+    return oracle.grow_tree(root, rows, W, L), rows, root
+
+
+@pytest.mark.parametrize("W,L", [(1, 1), (1, 5), (2, 1), (2, 3), (3, 4), (10, 2), (4, 6)])
+def test_tree_size_closed_form(W, L):
+    tree, _, _ = _random_tree(W * 100 + L, W, L, vocab=64)
+    # 3.2 Candidate Token Selection: V_all = 1 + W + (D-2) W^2 with D = L + 1
+    assert tree.n_nodes == 1 + W + (L - 1) * W * W
+
+
+@pytest.mark.parametrize("seed", range(4))
+@pytest.mark.parametrize("ties", [False, True])
+def test_expand_against_scipy_and_brute_force(seed, ties):
+    W, L, vocab = 3, 4, 9
+    tree, rows, _ = _random_tree(seed, W, L, vocab, ties)
+    # every expanded row: scipy's log_softmax, normalisation, and the
+    # brute-force rank of each child among all tokens of its parent's row
+    for u in range(tree.n_nodes):
+        r = tree.xrow[u]
+        if r < 0:
+            continue
+        row = rows[r]
+        ref = scipy.special.logsumexp(row)
+        assert tree.xlse[u] == pytest.approx(ref, abs=1e-12)
+        assert np.exp(row - tree.xlse[u]).sum() == pytest.approx(1.0, abs=1e-12)
+        kids = [c for c in range(tree.n_nodes) if tree.parent[c] == u]
+        assert len(kids) == W
+        for rank, c in enumerate(kids):
+            t = tree.token[c]
+            better = sum(1 for s in range(vocab)
+                         if row[s] > row[t] or (row[s] == row[t] and s < t))
+            assert better == rank
+    # cum of every node is the sum of scipy log-probs along its path
+    for c in range(1, tree.n_nodes):
+        total, a = 0.0, c
+        while tree.parent[a] >= 0:
+            p = tree.parent[a]
+            total += scipy.special.log_softmax(rows[tree.xrow[p]])[tree.token[a]]
+            a = p
+        assert tree.cum[c] == pytest.approx(total, abs=1e-12)
+        assert tree.depth[c] == tree.depth[tree.parent[c]] + 1
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_beam_frontier_is_top_w_of_pool(seed):
+    W, L = 3, 5
+    tree, rows, _ = _random_tree(seed, W, L, vocab=11, ties=(seed % 2 == 1))
+    # brute force: frontier after the last level is the W best of the last
+    # level's W^2 children by (cum desc, id asc)
+    last = [i for i in range(tree.n_nodes) if tree.depth[i] == L]
+    assert len(last) == W * W
+    best = sorted(last, key=lambda i: (-tree.cum[i], i))[:W]
+    assert tree.frontier == best
+    # only frontier nodes of level l have children at level l + 1
+    for lvl in range(2, L):
+        parents = {tree.parent[i] for i in range(tree.n_nodes) if tree.depth[i] == lvl + 1}
+        lvl_nodes = [i for i in range(tree.n_nodes) if tree.depth[i] == lvl]
+        ranked = sorted(lvl_nodes, key=lambda i: (-tree.cum[i], i))[:W]
+        assert parents == set(ranked)
+
+
+def test_expand_row_indexing_follows_frontier_rank():
+    W, L = 2, 3
+    tree, rows, _ = _random_tree(11, W, L, vocab=7)
+    # level 3 rows are 1 + W + r for frontier rank r of level 2
+    lvl2_frontier = sorted([i for i in range(tree.n_nodes) if tree.depth[i] == 2],
+                           key=lambda i: (-tree.cum[i], i))[:W]
+    for r, f in enumerate(lvl2_frontier):
+        assert tree.xrow[f] == 1 + (3 - 2) * W + r
+
+
+# ------------------------------------------------------------- selection pins
+def _ancestry_closure(parent):
+    n = len(parent)
+    A = np.eye(n, dtype=np.int64)
+    adj = np.zeros((n, n), dtype=np.int64)
+    for c, p in enumerate(parent):
+        if p >= 0:
+            adj[c, p] = 1
+    step = adj.copy()
+    for _ in range(n):
+        A = np.minimum(A + step, 1)
+        step = np.minimum(step @ adj, 1)
+    return A  # A[c, a] = 1 iff a is an ancestor-or-self of c
+
+
+@pytest.mark.parametrize("seed", range(5))
+@pytest.mark.parametrize("N", [1, 2, 5, 13, 30])
+def test_select_brute_force(seed, N):
+    W, L = 3, 4
+    tree, _, _ = _random_tree(seed, W, L, vocab=10, ties=(seed % 2 == 0))
+    N = min(N, tree.n_nodes)
+    ctx = 37
+    ids, pos, mask, _ = oracle.select_verify(tree, N, ctx)
+    chosen = set(int(i) for i in ids)
+    assert 0 in chosen and len(chosen) == N
+    assert list(ids) == sorted(ids)
+    key = lambda i: (-tree.cum[i], i)  # noqa: E731
+    inside = [i for i in chosen if i != 0]
+    outside = [i for i in range(1, tree.n_nodes) if i not in chosen]
+    for i in inside:
+        for j in outside:
+            assert key(i) < key(j)
+    A = _ancestry_closure(tree.parent)
+    for si, ni in enumerate(ids):
+        assert pos[si] == ctx + tree.depth[ni]
+        for sj, nj in enumerate(ids):
+            assert bool(mask[si, sj]) == bool(A[ni, nj])
+        # ancestor-closed and topological: every ancestor is verified, earlier
+        a = tree.parent[ni]
+        while a >= 0:
+            assert a in chosen and list(ids).index(a) < si
+            a = tree.parent[a]
+
+
+def test_select_special_cases():
+    tree, _, _ = _random_tree(3, 3, 3, vocab=8)
+    ids, pos, mask, _ = oracle.select_verify(tree, 1, 5)
+    assert list(ids) == [0] and list(pos) == [5] and mask.tolist() == [[True]]
+    ids, _, mask, _ = oracle.select_verify(tree, tree.n_nodes, 5)
+    assert list(ids) == list(range(tree.n_nodes))
+    # W = 1 is a chain: the mask is lower-triangular
+    chain, _, _ = _random_tree(4, 1, 7, vocab=8)
+    ids, _, mask, _ = oracle.select_verify(chain, chain.n_nodes, 0)
+    assert np.array_equal(mask, np.tril(np.ones((8, 8), dtype=bool)))
+
+
+def test_mask_words_layout():
+    m = np.zeros((2, 70), dtype=bool)
+    m[0, 0] = m[0, 31] = m[0, 32] = m[1, 69] = True
+    w = oracle.mask_words(m)
+    assert w.shape == (2, 3)
+    assert w[0].tolist() == [1 | (1 << 31), 1, 0]
+    assert w[1].tolist() == [0, 0, 1 << 5]
+
+
+# ------------------------------------------------------------- attention pins
+def _sdpa(q, k, v, mask=None, causal=False, scale=None):
+    return torch.nn.functional.scaled_dot_product_attention(
+        torch.from_numpy(q), torch.from_numpy(k), torch.from_numpy(v),
+        attn_mask=None if mask is None else torch.from_numpy(mask),
+        is_causal=causal, scale=scale).numpy()
+
+
+def _att_inputs(seed, N, Hq, Hkv, d, ctx, s_cap=None):
+    rng = np.random.default_rng(seed)
+    s_cap = s_cap or ctx + N + 5
+    q = rng.standard_normal((N, Hq, d))
+    k = rng.standard_normal((Hkv, s_cap, d))
+    v = rng.standard_normal((Hkv, s_cap, d))
+    return q, k, v
+
+
+def test_attention_chain_equals_causal():
+    N, Hq, Hkv, d, ctx = 6, 4, 2, 16, 9
+    q, k, v = _att_inputs(0, N, Hq, Hkv, d, ctx)
+    mask = np.tril(np.ones((N, N), dtype=bool))
+    scale = 1 / math.sqrt(d)
+    out = oracle.tree_attention(q, k, v, ctx, mask, scale)
+    # causal attention over the ctx + N sequence; prefix queries are arbitrary
+    rng = np.random.default_rng(1)
+    qfull = np.concatenate([rng.standard_normal((ctx, Hq, d)), q], axis=0)
+    G = Hq // Hkv
+    kk = np.repeat(k[:, :ctx + N], G, axis=0)
+    vv = np.repeat(v[:, :ctx + N], G, axis=0)
+    ref = _sdpa(qfull.transpose(1, 0, 2), kk, vv, causal=True, scale=scale)
+    np.testing.assert_allclose(out, ref.transpose(1, 0, 2)[ctx:], atol=1e-12)
+
+
+def test_attention_all_ones_equals_unmasked():
+    N, Hq, Hkv, d, ctx = 5, 2, 2, 8, 11
+    q, k, v = _att_inputs(2, N, Hq, Hkv, d, ctx)
+    out = oracle.tree_attention(q, k, v, ctx, np.ones((N, N), bool), 0.3)
+    ref = _sdpa(q.transpose(1, 0, 2), k[:, :ctx + N], v[:, :ctx + N], scale=0.3)
+    np.testing.assert_allclose(out, ref.transpose(1, 0, 2), atol=1e-12)
+
+
+def test_attention_single_token_is_decode():
+    Hq, Hkv, d, ctx = 8, 2, 32, 50
+    q, k, v = _att_inputs(3, 1, Hq, Hkv, d, ctx)
+    out = oracle.tree_attention(q, k, v, ctx, np.ones((1, 1), bool), 1 / math.sqrt(d))
+    G = Hq // Hkv
+    ref = _sdpa(q.transpose(1, 0, 2), np.repeat(k[:, :ctx + 1], G, 0),
+                np.repeat(v[:, :ctx + 1], G, 0), scale=1 / math.sqrt(d))
+    np.testing.assert_allclose(out, ref.transpose(1, 0, 2), atol=1e-12)
+
+
+@pytest.mark.parametrize("seed", range(3))
+def test_attention_tree_mask_and_gqa(seed):
+    W, L = 2, 3
+    tree, _, _ = _random_tree(seed, W, L, vocab=6)
+    N = 7
+    ids, _, mask, _ = oracle.select_verify(tree, N, 0)
+    Hq, Hkv, d, ctx = 8, 2, 16, 13
+    q, k, v = _att_inputs(seed + 10, N, Hq, Hkv, d, ctx)
+    out = oracle.tree_attention(q, k, v, ctx, mask, 0.25)
+    # independent mask from parent pointers, GQA as MHA with repeated KV heads
+    A = _ancestry_closure(tree.parent)
+    allowed = np.zeros((N, ctx + N), dtype=bool)
+    allowed[:, :ctx] = True
+    for i, ni in enumerate(ids):
+        for j, nj in enumerate(ids):
+            allowed[i, ctx + j] = bool(A[ni, nj])
+    G = Hq // Hkv
+    ref = _sdpa(q.transpose(1, 0, 2), np.repeat(k[:, :ctx + N], G, 0),
+                np.repeat(v[:, :ctx + N], G, 0), mask=allowed, scale=0.25)
+    np.testing.assert_allclose(out, ref.transpose(1, 0, 2), atol=1e-12)
+
+
+# -------------------------------------------------------- greedy accept pins
+def _brute_force_greedy(tree, ids, target):
+    """Enumerate every root path inside the verified set; the accepted one is
+    the longest whose every edge matches the target argmax at its parent."""
+    slot_of = {int(n): s for s, n in enumerate(ids)}
+    best = [0]
+    for s, n in enumerate(ids):
+        path, a = [], int(n)
+        while a >= 0:
+            path.append(slot_of[a])
+            a = tree.parent[a]
+        path = path[::-1]
+        ok = all(tree.token[int(ids[path[t + 1]])] == int(np.argmax(target[path[t]]))
+                 for t in range(len(path) - 1))
+        if ok and len(path) > len(best):
+            best = path
+    return best, int(np.argmax(target[best[-1]]))
+
+
+@pytest.mark.parametrize("seed", range(12))
+def test_greedy_accept_brute_force(seed):
+    W, L = 3, 4
+    rng = np.random.default_rng(seed + 100)
+    tree, _, _ = _random_tree(seed, W, L, vocab=5, ties=True)
+    N = int(rng.integers(1, tree.n_nodes + 1))
+    ids, _, _, _ = oracle.select_verify(tree, N, 0)
+    target = np.round(rng.standard_normal((N, 5)) * 2) / 2  # ties in argmax
+    # plant agreement on a random subset so long paths occur
+    for s, n in enumerate(ids):
+        kids = [t for t, m in enumerate(ids) if tree.parent[int(m)] == int(n)]
+        if kids and rng.random() < 0.8:
+            target[s, tree.token[int(ids[kids[0]])]] = 10.0
+    path, a, bonus = oracle.accept_greedy(tree, ids, target)
+    ref_path, ref_bonus = _brute_force_greedy(tree, ids, target)
+    assert path == ref_path and bonus == ref_bonus and a == len(path) - 1
+    assert a <= L
+
+
+def test_greedy_single_node_is_autoregressive():
+    tree, _, _ = _random_tree(9, 4, 3, vocab=30)
+    ids, _, _, _ = oracle.select_verify(tree, 1, 0)
+    row = np.random.default_rng(0).standard_normal((1, 30))
+    path, a, bonus = oracle.accept_greedy(tree, ids, row)
+    assert path == [0] and a == 0 and bonus == int(np.argmax(row[0]))
+
+
+# ---------------------------------------------------- stochastic accept pins
+def _star_tree(root_tok, child_tokens, W):
+    """Root with the given children (may repeat tokens); the root was expanded
+    from draft row 0."""
+    t = O.OracleTree.rooted(root_tok, W)
+    t.xrow[0] = 0
+    for tok in child_tokens:
+        t._add(tok, 0, 1, 0.0)
+    return t
+
+
+def test_stochastic_preserves_target_distribution():
+    """Lossless theorem (speculative sampling): with children drawn i.i.d.
+    from q, the first emitted token is distributed as p = softmax(target)."""
+    vocab, k, trials = 6, 3, 30000
+    rng = np.random.default_rng(123)
+    xt = rng.standard_normal(vocab) * 1.5
+    xq = rng.standard_normal(vocab) * 1.5
+    p = scipy.special.softmax(xt)
+    q = scipy.special.softmax(xq)
+    draft_rows = xq[None, :]
+    counts = np.zeros(vocab)
+    for trial in range(trials):
+        kids = rng.choice(vocab, size=k, p=q)
+        tree = _star_tree(0, kids, k)
+        ids = np.arange(k + 1)
+        target = np.vstack([xt] + [rng.standard_normal(vocab) for _ in range(k)])
+        path, a, bonus, _ = oracle.accept_stochastic(tree, ids, target, draft_rows,
+                                                     seed=7, b=0, cycle_no=trial)
+        first = tree.token[path[1]] if a >= 1 else bonus
+        counts[first] += 1
+    chi2 = ((counts - trials * p) ** 2 / (trials * p)).sum()
+    pval = scipy.stats.chi2.sf(chi2, vocab - 1)
+    assert pval > 1e-4, (counts / trials, p, pval)
+
+
+def test_stochastic_bonus_is_exact_sample():
+    """No children: the bonus alone is a Gumbel-max draw from p."""
+    vocab, trials = 5, 20000
+    xt = np.array([0.3, -1.0, 2.0, 0.0, 1.1])
+    p = scipy.special.softmax(xt)
+    tree = _star_tree(0, [], 1)
+    counts = np.zeros(vocab)
+    for trial in range(trials):
+        _, a, bonus, _ = oracle.accept_stochastic(tree, np.array([0]), xt[None, :],
+                                                  xt[None, :], seed=3, b=1, cycle_no=trial)
+        assert a == 0
+        counts[bonus] += 1
+    chi2 = ((counts - trials * p) ** 2 / (trials * p)).sum()
+    assert scipy.stats.chi2.sf(chi2, vocab - 1) > 1e-4
+
+
+def test_stochastic_identical_draft_and_target_accepts_first_child():
+    """q == p: the ratio test r q(x) < p(x) holds for every r < 1."""
+    vocab = 7
+    x = np.random.default_rng(5).standard_normal(vocab)
+    tree = _star_tree(0, [3, 1], 2)
+    path, a, _, _ = oracle.accept_stochastic(tree, np.arange(3), np.vstack([x, x, x]),
+                                             x[None, :], seed=1, b=0, cycle_no=0)
+    assert path == [0, 1] and a == 1
+
+
+def test_stochastic_zero_probability_child_rejected():
+    """p(x) = 0 up to fp64 underflow: the child is always rejected."""
+    vocab = 4
+    xt = np.array([0.0, -1e4, 0.0, 0.0])
+    xq = np.zeros(vocab)
+    tree = _star_tree(0, [1], 1)
+    for c in range(50):
+        path, a, bonus, _ = oracle.accept_stochastic(tree, np.arange(2), np.vstack([xt, xt]),
+                                                     xq[None, :], seed=9, b=0, cycle_no=c)
+        assert a == 0 and bonus != 1
+
+
+# ------------------------------------------------------------------ RNG pins
+def test_splitmix64_published_vector():
+    with open(os.path.join(GOLDEN, "splitmix64_seed0.txt")) as f:
+        vals = [int(line, 16) for line in f if line.strip() and not line.startswith("#")]
+    assert oracle.splitmix64_stream(0, 4) == vals
+
+
+def test_uniforms_exact_and_in_range():
+    for s in range(200):
+        u = oracle.uniform_ratio(11, 2, 3, s % 7, s)
+        assert 0.0 <= u < 1.0 and float(np.float32(u)) == u and (u * 2 ** 24).is_integer()
+    g = oracle.uniform_gumbel(11, 2, 3, 4, np.arange(5000))
+    assert (g > 0).all() and (g < 1).all()
+    assert np.array_equal(g.astype(np.float32).astype(np.float64), g)
+    # roughly uniform
+    assert scipy.stats.kstest(g, "uniform").pvalue > 1e-4
+
+
+# ----------------------------------------------------------- compaction pins
+def test_compaction_copies_and_preserves():
+    rng = np.random.default_rng(0)
+    cache = rng.standard_normal((2, 3, 20, 4))
+    ctx, path = 10, [0, 2, 3]  # destination 1 reads slot 2 while 2 is a destination
+    out = oracle.compact_kv(cache, ctx, path)
+    for t, s in enumerate(path):
+        assert np.array_equal(out[..., ctx + t, :], cache[..., ctx + s, :])
+    untouched = [r for r in range(20) if not (ctx <= r < ctx + len(path))]
+    assert np.array_equal(out[..., untouched, :], cache[..., untouched, :])
+
+
+def test_compaction_identity_path():
+    cache = np.arange(2 * 12 * 3, dtype=np.float64).reshape(2, 12, 3)
+    assert np.array_equal(oracle.compact_kv(cache, 4, [0, 1, 2, 3]), cache)
+
+
+# ------------------------------------------------- planted mistakes are caught
+def _mutant_log_softmax_dropped_lse(x):
+    x = np.asarray(x, np.float64)
+    return x - x.max(), float(x.max())  # mistake: drops log sum exp(x - m)
+
+
+def test_planted_mistake_in_log_softmax_is_caught(monkeypatch):
+    monkeypatch.setattr(O, "log_softmax", _mutant_log_softmax_dropped_lse)
+    with pytest.raises(AssertionError):
+        test_worked_example_tree()
+
+
+def test_planted_mistake_in_tiebreak_is_caught(monkeypatch):
+    def rank_hi_first(x, W):
+        x = np.asarray(x, np.float64)
+        return np.lexsort((-np.arange(x.size), -x))[:W]  # mistake: ties to higher id
+    monkeypatch.setattr(O, "rank_by_logit", rank_hi_first)
+    with pytest.raises(AssertionError):
+        test_worked_example_tree()
+
+
+def test_planted_mistake_in_attention_scale_is_caught(monkeypatch):
+    real = O.tree_attention
+
+    def wrong(q, k, v, ctx, mask, scale):
+        return real(q, k, v, ctx, mask, scale * 1.0001)
+    monkeypatch.setattr(oracle, "tree_attention", wrong)
+    with pytest.raises(AssertionError):
+        test_attention_all_ones_equals_unmasked()
+
+
+def test_planted_mistake_in_attention_mask_transpose_is_caught(monkeypatch):
+    real = O.tree_attention
+
+    def wrong(q, k, v, ctx, mask, scale):
+        return real(q, k, v, ctx, np.asarray(mask).T, scale)
+    monkeypatch.setattr(oracle, "tree_attention", wrong)
+    with pytest.raises(AssertionError):
+        test_attention_chain_equals_causal()
+
+
+def test_planted_mistake_in_residual_is_caught(monkeypatch):
+    """A sign error in the residual max(p - q, 0) breaks losslessness."""
+    real_max = np.maximum
+
+    def accept_wrong(tree, chosen, target_rows, draft_rows, seed, b, cycle_no):
+        orig = O.np.maximum
+        O.np.maximum = lambda a, c: real_max(-a, c)  # mistake: max(q - p, 0)
+        try:
+            return real_accept(tree, chosen, target_rows, draft_rows, seed, b, cycle_no)
+        finally:
+            O.np.maximum = orig
+    real_accept = O.accept_stochastic
+    monkeypatch.setattr(oracle, "accept_stochastic", accept_wrong)
+    with pytest.raises(AssertionError):
+        test_stochastic_preserves_target_distribution()
+
+
+def test_planted_mistake_in_greedy_walk_is_caught(monkeypatch):
+    real = O.accept_greedy
+
+    def wrong(tree, chosen, target_rows):
+        path, a, bonus = real(tree, chosen, target_rows)
+        return path[:-1] or path, max(a - 1, 0), bonus  # mistake: off by one
+    monkeypatch.setattr(oracle, "accept_greedy", wrong)
+    with pytest.raises(AssertionError):
+        test_worked_example_select_and_accept()
+
+
+def test_brute_force_enumeration_is_exhaustive():
+    """Self-check of the brute-force helper on a hand-made tree."""
+    t = _star_tree(0, [1, 2], 2)
+    t._add(3, 1, 2, 0.0)  # node 3 under node 1
+    ids = np.arange(4)
+    target = np.zeros((4, 4))
+    target[0, 1] = 1  # root predicts 1 -> slot 1
+    target[1, 3] = 1  # slot 1 predicts 3 -> slot 3
+    target[3, 2] = 1
+    best, bonus = _brute_force_greedy(t, ids, target)
+    assert best == [0, 1, 3] and bonus == 2

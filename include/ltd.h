@@ -1,0 +1,254 @@
+/*
+ * ltd.h -- C ABI of the GB300 (sm_103a) hot path of one draft-and-verify
+ * cycle of "Learning To Draft" (Zhang et al., LTD), section 3.2
+ * "Draft-and-Verify Cycle": draft tree generation, candidate token
+ * selection, tree-attention verification and acceptance.
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ *  - Every pointer named d_* is DEVICE memory owned by the caller.  The
+ *    library never allocates, frees or retains caller memory; the only
+ *    device memory it owns is one 4-byte error word per device.
+ *  - Every call is asynchronous on the given stream and never synchronises,
+ *    except ltd_check().  Arguments are validated on the host before any
+ *    launch; a bad argument returns an error status and launches nothing.
+ *  - Problems only the device can see (a sequence whose per-sequence size
+ *    breaks a bound, a bounded wait that gave up) set bits in the device
+ *    error word; the kernel skips the offending work and returns.  No kernel
+ *    traps or aborts.  ltd_check() synchronises the stream, reads and clears
+ *    the word, and maps it to a status.
+ *  - Tensors are dense, row-major, innermost dimension last.  Integers are
+ *    int32; bit masks are uint32 words, bit j of a row in word j/32 at bit
+ *    j%32.  Floating inputs are LTD_F32 or LTD_BF16 as stated per call.
+ *  - Batch entries are independent sequences ("b").  Sizes that may differ
+ *    per sequence (context, verify size, mode) are device arrays [batch].
+ *
+ * Readings of the paper (it leaves these open):
+ *  - depth L counts the levels below the root, so a tree of L levels holds
+ *    V_all = 1 + k + (L-1) k^2 nodes (the paper's formula with D = L + 1);
+ *  - the verify size N counts the root, which always occupies slot 0;
+ *  - ties break toward the lower token id within a row and toward the lower
+ *    node id across nodes.
+ */
+#ifndef LTD_H
+#define LTD_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* cudaStream_t without pulling in the CUDA headers. */
+typedef struct CUstream_st* ltd_stream_t;
+
+typedef enum ltd_status {
+  LTD_OK = 0,
+  LTD_ERR_INVALID_ARG = 1, /* null pointer, bad enum, non-positive size   */
+  LTD_ERR_SHAPE = 2,       /* sizes inconsistent with each other/limits   */
+  LTD_ERR_UNSUPPORTED = 3, /* valid request this build does not implement */
+  LTD_ERR_CUDA = 4,        /* a CUDA runtime call failed                  */
+  LTD_ERR_DEVICE = 5,      /* a kernel flagged bad per-sequence data      */
+  LTD_ERR_TIMEOUT = 6      /* a bounded device wait gave up               */
+} ltd_status;
+
+typedef enum ltd_dtype { LTD_F32 = 0, LTD_BF16 = 1 } ltd_dtype;
+typedef enum ltd_mode { LTD_GREEDY = 0, LTD_STOCHASTIC = 1 } ltd_mode;
+
+/* Limits of this build. */
+#define LTD_MAX_K 32          /* beam width k                              */
+#define LTD_MAX_DEPTH 16      /* levels below the root                     */
+#define LTD_MAX_N 256         /* verify size, root included               */
+#define LTD_MAX_TREE_NODES 4096
+
+/* Device error word bits (ltd_check folds them into one status). */
+#define LTD_DEVERR_LEVEL 0x1u     /* expand called out of level order    */
+#define LTD_DEVERR_NVERIFY 0x2u   /* N < 1, N > tree size or N > n_max   */
+#define LTD_DEVERR_CTX 0x4u       /* ctx < 0, ctx > max_ctx, ctx+N > s_cap */
+#define LTD_DEVERR_TREE 0x8u      /* selection not ancestor-closed        */
+#define LTD_DEVERR_TIMEOUT 0x10u  /* a bounded wait gave up               */
+#define LTD_DEVERR_MODE 0x20u     /* mode other than greedy/stochastic    */
+
+/* ------------------------------------------------------------------------
+ * Draft tree (section 3.2, "Draft Tree Generation").
+ *
+ * Structure-of-arrays state of `batch` trees, carved by ltd_tree_init() out
+ * of ONE caller-owned device buffer of ltd_tree_bytes() bytes.  Node ids are
+ * assigned in expansion order: the root is id 0; level 1 gives ids 1..k in
+ * rank order; level l >= 2 gives the child of rank c of the frontier node of
+ * rank r the id 1 + k + (l-2) k^2 + r k + c.  All arrays are [batch][...]:
+ *   token[max_nodes]        token id of the node
+ *   parent[max_nodes]       parent node id, -1 for the root
+ *   depth[max_nodes]        0 for the root
+ *   cum_logprob[max_nodes]  float, sum of log p along the root->node path
+ *   xrow[max_nodes]         draft row that expanded the node, -1 if none
+ *   xlse[max_nodes]         float, log-sum-exp of that row
+ *   frontier[k]             frontier node ids in rank order
+ *   n_nodes[1], n_levels[1] node count and levels built so far
+ * The scratch area holds per-CTA partial results of ltd_expand_tree; it is
+ * zeroed by ltd_tree_reset and left zeroed by every expansion.
+ * ------------------------------------------------------------------------ */
+typedef struct ltd_tree {
+  int32_t batch, max_depth, k, max_nodes;
+  int64_t max_vocab;
+  int32_t* token;
+  int32_t* parent;
+  int32_t* depth;
+  float* cum_logprob;
+  int32_t* xrow;
+  float* xlse;
+  int32_t* frontier;
+  int32_t* n_nodes;
+  int32_t* n_levels;
+  void* scratch;
+  size_t scratch_bytes;
+} ltd_tree;
+
+/* Bytes of device memory a tree of these dimensions needs (0 on bad sizes:
+ * batch >= 1, 1 <= max_depth <= LTD_MAX_DEPTH, 1 <= k <= LTD_MAX_K,
+ * 1 + k + (max_depth-1) k^2 <= LTD_MAX_TREE_NODES, k <= max_vocab). */
+size_t ltd_tree_bytes(int32_t batch, int32_t max_depth, int32_t k, int64_t max_vocab);
+
+/* Fill *tree with views into d_mem (host-side pointer arithmetic only; no
+ * CUDA call).  d_mem must be 256-byte aligned and hold ltd_tree_bytes(). */
+ltd_status ltd_tree_init(ltd_tree* tree, void* d_mem, size_t bytes, int32_t batch,
+                         int32_t max_depth, int32_t k, int64_t max_vocab);
+
+/* Start a new cycle: every tree becomes the single root node holding
+ * d_root_tokens[b] (the target's bonus token of the previous cycle, section
+ * 3.2 "Draft Tree Verification"), and the scratch area is zeroed. */
+ltd_status ltd_tree_reset(const ltd_tree* tree, const int32_t* d_root_tokens, ltd_stream_t stream);
+
+/* Expand every active tree by one level (section 3.2, "Draft Tree
+ * Generation"): level 1 takes the top-k tokens of the root's row; level
+ * l >= 2 gives each of the k frontier nodes its top-k tokens as children
+ * (a k^2 pool, all kept) and makes the k children with the largest
+ * cumulative log-probability the new frontier.
+ *
+ *  level           1-based level being built; all active sequences must have
+ *                  exactly level-1 levels (else LTD_DEVERR_LEVEL)
+ *  d_draft_rows    draft logits [batch][rows_per_seq][vocab] (dtype): row 0
+ *                  is the root's distribution, row 1+(l-2)k+r that of the
+ *                  frontier node of rank r at level l-1 (read for level l)
+ *  rows_per_seq    >= 1 + (max_depth-1) k
+ *  d_active        [batch] 0/1, NULL = all sequences expand
+ * Per node: cum = cum(parent) + x - logsumexp(row), computed in fp32.
+ * Rows must start 16-byte aligned (vocab * sizeof(dtype) % 16 == 0). */
+ltd_status ltd_expand_tree(const ltd_tree* tree, int32_t level, const void* d_draft_rows,
+                           ltd_dtype dtype, int64_t vocab, int64_t rows_per_seq,
+                           const int32_t* d_active, ltd_stream_t stream);
+
+/* Candidate token selection (section 3.2): the N-1 non-root nodes with the
+ * largest cum_logprob (ties to the lower id) plus the root, flattened in
+ * ascending id order ("slots"), with positions and the tree attention mask.
+ *  d_n_verify  [batch] N_b, 1 <= N_b <= min(n_max, n_nodes[b])
+ *  d_ctx       [batch] context length before the cycle
+ *  d_node_ids  out [batch][n_max]   node id per slot, -1 past N_b
+ *  d_pos       out [batch][n_max]   ctx + depth, -1 past N_b
+ *  d_mask      out [batch][n_max][ceil(n_max/32)]  bit j of row i set iff
+ *              slot j is an ancestor of slot i or i itself; zero past N_b. */
+ltd_status ltd_select_verify(const ltd_tree* tree, const int32_t* d_n_verify, int32_t n_max,
+                             const int32_t* d_ctx, int32_t* d_node_ids, int32_t* d_pos,
+                             uint32_t* d_mask, ltd_stream_t stream);
+
+/* Tree attention of the verified tokens against the KV cache (section 3.2
+ * "Draft Tree Verification"; tree attention as in SpecInfer, section 2.1).
+ * For slot i < N_b and query head h, KV head g = h / (hq/hkv):
+ *   out[b][i][h] = sum_k softmax_k(scale * q[b][i][h] . K[b][g][k]) V[b][g][k]
+ * over k in {0..ctx_b-1} and {ctx_b + j : mask bit (i, j)}; the caller has
+ * written the N_b new tokens' keys and values at rows ctx_b..ctx_b+N_b-1.
+ * Accumulation is fp32.  Rows i >= N_b of out are left untouched.
+ *  d_q, d_out   [batch][n_max][hq][head_dim] (dtype)
+ *  d_k, d_v     [batch][hkv][s_cap][head_dim] (dtype)
+ *  max_ctx      host-side bound on every ctx_b (sizes the work split)
+ *  d_workspace  ltd_attention_workspace_bytes() bytes of caller memory
+ * bf16 with head_dim 128 runs on the tcgen05 tensor cores; other shapes
+ * (f32, head_dim in {32, 64, 96, 128}) run on a CUDA-core kernel. */
+size_t ltd_attention_workspace_bytes(int32_t batch, int32_t hq, int32_t hkv, int32_t head_dim,
+                                     int32_t n_max, int32_t max_ctx, ltd_dtype dtype);
+ltd_status ltd_tree_attention(const void* d_q, const void* d_k, const void* d_v, void* d_out,
+                              ltd_dtype dtype, int32_t batch, int32_t hq, int32_t hkv,
+                              int32_t head_dim, int32_t s_cap, const int32_t* d_ctx,
+                              int32_t max_ctx, const int32_t* d_n_verify, int32_t n_max,
+                              const uint32_t* d_mask, float scale, void* d_workspace,
+                              size_t workspace_bytes, ltd_stream_t stream);
+
+/* Which kernel ltd_tree_attention runs for this dtype and head_dim:
+ * returns 1 for the tcgen05 tensor-core kernel, 0 for the CUDA-core kernel,
+ * -1 if the combination is unsupported.  *launches (if not NULL) receives
+ * the number of kernel launches one ltd_tree_attention call makes. */
+int32_t ltd_attention_kernel(ltd_dtype dtype, int32_t head_dim, int32_t* launches);
+
+/* KV cache views for compaction: device arrays of n_layers device pointers,
+ * each layer [batch][hkv][s_cap][head_dim] of dtype. */
+typedef struct ltd_kv_cache {
+  void* const* d_k_layers;
+  void* const* d_v_layers;
+  int32_t n_layers, hkv, head_dim, s_cap;
+  ltd_dtype dtype;
+} ltd_kv_cache;
+
+/* Acceptance (section 3.2 "Draft Tree Verification").
+ * Greedy (d_mode[b] == LTD_GREEDY): from slot 0, repeatedly take the
+ * target's argmax at the current slot (ties to the lower token id) and move
+ * to the verified child carrying that token; stop at the first mismatch, the
+ * argmax there is the bonus token.
+ * Stochastic (LTD_STOCHASTIC, temperature 1; the paper only requires the
+ * target distribution be preserved): at the current slot u, p = softmax of
+ * the target row, q = softmax of the draft row that expanded u; each verified
+ * child x_i in slot order is accepted if r_i q(x_i) < p(x_i), else
+ * p <- max(p - q, 0) / sum; with no child accepted the bonus is the
+ * Gumbel-max draw argmax_t log p(t) - log(-log g_t).  r_i and g_t are
+ * counter-based uniforms: h = seed; h = mix64(h + 0x9E3779B97F4A7C15 (j+1)
+ * + w_j) over the words (b, cycle, stream, slot, i-or-token), mix64 being the
+ * splitmix64 finaliser; r = (h >> 40) 2^-24 (stream 0), g = (2 (h >> 41) + 1)
+ * 2^-24 (stream 1).
+ *  d_target_logits  [batch][n_max][vocab] (dtype), row i = target at slot i
+ *  d_draft_rows     the row store given to ltd_expand_tree (stochastic only)
+ *  d_node_ids       ltd_select_verify output
+ *  d_ctx            [batch] in; d_new_ctx [batch] out = ctx + 1 + accept_len
+ *  d_path           out [batch][max_depth+1] accepted slots, -1 after the end
+ *  d_accept_len     out [batch] accepted draft tokens (root excluded)
+ *  d_bonus          out [batch]
+ *  kv               if not NULL, the accepted rows are compacted in every
+ *                   layer: row ctx+t <- row ctx+path[t] (ltd_kv_compact).
+ *  d_workspace      ltd_accept_workspace_bytes() bytes of caller memory,
+ *                   zero-filled before its first use; every call leaves it
+ *                   zero-filled again. */
+size_t ltd_accept_workspace_bytes(int32_t batch, int32_t n_max, int64_t vocab);
+ltd_status ltd_accept(const ltd_tree* tree, const void* d_target_logits,
+                      const void* d_draft_rows, ltd_dtype dtype, int64_t vocab,
+                      int64_t rows_per_seq, const int32_t* d_node_ids,
+                      const int32_t* d_n_verify, int32_t n_max, const int32_t* d_mode,
+                      uint64_t seed, uint64_t cycle, const int32_t* d_ctx, int32_t* d_new_ctx,
+                      int32_t* d_path, int32_t* d_accept_len, int32_t* d_bonus,
+                      const ltd_kv_cache* kv, void* d_workspace, size_t workspace_bytes,
+                      ltd_stream_t stream);
+
+/* In-place KV compaction ("discards the remainder", section 3.2): for every
+ * layer, sequence, KV head and K/V tensor, row ctx+t <- row ctx+path[t] for
+ * t = 0..accept_len, every source read before any row is written.  Rows
+ * below ctx and from ctx+accept_len+1 up are left as they are.
+ *  d_path [batch][path_stride], d_accept_len [batch], d_ctx [batch] (the
+ *  context before the cycle). */
+ltd_status ltd_kv_compact(const ltd_kv_cache* kv, int32_t batch, const int32_t* d_path,
+                          int32_t path_stride, const int32_t* d_accept_len,
+                          const int32_t* d_ctx, ltd_stream_t stream);
+
+/* Synchronise the stream, read and clear this device's error word.
+ * Returns LTD_OK, LTD_ERR_TIMEOUT, LTD_ERR_DEVICE or LTD_ERR_CUDA; if
+ * out_bits is not NULL it receives the raw LTD_DEVERR_* bits. */
+ltd_status ltd_check(ltd_stream_t stream, uint32_t* out_bits);
+
+/* Human-readable name of a status. */
+const char* ltd_status_string(ltd_status status);
+
+/* Version of this library as major*10000 + minor*100 + patch. */
+int32_t ltd_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* LTD_H */

@@ -1,0 +1,385 @@
+// C ABI glue: argument validation, memory carving and kernel launches for the
+// entry points declared in include/ltd.h.  Nothing here allocates device
+// memory; the per-device error word is a file-scope __device__ variable.
+#include <cuda_runtime.h>
+
+#include <mutex>
+
+#include "ltd.h"
+#include "ltd_internal.h"
+
+namespace ltd {
+
+__device__ uint32_t g_error_word;
+
+uint32_t* device_error_word() {
+  static std::mutex mu;
+  static uint32_t* ptrs[128] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 128) return nullptr;
+  std::lock_guard<std::mutex> lock(mu);
+  if (ptrs[dev] == nullptr) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_error_word) != cudaSuccess) return nullptr;
+    ptrs[dev] = static_cast<uint32_t*>(p);
+  }
+  return ptrs[dev];
+}
+
+namespace {
+
+size_t align256(size_t x) { return (x + 255) / 256 * 256; }
+
+size_t dtype_size(ltd_dtype d) { return d == LTD_BF16 ? 2 : 4; }
+
+bool dtype_ok(ltd_dtype d) { return d == LTD_F32 || d == LTD_BF16; }
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int64_t tree_nodes(int32_t max_depth, int32_t k) {
+  return 1 + static_cast<int64_t>(k) + static_cast<int64_t>(max_depth - 1) * k * k;
+}
+
+bool tree_dims_ok(int32_t batch, int32_t max_depth, int32_t k, int64_t max_vocab) {
+  return batch >= 1 && max_depth >= 1 && max_depth <= LTD_MAX_DEPTH && k >= 1 &&
+         k <= LTD_MAX_K && max_vocab >= k && max_vocab <= 0x7FFFFFFF &&
+         tree_nodes(max_depth, k) <= LTD_MAX_TREE_NODES;
+}
+
+bool tree_ok(const ltd_tree* t) {
+  return t != nullptr && tree_dims_ok(t->batch, t->max_depth, t->k, t->max_vocab) &&
+         t->max_nodes == tree_nodes(t->max_depth, t->k) && t->token && t->parent && t->depth &&
+         t->cum_logprob && t->xrow && t->xlse && t->frontier && t->n_nodes && t->n_levels &&
+         t->scratch;
+}
+
+ltd_status from_cuda(cudaError_t e) { return e == cudaSuccess ? LTD_OK : LTD_ERR_CUDA; }
+
+}  // namespace
+}  // namespace ltd
+
+using namespace ltd;
+
+extern "C" {
+
+int32_t ltd_version(void) { return 100; }
+
+const char* ltd_status_string(ltd_status s) {
+  switch (s) {
+    case LTD_OK: return "LTD_OK";
+    case LTD_ERR_INVALID_ARG: return "LTD_ERR_INVALID_ARG";
+    case LTD_ERR_SHAPE: return "LTD_ERR_SHAPE";
+    case LTD_ERR_UNSUPPORTED: return "LTD_ERR_UNSUPPORTED";
+    case LTD_ERR_CUDA: return "LTD_ERR_CUDA";
+    case LTD_ERR_DEVICE: return "LTD_ERR_DEVICE";
+    case LTD_ERR_TIMEOUT: return "LTD_ERR_TIMEOUT";
+  }
+  return "LTD_ERR_UNKNOWN";
+}
+
+size_t ltd_tree_bytes(int32_t batch, int32_t max_depth, int32_t k, int64_t max_vocab) {
+  if (!tree_dims_ok(batch, max_depth, k, max_vocab)) return 0;
+  const size_t nodes = static_cast<size_t>(batch) * tree_nodes(max_depth, k);
+  return 6 * align256(nodes * 4) + align256(static_cast<size_t>(batch) * k * 4) +
+         2 * align256(static_cast<size_t>(batch) * 4) + expand_layout(batch, k, max_vocab).total;
+}
+
+ltd_status ltd_tree_init(ltd_tree* tree, void* d_mem, size_t bytes, int32_t batch,
+                         int32_t max_depth, int32_t k, int64_t max_vocab) {
+  if (tree == nullptr || d_mem == nullptr) return LTD_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(d_mem) & 255u) != 0) return LTD_ERR_INVALID_ARG;
+  const size_t need = ltd_tree_bytes(batch, max_depth, k, max_vocab);
+  if (need == 0) return LTD_ERR_SHAPE;
+  if (bytes < need) return LTD_ERR_SHAPE;
+  const int64_t mn = tree_nodes(max_depth, k);
+  const size_t nodes = static_cast<size_t>(batch) * mn;
+  char* p = static_cast<char*>(d_mem);
+  auto take = [&p](size_t n) {
+    char* r = p;
+    p += align256(n);
+    return r;
+  };
+  tree->batch = batch;
+  tree->max_depth = max_depth;
+  tree->k = k;
+  tree->max_nodes = static_cast<int32_t>(mn);
+  tree->max_vocab = max_vocab;
+  tree->token = reinterpret_cast<int32_t*>(take(nodes * 4));
+  tree->parent = reinterpret_cast<int32_t*>(take(nodes * 4));
+  tree->depth = reinterpret_cast<int32_t*>(take(nodes * 4));
+  tree->cum_logprob = reinterpret_cast<float*>(take(nodes * 4));
+  tree->xrow = reinterpret_cast<int32_t*>(take(nodes * 4));
+  tree->xlse = reinterpret_cast<float*>(take(nodes * 4));
+  tree->frontier = reinterpret_cast<int32_t*>(take(static_cast<size_t>(batch) * k * 4));
+  tree->n_nodes = reinterpret_cast<int32_t*>(take(static_cast<size_t>(batch) * 4));
+  tree->n_levels = reinterpret_cast<int32_t*>(take(static_cast<size_t>(batch) * 4));
+  tree->scratch_bytes = expand_layout(batch, k, max_vocab).total;
+  tree->scratch = take(tree->scratch_bytes);
+  return LTD_OK;
+}
+
+ltd_status ltd_tree_reset(const ltd_tree* tree, const int32_t* d_root_tokens,
+                          ltd_stream_t stream) {
+  if (!tree_ok(tree) || d_root_tokens == nullptr) return LTD_ERR_INVALID_ARG;
+  return from_cuda(launch_tree_reset(tree, d_root_tokens, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+ltd_status ltd_expand_tree(const ltd_tree* tree, int32_t level, const void* d_draft_rows,
+                           ltd_dtype dtype, int64_t vocab, int64_t rows_per_seq,
+                           const int32_t* d_active, ltd_stream_t stream) {
+  if (!tree_ok(tree) || d_draft_rows == nullptr || !dtype_ok(dtype)) return LTD_ERR_INVALID_ARG;
+  if (level < 1 || level > tree->max_depth) return LTD_ERR_SHAPE;
+  if (vocab < tree->k || vocab > tree->max_vocab) return LTD_ERR_SHAPE;
+  if (rows_per_seq < 1 + static_cast<int64_t>(tree->max_depth - 1) * tree->k) return LTD_ERR_SHAPE;
+  if (!aligned16(d_draft_rows) || (vocab * static_cast<int64_t>(dtype_size(dtype))) % 16 != 0)
+    return LTD_ERR_SHAPE;
+  uint32_t* err = device_error_word();
+  if (err == nullptr) return LTD_ERR_CUDA;
+  const int32_t F = (level == 1) ? 1 : tree->k;
+  const VocabSplit vs = vocab_split(static_cast<int64_t>(tree->batch) * F, vocab,
+                                    kExpandTargetCtas, kExpandMinElems);
+  const ExpandRecordLayout l = expand_layout(tree->batch, tree->k, tree->max_vocab);
+  if (static_cast<int64_t>(tree->batch) * F * vs.chunks > l.records) return LTD_ERR_SHAPE;
+  char* base = static_cast<char*>(tree->scratch);
+  ExpandParams p{};
+  p.token = tree->token;
+  p.parent = tree->parent;
+  p.depth = tree->depth;
+  p.cum = tree->cum_logprob;
+  p.xrow = tree->xrow;
+  p.xlse = tree->xlse;
+  p.frontier = tree->frontier;
+  p.n_nodes = tree->n_nodes;
+  p.n_levels = tree->n_levels;
+  p.max_nodes = tree->max_nodes;
+  p.k = tree->k;
+  p.part_ms = reinterpret_cast<float2*>(base);
+  p.part_keys = reinterpret_cast<uint64_t*>(base + l.ms_bytes);
+  p.row_ticket = reinterpret_cast<uint32_t*>(base + l.ms_bytes + l.keys_bytes);
+  p.seq_ticket = reinterpret_cast<uint32_t*>(base + l.ms_bytes + l.keys_bytes + l.row_ticket_bytes);
+  p.rows = d_draft_rows;
+  p.vocab = vocab;
+  p.rows_per_seq = rows_per_seq;
+  p.active = d_active;
+  p.level = level;
+  p.F = F;
+  p.chunks = vs.chunks;
+  p.chunk_elems = vs.chunk_elems;
+  p.err = err;
+  return from_cuda(launch_expand(p, tree->batch, dtype, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+ltd_status ltd_select_verify(const ltd_tree* tree, const int32_t* d_n_verify, int32_t n_max,
+                             const int32_t* d_ctx, int32_t* d_node_ids, int32_t* d_pos,
+                             uint32_t* d_mask, ltd_stream_t stream) {
+  if (!tree_ok(tree) || !d_n_verify || !d_ctx || !d_node_ids || !d_pos || !d_mask)
+    return LTD_ERR_INVALID_ARG;
+  if (n_max < 1 || n_max > LTD_MAX_N) return LTD_ERR_SHAPE;
+  uint32_t* err = device_error_word();
+  if (err == nullptr) return LTD_ERR_CUDA;
+  SelectParams p{};
+  p.token = tree->token;
+  p.parent = tree->parent;
+  p.depth = tree->depth;
+  p.cum = tree->cum_logprob;
+  p.n_nodes = tree->n_nodes;
+  p.max_nodes = tree->max_nodes;
+  p.n_verify = d_n_verify;
+  p.n_max = n_max;
+  p.ctx = d_ctx;
+  p.node_ids = d_node_ids;
+  p.pos = d_pos;
+  p.mask = d_mask;
+  p.err = err;
+  return from_cuda(launch_select(p, tree->batch, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+size_t ltd_attention_workspace_bytes(int32_t batch, int32_t hq, int32_t hkv, int32_t head_dim,
+                                     int32_t n_max, int32_t max_ctx, ltd_dtype dtype) {
+  if (batch < 1 || hq < 1 || hkv < 1 || hq % hkv != 0 || n_max < 1 || max_ctx < 0) return 0;
+  AttnParams p{};
+  p.batch = batch;
+  p.hq = hq;
+  p.hkv = hkv;
+  p.d = head_dim;
+  p.n_max = n_max;
+  p.max_ctx = max_ctx;
+  size_t ws = 256;  // never zero, so 0 can mean "bad sizes"
+  if (attn_tc_supported(p, dtype)) {
+    const size_t t = attn_tc_workspace(batch, hq, hkv, head_dim, n_max, max_ctx);
+    ws = t > ws ? t : ws;
+  }
+  return ws;
+}
+
+ltd_status ltd_tree_attention(const void* d_q, const void* d_k, const void* d_v, void* d_out,
+                              ltd_dtype dtype, int32_t batch, int32_t hq, int32_t hkv,
+                              int32_t head_dim, int32_t s_cap, const int32_t* d_ctx,
+                              int32_t max_ctx, const int32_t* d_n_verify, int32_t n_max,
+                              const uint32_t* d_mask, float scale, void* d_workspace,
+                              size_t workspace_bytes, ltd_stream_t stream) {
+  if (!d_q || !d_k || !d_v || !d_out || !d_ctx || !d_n_verify || !d_mask || !dtype_ok(dtype))
+    return LTD_ERR_INVALID_ARG;
+  if (batch < 1 || hq < 1 || hkv < 1 || hq % hkv != 0 || n_max < 1 || n_max > LTD_MAX_N ||
+      max_ctx < 0 || s_cap < 1 || static_cast<int64_t>(max_ctx) + n_max > s_cap)
+    return LTD_ERR_SHAPE;
+  if (head_dim != 32 && head_dim != 64 && head_dim != 96 && head_dim != 128)
+    return LTD_ERR_UNSUPPORTED;
+  if (!(scale > 0.f)) return LTD_ERR_INVALID_ARG;
+  if (!aligned16(d_q) || !aligned16(d_k) || !aligned16(d_v) || !aligned16(d_out))
+    return LTD_ERR_SHAPE;
+  const size_t need =
+      ltd_attention_workspace_bytes(batch, hq, hkv, head_dim, n_max, max_ctx, dtype);
+  if (d_workspace == nullptr || workspace_bytes < need) return LTD_ERR_SHAPE;
+  uint32_t* err = device_error_word();
+  if (err == nullptr) return LTD_ERR_CUDA;
+  AttnParams p{};
+  p.q = d_q;
+  p.k = d_k;
+  p.v = d_v;
+  p.out = d_out;
+  p.batch = batch;
+  p.hq = hq;
+  p.hkv = hkv;
+  p.d = head_dim;
+  p.s_cap = s_cap;
+  p.ctx = d_ctx;
+  p.max_ctx = max_ctx;
+  p.n_verify = d_n_verify;
+  p.n_max = n_max;
+  p.mask = d_mask;
+  p.scale = scale;
+  p.ws = d_workspace;
+  p.ws_bytes = workspace_bytes;
+  p.err = err;
+  const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (attn_tc_supported(p, dtype)) return from_cuda(launch_attn_tc(p, s));
+  return from_cuda(launch_attn_simt(p, dtype, s));
+}
+
+int32_t ltd_attention_kernel(ltd_dtype dtype, int32_t head_dim, int32_t* launches) {
+  if (!dtype_ok(dtype) || (head_dim != 32 && head_dim != 64 && head_dim != 96 && head_dim != 128))
+    return -1;
+  AttnParams p{};
+  p.batch = 1;
+  p.hq = 1;
+  p.hkv = 1;
+  p.d = head_dim;
+  p.n_max = 1;
+  const bool tc = attn_tc_supported(p, dtype);
+  if (launches) *launches = tc ? attn_tc_launches() : 1;
+  return tc ? 1 : 0;
+}
+
+size_t ltd_accept_workspace_bytes(int32_t batch, int32_t n_max, int64_t vocab) {
+  if (batch < 1 || n_max < 1 || n_max > LTD_MAX_N || vocab < 1) return 0;
+  return accept_workspace(batch, n_max, vocab);
+}
+
+ltd_status ltd_kv_compact(const ltd_kv_cache* kv, int32_t batch, const int32_t* d_path,
+                          int32_t path_stride, const int32_t* d_accept_len, const int32_t* d_ctx,
+                          ltd_stream_t stream) {
+  if (kv == nullptr || !kv->d_k_layers || !kv->d_v_layers || !d_path || !d_accept_len || !d_ctx ||
+      !dtype_ok(kv->dtype))
+    return LTD_ERR_INVALID_ARG;
+  if (batch < 1 || kv->n_layers < 1 || kv->hkv < 1 || kv->s_cap < 1 || path_stride < 1)
+    return LTD_ERR_SHAPE;
+  const int64_t row_bytes = static_cast<int64_t>(kv->head_dim) * dtype_size(kv->dtype);
+  if (kv->head_dim < 1 || row_bytes % 16 != 0 || row_bytes > 512) return LTD_ERR_UNSUPPORTED;
+  uint32_t* err = device_error_word();
+  if (err == nullptr) return LTD_ERR_CUDA;
+  CompactParams p{};
+  p.k_layers = kv->d_k_layers;
+  p.v_layers = kv->d_v_layers;
+  p.n_layers = kv->n_layers;
+  p.hkv = kv->hkv;
+  p.s_cap = kv->s_cap;
+  p.row_bytes = static_cast<int32_t>(row_bytes);
+  p.path = d_path;
+  p.path_stride = path_stride;
+  p.accept_len = d_accept_len;
+  p.ctx = d_ctx;
+  p.err = err;
+  return from_cuda(launch_compact(p, batch, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+ltd_status ltd_accept(const ltd_tree* tree, const void* d_target_logits, const void* d_draft_rows,
+                      ltd_dtype dtype, int64_t vocab, int64_t rows_per_seq,
+                      const int32_t* d_node_ids, const int32_t* d_n_verify, int32_t n_max,
+                      const int32_t* d_mode, uint64_t seed, uint64_t cycle, const int32_t* d_ctx,
+                      int32_t* d_new_ctx, int32_t* d_path, int32_t* d_accept_len,
+                      int32_t* d_bonus, const ltd_kv_cache* kv, void* d_workspace,
+                      size_t workspace_bytes, ltd_stream_t stream) {
+  if (!tree_ok(tree) || !d_target_logits || !d_draft_rows || !dtype_ok(dtype) || !d_node_ids ||
+      !d_n_verify || !d_mode || !d_ctx || !d_new_ctx || !d_path || !d_accept_len || !d_bonus)
+    return LTD_ERR_INVALID_ARG;
+  if (n_max < 1 || n_max > LTD_MAX_N || vocab < 1 || vocab > tree->max_vocab) return LTD_ERR_SHAPE;
+  if (rows_per_seq < 1 + static_cast<int64_t>(tree->max_depth - 1) * tree->k) return LTD_ERR_SHAPE;
+  if (!aligned16(d_target_logits) || (vocab * static_cast<int64_t>(dtype_size(dtype))) % 16 != 0)
+    return LTD_ERR_SHAPE;
+  const size_t need = accept_workspace(tree->batch, n_max, vocab);
+  if (d_workspace == nullptr || workspace_bytes < need) return LTD_ERR_SHAPE;
+  if (kv != nullptr) {
+    if (!kv->d_k_layers || !kv->d_v_layers || !dtype_ok(kv->dtype)) return LTD_ERR_INVALID_ARG;
+    const int64_t row_bytes = static_cast<int64_t>(kv->head_dim) * dtype_size(kv->dtype);
+    if (kv->n_layers < 1 || kv->hkv < 1 || kv->s_cap < 1) return LTD_ERR_SHAPE;
+    if (kv->head_dim < 1 || row_bytes % 16 != 0 || row_bytes > 512) return LTD_ERR_UNSUPPORTED;
+  }
+  uint32_t* err = device_error_word();
+  if (err == nullptr) return LTD_ERR_CUDA;
+  const VocabSplit vs = vocab_split(static_cast<int64_t>(tree->batch) * n_max, vocab,
+                                    kAcceptTargetCtas, kAcceptMinElems);
+  const size_t rec_bytes =
+      static_cast<size_t>(tree->batch) * n_max * vs.chunks * sizeof(AcceptRecord);
+  AcceptParams p{};
+  p.token = tree->token;
+  p.parent = tree->parent;
+  p.xrow = tree->xrow;
+  p.xlse = tree->xlse;
+  p.max_nodes = tree->max_nodes;
+  p.max_depth = tree->max_depth;
+  p.target = d_target_logits;
+  p.draft = d_draft_rows;
+  p.vocab = vocab;
+  p.rows_per_seq = rows_per_seq;
+  p.node_ids = d_node_ids;
+  p.n_verify = d_n_verify;
+  p.n_max = n_max;
+  p.mode = d_mode;
+  p.seed = seed;
+  p.cycle = cycle;
+  p.ctx = d_ctx;
+  p.new_ctx = d_new_ctx;
+  p.path = d_path;
+  p.accept_len = d_accept_len;
+  p.bonus = d_bonus;
+  p.rec = static_cast<AcceptRecord*>(d_workspace);
+  p.ticket = reinterpret_cast<uint32_t*>(static_cast<char*>(d_workspace) + align256(rec_bytes));
+  p.chunks = vs.chunks;
+  p.chunk_elems = vs.chunk_elems;
+  p.err = err;
+  const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  cudaError_t e = launch_accept(p, tree->batch, dtype, s);
+  if (e != cudaSuccess || kv == nullptr) return from_cuda(e);
+  return ltd_kv_compact(kv, tree->batch, d_path, tree->max_depth + 1, d_accept_len, d_ctx, stream);
+}
+
+ltd_status ltd_check(ltd_stream_t stream, uint32_t* out_bits) {
+  const cudaError_t e = cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return LTD_ERR_CUDA;
+  uint32_t* w = device_error_word();
+  if (w == nullptr) return LTD_ERR_CUDA;
+  uint32_t bits = 0;
+  if (cudaMemcpy(&bits, w, sizeof(bits), cudaMemcpyDeviceToHost) != cudaSuccess) return LTD_ERR_CUDA;
+  if (bits != 0) {
+    const uint32_t zero = 0;
+    if (cudaMemcpy(w, &zero, sizeof(zero), cudaMemcpyHostToDevice) != cudaSuccess)
+      return LTD_ERR_CUDA;
+  }
+  if (out_bits) *out_bits = bits;
+  if (bits & LTD_DEVERR_TIMEOUT) return LTD_ERR_TIMEOUT;
+  if (bits) return LTD_ERR_DEVICE;
+  return LTD_OK;
+}
+
+}  // extern "C"

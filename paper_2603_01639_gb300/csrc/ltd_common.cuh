@@ -1,0 +1,268 @@
+// Device helpers shared by the LTD kernels: ordered 64-bit keys for
+// (value desc, index asc) selection, register-resident top-k lists, warp and
+// block reductions, the splitmix64-keyed uniforms, and vector loads.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <math_constants.h>
+#include <stdint.h>
+
+#include "ltd.h"
+
+namespace ltd {
+
+constexpr int kWarp = 32;
+constexpr uint64_t kGamma = 0x9E3779B97F4A7C15ull;
+
+// ---------------------------------------------------------------- keys
+// Monotone map of a float to uint32 (larger float -> larger code); -0 and +0
+// map to the same code so that equal values tie exactly as in the oracle.
+__device__ __forceinline__ uint32_t float_order_bits(float f) {
+  uint32_t u = __float_as_uint(f);
+  if (u == 0x80000000u) u = 0u;
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+__device__ __forceinline__ float order_bits_float(uint32_t o) {
+  const uint32_t u = (o & 0x80000000u) ? (o & 0x7FFFFFFFu) : ~o;
+  return __uint_as_float(u);
+}
+
+// Larger key = better: value descending, then index ascending.  Every real
+// key is > 0, so 0 serves as the empty slot.
+__device__ __forceinline__ uint64_t make_key(float v, uint32_t idx) {
+  return (static_cast<uint64_t>(float_order_bits(v)) << 32) |
+         static_cast<uint64_t>(0xFFFFFFFFu - idx);
+}
+__device__ __forceinline__ uint32_t key_index(uint64_t k) {
+  return 0xFFFFFFFFu - static_cast<uint32_t>(k);
+}
+__device__ __forceinline__ float key_value(uint64_t k) {
+  return order_bits_float(static_cast<uint32_t>(k >> 32));
+}
+
+// A descending list of the K largest keys seen, kept in registers (all
+// indices are compile-time after unrolling).
+template <int K>
+struct TopK {
+  uint64_t v[K];
+  __device__ __forceinline__ void init() {
+#pragma unroll
+    for (int i = 0; i < K; ++i) v[i] = 0ull;
+  }
+  __device__ __forceinline__ void insert(uint64_t key) {
+    if (key <= v[K - 1]) return;
+#pragma unroll
+    for (int i = K - 1; i > 0; --i) {
+      const uint64_t up = v[i - 1];
+      v[i] = (key > up) ? up : ((key > v[i]) ? key : v[i]);
+    }
+    v[0] = (key > v[0]) ? key : v[0];
+  }
+  __device__ __forceinline__ void pop() {
+#pragma unroll
+    for (int i = 0; i < K - 1; ++i) v[i] = v[i + 1];
+    v[K - 1] = 0ull;
+  }
+};
+
+// -------------------------------------------------------------- reductions
+__device__ __forceinline__ uint64_t warp_max_u64(uint64_t x) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const uint64_t y = __shfl_xor_sync(0xFFFFFFFFu, x, o);
+    x = (y > x) ? y : x;
+  }
+  return x;
+}
+
+__device__ __forceinline__ float warp_max_f(float x) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) x = fmaxf(x, __shfl_xor_sync(0xFFFFFFFFu, x, o));
+  return x;
+}
+
+__device__ __forceinline__ float warp_sum_f(float x) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xFFFFFFFFu, x, o);
+  return x;
+}
+
+// (max, sum of exp(x - max)) pairs: the merge of two partial softmax
+// normalisers.  An empty side has max = -inf and sum = 0.
+__device__ __forceinline__ void ms_merge(float& m, float& s, float m2, float s2) {
+  if (m2 == -CUDART_INF_F) return;
+  if (m == -CUDART_INF_F) {
+    m = m2;
+    s = s2;
+    return;
+  }
+  const float mm = fmaxf(m, m2);
+  s = s * __expf(m - mm) + s2 * __expf(m2 - mm);
+  m = mm;
+}
+
+__device__ __forceinline__ void warp_ms(float& m, float& s) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float m2 = __shfl_xor_sync(0xFFFFFFFFu, m, o);
+    const float s2 = __shfl_xor_sync(0xFFFFFFFFu, s, o);
+    ms_merge(m, s, m2, s2);
+  }
+}
+
+// Block-wide (max, sumexp) merge; the result is valid in every thread.
+// `red` needs 2 * (blockDim.x / 32) floats of shared memory.
+template <int NT>
+__device__ __forceinline__ void block_ms(float& m, float& s, float* red) {
+  constexpr int NW = NT / kWarp;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  warp_ms(m, s);
+  __syncthreads();
+  if (lane == 0) {
+    red[warp] = m;
+    red[NW + warp] = s;
+  }
+  __syncthreads();
+  m = -CUDART_INF_F;
+  s = 0.f;
+  for (int w = 0; w < NW; ++w) ms_merge(m, s, red[w], red[NW + w]);
+}
+
+template <int NT>
+__device__ __forceinline__ float block_sum(float x, float* red) {
+  constexpr int NW = NT / kWarp;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  x = warp_sum_f(x);
+  __syncthreads();
+  if (lane == 0) red[warp] = x;
+  __syncthreads();
+  float t = 0.f;
+  for (int w = 0; w < NW; ++w) t += red[w];
+  return t;
+}
+
+template <int NT>
+__device__ __forceinline__ uint64_t block_max_u64(uint64_t x, uint64_t* red) {
+  constexpr int NW = NT / kWarp;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  x = warp_max_u64(x);
+  __syncthreads();
+  if (lane == 0) red[warp] = x;
+  __syncthreads();
+  uint64_t t = 0;
+  for (int w = 0; w < NW; ++w) t = red[w] > t ? red[w] : t;
+  return t;
+}
+
+// Block-wide top-k of the keys held in every thread's TopK list.  Writes the
+// k best keys, descending, to out[0..k) (shared memory) and returns after a
+// barrier.  `stage` needs NW * K uint64 of shared memory.
+template <int K, int NT>
+__device__ __forceinline__ void block_topk(TopK<K>& tk, int k, uint64_t* stage, uint64_t* out) {
+  constexpr int NW = NT / kWarp;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  for (int r = 0; r < k; ++r) {
+    const uint64_t head = tk.v[0];
+    const uint64_t best = warp_max_u64(head);
+    if (lane == 0) stage[warp * K + r] = best;
+    if (best != 0ull && head == best) tk.pop();
+  }
+  __syncthreads();
+  if (warp == 0) {
+    TopK<K> t2;
+    t2.init();
+    for (int j = lane; j < NW * k; j += kWarp) t2.insert(stage[(j / k) * K + (j % k)]);
+    for (int r = 0; r < k; ++r) {
+      const uint64_t head = t2.v[0];
+      const uint64_t best = warp_max_u64(head);
+      if (lane == 0) out[r] = best;
+      if (best != 0ull && head == best) t2.pop();
+    }
+  }
+  __syncthreads();
+}
+
+// -------------------------------------------------------- counter uniforms
+// splitmix64 output finaliser (Steele, Lea & Flood 2014).
+__device__ __forceinline__ uint64_t mix64(uint64_t z) {
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+// h_0 = seed; h_{j+1} = mix64(h_j + gamma (j+1) + w_j), for words w_0..w_{n-1}
+// starting at position j0 (so a prefix hash can be extended later).
+__device__ __forceinline__ uint64_t hash_step(uint64_t h, int j, uint64_t w) {
+  return mix64(h + kGamma * static_cast<uint64_t>(j + 1) + w);
+}
+
+constexpr uint64_t kStreamRatio = 0;
+constexpr uint64_t kStreamBonus = 1;
+
+// Prefix (seed, b, cycle, stream, slot) -> 4 hash steps.
+__device__ __forceinline__ uint64_t hash_prefix(uint64_t seed, uint64_t b, uint64_t cycle,
+                                                uint64_t stream, uint64_t slot) {
+  uint64_t h = seed;
+  h = hash_step(h, 0, b);
+  h = hash_step(h, 1, cycle);
+  h = hash_step(h, 2, stream);
+  h = hash_step(h, 3, slot);
+  return h;
+}
+
+// Top 24 bits times 2^-24: exact in fp32.
+__device__ __forceinline__ float uniform_ratio(uint64_t prefix, uint64_t i) {
+  const uint64_t h = hash_step(prefix, 4, i);
+  return static_cast<float>(h >> 40) * 5.9604644775390625e-8f;
+}
+// (2 (h >> 41) + 1) 2^-24, in (0, 1), exact in fp32.
+__device__ __forceinline__ float uniform_gumbel(uint64_t prefix, uint64_t t) {
+  const uint64_t h = hash_step(prefix, 4, t);
+  return static_cast<float>(2ull * (h >> 41) + 1ull) * 5.9604644775390625e-8f;
+}
+
+// -------------------------------------------------------------- loads
+template <typename T>
+__device__ __forceinline__ float to_f(T x);
+template <>
+__device__ __forceinline__ float to_f<float>(float x) {
+  return x;
+}
+template <>
+__device__ __forceinline__ float to_f<__nv_bfloat16>(__nv_bfloat16 x) {
+  return __bfloat162float(x);
+}
+
+// 16-byte vector of VEC elements, converted to float.
+template <typename T>
+struct Vec16 {
+  static constexpr int N = 16 / sizeof(T);
+};
+
+__device__ __forceinline__ void unpack16(const uint4& u, float* out, const float*) {
+  out[0] = __uint_as_float(u.x);
+  out[1] = __uint_as_float(u.y);
+  out[2] = __uint_as_float(u.z);
+  out[3] = __uint_as_float(u.w);
+}
+__device__ __forceinline__ void unpack16(const uint4& u, float* out, const __nv_bfloat16*) {
+  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    out[2 * i] = __uint_as_float(w[i] << 16);
+    out[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+  }
+}
+
+// Streaming 16-byte load that bypasses L1 (data read once).
+__device__ __forceinline__ uint4 ld_stream16(const void* p) {
+  return __ldcs(reinterpret_cast<const uint4*>(p));
+}
+
+__device__ __forceinline__ void flag_error(uint32_t* err, uint32_t bits) {
+  if (err) atomicOr(err, bits);
+}
+
+}  // namespace ltd

@@ -1,0 +1,159 @@
+// Internal launch interfaces between the C ABI glue (ltd_api.cu) and the
+// kernel translation units.  Not part of the public ABI.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "ltd.h"
+
+namespace ltd {
+
+// Address of this device's error word (lives in ltd_api.cu).
+uint32_t* device_error_word();
+
+// Work split of a vocabulary scan: `chunks` CTAs per row, each covering
+// `chunk_elems` elements (a multiple of 8, so chunk starts stay 16-byte
+// aligned for both dtypes).
+struct VocabSplit {
+  int32_t chunks;
+  int64_t chunk_elems;
+};
+VocabSplit vocab_split(int64_t rows, int64_t vocab, int64_t target_ctas, int64_t min_elems);
+
+// ------------------------------------------------------------- expansion
+constexpr int64_t kExpandTargetCtas = 304;  // two CTAs per SM of a 152-SM GB300
+constexpr int64_t kExpandMinElems = 2048;
+
+struct ExpandRecordLayout {
+  size_t ms_bytes, keys_bytes, row_ticket_bytes, seq_ticket_bytes, total;
+  int64_t records;
+};
+ExpandRecordLayout expand_layout(int32_t batch, int32_t k, int64_t max_vocab);
+
+struct ExpandParams {
+  int32_t* token;
+  int32_t* parent;
+  int32_t* depth;
+  float* cum;
+  int32_t* xrow;
+  float* xlse;
+  int32_t* frontier;
+  int32_t* n_nodes;
+  int32_t* n_levels;
+  int32_t max_nodes;
+  int32_t k;
+  float2* part_ms;       // [records]
+  uint64_t* part_keys;   // [records][k]
+  uint32_t* row_ticket;  // [batch][k]
+  uint32_t* seq_ticket;  // [batch]
+  const void* rows;
+  int64_t vocab;
+  int64_t rows_per_seq;
+  const int32_t* active;
+  int32_t level;
+  int32_t F;
+  int32_t chunks;
+  int64_t chunk_elems;
+  uint32_t* err;
+};
+cudaError_t launch_tree_reset(const ltd_tree* t, const int32_t* roots, cudaStream_t s);
+cudaError_t launch_expand(const ExpandParams& p, int32_t batch, ltd_dtype dtype, cudaStream_t s);
+
+// ------------------------------------------------------------- selection
+struct SelectParams {
+  const int32_t* token;
+  const int32_t* parent;
+  const int32_t* depth;
+  const float* cum;
+  const int32_t* n_nodes;
+  int32_t max_nodes;
+  const int32_t* n_verify;
+  int32_t n_max;
+  const int32_t* ctx;
+  int32_t* node_ids;
+  int32_t* pos;
+  uint32_t* mask;
+  uint32_t* err;
+};
+cudaError_t launch_select(const SelectParams& p, int32_t batch, cudaStream_t s);
+
+// ------------------------------------------------------------- attention
+struct AttnParams {
+  const void* q;
+  const void* k;
+  const void* v;
+  void* out;
+  int32_t batch, hq, hkv, d, s_cap;
+  const int32_t* ctx;
+  int32_t max_ctx;
+  const int32_t* n_verify;
+  int32_t n_max;
+  const uint32_t* mask;
+  float scale;
+  void* ws;
+  size_t ws_bytes;
+  uint32_t* err;
+};
+size_t attn_simt_workspace(const AttnParams& p);
+cudaError_t launch_attn_simt(const AttnParams& p, ltd_dtype dtype, cudaStream_t s);
+bool attn_tc_supported(const AttnParams& p, ltd_dtype dtype);
+size_t attn_tc_workspace(int32_t batch, int32_t hq, int32_t hkv, int32_t d, int32_t n_max,
+                         int32_t max_ctx);
+cudaError_t launch_attn_tc(const AttnParams& p, cudaStream_t s);
+int32_t attn_tc_launches();
+
+// ------------------------------------------------------------- acceptance
+constexpr int64_t kAcceptTargetCtas = 608;
+constexpr int64_t kAcceptMinElems = 4096;
+
+struct AcceptRecord {
+  float m, s;
+  unsigned long long key;
+};
+
+struct AcceptParams {
+  const int32_t* token;
+  const int32_t* parent;
+  const int32_t* xrow;
+  const float* xlse;
+  int32_t max_nodes;
+  int32_t max_depth;
+  const void* target;
+  const void* draft;
+  int64_t vocab;
+  int64_t rows_per_seq;
+  const int32_t* node_ids;
+  const int32_t* n_verify;
+  int32_t n_max;
+  const int32_t* mode;
+  unsigned long long seed, cycle;
+  const int32_t* ctx;
+  int32_t* new_ctx;
+  int32_t* path;
+  int32_t* accept_len;
+  int32_t* bonus;
+  AcceptRecord* rec;  // [batch][n_max][chunks]
+  uint32_t* ticket;   // [batch]
+  int32_t chunks;
+  int64_t chunk_elems;
+  uint32_t* err;
+};
+size_t accept_workspace(int32_t batch, int32_t n_max, int64_t vocab);
+cudaError_t launch_accept(const AcceptParams& p, int32_t batch, ltd_dtype dtype, cudaStream_t s);
+
+struct CompactParams {
+  void* const* k_layers;
+  void* const* v_layers;
+  int32_t n_layers, hkv, s_cap;
+  int32_t row_bytes;
+  const int32_t* path;
+  int32_t path_stride;
+  const int32_t* accept_len;
+  const int32_t* ctx;
+  uint32_t* err;
+};
+cudaError_t launch_compact(const CompactParams& p, int32_t batch, cudaStream_t s);
+
+}  // namespace ltd

@@ -1,0 +1,328 @@
+"""Thin ctypes binding of ``libltd.so`` (the C ABI in ``include/ltd.h``).
+
+Functions carry the C names and only marshal arguments: torch tensors become
+device pointers, the current torch stream becomes the ``cudaStream_t``, and
+output tensors are allocated with torch.  Every step of the cycle runs in the
+library's CUDA kernels; there is no fallback of any kind -- if the library is
+missing or no GPU is present, calls raise.
+"""
+
+from __future__ import annotations
+
+import ctypes as C
+import os
+import threading
+
+import torch
+
+_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libltd.so")
+_lib = None
+_lock = threading.Lock()
+
+LTD_F32, LTD_BF16 = 0, 1
+LTD_GREEDY, LTD_STOCHASTIC = 0, 1
+LTD_MAX_K, LTD_MAX_DEPTH, LTD_MAX_N, LTD_MAX_TREE_NODES = 32, 16, 256, 4096
+DEVERR = {0x1: "LEVEL", 0x2: "NVERIFY", 0x4: "CTX", 0x8: "TREE", 0x10: "TIMEOUT", 0x20: "MODE"}
+
+# Every symbol declared in include/ltd.h.
+EXPORTS = [
+    "ltd_tree_bytes", "ltd_tree_init", "ltd_tree_reset", "ltd_expand_tree", "ltd_select_verify",
+    "ltd_attention_workspace_bytes", "ltd_tree_attention", "ltd_accept_workspace_bytes",
+    "ltd_accept", "ltd_kv_compact", "ltd_check", "ltd_status_string", "ltd_version",
+    "ltd_attention_kernel",
+]
+
+
+class LtdError(RuntimeError):
+    pass
+
+
+class ltd_tree(C.Structure):
+    _fields_ = [("batch", C.c_int32), ("max_depth", C.c_int32), ("k", C.c_int32),
+                ("max_nodes", C.c_int32), ("max_vocab", C.c_int64),
+                ("token", C.c_void_p), ("parent", C.c_void_p), ("depth", C.c_void_p),
+                ("cum_logprob", C.c_void_p), ("xrow", C.c_void_p), ("xlse", C.c_void_p),
+                ("frontier", C.c_void_p), ("n_nodes", C.c_void_p), ("n_levels", C.c_void_p),
+                ("scratch", C.c_void_p), ("scratch_bytes", C.c_size_t)]
+
+
+class ltd_kv_cache(C.Structure):
+    _fields_ = [("d_k_layers", C.c_void_p), ("d_v_layers", C.c_void_p),
+                ("n_layers", C.c_int32), ("hkv", C.c_int32), ("head_dim", C.c_int32),
+                ("s_cap", C.c_int32), ("dtype", C.c_int32)]
+
+
+def lib():
+    """Load libltd.so once; raise if it is not built."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(_LIB_PATH):
+                raise LtdError(f"{_LIB_PATH} is missing: build it with "
+                               "`python -c 'import __graft_entry__ as g; g.build()'`")
+            L = C.CDLL(_LIB_PATH)
+            vp, i32, i64, u64, sz = C.c_void_p, C.c_int32, C.c_int64, C.c_uint64, C.c_size_t
+            tp = C.POINTER(ltd_tree)
+            sig = {
+                "ltd_tree_bytes": (sz, [i32, i32, i32, i64]),
+                "ltd_tree_init": (C.c_int, [tp, vp, sz, i32, i32, i32, i64]),
+                "ltd_tree_reset": (C.c_int, [tp, vp, vp]),
+                "ltd_expand_tree": (C.c_int, [tp, i32, vp, C.c_int, i64, i64, vp, vp]),
+                "ltd_select_verify": (C.c_int, [tp, vp, i32, vp, vp, vp, vp, vp]),
+                "ltd_attention_workspace_bytes": (sz, [i32, i32, i32, i32, i32, i32, C.c_int]),
+                "ltd_tree_attention": (C.c_int, [vp, vp, vp, vp, C.c_int, i32, i32, i32, i32, i32,
+                                                 vp, i32, vp, i32, vp, C.c_float, vp, sz, vp]),
+                "ltd_accept_workspace_bytes": (sz, [i32, i32, i64]),
+                "ltd_accept": (C.c_int, [tp, vp, vp, C.c_int, i64, i64, vp, vp, i32, vp, u64, u64,
+                                         vp, vp, vp, vp, vp, C.POINTER(ltd_kv_cache), vp, sz, vp]),
+                "ltd_kv_compact": (C.c_int, [C.POINTER(ltd_kv_cache), i32, vp, i32, vp, vp, vp]),
+                "ltd_check": (C.c_int, [vp, C.POINTER(C.c_uint32)]),
+                "ltd_status_string": (C.c_char_p, [C.c_int]),
+                "ltd_version": (i32, []),
+                "ltd_attention_kernel": (i32, [C.c_int, i32, C.POINTER(i32)]),
+            }
+            for name, (res, args) in sig.items():
+                fn = getattr(L, name)
+                fn.restype = res
+                fn.argtypes = args
+            _lib = L
+    return _lib
+
+
+def _ok(status: int, what: str):
+    if status != 0:
+        raise LtdError(f"{what}: {lib().ltd_status_string(status).decode()}")
+
+
+def _stream(stream=None):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return C.c_void_p(s.cuda_stream)
+
+
+def _ptr(t):
+    return None if t is None else C.c_void_p(t.data_ptr())
+
+
+def _dtype(t: torch.Tensor) -> int:
+    if t.dtype == torch.bfloat16:
+        return LTD_BF16
+    if t.dtype == torch.float32:
+        return LTD_F32
+    raise LtdError(f"unsupported dtype {t.dtype}")
+
+
+def _need(t: torch.Tensor, name: str, dtype=None):
+    if not t.is_cuda:
+        raise LtdError(f"{name} must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise LtdError(f"{name} must be contiguous")
+    if dtype is not None and t.dtype != dtype:
+        raise LtdError(f"{name} must be {dtype}, got {t.dtype}")
+
+
+# ------------------------------------------------------------------ tree
+class Tree:
+    """A batch of draft trees in one torch-owned device buffer."""
+
+    def __init__(self, batch: int, max_depth: int, k: int, max_vocab: int, device="cuda"):
+        L = lib()
+        n = L.ltd_tree_bytes(batch, max_depth, k, max_vocab)
+        if n == 0:
+            raise LtdError("ltd_tree_bytes: bad tree dimensions")
+        self.buf = torch.empty(n + 256, dtype=torch.uint8, device=device)
+        off = (-self.buf.data_ptr()) % 256
+        self.mem = self.buf[off:off + n]
+        self.s = ltd_tree()
+        _ok(L.ltd_tree_init(C.byref(self.s), C.c_void_p(self.mem.data_ptr()), n, batch, max_depth,
+                            k, max_vocab), "ltd_tree_init")
+
+    @property
+    def batch(self):
+        return self.s.batch
+
+    @property
+    def k(self):
+        return self.s.k
+
+    @property
+    def max_depth(self):
+        return self.s.max_depth
+
+    @property
+    def max_nodes(self):
+        return self.s.max_nodes
+
+    def _view(self, ptr, count, dtype):
+        off = ptr - self.mem.data_ptr()
+        nbytes = count * 4
+        return self.mem[off:off + nbytes].view(dtype)
+
+    def view(self) -> dict:
+        """Device views of the tree arrays ([batch][max_nodes] etc.)."""
+        B, mn, k = self.batch, self.max_nodes, self.k
+        s = self.s
+        i32, f32 = torch.int32, torch.float32
+        return {
+            "token": self._view(s.token, B * mn, i32).view(B, mn),
+            "parent": self._view(s.parent, B * mn, i32).view(B, mn),
+            "depth": self._view(s.depth, B * mn, i32).view(B, mn),
+            "cum_logprob": self._view(s.cum_logprob, B * mn, f32).view(B, mn),
+            "xrow": self._view(s.xrow, B * mn, i32).view(B, mn),
+            "xlse": self._view(s.xlse, B * mn, f32).view(B, mn),
+            "frontier": self._view(s.frontier, B * k, i32).view(B, k),
+            "n_nodes": self._view(s.n_nodes, B, i32),
+            "n_levels": self._view(s.n_levels, B, i32),
+        }
+
+
+def ltd_tree_reset(tree: Tree, root_tokens: torch.Tensor, stream=None):
+    _need(root_tokens, "root_tokens", torch.int32)
+    _ok(lib().ltd_tree_reset(C.byref(tree.s), _ptr(root_tokens), _stream(stream)), "ltd_tree_reset")
+
+
+def ltd_expand_tree(tree: Tree, level: int, draft_rows: torch.Tensor, active=None, stream=None):
+    """draft_rows: [batch][rows_per_seq][vocab] bf16/f32."""
+    _need(draft_rows, "draft_rows")
+    if active is not None:
+        _need(active, "active", torch.int32)
+    B, R, V = draft_rows.shape
+    _ok(lib().ltd_expand_tree(C.byref(tree.s), level, _ptr(draft_rows), _dtype(draft_rows), V, R,
+                              _ptr(active), _stream(stream)), "ltd_expand_tree")
+
+
+def ltd_select_verify(tree: Tree, n_verify: torch.Tensor, n_max: int, ctx: torch.Tensor,
+                      out=None, stream=None):
+    """Returns (node_ids [B][n_max], pos [B][n_max], mask [B][n_max][ceil(n_max/32)])."""
+    _need(n_verify, "n_verify", torch.int32)
+    _need(ctx, "ctx", torch.int32)
+    B = tree.batch
+    w32 = (n_max + 31) // 32
+    dev = n_verify.device
+    if out is None:
+        out = (torch.empty(B, n_max, dtype=torch.int32, device=dev),
+               torch.empty(B, n_max, dtype=torch.int32, device=dev),
+               torch.empty(B, n_max, w32, dtype=torch.int32, device=dev))
+    ids, pos, mask = out
+    _ok(lib().ltd_select_verify(C.byref(tree.s), _ptr(n_verify), n_max, _ptr(ctx), _ptr(ids),
+                                _ptr(pos), _ptr(mask), _stream(stream)), "ltd_select_verify")
+    return ids, pos, mask
+
+
+def attention_workspace(batch, hq, hkv, head_dim, n_max, max_ctx, dtype, device="cuda"):
+    n = lib().ltd_attention_workspace_bytes(batch, hq, hkv, head_dim, n_max, max_ctx,
+                                            LTD_BF16 if dtype == torch.bfloat16 else LTD_F32)
+    if n == 0:
+        raise LtdError("ltd_attention_workspace_bytes: bad sizes")
+    return torch.zeros(n, dtype=torch.uint8, device=device)
+
+
+def ltd_tree_attention(q, k_cache, v_cache, ctx, max_ctx, n_verify, mask, scale=None,
+                       out=None, workspace=None, stream=None):
+    """q [B][n_max][hq][d]; k/v [B][hkv][s_cap][d]; returns out like q."""
+    for t, n in ((q, "q"), (k_cache, "k_cache"), (v_cache, "v_cache")):
+        _need(t, n, q.dtype)
+    _need(ctx, "ctx", torch.int32)
+    _need(n_verify, "n_verify", torch.int32)
+    _need(mask, "mask")
+    B, n_max, hq, d = q.shape
+    hkv, s_cap = k_cache.shape[1], k_cache.shape[2]
+    if scale is None:
+        scale = d ** -0.5
+    if out is None:
+        out = torch.zeros_like(q)
+    if workspace is None:
+        workspace = attention_workspace(B, hq, hkv, d, n_max, max_ctx, q.dtype, q.device)
+    _ok(lib().ltd_tree_attention(_ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(out), _dtype(q), B,
+                                 hq, hkv, d, s_cap, _ptr(ctx), max_ctx, _ptr(n_verify), n_max,
+                                 _ptr(mask), float(scale), _ptr(workspace), workspace.numel(),
+                                 _stream(stream)), "ltd_tree_attention")
+    return out
+
+
+def accept_workspace(batch, n_max, vocab, device="cuda"):
+    n = lib().ltd_accept_workspace_bytes(batch, n_max, vocab)
+    if n == 0:
+        raise LtdError("ltd_accept_workspace_bytes: bad sizes")
+    return torch.zeros(n, dtype=torch.uint8, device=device)
+
+
+class KVCache:
+    """Per-layer K/V tensors [B][hkv][s_cap][d] plus the device pointer arrays
+    ltd_kv_compact reads."""
+
+    def __init__(self, k_layers, v_layers):
+        self.k_layers, self.v_layers = list(k_layers), list(v_layers)
+        dev = self.k_layers[0].device
+        self.k_ptrs = torch.tensor([t.data_ptr() for t in self.k_layers], dtype=torch.int64, device=dev)
+        self.v_ptrs = torch.tensor([t.data_ptr() for t in self.v_layers], dtype=torch.int64, device=dev)
+        k0 = self.k_layers[0]
+        self.s = ltd_kv_cache(C.c_void_p(self.k_ptrs.data_ptr()), C.c_void_p(self.v_ptrs.data_ptr()),
+                              len(self.k_layers), k0.shape[1], k0.shape[3], k0.shape[2], _dtype(k0))
+
+
+def ltd_accept(tree: Tree, target, draft_rows, node_ids, n_verify, mode, ctx, seed=0, cycle=0,
+               kv: KVCache | None = None, workspace=None, out=None, stream=None):
+    """Returns dict(path [B][max_depth+1], accept_len [B], bonus [B], new_ctx [B])."""
+    _need(target, "target")
+    _need(draft_rows, "draft_rows", target.dtype)
+    for t, n in ((node_ids, "node_ids"), (n_verify, "n_verify"), (mode, "mode"), (ctx, "ctx")):
+        _need(t, n, torch.int32)
+    B, n_max, V = target.shape
+    R = draft_rows.shape[1]
+    dev = target.device
+    if workspace is None:
+        workspace = accept_workspace(B, n_max, V, dev)
+    if out is None:
+        out = {"path": torch.empty(B, tree.max_depth + 1, dtype=torch.int32, device=dev),
+               "accept_len": torch.empty(B, dtype=torch.int32, device=dev),
+               "bonus": torch.empty(B, dtype=torch.int32, device=dev),
+               "new_ctx": torch.empty(B, dtype=torch.int32, device=dev)}
+    kvp = C.byref(kv.s) if kv is not None else None
+    _ok(lib().ltd_accept(C.byref(tree.s), _ptr(target), _ptr(draft_rows), _dtype(target), V, R,
+                         _ptr(node_ids), _ptr(n_verify), n_max, _ptr(mode), seed, cycle, _ptr(ctx),
+                         _ptr(out["new_ctx"]), _ptr(out["path"]), _ptr(out["accept_len"]),
+                         _ptr(out["bonus"]), kvp, _ptr(workspace), workspace.numel(),
+                         _stream(stream)), "ltd_accept")
+    return out
+
+
+def ltd_kv_compact(kv: KVCache, path, accept_len, ctx, stream=None):
+    _need(path, "path", torch.int32)
+    _ok(lib().ltd_kv_compact(C.byref(kv.s), path.shape[0], _ptr(path), path.shape[1],
+                             _ptr(accept_len), _ptr(ctx), _stream(stream)), "ltd_kv_compact")
+
+
+def ltd_check(stream=None, raise_on_error=True) -> int:
+    """Synchronise, read and clear the device error word; returns its bits."""
+    bits = C.c_uint32(0)
+    st = lib().ltd_check(_stream(stream), C.byref(bits))
+    if raise_on_error and st != 0:
+        names = [v for k, v in DEVERR.items() if bits.value & k]
+        raise LtdError(f"ltd_check: {lib().ltd_status_string(st).decode()} {names}")
+    return bits.value
+
+
+def ltd_version() -> int:
+    return lib().ltd_version()
+
+
+def ltd_attention_kernel(head_dim: int, dtype) -> tuple:
+    """(1 tensor cores / 0 CUDA cores / -1 unsupported, launches per call)."""
+    n = C.c_int32(0)
+    code = lib().ltd_attention_kernel(LTD_BF16 if dtype == torch.bfloat16 else LTD_F32, head_dim,
+                                      C.byref(n))
+    return code, n.value
+
+
+def attention_launches(head_dim: int, dtype) -> int:
+    return ltd_attention_kernel(head_dim, dtype)[1]
+
+
+def attention_kernel_tag(head_dim: int, dtype) -> str:
+    return "attn_tc" if ltd_attention_kernel(head_dim, dtype)[0] == 1 else "attn_simt"
+
+
+def attention_kernel_sources(head_dim: int, dtype) -> list:
+    """Source files of the attention kernel this call dispatches to."""
+    main = "k_attn_tc.cu" if ltd_attention_kernel(head_dim, dtype)[0] == 1 else "k_attn_simt.cu"
+    return [main, "ltd_common.cuh"]

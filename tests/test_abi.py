@@ -1,0 +1,100 @@
+"""libltd.so loads, exports every function include/ltd.h declares, and rejects
+bad arguments on the host before touching a GPU (no compute calls here)."""
+
+import ctypes as C
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def L():
+    from paper_2603_01639_gb300 import build, ltd
+    build.build()
+    return ltd.lib()
+
+
+def _declared():
+    with open(os.path.join(ROOT, "include", "ltd.h")) as f:
+        text = f.read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(ltd_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_every_declared_symbol_is_exported(L):
+    from paper_2603_01639_gb300 import ltd
+    declared = _declared()
+    assert declared, "no declarations parsed"
+    for name in declared:
+        assert hasattr(L, name), f"{name} declared in ltd.h but not exported"
+    assert sorted(ltd.EXPORTS) == declared
+
+
+def test_version_and_status_strings(L):
+    assert L.ltd_version() == 100
+    for s, name in enumerate(["LTD_OK", "LTD_ERR_INVALID_ARG", "LTD_ERR_SHAPE",
+                              "LTD_ERR_UNSUPPORTED", "LTD_ERR_CUDA", "LTD_ERR_DEVICE",
+                              "LTD_ERR_TIMEOUT"]):
+        assert L.ltd_status_string(s).decode() == name
+
+
+def test_tree_bytes_and_init_validate_on_host(L):
+    from paper_2603_01639_gb300 import ltd
+    assert L.ltd_tree_bytes(1, 6, 10, 128256) > 0
+    assert L.ltd_tree_bytes(0, 6, 10, 128256) == 0
+    assert L.ltd_tree_bytes(1, 17, 10, 128256) == 0          # depth over LTD_MAX_DEPTH
+    assert L.ltd_tree_bytes(1, 6, 33, 128256) == 0           # k over LTD_MAX_K
+    assert L.ltd_tree_bytes(1, 16, 32, 128256) == 0          # more than 4096 nodes
+    assert L.ltd_tree_bytes(1, 3, 8, 4) == 0                 # k > vocab
+    t = ltd.ltd_tree()
+    n = L.ltd_tree_bytes(2, 3, 4, 1000)
+    assert L.ltd_tree_init(None, C.c_void_p(256), n, 2, 3, 4, 1000) == 1
+    assert L.ltd_tree_init(C.byref(t), None, n, 2, 3, 4, 1000) == 1
+    assert L.ltd_tree_init(C.byref(t), C.c_void_p(257), n, 2, 3, 4, 1000) == 1  # misaligned
+    assert L.ltd_tree_init(C.byref(t), C.c_void_p(4096), n - 1, 2, 3, 4, 1000) == 2
+    # carving is pure pointer arithmetic on the host
+    assert L.ltd_tree_init(C.byref(t), C.c_void_p(1 << 20), n, 2, 3, 4, 1000) == 0
+    assert t.max_nodes == 1 + 4 + 2 * 16
+    ptrs = [t.token, t.parent, t.depth, t.cum_logprob, t.xrow, t.xlse, t.frontier, t.n_nodes,
+            t.n_levels, t.scratch]
+    assert all(p % 256 == 0 for p in ptrs)
+    assert ptrs == sorted(ptrs) and ptrs[-1] + t.scratch_bytes <= (1 << 20) + n
+
+
+def test_entry_points_reject_bad_arguments_before_launch(L):
+    from paper_2603_01639_gb300 import ltd
+    t = ltd.ltd_tree()
+    n = L.ltd_tree_bytes(1, 3, 4, 1000)
+    assert L.ltd_tree_init(C.byref(t), C.c_void_p(1 << 20), n, 1, 3, 4, 1000) == 0
+    fake = C.c_void_p(1 << 24)
+    s = C.c_void_p(0)
+    assert L.ltd_tree_reset(None, fake, s) == 1
+    assert L.ltd_tree_reset(C.byref(t), None, s) == 1
+    assert L.ltd_expand_tree(C.byref(t), 0, fake, 0, 1000, 9, None, s) == 2       # level 0
+    assert L.ltd_expand_tree(C.byref(t), 4, fake, 0, 1000, 9, None, s) == 2       # > max_depth
+    assert L.ltd_expand_tree(C.byref(t), 1, fake, 0, 1001, 9, None, s) == 2       # > max_vocab
+    assert L.ltd_expand_tree(C.byref(t), 1, fake, 0, 1000, 8, None, s) == 2       # row store short
+    assert L.ltd_expand_tree(C.byref(t), 1, fake, 7, 1000, 9, None, s) == 1       # bad dtype
+    assert L.ltd_expand_tree(C.byref(t), 1, fake, 1, 996, 9, None, s) == 2        # bf16 row not 16B
+    assert L.ltd_select_verify(C.byref(t), fake, 257, fake, fake, fake, fake, s) == 2
+    assert L.ltd_select_verify(C.byref(t), None, 8, fake, fake, fake, fake, s) == 1
+    ws = L.ltd_attention_workspace_bytes(1, 4, 1, 64, 8, 128, 0)
+    assert ws > 0
+    assert L.ltd_attention_workspace_bytes(1, 5, 2, 64, 8, 128, 0) == 0          # hq % hkv
+    args = [fake, fake, fake, fake, 0, 1, 4, 1, 64, 256, fake, 128, fake, 8, fake, 0.125, fake, ws, s]
+    bad = list(args); bad[8] = 80                                                  # head_dim
+    assert L.ltd_tree_attention(*bad) == 3
+    bad = list(args); bad[9] = 130                                                 # s_cap < ctx + n
+    assert L.ltd_tree_attention(*bad) == 2
+    bad = list(args); bad[17] = ws - 1
+    assert L.ltd_tree_attention(*bad) == 2
+    bad = list(args); bad[15] = 0.0
+    assert L.ltd_tree_attention(*bad) == 1
+    assert L.ltd_accept_workspace_bytes(1, 8, 1000) > 0
+    assert L.ltd_accept_workspace_bytes(1, 300, 1000) == 0
+    kv = ltd.ltd_kv_cache(fake, fake, 1, 1, 70, 256, 1)                            # 140-byte rows
+    assert L.ltd_kv_compact(C.byref(kv), 1, fake, 4, fake, fake, s) == 3
+    assert L.ltd_kv_compact(None, 1, fake, 4, fake, fake, s) == 1

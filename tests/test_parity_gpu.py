@@ -1,0 +1,271 @@
+"""GPU (C ABI) vs oracle parity on the seeded workloads, plus edge cases.
+
+Sizes: the tiny workload end to end; the draft, selection and acceptance of
+every workload at full size (vocab 32k-152k, trees up to 711 nodes, batch 16
+ragged); tree attention at full size for one layer, compared on every output
+where the oracle is affordable and on sampled KV heads for the 32B and 70B
+shapes.
+"""
+
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2603_01639_gb300 import ltd
+from paper_2603_01639_gb300 import workload as wl
+
+from . import harness as H
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2603_01639_gb300 import build
+    build.build()
+    ltd.lib()
+    torch.cuda.init()
+
+
+def _draft_select_accept(name, seed, cycle_no=0, acc_seed=1234):
+    cfg = wl.config(name)
+    ci = wl.draw_cycle(cfg, seed)
+    trees, sels, target = H.oracle_side(cfg, ci)
+    draft = H.dev(ci.draft_rows, cfg.dtype)
+    tree = H.gpu_draft(cfg, ci, draft)
+    cut = H.compare_trees(cfg, ci, tree, trees)
+    assert cut > H.CUT_MARGIN, f"near-tie at a frontier cut ({cut}); pick another seed"
+    got = H.gpu_select(cfg, ci, tree)
+    sel_margin = H.compare_select(cfg, ci, got, sels)
+    assert sel_margin > H.CUT_MARGIN
+    ref = H.oracle_accept(cfg, ci, trees, sels, target, acc_seed, cycle_no)
+    assert H.stochastic_margins_ok(ref), "near-tie in a stochastic decision; pick another seed"
+    tgt = H.dev(target, cfg.dtype)
+    out = ltd.ltd_accept(tree, tgt, draft, got[0], H.i32(ci.n_verify), H.i32(ci.mode),
+                         H.i32(ci.ctx), seed=acc_seed, cycle=cycle_no)
+    assert ltd.ltd_check() == 0
+    H.compare_accept(cfg, out, ref)
+    return cfg, ci, ref
+
+
+# ------------------------------------------------------------ draft/select/accept
+def test_tiny_cycle():
+    cfg, ci, ref = _draft_select_accept("tiny", 0)
+    assert 0 <= ref[0]["accept_len"] <= 3
+
+
+@pytest.mark.parametrize("seed", [0, 1])
+def test_8b_cycle_full_size(seed):
+    cfg, ci, ref = _draft_select_accept("8b", seed)
+    assert ref[0]["accept_len"] >= 0
+
+
+@pytest.mark.parametrize("seed", [0, 1, 2, 3, 4])
+def test_13b_stochastic_cycles(seed):
+    _draft_select_accept("13b", seed, cycle_no=seed)
+
+
+def test_32b_cycle_full_size():
+    _draft_select_accept("32b", 0)
+
+
+def test_70b_batched_ragged_mixed():
+    cfg, ci, ref = _draft_select_accept("70b", 0)
+    assert set(ci.mode.tolist()) == {0, 1}
+    assert len(set(ci.depth.tolist())) > 1 and len(set(ci.ctx.tolist())) > 1
+
+
+def test_determinism_and_reuse_of_scratch():
+    """Same inputs twice through the same tree and workspace: identical bits
+    (tickets and scratch are left ready for reuse)."""
+    cfg = wl.config("8b")
+    ci = wl.draw_cycle(cfg, 5)
+    draft = H.dev(ci.draft_rows, cfg.dtype)
+    tree = H.gpu_draft(cfg, ci, draft)
+    a = {k: v.clone() for k, v in tree.view().items()}
+    H.gpu_draft(cfg, ci, draft, tree)
+    b = tree.view()
+    for k in a:
+        assert torch.equal(a[k], b[k]), k
+
+
+# --------------------------------------------------------------------- edge cases
+def _small_tree(W, L, vocab, seed, dtype=wl.F32):
+    rng = np.random.default_rng(seed)
+    R = 1 + (L - 1) * W
+    rows = wl.round_to(rng.standard_normal((1, R, vocab)).astype(np.float32), dtype)
+    root = int(rng.integers(vocab))
+    ci = wl.CycleInputs(wl.config("tiny", W=W, vocab=vocab, depth_range=(L, L), dtype=dtype),
+                        seed, np.array([root], np.int32), np.array([L], np.int32),
+                        np.array([1], np.int32), np.array([0], np.int32),
+                        np.array([0], np.int32), rows)
+    return ci
+
+
+@pytest.mark.parametrize("W,L,vocab", [(1, 6, 64), (2, 1, 8), (3, 4, 24), (32, 2, 4096),
+                                       (5, 3, 1000 + 8 * 37)])
+def test_expand_and_select_shapes(W, L, vocab):
+    """k = 1 chains, a single level, k = 32, vocab not a multiple of the chunk."""
+    ci = _small_tree(W, L, vocab, seed=W * 7 + L)
+    cfg = ci.cfg
+    tree = H.gpu_draft(cfg, ci, H.dev(ci.draft_rows, wl.F32))
+    otree = oracle.grow_tree(int(ci.root[0]), ci.draft_rows[0], W, L)
+    H.compare_trees(cfg, ci, tree, [otree])
+    n = otree.n_nodes
+    for N in sorted({1, 2, min(7, n), min(n, ltd.LTD_MAX_N)}):
+        ids, pos, mask = ltd.ltd_select_verify(tree, H.i32([N]), max(N, 1), H.i32([11]))
+        rids, rpos, rmask, _ = oracle.select_verify(otree, N, 11)
+        assert ids.cpu().numpy()[0].tolist() == rids.tolist()
+        assert pos.cpu().numpy()[0].tolist() == rpos.tolist()
+        words = oracle.mask_words(rmask)
+        assert np.array_equal(mask.cpu().numpy()[0].view(np.uint32), words)
+        if W == 1:
+            assert np.array_equal(rmask, np.tril(np.ones((N, N), bool)))
+
+
+def test_single_node_verify_is_autoregressive():
+    cfg = wl.config("tiny")
+    ci = wl.draw_cycle(cfg, 3)
+    ci.n_verify[:] = 1
+    draft = H.dev(ci.draft_rows, cfg.dtype)
+    tree = H.gpu_draft(cfg, ci, draft)
+    ids, pos, mask = H.gpu_select(cfg, ci, tree)
+    tgt = torch.randn(1, cfg.max_n, cfg.vocab, device="cuda")
+    out = ltd.ltd_accept(tree, tgt, draft, ids, H.i32([1]), H.i32([0]), H.i32(ci.ctx))
+    assert out["accept_len"].item() == 0
+    assert out["bonus"].item() == int(torch.argmax(tgt[0, 0]).item())
+    assert out["new_ctx"].item() == int(ci.ctx[0]) + 1
+
+
+def test_device_flags_bad_per_sequence_sizes():
+    """N larger than the tree is a device-side error: flagged, not trapped, and
+    the context stays usable."""
+    cfg = wl.config("tiny")
+    ci = wl.draw_cycle(cfg, 4)
+    draft = H.dev(ci.draft_rows, cfg.dtype)
+    tree = H.gpu_draft(cfg, ci, draft)
+    ltd.ltd_check()
+    ids, pos, mask = ltd.ltd_select_verify(tree, H.i32([12]), 16, H.i32(ci.ctx))  # V_all = 11
+    bits = ltd.ltd_check(raise_on_error=False)
+    assert bits & 0x2
+    assert (ids == -1).all()
+    # expanding out of order is flagged too
+    ltd.ltd_expand_tree(tree, 2, draft)
+    assert ltd.ltd_check(raise_on_error=False) & 0x1
+    # and the device still works
+    tree = H.gpu_draft(cfg, ci, draft)
+    assert ltd.ltd_check() == 0
+
+
+def test_compaction_race_pattern_and_untouched_rows():
+    B, hkv, s_cap, d, layers = 2, 3, 64, 128, 2
+    g = torch.Generator(device="cuda").manual_seed(0)
+    ks = [torch.randn(B, hkv, s_cap, d, device="cuda", generator=g).to(torch.bfloat16)
+          for _ in range(layers)]
+    vs = [torch.randn(B, hkv, s_cap, d, device="cuda", generator=g).to(torch.bfloat16)
+          for _ in range(layers)]
+    before_k = [k.cpu().float().numpy() for k in ks]
+    before_v = [v.cpu().float().numpy() for v in vs]
+    kv = ltd.KVCache(ks, vs)
+    path = H.i32([[0, 2, 3, -1, -1], [0, 1, 4, 6, 9]])
+    alen = H.i32([2, 4])
+    ctx = H.i32([10, 20])
+    ltd.ltd_kv_compact(kv, path, alen, ctx)
+    assert ltd.ltd_check() == 0
+    for arrs, before in ((ks, before_k), (vs, before_v)):
+        for l in range(layers):
+            got = arrs[l].cpu().float().numpy()
+            for b, (c, p, a) in enumerate([(10, [0, 2, 3], 2), (20, [0, 1, 4, 6, 9], 4)]):
+                ref = oracle.compact_kv(before[l][b], c, p[:a + 1])
+                assert np.array_equal(got[b], ref)
+
+
+# ---------------------------------------------------------------------- attention
+def _attention_case(name, seed, heads=None, seqs=None):
+    cfg = wl.config(name)
+    ci = wl.draw_cycle(cfg, seed, draft_rows=False)
+    rng = np.random.default_rng(seed + 5)
+    masks = []
+    for b in range(cfg.batch):
+        # a random valid tree over the verified slots: parent slot < slot
+        N = int(ci.n_verify[b])
+        par = [-1] + [int(rng.integers(0, i)) for i in range(1, N)]
+        m = np.zeros((N, N), bool)
+        for i in range(N):
+            a = i
+            while a >= 0:
+                m[i, a] = True
+                a = par[a]
+        masks.append(m)
+    q, k, v = wl.draw_attention(cfg, seed, ci.ctx, ci.n_verify)
+    W32 = (cfg.max_n + 31) // 32
+    mw = np.zeros((cfg.batch, cfg.max_n, W32), np.uint32)
+    for b in range(cfg.batch):
+        w = oracle.mask_words(masks[b])
+        mw[b, :w.shape[0], :w.shape[1]] = w
+    qd, kd, vd = H.dev(q, cfg.dtype), H.dev(k, cfg.dtype), H.dev(v, cfg.dtype)
+    out = ltd.ltd_tree_attention(qd, kd, vd, H.i32(ci.ctx), cfg.max_ctx, H.i32(ci.n_verify),
+                                 torch.from_numpy(mw.view(np.int32)).cuda())
+    assert ltd.ltd_check() == 0
+    got = out.float().cpu().numpy()
+    G = cfg.hq // cfg.hkv
+    scale = 1.0 / math.sqrt(cfg.head_dim)
+    worst_max, worst_mean = 0.0, 0.0
+    for b in (seqs if seqs is not None else range(cfg.batch)):
+        N, c = int(ci.n_verify[b]), int(ci.ctx[b])
+        for kvh in (heads if heads is not None else range(cfg.hkv)):
+            hs = list(range(kvh * G, kvh * G + G))
+            ref = oracle.tree_attention(q[b, :N][:, hs], k[b, kvh:kvh + 1], v[b, kvh:kvh + 1], c,
+                                        masks[b], scale)
+            mx, mn = H.attention_error(got[b, :N][:, hs], ref)
+            worst_max, worst_mean = max(worst_max, mx), max(worst_mean, mn)
+        # rows past N are untouched (zeros from torch.zeros_like)
+        assert not got[b, N:].any()
+    tol_max, tol_mean = H.ATT_TOL[cfg.dtype]
+    assert worst_max <= tol_max and worst_mean <= tol_mean, (worst_max, worst_mean)
+    return worst_max, worst_mean
+
+
+def test_attention_tiny():
+    _attention_case("tiny", 0)
+
+
+@pytest.mark.parametrize("seed", [0, 1])
+def test_attention_8b_layer(seed):
+    _attention_case("8b", seed)
+
+
+def test_attention_13b_mha():
+    _attention_case("13b", 2)
+
+
+def test_attention_32b_sampled_heads():
+    _attention_case("32b", 0, heads=[0, 7])
+
+
+def test_attention_70b_sampled():
+    _attention_case("70b", 0, heads=[3], seqs=[0, 5, 11, 15])
+
+
+def test_attention_all_ones_mask_equals_unmasked():
+    cfg = wl.config("8b", ctx_range=(300, 300), n_choices=(40,))
+    rng = np.random.default_rng(3)
+    q = wl.round_to(rng.standard_normal((1, 40, cfg.hq, 128)).astype(np.float32), wl.BF16)
+    k = wl.round_to(rng.standard_normal((1, cfg.hkv, cfg.s_cap, 128)).astype(np.float32), wl.BF16)
+    v = wl.round_to(rng.standard_normal((1, cfg.hkv, cfg.s_cap, 128)).astype(np.float32), wl.BF16)
+    ones = np.full((1, 40, 2), 0xFFFFFFFF, np.uint32)
+    ones[..., 1] = (1 << 8) - 1
+    out = ltd.ltd_tree_attention(H.dev(q, wl.BF16), H.dev(k, wl.BF16), H.dev(v, wl.BF16),
+                                 H.i32([300]), 300, H.i32([40]),
+                                 torch.from_numpy(ones.view(np.int32)).cuda())
+    G = cfg.hq // cfg.hkv
+    ref = torch.nn.functional.scaled_dot_product_attention(
+        torch.from_numpy(q[0].astype(np.float64)).transpose(0, 1),
+        torch.from_numpy(np.repeat(k[0, :, :340], G, 0).astype(np.float64)),
+        torch.from_numpy(np.repeat(v[0, :, :340], G, 0).astype(np.float64)),
+        scale=1 / math.sqrt(128)).transpose(0, 1).numpy()
+    mx, mn = H.attention_error(out[0].float().cpu().numpy(), ref)
+    assert mx <= 2e-2 and mn <= 2e-3

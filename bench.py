@@ -178,9 +178,13 @@ class Cycle:
                             self.mode, self.ctx, seed=1234, cycle=cycle_no, kv=self.kv,
                             workspace=self.acc_ws, out=self.acc)
 
+    def attention_kernel(self):
+        cfg = self.cfg
+        return self.ltd.ltd_attention_kernel(self.tdt, cfg.batch, cfg.hq, cfg.hkv, cfg.head_dim,
+                                             cfg.max_n, cfg.max_ctx)
+
     def launches_per_step(self):
-        return 1 + self.max_depth + 1 + self.layers * self.ltd.attention_launches(
-            self.cfg.head_dim, self.tdt) + 2
+        return 1 + self.max_depth + 1 + self.layers * self.attention_kernel()[1] + 2
 
     # algorithmic bytes / flops of one attention launch
     def attention_algorithmic(self):
@@ -392,8 +396,9 @@ def run_ours(args):
     except (OSError, ValueError, KeyError):
         hbm_peak, peak_note = 6800.0, "fallback"
     achieved = att_bytes / (att_launch_ms * 1e-3) / 1e9
-    tag = ltd.attention_kernel_tag(cfg.head_dim, cyc.tdt)
-    sha = _source_sha(ltd.attention_kernel_sources(cfg.head_dim, cyc.tdt))
+    code, _ = cyc.attention_kernel()
+    tag = "attn_tc" if code == 1 else "attn_simt"
+    sha = _source_sha(ltd.attention_kernel_sources(code))
     traffic = _traffic_from_profiles(f"{tag}:{cfg.name}", sha)
     roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": hbm_peak,
                 "unit": "GB/s", "frac": round(achieved / hbm_peak, 4), "traffic": traffic,

@@ -174,11 +174,12 @@ ltd_status ltd_tree_attention(const void* d_q, const void* d_k, const void* d_v,
                               const uint32_t* d_mask, float scale, void* d_workspace,
                               size_t workspace_bytes, ltd_stream_t stream);
 
-/* Which kernel ltd_tree_attention runs for this dtype and head_dim:
- * returns 1 for the tcgen05 tensor-core kernel, 0 for the CUDA-core kernel,
- * -1 if the combination is unsupported.  *launches (if not NULL) receives
- * the number of kernel launches one ltd_tree_attention call makes. */
-int32_t ltd_attention_kernel(ltd_dtype dtype, int32_t head_dim, int32_t* launches);
+/* Which kernel ltd_tree_attention runs for these sizes: returns 1 for the
+ * tcgen05 tensor-core kernel, 0 for the CUDA-core kernel, -1 if the sizes are
+ * unsupported.  *launches (if not NULL) receives the number of kernel
+ * launches one ltd_tree_attention call with these sizes makes. */
+int32_t ltd_attention_kernel(ltd_dtype dtype, int32_t batch, int32_t hq, int32_t hkv,
+                             int32_t head_dim, int32_t n_max, int32_t max_ctx, int32_t* launches);
 
 /* KV cache views for compaction: device arrays of n_layers device pointers,
  * each layer [batch][hkv][s_cap][head_dim] of dtype. */
@@ -235,6 +236,17 @@ ltd_status ltd_accept(const ltd_tree* tree, const void* d_target_logits,
 ltd_status ltd_kv_compact(const ltd_kv_cache* kv, int32_t batch, const int32_t* d_path,
                           int32_t path_stride, const int32_t* d_accept_len,
                           const int32_t* d_ctx, ltd_stream_t stream);
+
+/* Diagnostic of the tensor-core building blocks the attention kernel uses
+ * (TMA with 128-byte swizzle, tcgen05.mma from shared-memory descriptors
+ * into tensor memory, tcgen05.ld): one 128x128x128 bf16 GEMM with fp32
+ * output.  mode 0: C = A B^T with B stored [N][K]; mode 1: C = A B with B
+ * stored [K][N].  d_a, d_b row-major bf16 [128][128], d_c row-major fp32
+ * [128][128], all 16-byte aligned device memory.  No counterpart in the
+ * paper: it exists so a driver or toolkit change that breaks these
+ * instructions shows up as a wrong product, not a wrong attention. */
+ltd_status ltd_selftest_umma(int32_t mode, const void* d_a, const void* d_b, float* d_c,
+                             ltd_stream_t stream);
 
 /* Synchronise the stream, read and clear this device's error word.
  * Returns LTD_OK, LTD_ERR_TIMEOUT, LTD_ERR_DEVICE or LTD_ERR_CUDA; if

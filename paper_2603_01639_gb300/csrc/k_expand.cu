@@ -4,7 +4,7 @@
 // (chunks, F, batch) with F = 1 at level 1 and F = k afterwards: each CTA
 // scans one vocabulary chunk of one frontier row with 16-byte streaming loads,
 // computing the chunk's (max, sum exp) and its top-k (logit desc, token asc)
-// in registers.  The last CTA to finish a row (atomic ticket; nothing spins)
+// in warp-distributed lists (lane i holds the i-th best key).  The last CTA to finish a row (atomic ticket; nothing spins)
 // merges the chunk partials in a fixed order into the row's log-sum-exp and
 // top-k, appends the k children with cum = cum(parent) + x - lse, and the
 // last row of a sequence picks the new frontier: the k best of the k^2 pool
@@ -39,17 +39,18 @@ __global__ void tree_reset_kernel(ltd_tree t, const int32_t* __restrict__ roots,
   seq_ticket[b] = 0u;
 }
 
-template <typename T, int K>
+template <typename T>
 __global__ void __launch_bounds__(kNT) expand_kernel(const ExpandParams p) {
   constexpr int NW = kNT / kWarp;
   constexpr int VEC = 16 / sizeof(T);
   constexpr int U = 4;
   __shared__ float red[2 * NW];
-  __shared__ uint64_t stage[NW * K];
-  __shared__ uint64_t best[K];
+  __shared__ uint64_t stage[NW * kWarp];
+  __shared__ uint64_t best[kWarp];
   __shared__ int s_last;
 
   const int ch = blockIdx.x, f = blockIdx.y, b = blockIdx.z, tid = threadIdx.x;
+  const int lane = tid & 31, warp = tid >> 5;
   if (p.active != nullptr && p.active[b] == 0) return;
   if (p.n_levels[b] != p.level - 1) {
     if (tid == 0 && ch == 0 && f == 0) flag_error(p.err, LTD_DEVERR_LEVEL);
@@ -64,14 +65,16 @@ __global__ void __launch_bounds__(kNT) expand_kernel(const ExpandParams p) {
   const int64_t hi = min(lo + p.chunk_elems, p.vocab);
 
   float m = -CUDART_INF_F, s = 0.f;
-  TopK<K> tk;
-  tk.init();
-  for (int64_t base = lo + static_cast<int64_t>(tid) * VEC; base < hi;
-       base += static_cast<int64_t>(kNT) * VEC * U) {
+  WarpTopK wt;
+  wt.init();
+  // every lane of a warp runs the same number of iterations (offer() is
+  // warp-collective); out-of-range slots offer the empty key 0
+  for (int64_t wbase = lo + static_cast<int64_t>(warp) * kWarp * VEC; wbase < hi;
+       wbase += static_cast<int64_t>(kNT) * VEC * U) {
     float xv[U][VEC];
 #pragma unroll
     for (int u = 0; u < U; ++u) {
-      const int64_t i = base + static_cast<int64_t>(u) * kNT * VEC;
+      const int64_t i = wbase + (static_cast<int64_t>(u) * kNT + lane) * VEC;
       if (i + VEC <= hi) {
         unpack16(ld_stream16(x + i), xv[u], static_cast<const T*>(nullptr));
       } else {
@@ -81,7 +84,7 @@ __global__ void __launch_bounds__(kNT) expand_kernel(const ExpandParams p) {
     }
 #pragma unroll
     for (int u = 0; u < U; ++u) {
-      const int64_t i = base + static_cast<int64_t>(u) * kNT * VEC;
+      const int64_t i = wbase + (static_cast<int64_t>(u) * kNT + lane) * VEC;
       float vm = -CUDART_INF_F;
 #pragma unroll
       for (int j = 0; j < VEC; ++j) vm = fmaxf(vm, xv[u][j]);
@@ -91,16 +94,15 @@ __global__ void __launch_bounds__(kNT) expand_kernel(const ExpandParams p) {
       }
 #pragma unroll
       for (int j = 0; j < VEC; ++j) {
-        if (i + j < hi) {
-          const float xj = xv[u][j];
-          s += (xj == -CUDART_INF_F) ? 0.f : __expf(xj - m);
-          tk.insert(make_key(xj, static_cast<uint32_t>(i + j)));
-        }
+        const float xj = xv[u][j];
+        const bool in = i + j < hi;
+        s += (!in || xj == -CUDART_INF_F) ? 0.f : __expf(xj - m);
+        wt.offer(in ? make_key(xj, static_cast<uint32_t>(i + j)) : 0ull, p.k);
       }
     }
   }
   block_ms<kNT>(m, s, red);
-  block_topk<K, kNT>(tk, p.k, stage, best);
+  block_topk<kNT>(wt, p.k, stage, best);
 
   const int64_t rec_row = (static_cast<int64_t>(b) * p.F + f) * p.chunks;
   if (tid == 0) p.part_ms[rec_row + ch] = make_float2(m, s);
@@ -122,11 +124,11 @@ __global__ void __launch_bounds__(kNT) expand_kernel(const ExpandParams p) {
     ms_merge(M, S, ms.x, ms.y);
   }
   block_ms<kNT>(M, S, red);
-  TopK<K> t2;
+  WarpTopK t2;
   t2.init();
-  for (int64_t j = tid; j < static_cast<int64_t>(p.chunks) * p.k; j += kNT)
-    t2.insert(__ldcg(&p.part_keys[rec_row * p.k + j]));
-  block_topk<K, kNT>(t2, p.k, stage, best);
+  for (int c = warp; c < p.chunks; c += NW)
+    t2.offer(lane < p.k ? __ldcg(&p.part_keys[(rec_row + c) * p.k + lane]) : 0ull, p.k);
+  block_topk<kNT>(t2, p.k, stage, best);
   const float lse = M + logf(S);
 
   const int64_t nb = static_cast<int64_t>(b) * p.max_nodes;
@@ -162,13 +164,15 @@ __global__ void __launch_bounds__(kNT) expand_kernel(const ExpandParams p) {
   if (p.level == 1) {
     if (tid < p.k) p.frontier[b * p.k + tid] = 1 + tid;
   } else {
-    TopK<K> t3;
+    WarpTopK t3;
     t3.init();
-    for (int j = tid; j < p.k * p.k; j += kNT) {
+    const int pool = p.k * p.k;
+    for (int j0 = warp * kWarp; j0 < pool; j0 += kNT) {
+      const int j = j0 + lane;
       const int id = base + j;
-      t3.insert(make_key(__ldcg(&p.cum[nb + id]), static_cast<uint32_t>(id)));
+      t3.offer(j < pool ? make_key(__ldcg(&p.cum[nb + id]), static_cast<uint32_t>(id)) : 0ull, p.k);
     }
-    block_topk<K, kNT>(t3, p.k, stage, best);
+    block_topk<kNT>(t3, p.k, stage, best);
     if (tid < p.k) p.frontier[b * p.k + tid] = static_cast<int32_t>(key_index(best[tid]));
   }
   if (tid == 0) {
@@ -181,11 +185,7 @@ __global__ void __launch_bounds__(kNT) expand_kernel(const ExpandParams p) {
 template <typename T>
 cudaError_t launch_expand_t(const ExpandParams& p, int32_t batch, cudaStream_t s) {
   const dim3 grid(p.chunks, p.F, batch);
-  if (p.k <= 2) expand_kernel<T, 2><<<grid, kNT, 0, s>>>(p);
-  else if (p.k <= 4) expand_kernel<T, 4><<<grid, kNT, 0, s>>>(p);
-  else if (p.k <= 8) expand_kernel<T, 8><<<grid, kNT, 0, s>>>(p);
-  else if (p.k <= 16) expand_kernel<T, 16><<<grid, kNT, 0, s>>>(p);
-  else expand_kernel<T, 32><<<grid, kNT, 0, s>>>(p);
+  expand_kernel<T><<<grid, kNT, 0, s>>>(p);
   return cudaGetLastError();
 }
 

@@ -2,8 +2,8 @@
 //
 // One CTA per sequence.  Every node gets the key (cum desc, id asc) in
 // shared memory (the root gets the maximum key, so it always ranks first);
-// each thread counts, for its nodes, how many keys beat them -- a node is
-// verified iff that rank is below N.  A block-wide exclusive scan over the
+// one warp per node counts how many keys beat it -- a node is verified iff
+// that rank is below N.  A block-wide exclusive scan over the
 // flags in id order gives each verified node its slot, so slots are the
 // verified ids in ascending order.  Each slot then walks its parent chain
 // (at most max_depth steps) and sets one mask bit per ancestor.  Because a
@@ -51,25 +51,29 @@ __global__ void __launch_bounds__(kNT) select_kernel(const SelectParams p) {
   for (int i = tid; i < p.n_max * W32; i += kNT) words[i] = 0u;
   __syncthreads();
 
-  // rank = number of keys strictly greater; verified iff rank < N
-  // (each thread owns ids [4 tid, 4 tid + 4) so the scan below is in id order)
+  // rank = number of keys strictly greater; verified iff rank < N.  One warp
+  // per node, its lanes splitting the key scan; the flag lands in slot_of.
+  const int lane = tid & 31, warp = tid >> 5;
+  for (int i = warp; i < n; i += kNT / kWarp) {
+    const uint64_t ki = keys[i];
+    int cnt = 0;
+    for (int j = lane; j < n; j += kWarp) cnt += (keys[j] > ki) ? 1 : 0;
+    cnt = __reduce_add_sync(0xFFFFFFFFu, cnt);
+    if (lane == 0) slot_of[i] = (cnt < N) ? 1 : 0;
+  }
+  __syncthreads();
+  // each thread owns ids [4 tid, 4 tid + 4) so the scan below is in id order
   constexpr int PER = 4;
   int flags[PER];
   int local = 0;
 #pragma unroll
   for (int r = 0; r < PER; ++r) {
     const int i = tid * PER + r;
-    flags[r] = 0;
-    if (i < n) {
-      const uint64_t ki = keys[i];
-      int rank = 0;
-      for (int j = 0; j < n && rank < N; ++j) rank += (keys[j] > ki) ? 1 : 0;
-      flags[r] = (rank < N) ? 1 : 0;
-    }
+    flags[r] = (i < n) ? slot_of[i] : 0;
     local += flags[r];
   }
+  __syncthreads();
   // block exclusive scan of `local`
-  const int lane = tid & 31, warp = tid >> 5;
   int incl = local;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {

@@ -257,18 +257,32 @@ ltd_status ltd_tree_attention(const void* d_q, const void* d_k, const void* d_v,
   return from_cuda(launch_attn_simt(p, dtype, s));
 }
 
-int32_t ltd_attention_kernel(ltd_dtype dtype, int32_t head_dim, int32_t* launches) {
-  if (!dtype_ok(dtype) || (head_dim != 32 && head_dim != 64 && head_dim != 96 && head_dim != 128))
+int32_t ltd_attention_kernel(ltd_dtype dtype, int32_t batch, int32_t hq, int32_t hkv,
+                             int32_t head_dim, int32_t n_max, int32_t max_ctx, int32_t* launches) {
+  if (!dtype_ok(dtype) || (head_dim != 32 && head_dim != 64 && head_dim != 96 && head_dim != 128) ||
+      batch < 1 || hq < 1 || hkv < 1 || hq % hkv != 0 || n_max < 1 || n_max > LTD_MAX_N ||
+      max_ctx < 0)
     return -1;
   AttnParams p{};
-  p.batch = 1;
-  p.hq = 1;
-  p.hkv = 1;
+  p.batch = batch;
+  p.hq = hq;
+  p.hkv = hkv;
   p.d = head_dim;
-  p.n_max = 1;
+  p.n_max = n_max;
+  p.max_ctx = max_ctx;
   const bool tc = attn_tc_supported(p, dtype);
-  if (launches) *launches = tc ? attn_tc_launches() : 1;
+  if (launches) *launches = tc ? attn_tc_launches(batch, hq, hkv, n_max, max_ctx) : 1;
   return tc ? 1 : 0;
+}
+
+ltd_status ltd_selftest_umma(int32_t mode, const void* d_a, const void* d_b, float* d_c,
+                             ltd_stream_t stream) {
+  if ((mode != 0 && mode != 1) || !d_a || !d_b || !d_c) return LTD_ERR_INVALID_ARG;
+  if (!aligned16(d_a) || !aligned16(d_b) || !aligned16(d_c)) return LTD_ERR_SHAPE;
+  uint32_t* err = device_error_word();
+  if (err == nullptr) return LTD_ERR_CUDA;
+  return from_cuda(
+      launch_umma_selftest(mode, d_a, d_b, d_c, err, reinterpret_cast<cudaStream_t>(stream)));
 }
 
 size_t ltd_accept_workspace_bytes(int32_t batch, int32_t n_max, int64_t vocab) {

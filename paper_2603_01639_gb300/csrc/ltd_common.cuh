@@ -1,5 +1,5 @@
 // Device helpers shared by the LTD kernels: ordered 64-bit keys for
-// (value desc, index asc) selection, register-resident top-k lists, warp and
+// (value desc, index asc) selection, warp-distributed top-k lists, warp and
 // block reductions, the splitmix64-keyed uniforms, and vector loads.
 #pragma once
 
@@ -42,28 +42,26 @@ __device__ __forceinline__ float key_value(uint64_t k) {
   return order_bits_float(static_cast<uint32_t>(k >> 32));
 }
 
-// A descending list of the K largest keys seen, kept in registers (all
-// indices are compile-time after unrolling).
-template <int K>
-struct TopK {
-  uint64_t v[K];
-  __device__ __forceinline__ void init() {
-#pragma unroll
-    for (int i = 0; i < K; ++i) v[i] = 0ull;
-  }
-  __device__ __forceinline__ void insert(uint64_t key) {
-    if (key <= v[K - 1]) return;
-#pragma unroll
-    for (int i = K - 1; i > 0; --i) {
-      const uint64_t up = v[i - 1];
-      v[i] = (key > up) ? up : ((key > v[i]) ? key : v[i]);
+// Warp-distributed top-k (k <= 32): lane i holds the i-th largest key seen
+// so far (descending; 0 = empty).  Each call offers one key per lane; a
+// ballot against the current k-th key filters the offers, and each survivor
+// is inserted with one ballot and one shuffle.  All lanes must call.
+struct WarpTopK {
+  uint64_t v;
+  __device__ __forceinline__ void init() { v = 0ull; }
+  __device__ __forceinline__ void offer(uint64_t key, int k) {
+    const int lane = threadIdx.x & 31;
+    uint32_t cand = __ballot_sync(0xFFFFFFFFu, key > __shfl_sync(0xFFFFFFFFu, v, k - 1));
+    while (cand) {
+      const int src = __ffs(cand) - 1;
+      cand &= cand - 1;
+      const uint64_t kk = __shfl_sync(0xFFFFFFFFu, key, src);
+      if (kk <= __shfl_sync(0xFFFFFFFFu, v, k - 1)) continue;
+      const int pos = __popc(__ballot_sync(0xFFFFFFFFu, lane < k && v > kk));
+      const uint64_t up = __shfl_up_sync(0xFFFFFFFFu, v, 1);
+      if (lane > pos && lane < k) v = up;
+      if (lane == pos) v = kk;
     }
-    v[0] = (key > v[0]) ? key : v[0];
-  }
-  __device__ __forceinline__ void pop() {
-#pragma unroll
-    for (int i = 0; i < K - 1; ++i) v[i] = v[i + 1];
-    v[K - 1] = 0ull;
   }
 };
 
@@ -156,30 +154,21 @@ __device__ __forceinline__ uint64_t block_max_u64(uint64_t x, uint64_t* red) {
   return t;
 }
 
-// Block-wide top-k of the keys held in every thread's TopK list.  Writes the
-// k best keys, descending, to out[0..k) (shared memory) and returns after a
-// barrier.  `stage` needs NW * K uint64 of shared memory.
-template <int K, int NT>
-__device__ __forceinline__ void block_topk(TopK<K>& tk, int k, uint64_t* stage, uint64_t* out) {
+// Block-wide top-k of the per-warp lists: writes the k best keys,
+// descending, to out[0..k) (shared memory) and returns after a barrier.
+// `stage` needs (NT / 32) * 32 uint64 of shared memory.
+template <int NT>
+__device__ __forceinline__ void block_topk(const WarpTopK& wt, int k, uint64_t* stage,
+                                           uint64_t* out) {
   constexpr int NW = NT / kWarp;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  for (int r = 0; r < k; ++r) {
-    const uint64_t head = tk.v[0];
-    const uint64_t best = warp_max_u64(head);
-    if (lane == 0) stage[warp * K + r] = best;
-    if (best != 0ull && head == best) tk.pop();
-  }
+  stage[warp * kWarp + lane] = (lane < k) ? wt.v : 0ull;
   __syncthreads();
   if (warp == 0) {
-    TopK<K> t2;
-    t2.init();
-    for (int j = lane; j < NW * k; j += kWarp) t2.insert(stage[(j / k) * K + (j % k)]);
-    for (int r = 0; r < k; ++r) {
-      const uint64_t head = t2.v[0];
-      const uint64_t best = warp_max_u64(head);
-      if (lane == 0) out[r] = best;
-      if (best != 0ull && head == best) t2.pop();
-    }
+    WarpTopK t;
+    t.init();
+    for (int w = 0; w < NW; ++w) t.offer(stage[w * kWarp + lane], k);
+    if (lane < k) out[lane] = t.v;
   }
   __syncthreads();
 }

@@ -102,7 +102,10 @@ bool attn_tc_supported(const AttnParams& p, ltd_dtype dtype);
 size_t attn_tc_workspace(int32_t batch, int32_t hq, int32_t hkv, int32_t d, int32_t n_max,
                          int32_t max_ctx);
 cudaError_t launch_attn_tc(const AttnParams& p, cudaStream_t s);
-int32_t attn_tc_launches();
+int32_t attn_tc_launches(int32_t batch, int32_t hq, int32_t hkv, int32_t n_max,
+                         int32_t max_ctx);
+cudaError_t launch_umma_selftest(int mode, const void* a, const void* b, float* c, uint32_t* err,
+                                 cudaStream_t s);
 
 // ------------------------------------------------------------- acceptance
 constexpr int64_t kAcceptTargetCtas = 608;

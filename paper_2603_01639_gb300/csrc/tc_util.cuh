@@ -1,0 +1,204 @@
+// Blackwell (sm_103a) building blocks in inline PTX: mbarriers with bounded
+// waits, TMA tensor loads, tensor-memory allocation / loads / stores, and
+// tcgen05 MMA with shared-memory matrix descriptors (bf16 in, fp32 out).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace ltd {
+namespace tc {
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ uint64_t globaltimer() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+// ------------------------------------------------------------- mbarriers
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_init_fence() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Every wait gives up after this long (the caller then flags a timeout and
+// winds down instead of spinning forever).
+constexpr uint64_t kWaitLimitNs = 1000000000ull;
+
+// Wait until the phase with the given parity has completed; false on timeout.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+  if (mbar_try(bar, parity)) return true;
+  const uint64_t t0 = globaltimer();
+  while (true) {
+#pragma unroll 1
+    for (int i = 0; i < 64; ++i)
+      if (mbar_try(bar, parity)) return true;
+    if (globaltimer() - t0 > kWaitLimitNs) return false;
+  }
+}
+
+// ------------------------------------------------------------------- TMA
+__device__ __forceinline__ void tma_prefetch(const CUtensorMap* map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+// 3-D tiled load into shared memory; completes `bytes` on mbarrier `bar`.
+// The innermost coordinate c0 times the element size must be a multiple of
+// 16 bytes (every caller passes 0 or 64 bf16 elements).
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map, uint32_t bar,
+                                            int32_t c0, int32_t c1, int32_t c2) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1), "r"(c2)
+      : "memory");
+}
+
+// ------------------------------------------------------- tensor memory
+__device__ __forceinline__ void tmem_alloc(uint32_t holder_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(holder_smem),
+               "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void fence_before_sync() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void fence_after_sync() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+// Generic-proxy shared-memory writes become visible to the tensor core.
+__device__ __forceinline__ void fence_smem_async() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+// Arrive on `bar` once every MMA issued so far by this thread completes.
+__device__ __forceinline__ void mma_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                   bar)
+               : "memory");
+}
+
+// 32 consecutive 32-bit columns of this thread's TMEM lane.  The registers
+// are tied through the wait so no use can be scheduled before it.
+struct Frag32 {
+  uint32_t r[32];
+};
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, Frag32& f) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, "
+      "%12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, "
+      "%30, %31}, [%32];"
+      : "=r"(f.r[0]), "=r"(f.r[1]), "=r"(f.r[2]), "=r"(f.r[3]), "=r"(f.r[4]), "=r"(f.r[5]),
+        "=r"(f.r[6]), "=r"(f.r[7]), "=r"(f.r[8]), "=r"(f.r[9]), "=r"(f.r[10]), "=r"(f.r[11]),
+        "=r"(f.r[12]), "=r"(f.r[13]), "=r"(f.r[14]), "=r"(f.r[15]), "=r"(f.r[16]), "=r"(f.r[17]),
+        "=r"(f.r[18]), "=r"(f.r[19]), "=r"(f.r[20]), "=r"(f.r[21]), "=r"(f.r[22]), "=r"(f.r[23]),
+        "=r"(f.r[24]), "=r"(f.r[25]), "=r"(f.r[26]), "=r"(f.r[27]), "=r"(f.r[28]), "=r"(f.r[29]),
+        "=r"(f.r[30]), "=r"(f.r[31])
+      : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_wait_ld(Frag32& f) {
+  asm volatile(
+      "tcgen05.wait::ld.sync.aligned;"
+      : "+r"(f.r[0]), "+r"(f.r[1]), "+r"(f.r[2]), "+r"(f.r[3]), "+r"(f.r[4]), "+r"(f.r[5]),
+        "+r"(f.r[6]), "+r"(f.r[7]), "+r"(f.r[8]), "+r"(f.r[9]), "+r"(f.r[10]), "+r"(f.r[11]),
+        "+r"(f.r[12]), "+r"(f.r[13]), "+r"(f.r[14]), "+r"(f.r[15]), "+r"(f.r[16]), "+r"(f.r[17]),
+        "+r"(f.r[18]), "+r"(f.r[19]), "+r"(f.r[20]), "+r"(f.r[21]), "+r"(f.r[22]), "+r"(f.r[23]),
+        "+r"(f.r[24]), "+r"(f.r[25]), "+r"(f.r[26]), "+r"(f.r[27]), "+r"(f.r[28]), "+r"(f.r[29]),
+        "+r"(f.r[30]), "+r"(f.r[31])
+      :
+      : "memory");
+}
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const Frag32& f) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
+      "%11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, "
+      "%29, %30, %31, %32};" ::"r"(taddr),
+      "r"(f.r[0]), "r"(f.r[1]), "r"(f.r[2]), "r"(f.r[3]), "r"(f.r[4]), "r"(f.r[5]), "r"(f.r[6]),
+      "r"(f.r[7]), "r"(f.r[8]), "r"(f.r[9]), "r"(f.r[10]), "r"(f.r[11]), "r"(f.r[12]),
+      "r"(f.r[13]), "r"(f.r[14]), "r"(f.r[15]), "r"(f.r[16]), "r"(f.r[17]), "r"(f.r[18]),
+      "r"(f.r[19]), "r"(f.r[20]), "r"(f.r[21]), "r"(f.r[22]), "r"(f.r[23]), "r"(f.r[24]),
+      "r"(f.r[25]), "r"(f.r[26]), "r"(f.r[27]), "r"(f.r[28]), "r"(f.r[29]), "r"(f.r[30]),
+      "r"(f.r[31])
+      : "memory");
+}
+__device__ __forceinline__ void tmem_wait_st() {
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+// ------------------------------------------------------- MMA descriptors
+// Shared-memory matrix descriptor, 128-byte swizzle (tcgen05 format):
+// start address >> 4 in bits 0-13, leading-dimension byte offset >> 4 in
+// 16-29, stride-dimension byte offset >> 4 in 32-45, the fixed 0b001 in
+// 46-48, base offset 0 (atoms are 1024-byte aligned), swizzle mode 2 (128B)
+// in 61-63.  K-major operands: SBO = 1024 (eight 128-byte rows), LBO unused.
+// MN-major operands: LBO = bytes between 64-element MN blocks, SBO = bytes
+// between groups of eight K rows.
+__device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  return static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4) |
+         (static_cast<uint64_t>((lbo >> 4) & 0x3FFFu) << 16) |
+         (static_cast<uint64_t>((sbo >> 4) & 0x3FFFu) << 32) | (1ull << 46) | (2ull << 61);
+}
+
+// Instruction descriptor of kind::f16 with bf16 A/B and fp32 accumulation:
+// D format (bits 4-5) = F32, A and B formats (7-9, 10-12) = BF16, A K-major,
+// B K-major or MN-major (bit 16), N >> 3 in bits 17-22, M >> 4 in 24-28.
+__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, bool b_mn_major) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((b_mn_major ? 1u : 0u) << 16) |
+         (static_cast<uint32_t>(N >> 3) << 17) | (static_cast<uint32_t>(M >> 4) << 24);
+}
+
+// D[tmem] (+)= A[smem] * B[smem], one elected thread issues it.
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                         uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+}  // namespace tc
+
+// Host: encode a 3-D bf16 tensor map with 128-byte swizzle (dims innermost
+// first, strides in bytes for dims 1 and 2).  Returns false on failure.
+bool encode_tmap_bf16_3d(CUtensorMap* map, const void* base, uint64_t d0, uint64_t d1, uint64_t d2,
+                         uint64_t stride1, uint64_t stride2, uint32_t b0, uint32_t b1, uint32_t b2);
+
+}  // namespace ltd

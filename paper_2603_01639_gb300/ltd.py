@@ -29,7 +29,7 @@ EXPORTS = [
     "ltd_tree_bytes", "ltd_tree_init", "ltd_tree_reset", "ltd_expand_tree", "ltd_select_verify",
     "ltd_attention_workspace_bytes", "ltd_tree_attention", "ltd_accept_workspace_bytes",
     "ltd_accept", "ltd_kv_compact", "ltd_check", "ltd_status_string", "ltd_version",
-    "ltd_attention_kernel",
+    "ltd_attention_kernel", "ltd_selftest_umma",
 ]
 
 
@@ -79,7 +79,9 @@ def lib():
                 "ltd_check": (C.c_int, [vp, C.POINTER(C.c_uint32)]),
                 "ltd_status_string": (C.c_char_p, [C.c_int]),
                 "ltd_version": (i32, []),
-                "ltd_attention_kernel": (i32, [C.c_int, i32, C.POINTER(i32)]),
+                "ltd_attention_kernel": (i32, [C.c_int, i32, i32, i32, i32, i32, i32,
+                                               C.POINTER(i32)]),
+                "ltd_selftest_umma": (C.c_int, [i32, vp, vp, vp, vp]),
             }
             for name, (res, args) in sig.items():
                 fn = getattr(L, name)
@@ -306,23 +308,26 @@ def ltd_version() -> int:
     return lib().ltd_version()
 
 
-def ltd_attention_kernel(head_dim: int, dtype) -> tuple:
+def ltd_attention_kernel(dtype, batch, hq, hkv, head_dim, n_max, max_ctx) -> tuple:
     """(1 tensor cores / 0 CUDA cores / -1 unsupported, launches per call)."""
     n = C.c_int32(0)
-    code = lib().ltd_attention_kernel(LTD_BF16 if dtype == torch.bfloat16 else LTD_F32, head_dim,
-                                      C.byref(n))
+    code = lib().ltd_attention_kernel(LTD_BF16 if dtype == torch.bfloat16 else LTD_F32, batch, hq,
+                                      hkv, head_dim, n_max, max_ctx, C.byref(n))
     return code, n.value
 
 
-def attention_launches(head_dim: int, dtype) -> int:
-    return ltd_attention_kernel(head_dim, dtype)[1]
+def attention_kernel_sources(code: int) -> list:
+    """Source files of the attention kernel selected by ltd_attention_kernel."""
+    if code == 1:
+        return ["k_attn_tc.cu", "tc_util.cuh", "ltd_common.cuh"]
+    return ["k_attn_simt.cu", "ltd_common.cuh"]
 
 
-def attention_kernel_tag(head_dim: int, dtype) -> str:
-    return "attn_tc" if ltd_attention_kernel(head_dim, dtype)[0] == 1 else "attn_simt"
-
-
-def attention_kernel_sources(head_dim: int, dtype) -> list:
-    """Source files of the attention kernel this call dispatches to."""
-    main = "k_attn_tc.cu" if ltd_attention_kernel(head_dim, dtype)[0] == 1 else "k_attn_simt.cu"
-    return [main, "ltd_common.cuh"]
+def ltd_selftest_umma(mode: int, a: torch.Tensor, b: torch.Tensor, stream=None) -> torch.Tensor:
+    """128x128x128 bf16 GEMM through TMA + tcgen05 (mode 0: a @ b.T, mode 1: a @ b)."""
+    _need(a, "a", torch.bfloat16)
+    _need(b, "b", torch.bfloat16)
+    c = torch.empty(128, 128, dtype=torch.float32, device=a.device)
+    _ok(lib().ltd_selftest_umma(mode, _ptr(a), _ptr(b), _ptr(c), _stream(stream)),
+        "ltd_selftest_umma")
+    return c

@@ -36,11 +36,13 @@ def _draft_select_accept(name, seed, cycle_no=0, acc_seed=1234):
     trees, sels, target = H.oracle_side(cfg, ci)
     draft = H.dev(ci.draft_rows, cfg.dtype)
     tree = H.gpu_draft(cfg, ci, draft)
-    cut = H.compare_trees(cfg, ci, tree, trees)
-    assert cut > H.CUT_MARGIN, f"near-tie at a frontier cut ({cut}); pick another seed"
+    margin = min(H.tree_margin(t, cfg.W) for t in trees)
+    assert margin > H.CUT_MARGIN, f"near-tie deciding a frontier ({margin}); pick another seed"
+    sel_margin = min(H.select_margin(t, int(n)) for t, n in zip(trees, ci.n_verify))
+    assert sel_margin > H.CUT_MARGIN, f"near-tie at the selection cut ({sel_margin})"
+    H.compare_trees(cfg, ci, tree, trees)
     got = H.gpu_select(cfg, ci, tree)
-    sel_margin = H.compare_select(cfg, ci, got, sels)
-    assert sel_margin > H.CUT_MARGIN
+    H.compare_select(cfg, ci, got, sels, trees)
     ref = H.oracle_accept(cfg, ci, trees, sels, target, acc_seed, cycle_no)
     assert H.stochastic_margins_ok(ref), "near-tie in a stochastic decision; pick another seed"
     tgt = H.dev(target, cfg.dtype)

@@ -55,7 +55,7 @@ struct TcArgs {
   const uint32_t* mask;
   float scale_log2;
   __nv_bfloat16* out;
-  float4* ws_o;   // [cta][32][128] float4
+  float4* ws_o;   // [cta][128 rows][32] float4
   float2* ws_ml;  // [cta][128] (max in log2 units, sum)
   uint32_t* err;
 };
@@ -335,7 +335,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       } else {
-        float4* wo = a.ws_o + cta * 32 * kBM;
+        float4* wo = a.ws_o + (cta * kBM + i) * 32;
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
           tc::Frag32 f;
@@ -343,7 +343,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc::tmem_wait_ld(f);
 #pragma unroll
           for (int c4 = 0; c4 < 8; ++c4)
-            wo[(8 * q + c4) * kBM + i] =
+            wo[8 * q + c4] =
                 make_float4(__uint_as_float(f.r[4 * c4]), __uint_as_float(f.r[4 * c4 + 1]),
                             __uint_as_float(f.r[4 * c4 + 2]), __uint_as_float(f.r[4 * c4 + 3]));
         }
@@ -363,16 +363,23 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-// Combine the split partials of every row: weights 2^(m_s - max m).
-__global__ void __launch_bounds__(kBM) attn_tc_merge_kernel(const TcArgs a) {
-  const int i = threadIdx.x;
-  const int tile = blockIdx.x % a.n_tiles;
-  const int bh = blockIdx.x / a.n_tiles;
+// Combine the split partials of every row: weights 2^(m_s - max m).  One
+// warp per row, lane c owns output dims 4c..4c+3, so both the partial reads
+// (row-major [cta][row][32 float4]) and the bf16 output writes coalesce.
+constexpr int kMergeRows = 8;
+
+__global__ void __launch_bounds__(kMergeRows * 32) attn_tc_merge_kernel(const TcArgs a) {
+  const int lane = threadIdx.x & 31;
+  const int64_t grow = static_cast<int64_t>(blockIdx.x) * kMergeRows + (threadIdx.x >> 5);
+  const int64_t rows_per_bh = static_cast<int64_t>(a.n_tiles) * kBM;
+  const int bh = static_cast<int>(grow / rows_per_bh);
+  if (bh >= a.batch * a.hkv) return;
+  const int R = static_cast<int>(grow % rows_per_bh);
+  const int tile = R / kBM, i = R % kBM;
   const int b = bh / a.hkv, kvh = bh % a.hkv;
   const int ctx = a.ctx[b];
   const int N = a.n_verify[b];
   if (N < 1 || N > a.n_max || ctx < 0 || ctx > a.max_ctx || ctx + N > a.s_cap) return;
-  const int R = tile * kBM + i;
   if (R >= N * a.G) return;
   const int slot = R / a.G, g = R % a.G;
   const int64_t cta0 = (static_cast<int64_t>(bh) * a.n_tiles + tile) * a.splits;
@@ -381,36 +388,26 @@ __global__ void __launch_bounds__(kBM) attn_tc_merge_kernel(const TcArgs a) {
     const float2 ml = a.ws_ml[(cta0 + s) * kBM + i];
     if (ml.y > 0.f) mx = fmaxf(mx, ml.x);
   }
-  float acc[kD];
-#pragma unroll
-  for (int c = 0; c < kD; ++c) acc[c] = 0.f;
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
   float L = 0.f;
   for (int s = 0; s < a.splits; ++s) {
     const float2 ml = a.ws_ml[(cta0 + s) * kBM + i];
     if (!(ml.y > 0.f)) continue;
     const float w = tc::ex2(ml.x - mx);
     L += w * ml.y;
-    const float4* src = a.ws_o + (cta0 + s) * 32 * kBM;
-#pragma unroll
-    for (int c4 = 0; c4 < 32; ++c4) {
-      const float4 v = src[c4 * kBM + i];
-      acc[4 * c4] += w * v.x;
-      acc[4 * c4 + 1] += w * v.y;
-      acc[4 * c4 + 2] += w * v.z;
-      acc[4 * c4 + 3] += w * v.w;
-    }
+    const float4 v = a.ws_o[((cta0 + s) * kBM + i) * 32 + lane];
+    acc.x += w * v.x;
+    acc.y += w * v.y;
+    acc.z += w * v.z;
+    acc.w += w * v.w;
   }
   const float inv = L > 0.f ? 1.f / L : 0.f;
-  __nv_bfloat16* dst = a.out + ((static_cast<int64_t>(b) * a.n_max + slot) * a.hq + kvh * a.G + g) * kD;
-#pragma unroll
-  for (int c = 0; c < kD; c += 8) {
-    uint4 w;
-    w.x = pack_bf16(acc[c] * inv, acc[c + 1] * inv);
-    w.y = pack_bf16(acc[c + 2] * inv, acc[c + 3] * inv);
-    w.z = pack_bf16(acc[c + 4] * inv, acc[c + 5] * inv);
-    w.w = pack_bf16(acc[c + 6] * inv, acc[c + 7] * inv);
-    *reinterpret_cast<uint4*>(dst + c) = w;
-  }
+  __nv_bfloat16* dst =
+      a.out + ((static_cast<int64_t>(b) * a.n_max + slot) * a.hq + kvh * a.G + g) * kD + 4 * lane;
+  uint2 w2;
+  w2.x = pack_bf16(acc.x * inv, acc.y * inv);
+  w2.y = pack_bf16(acc.z * inv, acc.w * inv);
+  *reinterpret_cast<uint2*>(dst) = w2;
 }
 
 struct Plan {
@@ -528,7 +525,9 @@ cudaError_t launch_attn_tc(const AttnParams& p, cudaStream_t s) {
   attn_tc_kernel<<<grid, kThreads, kSmemBytes, s>>>(tq, tk, tv, a);
   e = cudaGetLastError();
   if (e != cudaSuccess || pl.splits == 1) return e;
-  attn_tc_merge_kernel<<<p.batch * p.hkv * pl.n_tiles, kBM, 0, s>>>(a);
+  const int64_t rows = static_cast<int64_t>(p.batch) * p.hkv * pl.n_tiles * kBM;
+  attn_tc_merge_kernel<<<static_cast<unsigned>((rows + kMergeRows - 1) / kMergeRows),
+                         kMergeRows * 32, 0, s>>>(a);
   return cudaGetLastError();
 }
 

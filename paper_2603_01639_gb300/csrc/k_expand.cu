@@ -3,8 +3,10 @@
 // One launch builds one level for every active sequence.  The grid is
 // (chunks, F, batch) with F = 1 at level 1 and F = k afterwards: each CTA
 // scans one vocabulary chunk of one frontier row with 16-byte streaming loads,
-// computing the chunk's (max, sum exp) and its top-k (logit desc, token asc)
-// in warp-distributed lists (lane i holds the i-th best key).  The last CTA to finish a row (atomic ticket; nothing spins)
+// computing the chunk's (max, sum exp) and, per thread, its four best
+// (logit desc, token asc) keys; bitonic warp networks turn those into the
+// chunk's top-k (with an exact rescan in the rare case a thread may hold
+// more than four of them).  The last CTA to finish a row (atomic ticket; nothing spins)
 // merges the chunk partials in a fixed order into the row's log-sum-exp and
 // top-k, appends the k children with cum = cum(parent) + x - lse, and the
 // last row of a sequence picks the new frontier: the k best of the k^2 pool
@@ -65,16 +67,14 @@ __global__ void __launch_bounds__(kNT) expand_kernel(const ExpandParams p) {
   const int64_t hi = min(lo + p.chunk_elems, p.vocab);
 
   float m = -CUDART_INF_F, s = 0.f;
-  WarpTopK wt;
-  wt.init();
-  // every lane of a warp runs the same number of iterations (offer() is
-  // warp-collective); out-of-range slots offer the empty key 0
-  for (int64_t wbase = lo + static_cast<int64_t>(warp) * kWarp * VEC; wbase < hi;
-       wbase += static_cast<int64_t>(kNT) * VEC * U) {
+  Top4 t4;
+  t4.init();
+  for (int64_t base = lo + static_cast<int64_t>(tid) * VEC; base < hi;
+       base += static_cast<int64_t>(kNT) * VEC * U) {
     float xv[U][VEC];
 #pragma unroll
     for (int u = 0; u < U; ++u) {
-      const int64_t i = wbase + (static_cast<int64_t>(u) * kNT + lane) * VEC;
+      const int64_t i = base + static_cast<int64_t>(u) * kNT * VEC;
       if (i + VEC <= hi) {
         unpack16(ld_stream16(x + i), xv[u], static_cast<const T*>(nullptr));
       } else {
@@ -84,7 +84,7 @@ __global__ void __launch_bounds__(kNT) expand_kernel(const ExpandParams p) {
     }
 #pragma unroll
     for (int u = 0; u < U; ++u) {
-      const int64_t i = wbase + (static_cast<int64_t>(u) * kNT + lane) * VEC;
+      const int64_t i = base + static_cast<int64_t>(u) * kNT * VEC;
       float vm = -CUDART_INF_F;
 #pragma unroll
       for (int j = 0; j < VEC; ++j) vm = fmaxf(vm, xv[u][j]);
@@ -94,15 +94,35 @@ __global__ void __launch_bounds__(kNT) expand_kernel(const ExpandParams p) {
       }
 #pragma unroll
       for (int j = 0; j < VEC; ++j) {
-        const float xj = xv[u][j];
-        const bool in = i + j < hi;
-        s += (!in || xj == -CUDART_INF_F) ? 0.f : __expf(xj - m);
-        wt.offer(in ? make_key(xj, static_cast<uint32_t>(i + j)) : 0ull, p.k);
+        if (i + j < hi) {
+          const float xj = xv[u][j];
+          s += (xj == -CUDART_INF_F) ? 0.f : __expf(xj - m);
+          t4.insert(make_key(xj, static_cast<uint32_t>(i + j)));
+        }
       }
     }
   }
   block_ms<kNT>(m, s, red);
-  block_topk<kNT>(wt, p.k, stage, best);
+  // warp lists from the per-thread top-4s, then the block list
+  WarpTopK wt;
+  wt.init();
+  wt.offer(t4.t0, p.k);
+  wt.offer(t4.t1, p.k);
+  wt.offer(t4.t2, p.k);
+  wt.offer(t4.t3, p.k);
+  block_topk<kNT>(wt, stage, best);
+  // exactness: a thread whose 4th key made the top-k may hold more of it;
+  // then every thread offers its whole chunk again (rare: needs 4 of the
+  // chunk's top-k in one thread's 1/256 of the chunk)
+  if (__syncthreads_or(t4.t3 != 0ull && t4.t3 >= best[p.k - 1])) {
+    wt.init();
+    for (int64_t wbase = lo + static_cast<int64_t>(warp) * kWarp; wbase < hi;
+         wbase += static_cast<int64_t>(kNT)) {
+      const int64_t i = wbase + lane;
+      wt.offer(i < hi ? make_key(to_f<T>(x[i]), static_cast<uint32_t>(i)) : 0ull, p.k);
+    }
+    block_topk<kNT>(wt, stage, best);
+  }
 
   const int64_t rec_row = (static_cast<int64_t>(b) * p.F + f) * p.chunks;
   if (tid == 0) p.part_ms[rec_row + ch] = make_float2(m, s);
@@ -127,8 +147,8 @@ __global__ void __launch_bounds__(kNT) expand_kernel(const ExpandParams p) {
   WarpTopK t2;
   t2.init();
   for (int c = warp; c < p.chunks; c += NW)
-    t2.offer(lane < p.k ? __ldcg(&p.part_keys[(rec_row + c) * p.k + lane]) : 0ull, p.k);
-  block_topk<kNT>(t2, p.k, stage, best);
+    t2.merge_sorted(lane < p.k ? __ldcg(&p.part_keys[(rec_row + c) * p.k + lane]) : 0ull);
+  block_topk<kNT>(t2, stage, best);
   const float lse = M + logf(S);
 
   const int64_t nb = static_cast<int64_t>(b) * p.max_nodes;
@@ -172,7 +192,7 @@ __global__ void __launch_bounds__(kNT) expand_kernel(const ExpandParams p) {
       const int id = base + j;
       t3.offer(j < pool ? make_key(__ldcg(&p.cum[nb + id]), static_cast<uint32_t>(id)) : 0ull, p.k);
     }
-    block_topk<kNT>(t3, p.k, stage, best);
+    block_topk<kNT>(t3, stage, best);
     if (tid < p.k) p.frontier[b * p.k + tid] = static_cast<int32_t>(key_index(best[tid]));
   }
   if (tid == 0) {

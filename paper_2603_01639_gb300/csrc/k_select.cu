@@ -23,7 +23,8 @@ __global__ void __launch_bounds__(kNT) select_kernel(const SelectParams p) {
   const int W32 = (p.n_max + 31) / 32;
   uint64_t* keys = reinterpret_cast<uint64_t*>(smem);                          // [max_nodes]
   int32_t* slot_of = reinterpret_cast<int32_t*>(keys + p.max_nodes);          // [max_nodes]
-  uint32_t* words = reinterpret_cast<uint32_t*>(slot_of + p.max_nodes);       // [n_max][W32]
+  int32_t* par_s = slot_of + p.max_nodes;                                     // [max_nodes]
+  uint32_t* words = reinterpret_cast<uint32_t*>(par_s + p.max_nodes);         // [n_max][W32]
   __shared__ int32_t warp_tot[kNT / kWarp];
 
   const int b = blockIdx.x, tid = threadIdx.x;
@@ -46,8 +47,10 @@ __global__ void __launch_bounds__(kNT) select_kernel(const SelectParams p) {
     return;
   }
 
-  for (int i = tid; i < n; i += kNT)
+  for (int i = tid; i < n; i += kNT) {
     keys[i] = (i == 0) ? ~0ull : make_key(p.cum[nb + i], static_cast<uint32_t>(i));
+    par_s[i] = p.parent[nb + i];
+  }
   for (int i = tid; i < p.n_max * W32; i += kNT) words[i] = 0u;
   __syncthreads();
 
@@ -122,7 +125,7 @@ __global__ void __launch_bounds__(kNT) select_kernel(const SelectParams p) {
         break;
       }
       row[sa >> 5] |= 1u << (sa & 31);
-      a = p.parent[nb + a];
+      a = par_s[a];
       ++guard;
     }
   }
@@ -138,7 +141,7 @@ __global__ void __launch_bounds__(kNT) select_kernel(const SelectParams p) {
 
 cudaError_t launch_select(const SelectParams& p, int32_t batch, cudaStream_t s) {
   const int W32 = (p.n_max + 31) / 32;
-  const size_t smem = static_cast<size_t>(p.max_nodes) * (sizeof(uint64_t) + sizeof(int32_t)) +
+  const size_t smem = static_cast<size_t>(p.max_nodes) * (sizeof(uint64_t) + 2 * sizeof(int32_t)) +
                       static_cast<size_t>(p.n_max) * W32 * sizeof(uint32_t);
   cudaError_t e = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));

@@ -42,26 +42,61 @@ __device__ __forceinline__ float key_value(uint64_t k) {
   return order_bits_float(static_cast<uint32_t>(k >> 32));
 }
 
-// Warp-distributed top-k (k <= 32): lane i holds the i-th largest key seen
-// so far (descending; 0 = empty).  Each call offers one key per lane; a
-// ballot against the current k-th key filters the offers, and each survivor
-// is inserted with one ballot and one shuffle.  All lanes must call.
+// Warp bitonic sort of one key per lane, descending (lane 0 = largest).
+__device__ __forceinline__ uint64_t warp_sort_desc(uint64_t v) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int size = 2; size <= 32; size <<= 1) {
+#pragma unroll
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      const uint64_t o = __shfl_xor_sync(0xFFFFFFFFu, v, stride);
+      const bool keep_max = ((lane & stride) == 0) == ((lane & size) == 0);
+      v = keep_max ? (v > o ? v : o) : (v < o ? v : o);
+    }
+  }
+  return v;
+}
+
+// The 32 largest of two descending lane-sorted lists, descending: the
+// element-wise max of a and reversed b is bitonic and holds the 32 largest;
+// five half-cleaner steps sort it.
+__device__ __forceinline__ uint64_t warp_merge_desc(uint64_t a, uint64_t b) {
+  const int lane = threadIdx.x & 31;
+  const uint64_t br = __shfl_sync(0xFFFFFFFFu, b, 31 - lane);
+  uint64_t v = a > br ? a : br;
+#pragma unroll
+  for (int stride = 16; stride > 0; stride >>= 1) {
+    const uint64_t o = __shfl_xor_sync(0xFFFFFFFFu, v, stride);
+    v = ((lane & stride) == 0) ? (v > o ? v : o) : (v < o ? v : o);
+  }
+  return v;
+}
+
+// Warp-distributed top list: lane i holds the i-th largest key seen so far
+// (descending; 0 = empty); the first k lanes are the top-k (k <= 32).  All
+// lanes of the warp must call its members.
 struct WarpTopK {
   uint64_t v;
   __device__ __forceinline__ void init() { v = 0ull; }
+  // one unsorted key per lane; skipped when no key beats the k-th
   __device__ __forceinline__ void offer(uint64_t key, int k) {
-    const int lane = threadIdx.x & 31;
-    uint32_t cand = __ballot_sync(0xFFFFFFFFu, key > __shfl_sync(0xFFFFFFFFu, v, k - 1));
-    while (cand) {
-      const int src = __ffs(cand) - 1;
-      cand &= cand - 1;
-      const uint64_t kk = __shfl_sync(0xFFFFFFFFu, key, src);
-      if (kk <= __shfl_sync(0xFFFFFFFFu, v, k - 1)) continue;
-      const int pos = __popc(__ballot_sync(0xFFFFFFFFu, lane < k && v > kk));
-      const uint64_t up = __shfl_up_sync(0xFFFFFFFFu, v, 1);
-      if (lane > pos && lane < k) v = up;
-      if (lane == pos) v = kk;
-    }
+    const uint64_t kth = __shfl_sync(0xFFFFFFFFu, v, k - 1);
+    if (__any_sync(0xFFFFFFFFu, key > kth)) v = warp_merge_desc(v, warp_sort_desc(key));
+  }
+  // a list already sorted descending across the lanes
+  __device__ __forceinline__ void merge_sorted(uint64_t sorted) { v = warp_merge_desc(v, sorted); }
+};
+
+// Four largest keys seen by one thread, descending, in registers.
+struct Top4 {
+  uint64_t t0, t1, t2, t3;
+  __device__ __forceinline__ void init() { t0 = t1 = t2 = t3 = 0ull; }
+  __device__ __forceinline__ void insert(uint64_t key) {
+    if (key <= t3) return;
+    if (key > t0) { t3 = t2; t2 = t1; t1 = t0; t0 = key; }
+    else if (key > t1) { t3 = t2; t2 = t1; t1 = key; }
+    else if (key > t2) { t3 = t2; t2 = key; }
+    else { t3 = key; }
   }
 };
 
@@ -154,21 +189,20 @@ __device__ __forceinline__ uint64_t block_max_u64(uint64_t x, uint64_t* red) {
   return t;
 }
 
-// Block-wide top-k of the per-warp lists: writes the k best keys,
-// descending, to out[0..k) (shared memory) and returns after a barrier.
+// Block-wide top list from the per-warp lists: writes the 32 largest keys,
+// descending, to out[0..32) (shared memory) and returns after a barrier.
 // `stage` needs (NT / 32) * 32 uint64 of shared memory.
 template <int NT>
-__device__ __forceinline__ void block_topk(const WarpTopK& wt, int k, uint64_t* stage,
-                                           uint64_t* out) {
+__device__ __forceinline__ void block_topk(const WarpTopK& wt, uint64_t* stage, uint64_t* out) {
   constexpr int NW = NT / kWarp;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  stage[warp * kWarp + lane] = (lane < k) ? wt.v : 0ull;
+  stage[warp * kWarp + lane] = wt.v;
   __syncthreads();
   if (warp == 0) {
-    WarpTopK t;
-    t.init();
-    for (int w = 0; w < NW; ++w) t.offer(stage[w * kWarp + lane], k);
-    if (lane < k) out[lane] = t.v;
+    uint64_t v = stage[lane];
+#pragma unroll 1
+    for (int w = 1; w < NW; ++w) v = warp_merge_desc(v, stage[w * kWarp + lane]);
+    out[lane] = v;
   }
   __syncthreads();
 }

@@ -233,6 +233,26 @@ def _source_sha(files):
     return h.hexdigest()[:16]
 
 
+def replica_seed(seed: int, rank: int) -> int:
+    """Each rank drafts and verifies its own independent sequences."""
+    return seed + 1000 * rank
+
+
+def aggregate(total_ms: float, steps: int, batch: int, world: int, device=None):
+    """Job time = the slowest rank's time (max over ranks); value = job time
+    per cycle over the cycles all ranks completed.  Returns (ms per step,
+    µs per cycle)."""
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        t = torch.tensor([total_ms], dtype=torch.float64,
+                         device=device if dist.get_backend() == "nccl" else "cpu")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    ms_per_step = total_ms / steps
+    return ms_per_step, ms_per_step * 1e3 / (batch * world)
+
+
 # ----------------------------------------------------------- CPU baseline
 def time_oracle_cycle(cfg, layers, seed, budget_s):
     """The fp64 oracle on the same workload: draft, selection, acceptance and
@@ -335,7 +355,7 @@ def run_ours(args):
     build()
     cfg = wl.config(args.config)
     layers = N_LAYERS[args.config]
-    cyc = Cycle(cfg, layers, args.seed + rank, device)
+    cyc = Cycle(cfg, layers, replica_seed(args.seed, rank), device)
 
     def full():
         cyc.draft_phase()
@@ -377,13 +397,7 @@ def run_ours(args):
     draft_ms = statistics.mean(ev[i][0].elapsed_time(ev[i][1]) for i in range(K))
     verify_ms = statistics.mean(ev[i][1].elapsed_time(ev[i][2]) for i in range(K))
     accept_ms = statistics.mean(ev[i][2].elapsed_time(ev[i][3]) for i in range(K))
-    if world > 1:
-        t = torch.tensor([total_ms], device=device)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        total_ms = float(t.item())
-    ms_per_step = total_ms / K
-    cycles_per_step = cfg.batch * world
-    value_us = ms_per_step * 1e3 / cycles_per_step
+    ms_per_step, value_us = aggregate(total_ms, K, cfg.batch, world, device)
 
     # roofline of the dominant kernel (tree attention)
     att_bytes, att_flops = cyc.attention_algorithmic()

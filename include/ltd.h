@@ -227,6 +227,32 @@ ltd_status ltd_accept(const ltd_tree* tree, const void* d_target_logits,
                       const ltd_kv_cache* kv, void* d_workspace, size_t workspace_bytes,
                       ltd_stream_t stream);
 
+/* Acceptance for callers that cannot allocate device memory when they
+ * accept a draft -- a serving loop that reserved its memory up front and
+ * keeps allocation off the hot path, a plugin whose host framework owns all
+ * device buffers, code that must stay allocation-free so its stream can be
+ * captured with a fixed memory plan.  The paper has no counterpart; it is
+ * a deployment convenience.
+ *
+ * Same arguments and results as ltd_accept without the workspace: the
+ * scratch lives in a static device array of LTD_ACCEPT_NOALLOC_SCRATCH_BYTES
+ * (1 MiB) inside the library, held by every GPU that loads it until the
+ * process exits.  Sizes whose ltd_accept_workspace_bytes() exceeds that
+ * return LTD_ERR_SHAPE.  Allocates nothing (no cudaMalloc or cudaFree); each
+ * call clears the array's tickets with one cudaMemsetAsync on the stream.
+ * The first call on a device looks up the array's device address; make
+ * that first call before any stream capture.  All calls share the array,
+ * so calls whose kernels overlap on the GPU (for example on two streams)
+ * race; calls on one stream are ordered and safe. */
+#define LTD_ACCEPT_NOALLOC_SCRATCH_BYTES (1u << 20)
+ltd_status ltd_accept_noalloc(const ltd_tree* tree, const void* d_target_logits,
+                              const void* d_draft_rows, ltd_dtype dtype, int64_t vocab,
+                              int64_t rows_per_seq, const int32_t* d_node_ids,
+                              const int32_t* d_n_verify, int32_t n_max, const int32_t* d_mode,
+                              uint64_t seed, uint64_t cycle, const int32_t* d_ctx,
+                              int32_t* d_new_ctx, int32_t* d_path, int32_t* d_accept_len,
+                              int32_t* d_bonus, const ltd_kv_cache* kv, ltd_stream_t stream);
+
 /* In-place KV compaction ("discards the remainder", section 3.2): for every
  * layer, sequence, KV head and K/V tensor, row ctx+t <- row ctx+path[t] for
  * t = 0..accept_len, every source read before any row is written.  Rows

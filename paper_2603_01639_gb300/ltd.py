@@ -29,8 +29,9 @@ EXPORTS = [
     "ltd_tree_bytes", "ltd_tree_init", "ltd_tree_reset", "ltd_expand_tree", "ltd_select_verify",
     "ltd_attention_workspace_bytes", "ltd_tree_attention", "ltd_accept_workspace_bytes",
     "ltd_accept", "ltd_kv_compact", "ltd_check", "ltd_status_string", "ltd_version",
-    "ltd_attention_kernel", "ltd_selftest_umma",
+    "ltd_attention_kernel", "ltd_selftest_umma", "ltd_accept_noalloc",
 ]
+LTD_ACCEPT_NOALLOC_SCRATCH_BYTES = 1 << 20
 
 
 class LtdError(RuntimeError):
@@ -82,6 +83,9 @@ def lib():
                 "ltd_attention_kernel": (i32, [C.c_int, i32, i32, i32, i32, i32, i32,
                                                C.POINTER(i32)]),
                 "ltd_selftest_umma": (C.c_int, [i32, vp, vp, vp, vp]),
+                "ltd_accept_noalloc": (C.c_int, [tp, vp, vp, C.c_int, i64, i64, vp, vp, i32, vp, u64,
+                                                 u64, vp, vp, vp, vp, vp, C.POINTER(ltd_kv_cache),
+                                                 vp]),
             }
             for name, (res, args) in sig.items():
                 fn = getattr(L, name)
@@ -285,6 +289,33 @@ def ltd_accept(tree: Tree, target, draft_rows, node_ids, n_verify, mode, ctx, se
                          _ptr(out["new_ctx"]), _ptr(out["path"]), _ptr(out["accept_len"]),
                          _ptr(out["bonus"]), kvp, _ptr(workspace), workspace.numel(),
                          _stream(stream)), "ltd_accept")
+    return out
+
+
+def ltd_accept_noalloc(tree: Tree, target, draft_rows, node_ids, n_verify, mode, ctx, seed=0,
+                       cycle=0, kv: KVCache | None = None, out=None, stream=None):
+    """ltd_accept without a workspace, for callers that cannot allocate device
+    memory when they accept (the library keeps the scratch in a static 1 MiB
+    device array).  Output tensors are still the caller's: pass ``out`` (a
+    dict like ltd_accept returns) to keep this call allocation-free."""
+    _need(target, "target")
+    _need(draft_rows, "draft_rows", target.dtype)
+    for t, n in ((node_ids, "node_ids"), (n_verify, "n_verify"), (mode, "mode"), (ctx, "ctx")):
+        _need(t, n, torch.int32)
+    B, n_max, V = target.shape
+    R = draft_rows.shape[1]
+    dev = target.device
+    if out is None:
+        out = {"path": torch.empty(B, tree.max_depth + 1, dtype=torch.int32, device=dev),
+               "accept_len": torch.empty(B, dtype=torch.int32, device=dev),
+               "bonus": torch.empty(B, dtype=torch.int32, device=dev),
+               "new_ctx": torch.empty(B, dtype=torch.int32, device=dev)}
+    kvp = C.byref(kv.s) if kv is not None else None
+    _ok(lib().ltd_accept_noalloc(C.byref(tree.s), _ptr(target), _ptr(draft_rows), _dtype(target),
+                                 V, R, _ptr(node_ids), _ptr(n_verify), n_max, _ptr(mode), seed,
+                                 cycle, _ptr(ctx), _ptr(out["new_ctx"]), _ptr(out["path"]),
+                                 _ptr(out["accept_len"]), _ptr(out["bonus"]), kvp,
+                                 _stream(stream)), "ltd_accept_noalloc")
     return out
 
 

@@ -1,23 +1,32 @@
 // Tensor-core tree attention (LTD section 3.2, "Draft Tree Verification";
 // SpecInfer-style tree mask) for bf16 and head_dim 128 on sm_103a.
 //
-// Work split: a CTA owns one 128-row tile of the query rows of one KV head
-// (row r = slot * G + g, so all G query heads sharing the KV head ride on
-// every K/V byte) and one split of that head's keys.  Per 128-key chunk:
-//   TMA (warp 0)   K and V chunks -> a 2-stage shared-memory ring, 128-byte
-//                  swizzle, plus the Q tile once;
-//   MMA (warp 1)   S = Q K^T into tensor memory (double-buffered), then
-//                  O += P V into a tensor-memory accumulator, software-
-//                  pipelined so S of chunk j+1 overlaps the softmax of j;
-//   softmax (warps 4-7, one thread per row / TMEM lane)  read S, apply the
-//                  prefix + ancestor-bit mask, keep a running max that only
-//                  moves (rescaling O in TMEM) when it grows by more than
-//                  2^8, write P as bf16 into swizzled shared memory.
-// With one split the CTA normalises and writes bf16 output; otherwise it
-// writes (O, max, sum) partials and a small merge kernel combines splits.
+// Work split: a CTA owns two 128-row tiles ("a" and "b") of the query rows
+// of one KV head (row r = slot * G + g, so the G query heads of a KV head
+// share every K/V byte) and one split of that head's keys; the splits of one
+// (sequence, head, tile pair) form a thread-block cluster of up to 16 CTAs.
+//   warp 0      TMA: both Q tiles once, then 128-key K and V chunks into
+//               two-stage rings (128-byte swizzle);
+//   warp 1      tcgen05.mma: S_x = Q_x K^T into tensor memory, then
+//               O_x += P_x V with P_x read from tensor memory; the order
+//               PV_a(j), S_a(j+1), PV_b(j), S_b(j+1) lets one tile's
+//               softmax run while the tensor core works on the other;
+//   warps 4-7   softmax of tile a, warps 8-11 of tile b, one thread per row
+//               (= tensor-memory lane): read S, apply the prefix + ancestor
+//               mask, keep a running max that rescales O only when it grows
+//               by more than 2^8, write P as bf16 over S's columns.
+// Tensor memory (512 columns): S_a | S_b | O_a | O_b.
+// After the last MMA every CTA stages its rows as O/l in bf16 plus the
+// log-sum-exp, and (after one cluster barrier) bulk-copies each block of
+// rows to the cluster CTA that owns them through distributed shared memory;
+// each CTA then combines its rows across all splits locally and writes bf16
+// output.  No global workspace, no second kernel.
 // Every mbarrier wait is bounded: on timeout the CTA flags
-// LTD_DEVERR_TIMEOUT, drains its own TMA loads and MMAs, frees its tensor
-// memory and returns.
+// LTD_DEVERR_TIMEOUT, drains its own TMA loads and MMAs, and still joins
+// the cluster barrier and sends every block its peers expect (so no peer
+// waits on it forever), frees its tensor memory and returns.
+#include <mutex>
+
 #include "ltd_common.cuh"
 #include "ltd_internal.h"
 #include "tc_util.cuh"
@@ -26,37 +35,62 @@ namespace ltd {
 
 namespace {
 
-constexpr int kBM = 128;  // query rows per CTA = TMEM lanes
+constexpr int kBM = 128;  // rows per tile = TMEM lanes
 constexpr int kBN = 128;  // keys per chunk
 constexpr int kD = 128;
-constexpr int kThreads = 256;
+constexpr int kRows = 2 * kBM;
+constexpr int kThreads = 384;
+constexpr int kWarps = kThreads / 32;
 constexpr int kMaxW32 = LTD_MAX_N / 32;
-constexpr uint32_t kHalf = 16384;       // 128 rows x 128 bytes
-constexpr uint32_t kTile = 2 * kHalf;   // 128 x 128 bf16
-constexpr uint32_t kOffQ = 0;
-constexpr uint32_t kOffK = kOffQ + kTile;
-constexpr uint32_t kOffV = kOffK + 2 * kTile;
-constexpr uint32_t kOffP = kOffV + 2 * kTile;
-constexpr uint32_t kOffMask = kOffP + kTile;
-constexpr uint32_t kOffBar = kOffMask + kBM * kMaxW32 * 4;
-constexpr uint32_t kOffHolder = kOffBar + 16 * 8;
+constexpr int kMaxCluster = 16;
+constexpr uint32_t kHalf = 16384;      // 128 rows x 128 bytes
+constexpr uint32_t kTile = 2 * kHalf;  // 128 x 128 bf16
+constexpr uint32_t kOffQ = 0;                        // Q_a, Q_b
+constexpr uint32_t kOffK = kOffQ + 2 * kTile;        // two stages
+constexpr uint32_t kOffV = kOffK + 2 * kTile;        // two stages
+constexpr uint32_t kOffMask = kOffV + 2 * kTile;     // [256][8] words
+constexpr uint32_t kOffBar = kOffMask + kRows * kMaxW32 * 4;
+constexpr uint32_t kOffHolder = kOffBar + 32 * 8;
 constexpr uint32_t kSmemBytes = kOffHolder + 16 + 1024;  // + alignment slack
-constexpr uint32_t kTmemCols = 512;  // S0 | S1 | O (| unused)
+// Split reduction, over the Q/K/V space once the MMAs have finished.  CTA r
+// of the cluster owns rows [r R, r R + R), R = ceil(256 / splits) rounded up
+// to a multiple of 4, and receives every split's normalised O (bf16, 256
+// bytes per row, 16-byte chunks swizzled by row) and log-sum-exp for them.
+constexpr uint32_t kRowBytes = kD * 2;
+constexpr uint32_t kOffRecvO = 0;                           // [split][R] rows, <= 80 KB
+constexpr uint32_t kOffRecvL = 80 * 1024;                   // [split][R] float, <= 2 KB
+constexpr uint32_t kOffStgO = 96 * 1024;                    // [256] rows
+constexpr uint32_t kOffStgL = kOffStgO + kRows * kRowBytes;  // [256] float
+constexpr uint32_t kTmemCols = 512;
 constexpr float kRescaleThreshold = 8.f;  // log2 units
 
-enum Bar { QFULL = 0, KFULL = 1, VFULL = 3, KVEMPTY = 5, SFULL = 7, SFREE = 9, PFULL = 11,
-           PVDONE = 12, FIN = 13 };
+static_assert(kOffStgL + kRows * 4 <= kOffMask, "reduction buffers overlap the mask");
+
+enum Bar { QFULL = 0, KFULL = 1, VFULL = 3, KEMPTY = 5, VEMPTY = 7, SFULL = 9, PFULL = 11, FIN = 13,
+           RECV = 14 };
+
+// Optional phase timestamps for performance work (off in normal builds).
+#ifdef LTD_TRACE
+__device__ unsigned long long g_attn_trace[2048][24];
+#define TRACE(slot)                                                                           \
+  do {                                                                                        \
+    const int cta_ = blockIdx.x + gridDim.x * (blockIdx.y + gridDim.y * blockIdx.z);          \
+    if (cta_ < 2048) g_attn_trace[cta_][slot] = tc::globaltimer();                            \
+  } while (0)
+#else
+#define TRACE(slot) \
+  do {              \
+  } while (0)
+#endif
 
 struct TcArgs {
   int32_t batch, hq, hkv, G, n_max, s_cap, max_ctx, W32;
-  int32_t splits, n_tiles;
+  int32_t splits, n_pairs;
   const int32_t* ctx;
   const int32_t* n_verify;
   const uint32_t* mask;
   float scale_log2;
   __nv_bfloat16* out;
-  float4* ws_o;   // [cta][128 rows][32] float4
-  float2* ws_ml;  // [cta][128] (max in log2 units, sum)
   uint32_t* err;
 };
 
@@ -65,33 +99,55 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   return *reinterpret_cast<const uint32_t*>(&v);
 }
 
+// Visibility of keys kk0 .. kk0+31 for one row as a 32-bit mask: keys below
+// ctx are the prefix (always visible), key ctx + j is verified slot j (bit j
+// of the row's ancestor mask), keys from key_hi on are outside this split.
+__device__ __forceinline__ uint32_t low_bits(int n) {
+  return n <= 0 ? 0u : (n >= 32 ? 0xFFFFFFFFu : ((1u << n) - 1u));
+}
+__device__ __forceinline__ uint32_t visible32(int kk0, int ctx, int key_hi, int W32,
+                                              const uint32_t* mbits) {
+  const uint32_t in_range = low_bits(key_hi - kk0);
+  const uint32_t prefix = low_bits(ctx - kk0);
+  uint32_t tree = 0u;
+  const int js0 = kk0 - ctx;  // slot of bit 0 of the window (may be negative)
+  if (js0 > -32 && js0 < 32 * W32) {
+    const int w = js0 >> 5;  // floor division
+    const int sh = js0 & 31;
+    const uint32_t lo = (w >= 0 && w < W32) ? mbits[w] : 0u;
+    const uint32_t hi = (w + 1 >= 0 && w + 1 < W32) ? mbits[w + 1] : 0u;
+    tree = __funnelshift_r(lo, hi, sh);
+  }
+  return in_range & (prefix | tree);
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CUtensorMap tk,
                    const __grid_constant__ CUtensorMap tv, const TcArgs a) {
   extern __shared__ uint8_t smem_raw[];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int split = blockIdx.x, tile = blockIdx.y;
+  if (tid == 0) TRACE(0);
+  const int split = blockIdx.x, pair = blockIdx.y;
   const int b = blockIdx.z / a.hkv, kvh = blockIdx.z % a.hkv;
 
+  // Everything a CTA returns early on is shared by its whole cluster (same
+  // sequence, head and tile pair), so clusters return as a unit.
   const int ctx = a.ctx[b];
   const int N = a.n_verify[b];
   if (N < 1 || N > a.n_max || ctx < 0 || ctx > a.max_ctx || ctx + N > a.s_cap) {
-    if (tid == 0 && split == 0 && tile == 0 && kvh == 0)
+    if (tid == 0 && split == 0 && pair == 0 && kvh == 0)
       flag_error(a.err, (N < 1 || N > a.n_max) ? LTD_DEVERR_NVERIFY : LTD_DEVERR_CTX);
     return;
   }
   const int M = N * a.G;
-  if (tile * kBM >= M) return;
+  const int row0 = pair * kRows;
+  if (row0 >= M) return;
+  const bool has_b = row0 + kBM < M;
   const int nk = ctx + N;
   const int nch = (nk + kBN - 1) / kBN;
   const int cs = split * nch / a.splits, ce = (split + 1) * nch / a.splits;
   const int nc = ce - cs;
   const int key_lo = cs * kBN, key_hi = min(ce * kBN, nk);
-  const int64_t cta = ((static_cast<int64_t>(blockIdx.z) * a.n_tiles + tile) * a.splits) + split;
-  if (nc <= 0) {  // empty split: contributes nothing to the merge
-    if (tid >= 128) a.ws_ml[cta * kBM + (tid - 128)] = make_float2(-CUDART_INF_F, 0.f);
-    return;
-  }
 
   const uint32_t raw = tc::smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -105,256 +161,366 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int s = 0; s < 2; ++s) {
       tc::mbar_init(bar(KFULL + s), 1);
       tc::mbar_init(bar(VFULL + s), 1);
-      tc::mbar_init(bar(KVEMPTY + s), 1);
+      tc::mbar_init(bar(KEMPTY + s), 1);
+      tc::mbar_init(bar(VEMPTY + s), 1);
       tc::mbar_init(bar(SFULL + s), 1);
-      tc::mbar_init(bar(SFREE + s), 128);
+      tc::mbar_init(bar(PFULL + s), 128);
     }
-    tc::mbar_init(bar(PFULL), 128);
-    tc::mbar_init(bar(PVDONE), 1);
     tc::mbar_init(bar(FIN), 1);
+    tc::mbar_init(bar(RECV), 1);
     tc::mbar_init_fence();
   }
   if (warp == 1) {
     tc::tmem_alloc(tc::smem_u32(holder), kTmemCols);
     tc::tmem_relinquish();
   }
-  const int i = tid - 128;  // softmax row (TMEM lane) for warps 4-7
-  const int R = tile * kBM + i;
-  const bool row_ok = (tid >= 128) && (R < M);
-  const int slot = row_ok ? R / a.G : 0;
+  // softmax threads: tile x, TMEM lane rr % 128, staging row rr
+  const int rr = tid - 128;
+  const int x = rr >> 7;
+  const int R = row0 + rr;
+  const bool row_ok = tid >= 128 && R < M;
   if (tid >= 128) {
+    const int slot = row_ok ? R / a.G : 0;
     for (int w = 0; w < a.W32; ++w)
-      mask_s[i * kMaxW32 + w] =
+      mask_s[rr * kMaxW32 + w] =
           row_ok ? a.mask[(static_cast<int64_t>(b) * a.n_max + slot) * a.W32 + w] : 0u;
   }
   tc::fence_before_sync();
   __syncthreads();
   tc::fence_after_sync();
   const uint32_t tmem = *holder;
+  if (tid == 0) TRACE(1);
   bool ok = true;
+  const bool tile_active = tid >= 128 && (x == 0 || has_b) && nc > 0;
+  float m = -CUDART_INF_F, l = 0.f;
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
-    if (lane == 0) {
-      int issued[2] = {0, 0};
+    if (lane == 0 && nc > 0) {
+      int nk_issued[2] = {0, 0}, nv_issued[2] = {0, 0};
       tc::tma_prefetch(&tq);
       tc::tma_prefetch(&tk);
       tc::tma_prefetch(&tv);
-      tc::mbar_expect_tx(bar(QFULL), kTile);
-      const int qrow = b * a.n_max + tile * (kBM / a.G);
-      for (int h = 0; h < 2; ++h)
-        tc::tma_load_3d(base + kOffQ + h * kHalf, &tq, bar(QFULL), h * 64, kvh * a.G, qrow);
+      tc::mbar_expect_tx(bar(QFULL), has_b ? 2 * kTile : kTile);
+      for (int t = 0; t < (has_b ? 2 : 1); ++t) {
+        const int qrow = b * a.n_max + (row0 + t * kBM) / a.G;
+        for (int h = 0; h < 2; ++h)
+          tc::tma_load_3d(base + kOffQ + t * kTile + h * kHalf, &tq, bar(QFULL), h * 64, kvh * a.G,
+                          qrow);
+      }
       const int kvrow = b * a.hkv + kvh;
       for (int j = 0; j < nc && ok; ++j) {
         const int st = j & 1;
-        if (j >= 2) ok = tc::mbar_wait(bar(KVEMPTY + st), ((j >> 1) - 1) & 1);
-        if (!ok) break;
         const int key0 = key_lo + j * kBN;
+        if (j >= 2) ok = tc::mbar_wait(bar(KEMPTY + st), ((j >> 1) - 1) & 1);
+        if (!ok) break;
         tc::mbar_expect_tx(bar(KFULL + st), kTile);
         for (int h = 0; h < 2; ++h)
           tc::tma_load_3d(base + kOffK + st * kTile + h * kHalf, &tk, bar(KFULL + st), h * 64, key0,
                           kvrow);
+        ++nk_issued[st];
+        if (j >= 2) ok = tc::mbar_wait(bar(VEMPTY + st), ((j >> 1) - 1) & 1);
+        if (!ok) break;
         tc::mbar_expect_tx(bar(VFULL + st), kTile);
         for (int h = 0; h < 2; ++h)
           tc::tma_load_3d(base + kOffV + st * kTile + h * kHalf, &tv, bar(VFULL + st), h * 64, key0,
                           kvrow);
-        ++issued[st];
+        ++nv_issued[st];
       }
-      // drain: every load this CTA issued has landed before it can exit
+      // drain: every load this CTA issued has landed before shared memory is reused
       tc::mbar_wait(bar(QFULL), 0);
-      for (int st = 0; st < 2; ++st)
-        if (issued[st] > 0) {
-          tc::mbar_wait(bar(KFULL + st), (issued[st] - 1) & 1);
-          tc::mbar_wait(bar(VFULL + st), (issued[st] - 1) & 1);
-        }
+      for (int st = 0; st < 2; ++st) {
+        if (nk_issued[st] > 0) tc::mbar_wait(bar(KFULL + st), (nk_issued[st] - 1) & 1);
+        if (nv_issued[st] > 0) tc::mbar_wait(bar(VFULL + st), (nv_issued[st] - 1) & 1);
+      }
       if (!ok) flag_error(a.err, LTD_DEVERR_TIMEOUT);
     }
   } else if (warp == 1) {
     // ----------------------------------------------------------------- MMA
-    if (lane == 0) {
+    if (lane == 0 && nc > 0) {
       const uint32_t id_s = tc::idesc_bf16(kBM, kBN, false);
       const uint32_t id_o = tc::idesc_bf16(kBM, kD, true);
-      const uint32_t t_o = tmem + 2 * kBN;
+      const int ntile = has_b ? 2 : 1;
+      auto issue_s = [&](int t, int st) {
+        for (int ks = 0; ks < 8; ++ks) {
+          const uint64_t da =
+              tc::sdesc_sw128(base + kOffQ + t * kTile + (ks >> 2) * kHalf + (ks & 3) * 32, 16, 1024);
+          const uint64_t db =
+              tc::sdesc_sw128(base + kOffK + st * kTile + (ks >> 2) * kHalf + (ks & 3) * 32, 16, 1024);
+          tc::mma_bf16(tmem + t * kBN, da, db, id_s, ks > 0 ? 1u : 0u);
+        }
+      };
+      auto issue_pv = [&](int t, int st, bool acc) {
+        for (int ks = 0; ks < 8; ++ks) {
+          const uint64_t db = tc::sdesc_sw128(base + kOffV + st * kTile + ks * 2048, kHalf, 1024);
+          tc::mma_bf16_ts(tmem + 2 * kBN + t * kD, tmem + t * kBN + 8 * ks, db, id_o,
+                          (acc || ks > 0) ? 1u : 0u);
+        }
+      };
       ok = tc::mbar_wait(bar(QFULL), 0);
-      for (int j = 0; j <= nc && ok; ++j) {
-        if (j < nc) {
-          const int st = j & 1;
-          ok = tc::mbar_wait(bar(KFULL + st), (j >> 1) & 1);
-          if (ok && j >= 2) ok = tc::mbar_wait(bar(SFREE + st), ((j >> 1) - 1) & 1);
-          if (!ok) break;
-          tc::fence_after_sync();
-          for (int ks = 0; ks < 8; ++ks) {
-            const uint64_t da = tc::sdesc_sw128(base + kOffQ + (ks >> 2) * kHalf + (ks & 3) * 32, 16, 1024);
-            const uint64_t db =
-                tc::sdesc_sw128(base + kOffK + st * kTile + (ks >> 2) * kHalf + (ks & 3) * 32, 16, 1024);
-            tc::mma_bf16(tmem + st * kBN, da, db, id_s, ks > 0 ? 1u : 0u);
-          }
-          tc::mma_commit(bar(SFULL + st));
+      TRACE(2);
+      if (ok) ok = tc::mbar_wait(bar(KFULL + 0), 0);
+      if (ok) {
+        tc::fence_after_sync();
+        for (int t = 0; t < ntile; ++t) {
+          issue_s(t, 0);
+          tc::mma_commit(bar(SFULL + t));
         }
-        if (j >= 1) {
-          const int jj = j - 1, st = jj & 1;
-          ok = tc::mbar_wait(bar(PFULL), jj & 1);
-          if (ok) ok = tc::mbar_wait(bar(VFULL + st), (jj >> 1) & 1);
-          if (!ok) break;
-          tc::fence_after_sync();
-          for (int ks = 0; ks < 8; ++ks) {
-            const uint64_t da = tc::sdesc_sw128(base + kOffP + (ks >> 2) * kHalf + (ks & 3) * 32, 16, 1024);
-            const uint64_t db = tc::sdesc_sw128(base + kOffV + st * kTile + ks * 2048, kHalf, 1024);
-            tc::mma_bf16(t_o, da, db, id_o, (jj > 0 || ks > 0) ? 1u : 0u);
-          }
-          tc::mma_commit(bar(PVDONE));
-          tc::mma_commit(bar(KVEMPTY + st));
-        }
+        tc::mma_commit(bar(KEMPTY + 0));
       }
-      // all MMAs issued by this thread complete before tensor memory is freed
+      for (int j = 0; j < nc && ok; ++j) {
+        const int st = j & 1;
+        const bool nxt = j + 1 < nc;
+        ok = tc::mbar_wait(bar(VFULL + st), (j >> 1) & 1);
+        if (ok && nxt) ok = tc::mbar_wait(bar(KFULL + ((j + 1) & 1)), ((j + 1) >> 1) & 1);
+        for (int t = 0; t < ntile && ok; ++t) {
+          ok = tc::mbar_wait(bar(PFULL + t), j & 1);
+          if (!ok) break;
+          tc::fence_after_sync();
+          issue_pv(t, st, j > 0);
+          if (nxt) {
+            issue_s(t, (j + 1) & 1);
+            tc::mma_commit(bar(SFULL + t));
+          }
+        }
+        if (!ok) break;
+        if (nxt) tc::mma_commit(bar(KEMPTY + ((j + 1) & 1)));
+        tc::mma_commit(bar(VEMPTY + st));
+      }
+      // every MMA of this CTA completes before tensor memory is read or freed
       tc::mma_commit(bar(FIN));
       tc::mbar_wait(bar(FIN), 0);
       if (!ok) flag_error(a.err, LTD_DEVERR_TIMEOUT);
     }
-  } else if (warp >= 4) {
+  } else if (warp >= 4 && tile_active) {
     // ------------------------------------------------------------- softmax
-    const uint32_t t_lane = tmem + ((32u * (warp & 3)) << 16);
-    const uint32_t* mrow_bits = mask_s + i * kMaxW32;
-    float m = -CUDART_INF_F, l = 0.f;
+    const uint32_t lane_off = (32u * (warp & 3)) << 16;
+    const uint32_t t_s = tmem + x * kBN + lane_off;
+    const uint32_t t_o = tmem + 2 * kBN + x * kD + lane_off;
+    const uint32_t* mbits = mask_s + rr * kMaxW32;
     const int vis_all_below = min(ctx, key_hi);  // keys below this are all visible
+    const float sl2 = a.scale_log2;
+    const int w32 = a.W32;
     for (int j = 0; j < nc; ++j) {
-      const int sb = j & 1;
-      ok = tc::mbar_wait(bar(SFULL + sb), (j >> 1) & 1);
+      ok = tc::mbar_wait(bar(SFULL + x), j & 1);
       ok = __all_sync(0xFFFFFFFFu, ok);
+      if (tid == 128 && j == 0) TRACE(11);
+
       if (!ok) break;
       tc::fence_after_sync();
-      float s[kBN];
-#pragma unroll
+      const int kbase = key_lo + j * kBN;
+      const bool all_vis = kbase + kBN <= vis_all_below;
+      auto vis_of = [=](int q) {
+        return !row_ok ? 0u
+                       : (all_vis ? 0xFFFFFFFFu
+                                  : visible32(kbase + 32 * q, ctx, key_hi, w32, mbits));
+      };
+      // pass 1: the chunk's row max, 32 columns at a time, without branches
+      // per element; on fully visible fragments the max is taken on the raw
+      // scores (the scale is positive) and scaled once
+      float cm[4] = {-CUDART_INF_F, -CUDART_INF_F, -CUDART_INF_F, -CUDART_INF_F};
+#pragma unroll 1
       for (int q = 0; q < 4; ++q) {
         tc::Frag32 f;
-        tc::tmem_ld32(t_lane + sb * kBN + 32 * q, f);
+        tc::tmem_ld32(t_s + 32 * q, f);
+        const uint32_t vq = vis_of(q);
         tc::tmem_wait_ld(f);
+        if (tid == 128 && j == 0 && q < 2) TRACE(3 + 2 * q);
+        if (vq == 0xFFFFFFFFu) {
+          float r[4] = {-CUDART_INF_F, -CUDART_INF_F, -CUDART_INF_F, -CUDART_INF_F};
 #pragma unroll
-        for (int c = 0; c < 32; ++c) s[32 * q + c] = __uint_as_float(f.r[c]);
-      }
-      tc::fence_before_sync();
-      tc::mbar_arrive(bar(SFREE + sb));
-
-      const int kbase = key_lo + j * kBN;
-      float cmax = -CUDART_INF_F;
-      if (kbase + kBN <= vis_all_below) {
+          for (int c = 0; c < 32; ++c) r[c & 3] = fmaxf(r[c & 3], __uint_as_float(f.r[c]));
 #pragma unroll
-        for (int c = 0; c < kBN; ++c) {
-          s[c] = row_ok ? s[c] * a.scale_log2 : -CUDART_INF_F;
-          cmax = fmaxf(cmax, s[c]);
-        }
-      } else {
+          for (int u = 0; u < 4; ++u) cm[u] = fmaxf(cm[u], r[u] * sl2);
+        } else {
 #pragma unroll
-        for (int c = 0; c < kBN; ++c) {
-          const int kk = kbase + c;
-          bool vis = row_ok && kk < key_hi;
-          if (vis && kk >= ctx) {
-            const int js = kk - ctx;
-            vis = (mrow_bits[js >> 5] >> (js & 31)) & 1u;
+          for (int c = 0; c < 32; ++c) {
+            const float t = ((vq >> c) & 1u) ? __uint_as_float(f.r[c]) * sl2 : -CUDART_INF_F;
+            cm[c & 3] = fmaxf(cm[c & 3], t);
           }
-          s[c] = vis ? s[c] * a.scale_log2 : -CUDART_INF_F;
-          cmax = fmaxf(cmax, s[c]);
         }
+        if (tid == 128 && j == 0 && q < 2) TRACE(4 + 2 * q);
       }
-      // P buffer and O are free once the previous chunk's P V finished
-      if (j >= 1) {
-        ok = tc::mbar_wait(bar(PVDONE), (j - 1) & 1);
-        ok = __all_sync(0xFFFFFFFFu, ok);
-        if (!ok) break;
-      }
+      const float cmax = fmaxf(fmaxf(cm[0], cm[1]), fmaxf(cm[2], cm[3]));
+      if (tid == 128 && j == 0) TRACE(14);
+      // S(j) complete implies P_x(j-1) V finished, so O_x is stable here
       float mnew = m;
       if (cmax > m + kRescaleThreshold || (m == -CUDART_INF_F && cmax > -CUDART_INF_F)) mnew = cmax;
       const bool need = (mnew != m) && (m != -CUDART_INF_F) && (j >= 1);
       if (__any_sync(0xFFFFFFFFu, need)) {
         const float alpha = need ? tc::ex2(m - mnew) : 1.f;
         l *= alpha;
-        tc::fence_after_sync();
-#pragma unroll
+#pragma unroll 1
         for (int q = 0; q < 4; ++q) {
           tc::Frag32 f;
-          tc::tmem_ld32(t_lane + 2 * kBN + 32 * q, f);
+          tc::tmem_ld32(t_o + 32 * q, f);
           tc::tmem_wait_ld(f);
 #pragma unroll
           for (int c = 0; c < 32; ++c) f.r[c] = __float_as_uint(__uint_as_float(f.r[c]) * alpha);
-          tc::tmem_st32(t_lane + 2 * kBN + 32 * q, f);
+          tc::tmem_st32(t_o + 32 * q, f);
         }
-        tc::tmem_wait_st();
       }
       m = mnew;
-      // P row (bf16) into the K-major 128-byte-swizzled operand tile
-      uint8_t* prow = gbase + kOffP + i * 128;
-      float lsum = 0.f;
+      // pass 2: P = 2^(score - m) as bf16 pairs; fragment q (columns
+      // 32q..32q+31) becomes P columns 16q..16q+15, all already read
+      float2 ls2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+      const float mz = (m == -CUDART_INF_F) ? 0.f : m;  // m = -inf only if all are hidden
+      const float2 sl22 = make_float2(sl2, sl2), nm2 = make_float2(-mz, -mz);
+#pragma unroll 1
+      for (int q = 0; q < 4; ++q) {
+        tc::Frag32 f;
+        tc::tmem_ld32(t_s + 32 * q, f);
+        const uint32_t vq = vis_of(q);
+        tc::tmem_wait_ld(f);
+        tc::Frag16 pf;
+        if (vq == 0xFFFFFFFFu) {
 #pragma unroll
-      for (int c8 = 0; c8 < 16; ++c8) {
-        float p[8];
+          for (int c = 0; c < 16; ++c) {
+            const float2 t = __ffma2_rn(
+                make_float2(__uint_as_float(f.r[2 * c]), __uint_as_float(f.r[2 * c + 1])), sl22, nm2);
+            const float2 pp = make_float2(tc::ex2(t.x), tc::ex2(t.y));
+            ls2[c & 1] = __fadd2_rn(ls2[c & 1], pp);
+            pf.r[c] = pack_bf16(pp.x, pp.y);
+          }
+        } else {
 #pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          const float t = s[8 * c8 + e];
-          p[e] = (m == -CUDART_INF_F || t == -CUDART_INF_F) ? 0.f : tc::ex2(t - m);
-          lsum += p[e];
-        }
-        uint4 w;
-        w.x = pack_bf16(p[0], p[1]);
-        w.y = pack_bf16(p[2], p[3]);
-        w.z = pack_bf16(p[4], p[5]);
-        w.w = pack_bf16(p[6], p[7]);
-        const int half = c8 >> 3, cc = c8 & 7;
-        *reinterpret_cast<uint4*>(prow + half * kHalf + ((cc ^ (i & 7)) << 4)) = w;
-      }
-      l += lsum;
-      tc::fence_smem_async();
-      tc::fence_before_sync();
-      tc::mbar_arrive(bar(PFULL));
-    }
-    if (ok) {
-      ok = tc::mbar_wait(bar(PVDONE), (nc - 1) & 1);
-      ok = __all_sync(0xFFFFFFFFu, ok);
-    }
-    if (ok) {
-      tc::fence_after_sync();
-      const int g = row_ok ? R % a.G : 0;
-      if (a.splits == 1) {
-        const float inv = l > 0.f ? 1.f / l : 0.f;
-        __nv_bfloat16* dst =
-            a.out + ((static_cast<int64_t>(b) * a.n_max + slot) * a.hq + kvh * a.G + g) * kD;
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          tc::Frag32 f;
-          tc::tmem_ld32(t_lane + 2 * kBN + 32 * q, f);
-          tc::tmem_wait_ld(f);
-          if (row_ok) {
-#pragma unroll
-            for (int c = 0; c < 32; c += 8) {
-              uint4 w;
-              w.x = pack_bf16(__uint_as_float(f.r[c]) * inv, __uint_as_float(f.r[c + 1]) * inv);
-              w.y = pack_bf16(__uint_as_float(f.r[c + 2]) * inv, __uint_as_float(f.r[c + 3]) * inv);
-              w.z = pack_bf16(__uint_as_float(f.r[c + 4]) * inv, __uint_as_float(f.r[c + 5]) * inv);
-              w.w = pack_bf16(__uint_as_float(f.r[c + 6]) * inv, __uint_as_float(f.r[c + 7]) * inv);
-              *reinterpret_cast<uint4*>(dst + 32 * q + c) = w;
-            }
+          for (int c = 0; c < 16; ++c) {
+            const float t0 =
+                ((vq >> (2 * c)) & 1u) ? __uint_as_float(f.r[2 * c]) * sl2 : -CUDART_INF_F;
+            const float t1 =
+                ((vq >> (2 * c + 1)) & 1u) ? __uint_as_float(f.r[2 * c + 1]) * sl2 : -CUDART_INF_F;
+            const float2 pp = make_float2(tc::ex2(t0 - mz), tc::ex2(t1 - mz));
+            ls2[c & 1] = __fadd2_rn(ls2[c & 1], pp);
+            pf.r[c] = pack_bf16(pp.x, pp.y);
           }
         }
-      } else {
-        float4* wo = a.ws_o + (cta * kBM + i) * 32;
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          tc::Frag32 f;
-          tc::tmem_ld32(t_lane + 2 * kBN + 32 * q, f);
-          tc::tmem_wait_ld(f);
-#pragma unroll
-          for (int c4 = 0; c4 < 8; ++c4)
-            wo[8 * q + c4] =
-                make_float4(__uint_as_float(f.r[4 * c4]), __uint_as_float(f.r[4 * c4 + 1]),
-                            __uint_as_float(f.r[4 * c4 + 2]), __uint_as_float(f.r[4 * c4 + 3]));
-        }
-        a.ws_ml[cta * kBM + i] = make_float2(row_ok ? m : -CUDART_INF_F, row_ok ? l : 0.f);
+        tc::tmem_st16(t_s + 16 * q, pf);
       }
-    } else if (lane == 0) {
-      flag_error(a.err, LTD_DEVERR_TIMEOUT);
+      const float2 lsum = __fadd2_rn(ls2[0], ls2[1]);
+      l += lsum.x + lsum.y;
+      if (tid == 128 && j == 0) TRACE(15);
+      tc::tmem_wait_st();
+      tc::fence_before_sync();
+      tc::mbar_arrive(bar(PFULL + x));
+      if (tid == 128 && j == 0) TRACE(12);
     }
+    if (tid == 128) TRACE(13);
+    if (ok) {
+      ok = tc::mbar_wait(bar(FIN), 0);
+      ok = __all_sync(0xFFFFFFFFu, ok);
+    }
+    if (!ok && lane == 0) flag_error(a.err, LTD_DEVERR_TIMEOUT);
   }
 
+  // --------------------- exchange partials with the cluster (bulk DSMEM)
   tc::fence_before_sync();
+  __syncthreads();
+  if (tid == 0) TRACE(16);
+  const int S = a.splits;
+  const int rank = static_cast<int>(tc::cluster_rank());
+  const int R4 = (((kRows + S - 1) / S) + 3) & ~3;
+  const int n_own = max(0, min(R4, kRows - rank * R4));
+  if (tid == 0) tc::mbar_expect_tx(bar(RECV), static_cast<uint32_t>(S * n_own) * (kRowBytes + 4));
+  // stage this split's rows: O / l in bf16 and lse = m + log2(l)
+  if (tid >= 128) {
+    float lse = -CUDART_INF_F;
+    uint8_t* srow = gbase + kOffStgO + rr * kRowBytes;
+    if (tile_active && ok) {
+      tc::fence_after_sync();
+      const uint32_t t_o = tmem + 2 * kBN + x * kD + ((32u * (warp & 3)) << 16);
+      const float inv = l > 0.f ? 1.f / l : 0.f;
+#pragma unroll 1
+      for (int q = 0; q < 4; ++q) {
+        tc::Frag32 f;
+        tc::tmem_ld32(t_o + 32 * q, f);
+        tc::tmem_wait_ld(f);
+#pragma unroll
+        for (int c16 = 0; c16 < 4; ++c16) {
+          const int c = 4 * q + c16;  // 16-byte chunk (8 values) of the row
+          uint4 w;
+          w.x = pack_bf16(__uint_as_float(f.r[8 * c16]) * inv, __uint_as_float(f.r[8 * c16 + 1]) * inv);
+          w.y = pack_bf16(__uint_as_float(f.r[8 * c16 + 2]) * inv, __uint_as_float(f.r[8 * c16 + 3]) * inv);
+          w.z = pack_bf16(__uint_as_float(f.r[8 * c16 + 4]) * inv, __uint_as_float(f.r[8 * c16 + 5]) * inv);
+          w.w = pack_bf16(__uint_as_float(f.r[8 * c16 + 6]) * inv, __uint_as_float(f.r[8 * c16 + 7]) * inv);
+          *reinterpret_cast<uint4*>(srow + ((c ^ (rr & 15)) << 4)) = w;
+        }
+      }
+      if (row_ok && l > 0.f) lse = m + __log2f(l);
+    }
+    reinterpret_cast<float*>(gbase + kOffStgL)[rr] = lse;
+    tc::fence_smem_async();  // staging becomes visible to the bulk copies
+  }
+  __syncthreads();
+  // every CTA has registered its receive count and is past its last MMA and
+  // TMA load, so its ring buffers can now be written by peers
+  tc::cluster_sync();
+  if (tid == 0) TRACE(7);
+  if (tid == 0) {
+    for (int r = 0; r < S; ++r) {
+      const int n = max(0, min(R4, kRows - r * R4));
+      if (n == 0) continue;
+      const uint32_t pbar = tc::mapa(bar(RECV), r);
+      tc::bulk_s2cluster(tc::mapa(base + kOffRecvO + (rank * R4) * kRowBytes, r),
+                         base + kOffStgO + (r * R4) * kRowBytes, n * kRowBytes, pbar);
+      tc::bulk_s2cluster(tc::mapa(base + kOffRecvL + (rank * R4) * 4, r),
+                         base + kOffStgL + (r * R4) * 4, n * 4, pbar);
+    }
+    tc::bulk_commit();
+  }
+  const bool got = tc::mbar_wait(bar(RECV), 0);
+  if (!got && tid == 0) flag_error(a.err, LTD_DEVERR_TIMEOUT);
+  if (tid == 0) TRACE(8);
+
+  // ------------------------- combine the splits of this CTA's rows (local)
+  if (got) {
+    const uint8_t* recv_o = gbase + kOffRecvO;
+    const float* recv_l = reinterpret_cast<const float*>(gbase + kOffRecvL);
+    const int ch = lane >> 1, half = lane & 1;  // lane owns output dims 4 lane .. 4 lane + 3
+    for (int lr = warp; lr < n_own; lr += kWarps) {
+      const int r = rank * R4 + lr;
+      const int Rr = row0 + r;
+      if (Rr >= M) continue;
+      const uint32_t coff = (((ch ^ (r & 15)) << 4) + half * 8);
+      float lp[kMaxCluster];
+      uint2 vp[kMaxCluster];
+#pragma unroll
+      for (int p = 0; p < kMaxCluster; ++p) {
+        if (p < S) {
+          lp[p] = recv_l[p * R4 + lr];
+          vp[p] = *reinterpret_cast<const uint2*>(recv_o + (p * R4 + lr) * kRowBytes + coff);
+        }
+      }
+      float mx = -CUDART_INF_F;
+#pragma unroll
+      for (int p = 0; p < kMaxCluster; ++p)
+        if (p < S) mx = fmaxf(mx, lp[p]);
+      float acc[4] = {0.f, 0.f, 0.f, 0.f};
+      float L = 0.f;
+#pragma unroll
+      for (int p = 0; p < kMaxCluster; ++p) {
+        if (p < S && lp[p] > -CUDART_INF_F) {
+          const float w = tc::ex2(lp[p] - mx);
+          L += w;
+          acc[0] += w * __uint_as_float(vp[p].x << 16);
+          acc[1] += w * __uint_as_float(vp[p].x & 0xFFFF0000u);
+          acc[2] += w * __uint_as_float(vp[p].y << 16);
+          acc[3] += w * __uint_as_float(vp[p].y & 0xFFFF0000u);
+        }
+      }
+      const float inv = L > 0.f ? 1.f / L : 0.f;
+      const int slot = Rr / a.G, g = Rr % a.G;
+      __nv_bfloat16* dst = a.out +
+                           ((static_cast<int64_t>(b) * a.n_max + slot) * a.hq + kvh * a.G + g) * kD +
+                           4 * lane;
+      uint2 w2;
+      w2.x = pack_bf16(acc[0] * inv, acc[1] * inv);
+      w2.y = pack_bf16(acc[2] * inv, acc[3] * inv);
+      *reinterpret_cast<uint2*>(dst) = w2;
+    }
+  }
+  if (tid == 0) TRACE(9);
+  // the sources of this CTA's outgoing copies stay valid until read
+  if (tid == 0) tc::bulk_wait_read();
   __syncthreads();
   if (warp == 1) {
     __syncwarp();
@@ -363,68 +529,21 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-// Combine the split partials of every row: weights 2^(m_s - max m).  One
-// warp per row, lane c owns output dims 4c..4c+3, so both the partial reads
-// (row-major [cta][row][32 float4]) and the bf16 output writes coalesce.
-constexpr int kMergeRows = 8;
-
-__global__ void __launch_bounds__(kMergeRows * 32) attn_tc_merge_kernel(const TcArgs a) {
-  const int lane = threadIdx.x & 31;
-  const int64_t grow = static_cast<int64_t>(blockIdx.x) * kMergeRows + (threadIdx.x >> 5);
-  const int64_t rows_per_bh = static_cast<int64_t>(a.n_tiles) * kBM;
-  const int bh = static_cast<int>(grow / rows_per_bh);
-  if (bh >= a.batch * a.hkv) return;
-  const int R = static_cast<int>(grow % rows_per_bh);
-  const int tile = R / kBM, i = R % kBM;
-  const int b = bh / a.hkv, kvh = bh % a.hkv;
-  const int ctx = a.ctx[b];
-  const int N = a.n_verify[b];
-  if (N < 1 || N > a.n_max || ctx < 0 || ctx > a.max_ctx || ctx + N > a.s_cap) return;
-  if (R >= N * a.G) return;
-  const int slot = R / a.G, g = R % a.G;
-  const int64_t cta0 = (static_cast<int64_t>(bh) * a.n_tiles + tile) * a.splits;
-  float mx = -CUDART_INF_F;
-  for (int s = 0; s < a.splits; ++s) {
-    const float2 ml = a.ws_ml[(cta0 + s) * kBM + i];
-    if (ml.y > 0.f) mx = fmaxf(mx, ml.x);
-  }
-  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-  float L = 0.f;
-  for (int s = 0; s < a.splits; ++s) {
-    const float2 ml = a.ws_ml[(cta0 + s) * kBM + i];
-    if (!(ml.y > 0.f)) continue;
-    const float w = tc::ex2(ml.x - mx);
-    L += w * ml.y;
-    const float4 v = a.ws_o[((cta0 + s) * kBM + i) * 32 + lane];
-    acc.x += w * v.x;
-    acc.y += w * v.y;
-    acc.z += w * v.z;
-    acc.w += w * v.w;
-  }
-  const float inv = L > 0.f ? 1.f / L : 0.f;
-  __nv_bfloat16* dst =
-      a.out + ((static_cast<int64_t>(b) * a.n_max + slot) * a.hq + kvh * a.G + g) * kD + 4 * lane;
-  uint2 w2;
-  w2.x = pack_bf16(acc.x * inv, acc.y * inv);
-  w2.y = pack_bf16(acc.z * inv, acc.w * inv);
-  *reinterpret_cast<uint2*>(dst) = w2;
-}
-
 struct Plan {
-  int n_tiles, splits;
+  int n_pairs, splits;
 };
 
 Plan plan(int32_t batch, int32_t hq, int32_t hkv, int32_t n_max, int32_t max_ctx) {
   const int G = hq / hkv;
   Plan p{};
-  p.n_tiles = (n_max * G + kBM - 1) / kBM;
-  const int64_t base = static_cast<int64_t>(batch) * hkv * p.n_tiles;
+  p.n_pairs = (n_max * G + kRows - 1) / kRows;
+  const int64_t units = static_cast<int64_t>(batch) * hkv * p.n_pairs;
   const int nch = (max_ctx + n_max + kBN - 1) / kBN;
   constexpr int64_t kSMs = 152;
-  int s = base >= kSMs ? 1 : static_cast<int>(kSMs / base);
-  s = s < 1 ? 1 : s;
+  int s = units >= kSMs ? 1 : static_cast<int>(kSMs / units);
+  s = s > kMaxCluster ? kMaxCluster : s;
   s = s > nch ? nch : s;
-  p.splits = s;
+  p.splits = s < 1 ? 1 : s;
   return p;
 }
 
@@ -448,6 +567,52 @@ EncodeFn encode_fn() {
   return fn;
 }
 
+// Cluster size for `units` independent clusters: the largest s <= want for
+// which the device can keep all of them resident at once (one wave), else
+// the largest s it can run at all.  Asked once per device and size.
+int max_active_clusters(int s) {
+  static std::mutex mu;
+  static int known[128][kMaxCluster + 1];
+  static bool init = false;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 128) return 0;
+  std::lock_guard<std::mutex> lock(mu);
+  if (!init) {
+    for (auto& row : known)
+      for (int& v : row) v = -1;
+    init = true;
+  }
+  if (known[dev][s] < 0) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(s, 1, 1);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = kSmemBytes;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = s;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    const cudaError_t e = cudaOccupancyMaxActiveClusters(&n, attn_tc_kernel, &cfg);
+    if (e != cudaSuccess) {
+      (void)cudaGetLastError();
+      n = 0;
+    }
+    known[dev][s] = n;
+  }
+  return known[dev][s];
+}
+
+int fit_splits(int want, int64_t units) {
+  for (int s = want; s > 1; --s)
+    if (max_active_clusters(s) >= units) return s;
+  for (int s = want; s > 1; --s)
+    if (max_active_clusters(s) > 0) return s;
+  return 1;
+}
+
 }  // namespace
 
 bool encode_tmap_bf16_3d(CUtensorMap* map, const void* base, uint64_t d0, uint64_t d1, uint64_t d2,
@@ -469,18 +634,9 @@ bool attn_tc_supported(const AttnParams& p, ltd_dtype dtype) {
   return G >= 1 && G <= kBM && kBM % G == 0 && p.n_max <= LTD_MAX_N;
 }
 
-size_t attn_tc_workspace(int32_t batch, int32_t hq, int32_t hkv, int32_t d, int32_t n_max,
-                         int32_t max_ctx) {
-  (void)d;
-  const Plan pl = plan(batch, hq, hkv, n_max, max_ctx);
-  if (pl.splits == 1) return 0;
-  const size_t ctas = static_cast<size_t>(batch) * hkv * pl.n_tiles * pl.splits;
-  return ctas * (32 * kBM * sizeof(float4) + kBM * sizeof(float2));
-}
+size_t attn_tc_workspace(int32_t, int32_t, int32_t, int32_t, int32_t, int32_t) { return 0; }
 
-int32_t attn_tc_launches(int32_t batch, int32_t hq, int32_t hkv, int32_t n_max, int32_t max_ctx) {
-  return plan(batch, hq, hkv, n_max, max_ctx).splits > 1 ? 2 : 1;
-}
+int32_t attn_tc_launches(int32_t, int32_t, int32_t, int32_t, int32_t) { return 1; }
 
 cudaError_t launch_attn_tc(const AttnParams& p, cudaStream_t s) {
   const Plan pl = plan(p.batch, p.hq, p.hkv, p.n_max, p.max_ctx);
@@ -494,18 +650,13 @@ cudaError_t launch_attn_tc(const AttnParams& p, cudaStream_t s) {
   a.max_ctx = p.max_ctx;
   a.W32 = (p.n_max + 31) / 32;
   a.splits = pl.splits;
-  a.n_tiles = pl.n_tiles;
+  a.n_pairs = pl.n_pairs;
   a.ctx = p.ctx;
   a.n_verify = p.n_verify;
   a.mask = p.mask;
   a.scale_log2 = p.scale * 1.4426950408889634f;
   a.out = static_cast<__nv_bfloat16*>(p.out);
-  const size_t ctas = static_cast<size_t>(p.batch) * p.hkv * pl.n_tiles * pl.splits;
-  a.ws_o = static_cast<float4*>(p.ws);
-  a.ws_ml = reinterpret_cast<float2*>(static_cast<char*>(p.ws) + ctas * 32 * kBM * sizeof(float4));
   a.err = p.err;
-  if (pl.splits > 1 && p.ws_bytes < attn_tc_workspace(p.batch, p.hq, p.hkv, p.d, p.n_max, p.max_ctx))
-    return cudaErrorInvalidValue;
 
   CUtensorMap tq, tk, tv;
   const uint64_t row = kD * 2;
@@ -521,14 +672,33 @@ cudaError_t launch_attn_tc(const AttnParams& p, cudaStream_t s) {
   cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(kSmemBytes));
   if (e != cudaSuccess) return e;
-  const dim3 grid(pl.splits, pl.n_tiles, p.batch * p.hkv);
-  attn_tc_kernel<<<grid, kThreads, kSmemBytes, s>>>(tq, tk, tv, a);
-  e = cudaGetLastError();
-  if (e != cudaSuccess || pl.splits == 1) return e;
-  const int64_t rows = static_cast<int64_t>(p.batch) * p.hkv * pl.n_tiles * kBM;
-  attn_tc_merge_kernel<<<static_cast<unsigned>((rows + kMergeRows - 1) / kMergeRows),
-                         kMergeRows * 32, 0, s>>>(a);
-  return cudaGetLastError();
+  e = cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  if (e != cudaSuccess) return e;
+
+  const int splits =
+      fit_splits(pl.splits, static_cast<int64_t>(p.batch) * p.hkv * pl.n_pairs);
+  a.splits = splits;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(splits, pl.n_pairs, p.batch * p.hkv);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = splits;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, attn_tc_kernel, tq, tk, tv, a);
 }
 
 }  // namespace ltd
+
+#ifdef LTD_TRACE
+extern "C" int ltd_attn_trace_read(unsigned long long* host, int n) {
+  return cudaMemcpyFromSymbol(host, ltd::g_attn_trace, sizeof(unsigned long long) * n) == cudaSuccess
+             ? 0
+             : 1;
+}
+#endif

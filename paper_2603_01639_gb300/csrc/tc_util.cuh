@@ -109,7 +109,8 @@ __device__ __forceinline__ void mma_commit(uint32_t bar) {
 }
 
 // 32 consecutive 32-bit columns of this thread's TMEM lane.  The registers
-// are tied through the wait so no use can be scheduled before it.
+// are tied through the wait so no use can be scheduled before it; the wait
+// touches no memory, so it does not force reloads of anything else.
 struct Frag32 {
   uint32_t r[32];
 };
@@ -134,9 +135,7 @@ __device__ __forceinline__ void tmem_wait_ld(Frag32& f) {
         "+r"(f.r[12]), "+r"(f.r[13]), "+r"(f.r[14]), "+r"(f.r[15]), "+r"(f.r[16]), "+r"(f.r[17]),
         "+r"(f.r[18]), "+r"(f.r[19]), "+r"(f.r[20]), "+r"(f.r[21]), "+r"(f.r[22]), "+r"(f.r[23]),
         "+r"(f.r[24]), "+r"(f.r[25]), "+r"(f.r[26]), "+r"(f.r[27]), "+r"(f.r[28]), "+r"(f.r[29]),
-        "+r"(f.r[30]), "+r"(f.r[31])
-      :
-      : "memory");
+        "+r"(f.r[30]), "+r"(f.r[31]));
 }
 __device__ __forceinline__ void tmem_st32(uint32_t taddr, const Frag32& f) {
   asm volatile(
@@ -149,6 +148,18 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const Frag32& f) {
       "r"(f.r[19]), "r"(f.r[20]), "r"(f.r[21]), "r"(f.r[22]), "r"(f.r[23]), "r"(f.r[24]),
       "r"(f.r[25]), "r"(f.r[26]), "r"(f.r[27]), "r"(f.r[28]), "r"(f.r[29]), "r"(f.r[30]),
       "r"(f.r[31])
+      : "memory");
+}
+struct Frag16 {
+  uint32_t r[16];
+};
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const Frag16& f) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
+      "%11, %12, %13, %14, %15, %16};" ::"r"(taddr),
+      "r"(f.r[0]), "r"(f.r[1]), "r"(f.r[2]), "r"(f.r[3]), "r"(f.r[4]), "r"(f.r[5]), "r"(f.r[6]),
+      "r"(f.r[7]), "r"(f.r[8]), "r"(f.r[9]), "r"(f.r[10]), "r"(f.r[11]), "r"(f.r[12]),
+      "r"(f.r[13]), "r"(f.r[14]), "r"(f.r[15])
       : "memory");
 }
 __device__ __forceinline__ void tmem_wait_st() {
@@ -186,6 +197,80 @@ __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint6
       "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
       "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
       : "memory");
+}
+
+// D[tmem] (+)= A[tmem] * B[smem]: A (M x K, 16-bit, two K elements per
+// 32-bit column, row i in lane i) is read from tensor memory.
+__device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
+                                            uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// ------------------------------------------------- thread-block clusters
+// (a kernel launched without a cluster is a cluster of one CTA)
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// Every thread of every CTA in the cluster must call this.
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\t"
+               "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// Address of the same shared-memory location in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t mapa(uint32_t saddr, uint32_t rank) {
+  uint32_t r;
+  asm("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
+  return r;
+}
+// Plain loads (no volatile, no memory clobber): callers order them with a
+// cluster barrier, and independent loads can then be in flight together.
+__device__ __forceinline__ float4 ld_cluster_f4(uint32_t caddr) {
+  float4 v;
+  asm("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+      : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+      : "r"(caddr));
+  return v;
+}
+__device__ __forceinline__ float2 ld_cluster_f2(uint32_t caddr) {
+  float2 v;
+  asm("ld.shared::cluster.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(caddr));
+  return v;
+}
+
+__device__ __forceinline__ void st_cluster_f4(uint32_t caddr, float4 v) {
+  asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(caddr), "f"(v.x), "f"(v.y),
+               "f"(v.z), "f"(v.w)
+               : "memory");
+}
+__device__ __forceinline__ void st_cluster_f2(uint32_t caddr, float2 v) {
+  asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(caddr), "f"(v.x), "f"(v.y)
+               : "memory");
+}
+
+// Bulk copy of `bytes` (multiple of 16, both addresses 16-byte aligned)
+// from this CTA's shared memory to a cluster peer's shared memory; the
+// transfer completes `bytes` on the peer's mbarrier `peer_bar`.
+__device__ __forceinline__ void bulk_s2cluster(uint32_t peer_dst, uint32_t src, uint32_t bytes,
+                                               uint32_t peer_bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          peer_dst),
+      "r"(src), "r"(bytes), "r"(peer_bar)
+      : "memory");
+}
+__device__ __forceinline__ void bulk_commit() {
+  asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+// Wait until the sources of this thread's bulk copies have been read.
+__device__ __forceinline__ void bulk_wait_read() {
+  asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
 }
 
 __device__ __forceinline__ float ex2(float x) {

@@ -134,7 +134,9 @@ ltd_status ltd_tree_reset(const ltd_tree* tree, const int32_t* d_root_tokens, lt
  *  rows_per_seq    >= 1 + (max_depth-1) k
  *  d_active        [batch] 0/1, NULL = all sequences expand
  * Per node: cum = cum(parent) + x - logsumexp(row), computed in fp32.
- * Rows must start 16-byte aligned (vocab * sizeof(dtype) % 16 == 0). */
+ * Rows must start 16-byte aligned (vocab * sizeof(dtype) % 16 == 0).
+ * vocab <= 262,144 for LTD_BF16 and 131,072 for LTD_F32 (larger returns
+ * LTD_ERR_UNSUPPORTED). */
 ltd_status ltd_expand_tree(const ltd_tree* tree, int32_t level, const void* d_draft_rows,
                            ltd_dtype dtype, int64_t vocab, int64_t rows_per_seq,
                            const int32_t* d_active, ltd_stream_t stream);

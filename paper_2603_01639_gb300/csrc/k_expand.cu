@@ -1,28 +1,57 @@
 // Draft tree generation (LTD section 3.2, "Draft Tree Generation").
 //
 // One launch builds one level for every active sequence.  The grid is
-// (chunks, F, batch) with F = 1 at level 1 and F = k afterwards: each CTA
-// scans one vocabulary chunk of one frontier row with 16-byte streaming loads,
-// computing the chunk's (max, sum exp) and, per thread, its four best
-// (logit desc, token asc) keys; bitonic warp networks turn those into the
-// chunk's top-k (with an exact rescan in the rare case a thread may hold
-// more than four of them).  The last CTA to finish a row (atomic ticket; nothing spins)
-// merges the chunk partials in a fixed order into the row's log-sum-exp and
-// top-k, appends the k children with cum = cum(parent) + x - lse, and the
-// last row of a sequence picks the new frontier: the k best of the k^2 pool
-// by (cum desc, node id asc).  Tickets are reset to zero by their last user,
-// so the scratch is ready for the next launch.
+// (C, F, batch): F = 1 row at level 1, F = k rows (one per frontier node)
+// afterwards, and each row is split into C <= 8 vocabulary chunks whose CTAs
+// form one thread-block cluster.
+//
+// Per CTA (chunk): every thread loads its elements into registers with
+// 16-byte streaming loads and computes its own max and sum of exp -- no
+// per-element branches.  The k-th largest of the per-thread maxima, T, is a
+// lower bound of the chunk's k-th largest logit (at least k threads hold an
+// element >= T), so only elements >= T can be in the chunk's top-k: they
+// (typically about k of them) are appended to a shared list and ranked
+// exactly by (logit desc, token asc) with bitonic warp networks.  Inputs
+// that make that list overflow (huge tie sets) fall back to an exact
+// re-offer of the whole chunk.
+// Per row: rank 0 of the cluster gathers its peers' chunk lists and
+// (max, sum exp) through distributed shared memory, merges them, and
+// appends the k children with cum = cum(parent) + x - logsumexp(row) (fp32).
+// Per sequence: the last row to finish (one atomic ticket, nothing spins)
+// selects the new frontier: the k best of the k^2 children by (cum desc,
+// node id asc).  The ticket is reset by its last user.
 #include "ltd_common.cuh"
 #include "ltd_internal.h"
+#include "tc_util.cuh"
 
 namespace ltd {
 
 namespace {
 
-constexpr int kNT = 256;
+constexpr int kNT = 512;
+constexpr int kNW = kNT / kWarp;
+constexpr int kCand = 512;   // candidate list capacity per chunk
+constexpr int kMaxChunks = 8;
+constexpr int kMaxVec = 8;   // 16-byte vectors per thread
+
+// Optional phase timestamps for performance work (off in normal builds).
+#ifdef LTD_TRACE
+__device__ unsigned long long g_expand_trace[4096][8];
+#define TRACE(slot)                                                                  \
+  do {                                                                               \
+    const int cta_ = blockIdx.x + gridDim.x * (blockIdx.y + gridDim.y * blockIdx.z); \
+    unsigned long long t_;                                                           \
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t_));                          \
+    if (cta_ < 4096) g_expand_trace[cta_][slot] = t_;                                \
+  } while (0)
+#else
+#define TRACE(slot) \
+  do {              \
+  } while (0)
+#endif
 
 __global__ void tree_reset_kernel(ltd_tree t, const int32_t* __restrict__ roots,
-                                  uint32_t* row_ticket, uint32_t* seq_ticket) {
+                                  uint32_t* seq_ticket) {
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= t.batch) return;
   const int64_t nb = static_cast<int64_t>(b) * t.max_nodes;
@@ -34,130 +63,198 @@ __global__ void tree_reset_kernel(ltd_tree t, const int32_t* __restrict__ roots,
   t.xlse[nb] = 0.f;
   t.n_nodes[b] = 1;
   t.n_levels[b] = 0;
-  for (int i = 0; i < t.k; ++i) {
-    t.frontier[b * t.k + i] = (i == 0) ? 0 : -1;
-    row_ticket[b * t.k + i] = 0u;
-  }
+  for (int i = 0; i < t.k; ++i) t.frontier[b * t.k + i] = (i == 0) ? 0 : -1;
   seq_ticket[b] = 0u;
 }
 
-template <typename T>
-__global__ void __launch_bounds__(kNT) expand_kernel(const ExpandParams p) {
-  constexpr int NW = kNT / kWarp;
-  constexpr int VEC = 16 / sizeof(T);
-  constexpr int U = 4;
-  __shared__ float red[2 * NW];
-  __shared__ uint64_t stage[NW * kWarp];
-  __shared__ uint64_t best[kWarp];
-  __shared__ int s_last;
+// Warp bitonic sort of one float per lane, descending (lane 0 = largest).
+__device__ __forceinline__ float warp_sort_desc_f(float v) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int size = 2; size <= 32; size <<= 1) {
+#pragma unroll
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      const float o = __shfl_xor_sync(0xFFFFFFFFu, v, stride);
+      const bool keep_max = ((lane & stride) == 0) == ((lane & size) == 0);
+      v = keep_max ? fmaxf(v, o) : fminf(v, o);
+    }
+  }
+  return v;
+}
+// The 32 largest of two descending lane-sorted float lists, descending.
+__device__ __forceinline__ float warp_merge_desc_f(float a, float b) {
+  const int lane = threadIdx.x & 31;
+  const float br = __shfl_sync(0xFFFFFFFFu, b, 31 - lane);
+  float v = fmaxf(a, br);
+#pragma unroll
+  for (int stride = 16; stride > 0; stride >>= 1) {
+    const float o = __shfl_xor_sync(0xFFFFFFFFu, v, stride);
+    v = ((lane & stride) == 0) ? fmaxf(v, o) : fminf(v, o);
+  }
+  return v;
+}
 
+// Tree merge of one descending 32-entry list per warp (stage[w][lane]) into
+// stage[0][0..32).  All threads call; returns after a barrier.
+template <typename V, V (*Merge)(V, V)>
+__device__ __forceinline__ void tree_merge(V* stage) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll 1
+  for (int step = 1; step < kNW; step <<= 1) {
+    __syncthreads();
+    if ((warp % (2 * step)) == 0 && warp + step < kNW) {
+      const V m = Merge(stage[warp * kWarp + lane], stage[(warp + step) * kWarp + lane]);
+      __syncwarp();
+      stage[warp * kWarp + lane] = m;
+    }
+  }
+  __syncthreads();
+}
+
+struct ExpandShared {
+  uint64_t stage[kNW * kWarp];
+  float fstage[kNW * kWarp];
+  uint64_t cand[kCand];
+  float red[2 * kNW];
+  // published to the cluster: the chunk's sorted top list and (max, sum exp)
+  uint64_t top[kWarp];
+  float2 ms;
+  // gathered by rank 0
+  uint64_t peer_top[kMaxChunks][kWarp];
+  float2 peer_ms[kMaxChunks];
+  int n_cand;
+  int last;
+};
+
+template <typename T, int U>
+__global__ void __launch_bounds__(kNT) expand_kernel(const ExpandParams p) {
+  constexpr int VEC = 16 / sizeof(T);
+  __shared__ ExpandShared sh;
   const int ch = blockIdx.x, f = blockIdx.y, b = blockIdx.z, tid = threadIdx.x;
   const int lane = tid & 31, warp = tid >> 5;
+  if (tid == 0) TRACE(0);
+  // early exits are shared by the whole cluster (same row)
   if (p.active != nullptr && p.active[b] == 0) return;
   if (p.n_levels[b] != p.level - 1) {
     if (tid == 0 && ch == 0 && f == 0) flag_error(p.err, LTD_DEVERR_LEVEL);
     return;
   }
+  const int k = p.k;
 
-  // ---- phase 1: this CTA's chunk of row (b, f)
-  const int64_t row = (p.level == 1) ? 0 : 1 + static_cast<int64_t>(p.level - 2) * p.k + f;
+  // ---- stage 1: chunk elements into registers; per-thread max and sum exp
+  const int64_t row = (p.level == 1) ? 0 : 1 + static_cast<int64_t>(p.level - 2) * k + f;
   const T* x = reinterpret_cast<const T*>(p.rows) +
                (static_cast<int64_t>(b) * p.rows_per_seq + row) * p.vocab;
   const int64_t lo = static_cast<int64_t>(ch) * p.chunk_elems;
   const int64_t hi = min(lo + p.chunk_elems, p.vocab);
-
-  float m = -CUDART_INF_F, s = 0.f;
-  Top4 t4;
-  t4.init();
-  for (int64_t base = lo + static_cast<int64_t>(tid) * VEC; base < hi;
-       base += static_cast<int64_t>(kNT) * VEC * U) {
-    float xv[U][VEC];
+  float xv[U][VEC];
 #pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int64_t i = base + static_cast<int64_t>(u) * kNT * VEC;
-      if (i + VEC <= hi) {
-        unpack16(ld_stream16(x + i), xv[u], static_cast<const T*>(nullptr));
-      } else {
+  for (int u = 0; u < U; ++u) {
+    const int64_t i = lo + (static_cast<int64_t>(u) * kNT + tid) * VEC;
+    if (i + VEC <= hi) {
+      unpack16(ld_stream16(x + i), xv[u], static_cast<const T*>(nullptr));
+    } else {
 #pragma unroll
-        for (int j = 0; j < VEC; ++j) xv[u][j] = (i + j < hi) ? to_f<T>(x[i + j]) : -CUDART_INF_F;
-      }
+      for (int j = 0; j < VEC; ++j) xv[u][j] = (i + j < hi) ? to_f<T>(x[i + j]) : -CUDART_INF_F;
     }
+  }
+  float tmax = -CUDART_INF_F;
 #pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int64_t i = base + static_cast<int64_t>(u) * kNT * VEC;
-      float vm = -CUDART_INF_F;
+  for (int u = 0; u < U; ++u)
 #pragma unroll
-      for (int j = 0; j < VEC; ++j) vm = fmaxf(vm, xv[u][j]);
-      if (vm > m) {
-        s *= __expf(m - vm);
-        m = vm;
-      }
+    for (int j = 0; j < VEC; ++j) tmax = fmaxf(tmax, xv[u][j]);
+  float tsum = 0.f;
+  if (tmax > -CUDART_INF_F) {
+#pragma unroll
+    for (int u = 0; u < U; ++u)
+#pragma unroll
+      for (int j = 0; j < VEC; ++j) tsum += __expf(xv[u][j] - tmax);
+  }
+  if (tid == 0) TRACE(1);
+  float m = tmax, s = tsum;
+  block_ms<kNT>(m, s, sh.red);
+
+  // ---- stage 2: T = k-th largest per-thread max (a lower bound of the
+  // chunk's k-th largest logit)
+  sh.fstage[warp * kWarp + lane] = warp_sort_desc_f(tmax);
+  if (tid == 0) sh.n_cand = 0;
+  tree_merge<float, warp_merge_desc_f>(sh.fstage);
+  const float thr = sh.fstage[k - 1];
+
+  // ---- stage 3: the candidates >= T, ranked exactly by (logit desc, token asc)
+  if (tmax >= thr) {
+#pragma unroll
+    for (int u = 0; u < U; ++u)
 #pragma unroll
       for (int j = 0; j < VEC; ++j) {
-        if (i + j < hi) {
-          const float xj = xv[u][j];
-          s += (xj == -CUDART_INF_F) ? 0.f : __expf(xj - m);
-          t4.insert(make_key(xj, static_cast<uint32_t>(i + j)));
+        const int64_t i = lo + (static_cast<int64_t>(u) * kNT + tid) * VEC + j;
+        if (xv[u][j] >= thr && i < hi) {
+          const int slot = atomicAdd(&sh.n_cand, 1);
+          if (slot < kCand) sh.cand[slot] = make_key(xv[u][j], static_cast<uint32_t>(i));
         }
       }
-    }
   }
-  block_ms<kNT>(m, s, red);
-  // warp lists from the per-thread top-4s, then the block list
+  __syncthreads();
+  const int nc = sh.n_cand;
   WarpTopK wt;
   wt.init();
-  wt.offer(t4.t0, p.k);
-  wt.offer(t4.t1, p.k);
-  wt.offer(t4.t2, p.k);
-  wt.offer(t4.t3, p.k);
-  block_topk<kNT>(wt, stage, best);
-  // exactness: a thread whose 4th key made the top-k may hold more of it;
-  // then every thread offers its whole chunk again (rare: needs 4 of the
-  // chunk's top-k in one thread's 1/256 of the chunk)
-  if (__syncthreads_or(t4.t3 != 0ull && t4.t3 >= best[p.k - 1])) {
-    wt.init();
-    for (int64_t wbase = lo + static_cast<int64_t>(warp) * kWarp; wbase < hi;
-         wbase += static_cast<int64_t>(kNT)) {
-      const int64_t i = wbase + lane;
-      wt.offer(i < hi ? make_key(to_f<T>(x[i]), static_cast<uint32_t>(i)) : 0ull, p.k);
+  if (nc <= kCand) {
+    for (int c0 = warp * kWarp; c0 < nc; c0 += kNT) {
+      const int c = c0 + lane;
+      wt.offer(c < nc ? sh.cand[c] : 0ull, k);
     }
-    block_topk<kNT>(wt, stage, best);
+  } else {
+    // exact fallback: every element of the chunk is offered
+#pragma unroll
+    for (int u = 0; u < U; ++u)
+#pragma unroll
+      for (int j = 0; j < VEC; ++j) {
+        const int64_t i = lo + (static_cast<int64_t>(u) * kNT + tid) * VEC + j;
+        wt.offer(i < hi ? make_key(xv[u][j], static_cast<uint32_t>(i)) : 0ull, k);
+      }
   }
-
-  const int64_t rec_row = (static_cast<int64_t>(b) * p.F + f) * p.chunks;
-  if (tid == 0) p.part_ms[rec_row + ch] = make_float2(m, s);
-  if (tid < p.k) p.part_keys[(rec_row + ch) * p.k + tid] = best[tid];
-  __threadfence();
-  __syncthreads();
+  sh.stage[warp * kWarp + lane] = wt.v;
+  tree_merge<uint64_t, warp_merge_desc>(sh.stage);
+  if (tid < kWarp) sh.top[tid] = sh.stage[tid];
   if (tid == 0) {
-    const uint32_t prev = atomicAdd(&p.row_ticket[b * p.k + f], 1u);
-    s_last = (prev == static_cast<uint32_t>(p.chunks - 1));
+    sh.ms = make_float2(m, s);
+    TRACE(2);
   }
-  __syncthreads();
-  if (!s_last) return;
-  __threadfence();
 
-  // ---- phase 2: last CTA of the row merges its chunks (fixed order)
-  float M = -CUDART_INF_F, S = 0.f;
-  for (int c = tid; c < p.chunks; c += kNT) {
-    const float2 ms = __ldcg(&p.part_ms[rec_row + c]);
-    ms_merge(M, S, ms.x, ms.y);
+  // ---- row: rank 0 gathers the chunk results of its cluster
+  const int C = p.chunks;
+  tc::cluster_sync();
+  if (ch == 0) {
+    if (tid < C * kWarp) {
+      const int peer = tid / kWarp, e = tid % kWarp;
+      const uint32_t a = tc::mapa(tc::smem_u32(&sh.top[e]), peer);
+      uint64_t v;
+      asm volatile("ld.shared::cluster.u64 %0, [%1];" : "=l"(v) : "r"(a) : "memory");
+      sh.peer_top[peer][e] = v;
+    }
+    if (tid < C) sh.peer_ms[tid] = tc::ld_cluster_f2(tc::mapa(tc::smem_u32(&sh.ms), tid));
   }
-  block_ms<kNT>(M, S, red);
-  WarpTopK t2;
-  t2.init();
-  for (int c = warp; c < p.chunks; c += NW)
-    t2.merge_sorted(lane < p.k ? __ldcg(&p.part_keys[(rec_row + c) * p.k + lane]) : 0ull);
-  block_topk<kNT>(t2, stage, best);
-  const float lse = M + logf(S);
+  // no CTA leaves while rank 0 may still read its shared memory
+  tc::cluster_sync();
+  if (ch != 0) return;
+  if (tid == 0) TRACE(3);
+
+  if (tid == 0) {
+    float M = -CUDART_INF_F, S = 0.f;
+    for (int c = 0; c < C; ++c) ms_merge(M, S, sh.peer_ms[c].x, sh.peer_ms[c].y);
+    sh.red[0] = M + logf(S);
+  }
+  sh.stage[warp * kWarp + lane] = (warp < C) ? sh.peer_top[warp][lane] : 0ull;
+  tree_merge<uint64_t, warp_merge_desc>(sh.stage);
+  const float lse = sh.red[0];
 
   const int64_t nb = static_cast<int64_t>(b) * p.max_nodes;
-  const int parent = (p.level == 1) ? 0 : __ldcg(&p.frontier[b * p.k + f]);
+  const int parent = (p.level == 1) ? 0 : __ldcg(&p.frontier[b * k + f]);
   const float cum_p = (p.level == 1) ? 0.f : __ldcg(&p.cum[nb + parent]);
-  const int base = (p.level == 1) ? 1 : 1 + p.k + (p.level - 2) * p.k * p.k;
-  if (tid < p.k) {
-    const uint64_t key = best[tid];
-    const int64_t id = nb + base + f * p.k + tid;
+  const int base = (p.level == 1) ? 1 : 1 + k + (p.level - 2) * k * k;
+  if (tid < k) {
+    const uint64_t key = sh.stage[tid];
+    const int64_t id = nb + base + f * k + tid;
     p.token[id] = static_cast<int32_t>(key_index(key));
     p.parent[id] = parent;
     p.depth[id] = p.level;
@@ -168,45 +265,76 @@ __global__ void __launch_bounds__(kNT) expand_kernel(const ExpandParams p) {
   if (tid == 0) {
     p.xrow[nb + parent] = static_cast<int32_t>(row);
     p.xlse[nb + parent] = lse;
-    p.row_ticket[b * p.k + f] = 0u;
+    TRACE(4);
+  }
+
+  // ---- sequence: the frontier (level 1: all children; later: by the last row)
+  if (p.level == 1) {
+    if (tid < k) p.frontier[b * k + tid] = 1 + tid;
+    if (tid == 0) {
+      p.n_nodes[b] = 1 + k;
+      p.n_levels[b] = 1;
+    }
+    return;
   }
   __threadfence();
   __syncthreads();
   if (tid == 0) {
     const uint32_t prev = atomicAdd(&p.seq_ticket[b], 1u);
-    s_last = (prev == static_cast<uint32_t>(p.F - 1));
+    sh.last = (prev == static_cast<uint32_t>(p.F - 1));
   }
   __syncthreads();
-  if (!s_last) return;
+  if (!sh.last) return;
   __threadfence();
-
-  // ---- phase 3: last row of the sequence picks the frontier
-  if (p.level == 1) {
-    if (tid < p.k) p.frontier[b * p.k + tid] = 1 + tid;
-  } else {
-    WarpTopK t3;
-    t3.init();
-    const int pool = p.k * p.k;
+  if (tid == 0) TRACE(5);
+  {
+    WarpTopK pt;
+    pt.init();
+    const int pool = k * k;
     for (int j0 = warp * kWarp; j0 < pool; j0 += kNT) {
       const int j = j0 + lane;
       const int id = base + j;
-      t3.offer(j < pool ? make_key(__ldcg(&p.cum[nb + id]), static_cast<uint32_t>(id)) : 0ull, p.k);
+      pt.offer(j < pool ? make_key(__ldcg(&p.cum[nb + id]), static_cast<uint32_t>(id)) : 0ull, k);
     }
-    block_topk<kNT>(t3, stage, best);
-    if (tid < p.k) p.frontier[b * p.k + tid] = static_cast<int32_t>(key_index(best[tid]));
+    sh.stage[warp * kWarp + lane] = pt.v;
   }
+  tree_merge<uint64_t, warp_merge_desc>(sh.stage);
+  if (tid < k) p.frontier[b * k + tid] = static_cast<int32_t>(key_index(sh.stage[tid]));
   if (tid == 0) {
-    p.n_nodes[b] = base + p.F * p.k;
+    p.n_nodes[b] = base + p.F * k;
     p.n_levels[b] = p.level;
     p.seq_ticket[b] = 0u;
+    TRACE(6);
   }
 }
 
+template <typename T, int U>
+cudaError_t launch_u(const ExpandParams& p, int32_t batch, cudaStream_t s) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(p.chunks, p.F, batch);
+  cfg.blockDim = dim3(kNT);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = p.chunks;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, expand_kernel<T, U>, p);
+}
+
 template <typename T>
-cudaError_t launch_expand_t(const ExpandParams& p, int32_t batch, cudaStream_t s) {
-  const dim3 grid(p.chunks, p.F, batch);
-  expand_kernel<T><<<grid, kNT, 0, s>>>(p);
-  return cudaGetLastError();
+cudaError_t launch_t(const ExpandParams& p, int32_t batch, cudaStream_t s) {
+  constexpr int VEC = 16 / sizeof(T);
+  const int64_t vecs = (p.chunk_elems + static_cast<int64_t>(kNT) * VEC - 1) /
+                       (static_cast<int64_t>(kNT) * VEC);
+  if (vecs <= 1) return launch_u<T, 1>(p, batch, s);
+  if (vecs <= 2) return launch_u<T, 2>(p, batch, s);
+  if (vecs <= 4) return launch_u<T, 4>(p, batch, s);
+  if (vecs <= kMaxVec) return launch_u<T, kMaxVec>(p, batch, s);
+  return cudaErrorInvalidValue;
 }
 
 }  // namespace
@@ -223,38 +351,56 @@ VocabSplit vocab_split(int64_t rows, int64_t vocab, int64_t target_ctas, int64_t
   return VocabSplit{static_cast<int32_t>(chunks), elems};
 }
 
+int64_t expand_max_vocab(int elem_bytes) {
+  return static_cast<int64_t>(kMaxChunks) * kNT * kMaxVec * (16 / elem_bytes);
+}
+
+// At most 8 chunks (one cluster) per row of at most 512 threads x 8 vectors.
+VocabSplit expand_split(int64_t rows, int64_t vocab, int elem_bytes) {
+  const int64_t max_chunk = static_cast<int64_t>(kNT) * kMaxVec * (16 / elem_bytes);
+  VocabSplit v = vocab_split(rows, vocab, kExpandTargetCtas, kExpandMinElems);
+  if (v.chunks > kMaxChunks || v.chunk_elems > max_chunk) {
+    int64_t chunks = (vocab + max_chunk - 1) / max_chunk;
+    if (chunks < v.chunks) chunks = v.chunks;
+    if (chunks > kMaxChunks) chunks = kMaxChunks;
+    int64_t elems = (vocab + chunks - 1) / chunks;
+    elems = (elems + 7) / 8 * 8;
+    v.chunks = static_cast<int32_t>((vocab + elems - 1) / elems);
+    v.chunk_elems = elems;
+  }
+  return v;
+}
+
 ExpandRecordLayout expand_layout(int32_t batch, int32_t k, int64_t max_vocab) {
+  (void)k;
+  (void)max_vocab;
   ExpandRecordLayout l{};
-  const int64_t r1 = static_cast<int64_t>(batch) *
-                     vocab_split(batch, max_vocab, kExpandTargetCtas, kExpandMinElems).chunks;
-  const int64_t rk = static_cast<int64_t>(batch) * k *
-                     vocab_split(static_cast<int64_t>(batch) * k, max_vocab, kExpandTargetCtas,
-                                 kExpandMinElems).chunks;
-  l.records = r1 > rk ? r1 : rk;
-  auto up = [](size_t x) { return (x + 255) / 256 * 256; };
-  l.ms_bytes = up(l.records * sizeof(float2));
-  l.keys_bytes = up(l.records * k * sizeof(uint64_t));
-  l.row_ticket_bytes = up(static_cast<size_t>(batch) * k * sizeof(uint32_t));
-  l.seq_ticket_bytes = up(static_cast<size_t>(batch) * sizeof(uint32_t));
-  l.total = l.ms_bytes + l.keys_bytes + l.row_ticket_bytes + l.seq_ticket_bytes;
+  l.seq_ticket_bytes = (static_cast<size_t>(batch) * sizeof(uint32_t) + 255) / 256 * 256;
+  l.total = l.seq_ticket_bytes;
   return l;
 }
 
 cudaError_t launch_tree_reset(const ltd_tree* t, const int32_t* roots, cudaStream_t s) {
-  const ExpandRecordLayout l = expand_layout(t->batch, t->k, t->max_vocab);
-  char* base = static_cast<char*>(t->scratch);
-  uint32_t* row_ticket = reinterpret_cast<uint32_t*>(base + l.ms_bytes + l.keys_bytes);
-  uint32_t* seq_ticket = reinterpret_cast<uint32_t*>(base + l.ms_bytes + l.keys_bytes +
-                                                     l.row_ticket_bytes);
+  uint32_t* seq_ticket = static_cast<uint32_t*>(t->scratch);
   const int threads = 128;
-  tree_reset_kernel<<<(t->batch + threads - 1) / threads, threads, 0, s>>>(*t, roots, row_ticket,
-                                                                            seq_ticket);
+  tree_reset_kernel<<<(t->batch + threads - 1) / threads, threads, 0, s>>>(*t, roots, seq_ticket);
   return cudaGetLastError();
 }
 
 cudaError_t launch_expand(const ExpandParams& p, int32_t batch, ltd_dtype dtype, cudaStream_t s) {
-  return dtype == LTD_BF16 ? launch_expand_t<__nv_bfloat16>(p, batch, s)
-                           : launch_expand_t<float>(p, batch, s);
+  return dtype == LTD_BF16 ? launch_t<__nv_bfloat16>(p, batch, s) : launch_t<float>(p, batch, s);
 }
+
+#ifdef LTD_TRACE
+extern "C" int ltd_expand_trace_read(unsigned long long* host, int n) {
+  return cudaMemcpyFromSymbol(host, g_expand_trace, sizeof(unsigned long long) * n) == cudaSuccess
+             ? 0
+             : 1;
+}
+extern "C" int ltd_expand_trace_clear() {
+  static unsigned long long zeros[4096 * 8];
+  return cudaMemcpyToSymbol(g_expand_trace, zeros, sizeof(zeros)) == cudaSuccess ? 0 : 1;
+}
+#endif
 
 }  // namespace ltd

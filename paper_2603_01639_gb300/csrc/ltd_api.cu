@@ -136,11 +136,9 @@ ltd_status ltd_expand_tree(const ltd_tree* tree, int32_t level, const void* d_dr
   uint32_t* err = device_error_word();
   if (err == nullptr) return LTD_ERR_CUDA;
   const int32_t F = (level == 1) ? 1 : tree->k;
-  const VocabSplit vs = vocab_split(static_cast<int64_t>(tree->batch) * F, vocab,
-                                    kExpandTargetCtas, kExpandMinElems);
-  const ExpandRecordLayout l = expand_layout(tree->batch, tree->k, tree->max_vocab);
-  if (static_cast<int64_t>(tree->batch) * F * vs.chunks > l.records) return LTD_ERR_SHAPE;
-  char* base = static_cast<char*>(tree->scratch);
+  const int esize = static_cast<int>(dtype_size(dtype));
+  if (vocab > expand_max_vocab(esize)) return LTD_ERR_UNSUPPORTED;
+  const VocabSplit vs = expand_split(static_cast<int64_t>(tree->batch) * F, vocab, esize);
   ExpandParams p{};
   p.token = tree->token;
   p.parent = tree->parent;
@@ -153,10 +151,7 @@ ltd_status ltd_expand_tree(const ltd_tree* tree, int32_t level, const void* d_dr
   p.n_levels = tree->n_levels;
   p.max_nodes = tree->max_nodes;
   p.k = tree->k;
-  p.part_ms = reinterpret_cast<float2*>(base);
-  p.part_keys = reinterpret_cast<uint64_t*>(base + l.ms_bytes);
-  p.row_ticket = reinterpret_cast<uint32_t*>(base + l.ms_bytes + l.keys_bytes);
-  p.seq_ticket = reinterpret_cast<uint32_t*>(base + l.ms_bytes + l.keys_bytes + l.row_ticket_bytes);
+  p.seq_ticket = static_cast<uint32_t*>(tree->scratch);
   p.rows = d_draft_rows;
   p.vocab = vocab;
   p.rows_per_seq = rows_per_seq;

@@ -31,6 +31,8 @@ struct ExpandRecordLayout {
   int64_t records;
 };
 ExpandRecordLayout expand_layout(int32_t batch, int32_t k, int64_t max_vocab);
+VocabSplit expand_split(int64_t rows, int64_t vocab, int elem_bytes);
+int64_t expand_max_vocab(int elem_bytes);
 
 struct ExpandParams {
   int32_t* token;

@@ -216,9 +216,11 @@ typedef struct ltd_kv_cache {
  *  d_bonus          out [batch]
  *  kv               if not NULL, the accepted rows are compacted in every
  *                   layer: row ctx+t <- row ctx+path[t] (ltd_kv_compact).
- *  d_workspace      ltd_accept_workspace_bytes() bytes of caller memory,
- *                   zero-filled before its first use; every call leaves it
- *                   zero-filled again. */
+ *  d_workspace      ltd_accept_workspace_bytes() bytes of caller memory
+ *                   (per-slot, per-vocabulary-chunk statistics); its contents
+ *                   need no initial value and are overwritten by every call.
+ * vocab above 262144 returns LTD_ERR_UNSUPPORTED: the stochastic walk keeps
+ * p and q of one sequence in the shared memory of one 16-CTA cluster. */
 size_t ltd_accept_workspace_bytes(int32_t batch, int32_t n_max, int64_t vocab);
 ltd_status ltd_accept(const ltd_tree* tree, const void* d_target_logits,
                       const void* d_draft_rows, ltd_dtype dtype, int64_t vocab,
@@ -240,8 +242,8 @@ ltd_status ltd_accept(const ltd_tree* tree, const void* d_target_logits,
  * scratch lives in a static device array of LTD_ACCEPT_NOALLOC_SCRATCH_BYTES
  * (1 MiB) inside the library, held by every GPU that loads it until the
  * process exits.  Sizes whose ltd_accept_workspace_bytes() exceeds that
- * return LTD_ERR_SHAPE.  Allocates nothing (no cudaMalloc or cudaFree); each
- * call clears the array's tickets with one cudaMemsetAsync on the stream.
+ * return LTD_ERR_SHAPE.  Allocates nothing (no cudaMalloc or cudaFree) and
+ * needs no part of the array cleared between calls.
  * The first call on a device looks up the array's device address; make
  * that first call before any stream capture.  All calls share the array,
  * so calls whose kernels overlap on the GPU (for example on two streams)

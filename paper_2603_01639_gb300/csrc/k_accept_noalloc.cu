@@ -7,9 +7,8 @@
 // every device buffer, or code that must stay free of allocator calls so a
 // stream can later be captured into a CUDA graph with a fixed memory plan.
 // For them this entry point keeps the acceptance kernel's scratch (one
-// record per slot and vocabulary chunk, plus one ticket per sequence) in the
-// file-scope array below, which every GPU that loads the library holds
-// until the process exits.
+// record per slot and vocabulary chunk) in the file-scope array below,
+// which every GPU that loads the library holds until the process exits.
 //
 // Every call shares that one array: two calls whose kernels overlap on the
 // GPU (different streams, or a second call before the first finished on a
@@ -62,17 +61,6 @@ extern "C" ltd_status ltd_accept_noalloc(const ltd_tree* tree, const void* d_tar
   if (need == 0 || need > LTD_ACCEPT_NOALLOC_SCRATCH_BYTES) return LTD_ERR_SHAPE;
   unsigned char* scratch = scratch_address();
   if (scratch == nullptr) return LTD_ERR_CUDA;
-  // The tickets at the end of the scratch must start at zero.  A finished
-  // call leaves them zero, but a call that stopped early (for example on a
-  // sequence with a bad verify size) may not, so clear them every time.
-  const VocabSplit vs = vocab_split(static_cast<int64_t>(tree->batch) * n_max, vocab,
-                                    kAcceptTargetCtas, kAcceptMinElems);
-  const size_t rec_bytes =
-      static_cast<size_t>(tree->batch) * n_max * vs.chunks * sizeof(AcceptRecord);
-  const size_t ticket_off = (rec_bytes + 255) / 256 * 256;
-  if (cudaMemsetAsync(scratch + ticket_off, 0, static_cast<size_t>(tree->batch) * sizeof(uint32_t),
-                      reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
-    return LTD_ERR_CUDA;
   return ltd_accept(tree, d_target_logits, d_draft_rows, dtype, vocab, rows_per_seq, d_node_ids,
                     d_n_verify, n_max, d_mode, seed, cycle, d_ctx, d_new_ctx, d_path, d_accept_len,
                     d_bonus, kv, scratch, LTD_ACCEPT_NOALLOC_SCRATCH_BYTES, stream);

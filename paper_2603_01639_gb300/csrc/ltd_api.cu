@@ -326,6 +326,7 @@ ltd_status ltd_accept(const ltd_tree* tree, const void* d_target_logits, const v
   if (rows_per_seq < 1 + static_cast<int64_t>(tree->max_depth - 1) * tree->k) return LTD_ERR_SHAPE;
   if (!aligned16(d_target_logits) || (vocab * static_cast<int64_t>(dtype_size(dtype))) % 16 != 0)
     return LTD_ERR_SHAPE;
+  if (vocab > kAcceptMaxVocab) return LTD_ERR_UNSUPPORTED;
   const size_t need = accept_workspace(tree->batch, n_max, vocab);
   if (d_workspace == nullptr || workspace_bytes < need) return LTD_ERR_SHAPE;
   if (kv != nullptr) {
@@ -338,8 +339,6 @@ ltd_status ltd_accept(const ltd_tree* tree, const void* d_target_logits, const v
   if (err == nullptr) return LTD_ERR_CUDA;
   const VocabSplit vs = vocab_split(static_cast<int64_t>(tree->batch) * n_max, vocab,
                                     kAcceptTargetCtas, kAcceptMinElems);
-  const size_t rec_bytes =
-      static_cast<size_t>(tree->batch) * n_max * vs.chunks * sizeof(AcceptRecord);
   AcceptParams p{};
   p.token = tree->token;
   p.parent = tree->parent;
@@ -363,7 +362,6 @@ ltd_status ltd_accept(const ltd_tree* tree, const void* d_target_logits, const v
   p.accept_len = d_accept_len;
   p.bonus = d_bonus;
   p.rec = static_cast<AcceptRecord*>(d_workspace);
-  p.ticket = reinterpret_cast<uint32_t*>(static_cast<char*>(d_workspace) + align256(rec_bytes));
   p.chunks = vs.chunks;
   p.chunk_elems = vs.chunk_elems;
   p.err = err;

@@ -113,6 +113,9 @@ cudaError_t launch_umma_selftest(int mode, const void* a, const void* b, float* 
 constexpr int64_t kAcceptTargetCtas = 608;
 constexpr int64_t kAcceptMinElems = 4096;
 
+// Largest vocabulary the acceptance walk holds in one cluster's shared memory
+// (16 CTAs x 16384 fp32 entries of p and q each).
+constexpr int64_t kAcceptMaxVocab = 16 * 16384;
 struct AcceptRecord {
   float m, s;
   unsigned long long key;
@@ -140,7 +143,6 @@ struct AcceptParams {
   int32_t* accept_len;
   int32_t* bonus;
   AcceptRecord* rec;  // [batch][n_max][chunks]
-  uint32_t* ticket;   // [batch]
   int32_t chunks;
   int64_t chunk_elems;
   uint32_t* err;

@@ -229,6 +229,16 @@ __device__ __forceinline__ uint32_t mapa(uint32_t saddr, uint32_t rank) {
   asm("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
   return r;
 }
+__device__ __forceinline__ float ld_cluster_f1(uint32_t caddr) {
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(caddr) : "memory");
+  return v;
+}
+__device__ __forceinline__ uint64_t ld_cluster_u64(uint32_t caddr) {
+  uint64_t v;
+  asm volatile("ld.shared::cluster.u64 %0, [%1];" : "=l"(v) : "r"(caddr) : "memory");
+  return v;
+}
 // Plain loads (no volatile, no memory clobber): callers order them with a
 // cluster barrier, and independent loads can then be in flight together.
 __device__ __forceinline__ float4 ld_cluster_f4(uint32_t caddr) {

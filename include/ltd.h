@@ -164,7 +164,12 @@ ltd_status ltd_select_verify(const ltd_tree* tree, const int32_t* d_n_verify, in
  *  d_q, d_out   [batch][n_max][hq][head_dim] (dtype)
  *  d_k, d_v     [batch][hkv][s_cap][head_dim] (dtype)
  *  max_ctx      host-side bound on every ctx_b (sizes the work split)
- *  d_workspace  ltd_attention_workspace_bytes() bytes of caller memory
+ *  d_workspace  ltd_attention_workspace_bytes() bytes of caller memory,
+ *               zero-filled before its first use.  When the keys are split
+ *               it holds per-split partial rows and per-unit counters; every
+ *               call that ends without a device error leaves the counters
+ *               at zero (after LTD_DEVERR_TIMEOUT, zero it again).  The size
+ *               depends on the current device's SM count.
  * bf16 with head_dim 128 runs on the tcgen05 tensor cores; other shapes
  * (f32, head_dim in {32, 64, 96, 128}) run on a CUDA-core kernel. */
 size_t ltd_attention_workspace_bytes(int32_t batch, int32_t hq, int32_t hkv, int32_t head_dim,

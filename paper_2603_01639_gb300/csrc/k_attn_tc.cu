@@ -1,30 +1,39 @@
 // Tensor-core tree attention (LTD section 3.2, "Draft Tree Verification";
 // SpecInfer-style tree mask) for bf16 and head_dim 128 on sm_103a.
 //
-// Work split: a CTA owns two 128-row tiles ("a" and "b") of the query rows
-// of one KV head (row r = slot * G + g, so the G query heads of a KV head
-// share every K/V byte) and one split of that head's keys; the splits of one
-// (sequence, head, tile pair) form a thread-block cluster of up to 16 CTAs.
-//   warp 0      TMA: both Q tiles once, then 128-key K and V chunks into
-//               two-stage rings (128-byte swizzle);
+// Work unit: two 128-row tiles ("a" and "b") of the query rows of one KV
+// head of one sequence (row r = slot * G + g, so the G query heads of a KV
+// head share every K/V byte), over one split of that head's keys.
+//   warp 0      TMA: both Q tiles, then 128-key K and V chunks into
+//               two-stage rings (128-byte swizzle); the first two stages are
+//               issued before the setup barrier;
 //   warp 1      tcgen05.mma: S_x = Q_x K^T into tensor memory, then
 //               O_x += P_x V with P_x read from tensor memory; the order
 //               PV_a(j), S_a(j+1), PV_b(j), S_b(j+1) lets one tile's
 //               softmax run while the tensor core works on the other;
 //   warps 4-7   softmax of tile a, warps 8-11 of tile b, one thread per row
-//               (= tensor-memory lane): read S, apply the prefix + ancestor
-//               mask, keep a running max that rescales O only when it grows
-//               by more than 2^8, write P as bf16 over S's columns.
+//               (= tensor-memory lane): one 128-column load of S, the prefix
+//               + ancestor mask, a running max that rescales O only when it
+//               grows by more than 2^8, P written as bf16 over S's columns.
+//               The two tiles take turns chunk by chunk (a(j), b(j),
+//               a(j+1), ...), so one tile's softmax has the SM's exp and FMA
+//               pipes while the tensor core runs the other tile's MMAs.
 // Tensor memory (512 columns): S_a | S_b | O_a | O_b.
-// After the last MMA every CTA stages its rows as O/l in bf16 plus the
-// log-sum-exp, and (after one cluster barrier) bulk-copies each block of
-// rows to the cluster CTA that owns them through distributed shared memory;
-// each CTA then combines its rows across all splits locally and writes bf16
-// output.  No global workspace, no second kernel.
-// Every mbarrier wait is bounded: on timeout the CTA flags
-// LTD_DEVERR_TIMEOUT, drains its own TMA loads and MMAs, and still joins
-// the cluster barrier and sends every block its peers expect (so no peer
-// waits on it forever), frees its tensor memory and returns.
+//
+// Two launch shapes:
+//  - one split per unit (at least as many units as SMs): each CTA writes
+//    O / l straight to the output, and CTAs take the units longest first
+//    (every CTA ranks the (sequence, tile pair) groups by chunks x tiles
+//    from ctx and N), so the long sequences of a ragged batch start early;
+//  - several splits per unit (fewer units than SMs): a cooperative launch,
+//    so every CTA is resident at once.  Each split writes its rows' O / l
+//    (bf16) and log-sum-exp to the workspace and arrives on its unit's
+//    counter; when all splits have arrived, split s combines rows
+//    [s R, s R + R) of the unit from L2 and writes them; the last split to
+//    leave resets the unit's counters to zero.
+// Every wait is bounded (mbarrier waits and the counter spin): on timeout a
+// CTA flags LTD_DEVERR_TIMEOUT, drains its own TMA loads and MMAs, still
+// arrives and departs on its counter, frees its tensor memory and returns.
 #include <mutex>
 
 #include "ltd_common.cuh"
@@ -40,57 +49,60 @@ constexpr int kBN = 128;  // keys per chunk
 constexpr int kD = 128;
 constexpr int kRows = 2 * kBM;
 constexpr int kThreads = 384;
-constexpr int kWarps = kThreads / 32;
 constexpr int kMaxW32 = LTD_MAX_N / 32;
-constexpr int kMaxCluster = 16;
+constexpr int kMaxSplits = 64;
+constexpr int kMaxGroups = 1024;  // (sequence, tile pair) groups ranked on the device
 constexpr uint32_t kHalf = 16384;      // 128 rows x 128 bytes
 constexpr uint32_t kTile = 2 * kHalf;  // 128 x 128 bf16
-constexpr uint32_t kOffQ = 0;                        // Q_a, Q_b
-constexpr uint32_t kOffK = kOffQ + 2 * kTile;        // two stages
-constexpr uint32_t kOffV = kOffK + 2 * kTile;        // two stages
-constexpr uint32_t kOffMask = kOffV + 2 * kTile;     // [256][8] words
-constexpr uint32_t kOffBar = kOffMask + kRows * kMaxW32 * 4;
-constexpr uint32_t kOffHolder = kOffBar + 32 * 8;
+constexpr uint32_t kOffQ = 0;                                  // Q_a, Q_b
+constexpr uint32_t kOffK = kOffQ + 2 * kTile;                  // two stages
+constexpr uint32_t kOffV = kOffK + 2 * kTile;                  // two stages
+constexpr uint32_t kOffMask = kOffV + 2 * kTile;               // [256][8] words
+constexpr uint32_t kOffCost = kOffMask + kRows * kMaxW32 * 4;  // [kMaxGroups] int
+constexpr uint32_t kOffOrder = kOffCost + kMaxGroups * 4;      // [kMaxGroups] int
+constexpr uint32_t kOffBar = kOffOrder + kMaxGroups * 4;
+constexpr uint32_t kOffHolder = kOffBar + 24 * 8;
 constexpr uint32_t kSmemBytes = kOffHolder + 16 + 1024;  // + alignment slack
-// Split reduction, over the Q/K/V space once the MMAs have finished.  CTA r
-// of the cluster owns rows [r R, r R + R), R = ceil(256 / splits) rounded up
-// to a multiple of 4, and receives every split's normalised O (bf16, 256
-// bytes per row, 16-byte chunks swizzled by row) and log-sum-exp for them.
-constexpr uint32_t kRowBytes = kD * 2;
-constexpr uint32_t kOffRecvO = 0;                           // [split][R] rows, <= 80 KB
-constexpr uint32_t kOffRecvL = 80 * 1024;                   // [split][R] float, <= 2 KB
-constexpr uint32_t kOffStgO = 96 * 1024;                    // [256] rows
-constexpr uint32_t kOffStgL = kOffStgO + kRows * kRowBytes;  // [256] float
 constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kRowBytes = kD * 2;     // one bf16 output / partial row
 constexpr float kRescaleThreshold = 8.f;  // log2 units
 
-static_assert(kOffStgL + kRows * 4 <= kOffMask, "reduction buffers overlap the mask");
-
-enum Bar { QFULL = 0, KFULL = 1, VFULL = 3, KEMPTY = 5, VEMPTY = 7, SFULL = 9, PFULL = 11, FIN = 13,
-           RECV = 14 };
+enum Bar {
+  QFULL = 0, KFULL = 1, VFULL = 3, KEMPTY = 5, VEMPTY = 7, SFULL = 9, PFULL = 11, FIN = 13,
+  ADONE = 14, BDONE = 15, CBAR = 16
+};
 
 // Optional phase timestamps for performance work (off in normal builds).
 #ifdef LTD_TRACE
-__device__ unsigned long long g_attn_trace[2048][24];
-#define TRACE(slot)                                                                           \
+__device__ unsigned long long g_attn_trace[2048][32];
+#define TRACE_VAL(slot, v)                                                                    \
   do {                                                                                        \
     const int cta_ = blockIdx.x + gridDim.x * (blockIdx.y + gridDim.y * blockIdx.z);          \
-    if (cta_ < 2048) g_attn_trace[cta_][slot] = tc::globaltimer();                            \
+    if (cta_ < 2048) g_attn_trace[cta_][slot] = (v);                                          \
   } while (0)
+#define TRACE(slot) TRACE_VAL(slot, tc::globaltimer())
 #else
 #define TRACE(slot) \
   do {              \
+  } while (0)
+#define TRACE_VAL(slot, v) \
+  do {                     \
   } while (0)
 #endif
 
 struct TcArgs {
   int32_t batch, hq, hkv, G, n_max, s_cap, max_ctx, W32;
-  int32_t splits, n_pairs;
+  int32_t splits, n_pairs, lpt;
+  int32_t nch_h;  // host bound on chunks per sequence: ceil((max_ctx + n_max) / 128)
+  int32_t rs;     // rows per combining split: multiple of 4, >= 256 / splits
   const int32_t* ctx;
   const int32_t* n_verify;
   const uint32_t* mask;
   float scale_log2;
   __nv_bfloat16* out;
+  uint8_t* part_o;  // [unit][owner][split][rs][256 B] O / l, bf16 (splits > 1)
+  float* part_l;    // [unit][owner][split][rs] log2-sum-exp
+  uint32_t* sync;   // [unit][2] arrive, depart
   uint32_t* err;
 };
 
@@ -121,42 +133,28 @@ __device__ __forceinline__ uint32_t visible32(int kk0, int ctx, int key_hi, int 
   return in_range & (prefix | tree);
 }
 
+__device__ __forceinline__ bool seq_ok(const TcArgs& a, int ctx, int N) {
+  return N >= 1 && N <= a.n_max && ctx >= 0 && ctx <= a.max_ctx && ctx + N <= a.s_cap;
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CUtensorMap tk,
                    const __grid_constant__ CUtensorMap tv, const TcArgs a) {
   extern __shared__ uint8_t smem_raw[];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   if (tid == 0) TRACE(0);
-  const int split = blockIdx.x, pair = blockIdx.y;
-  const int b = blockIdx.z / a.hkv, kvh = blockIdx.z % a.hkv;
-
-  // Everything a CTA returns early on is shared by its whole cluster (same
-  // sequence, head and tile pair), so clusters return as a unit.
-  const int ctx = a.ctx[b];
-  const int N = a.n_verify[b];
-  if (N < 1 || N > a.n_max || ctx < 0 || ctx > a.max_ctx || ctx + N > a.s_cap) {
-    if (tid == 0 && split == 0 && pair == 0 && kvh == 0)
-      flag_error(a.err, (N < 1 || N > a.n_max) ? LTD_DEVERR_NVERIFY : LTD_DEVERR_CTX);
-    return;
-  }
-  const int M = N * a.G;
-  const int row0 = pair * kRows;
-  if (row0 >= M) return;
-  const bool has_b = row0 + kBM < M;
-  const int nk = ctx + N;
-  const int nch = (nk + kBN - 1) / kBN;
-  const int cs = split * nch / a.splits, ce = (split + 1) * nch / a.splits;
-  const int nc = ce - cs;
-  const int key_lo = cs * kBN, key_hi = min(ce * kBN, nk);
-
   const uint32_t raw = tc::smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
   uint8_t* gbase = smem_raw + (base - raw);
   uint32_t* mask_s = reinterpret_cast<uint32_t*>(gbase + kOffMask);
   uint32_t* holder = reinterpret_cast<uint32_t*>(gbase + kOffHolder);
   auto bar = [&](int i) { return base + kOffBar + 8u * i; };
+  const int S = a.splits;
 
   if (tid == 0) {
+    tc::tma_prefetch(&tq);
+    tc::tma_prefetch(&tk);
+    tc::tma_prefetch(&tv);
     tc::mbar_init(bar(QFULL), 1);
     for (int s = 0; s < 2; ++s) {
       tc::mbar_init(bar(KFULL + s), 1);
@@ -167,28 +165,153 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::mbar_init(bar(PFULL + s), 128);
     }
     tc::mbar_init(bar(FIN), 1);
-    tc::mbar_init(bar(RECV), 1);
+    tc::mbar_init(bar(ADONE), 128);
+    tc::mbar_init(bar(BDONE), 128);
+    tc::mbar_init(bar(CBAR), 1);
     tc::mbar_init_fence();
+    TRACE(19);
   }
+
+  // ------------------------------------------------------ which unit
+  int split = 0, pair, b, kvh;
+  if (S > 1) {
+    split = blockIdx.x;
+    pair = blockIdx.y;
+    b = blockIdx.z / a.hkv;
+    kvh = blockIdx.z % a.hkv;
+  } else {
+    const int i = blockIdx.x;
+    int g = i / a.hkv;
+    kvh = i % a.hkv;
+    if (a.lpt) {
+      // rank every (sequence, tile pair) group by its work, largest first
+      // (ties to the lower group, so equal pairs of one sequence, which
+      // read the same K/V, stay together), and take the group at this
+      // CTA's rank; bad sequences rank last and flag on their own CTAs
+      int* cost = reinterpret_cast<int*>(gbase + kOffCost);
+      int* order = reinterpret_cast<int*>(gbase + kOffOrder);
+      const int groups = a.batch * a.n_pairs;
+      for (int gi = tid; gi < groups; gi += kThreads) {
+        const int bb = gi / a.n_pairs, pp = gi % a.n_pairs;
+        const int c = a.ctx[bb], n = a.n_verify[bb];
+        int w = 0;
+        if (seq_ok(a, c, n)) {
+          const int rows = n * a.G - pp * kRows;
+          w = (rows <= 0 ? 0 : (rows > kBM ? 2 : 1)) * ((c + n + kBN - 1) / kBN);
+        }
+        cost[gi] = w;
+      }
+      __syncthreads();
+      for (int gi = tid; gi < groups; gi += kThreads) {
+        const int w = cost[gi];
+        int r = 0;
+        for (int o = 0; o < groups; ++o) {
+          const int wo = cost[o];
+          r += (wo > w) || (wo == w && o < gi);
+        }
+        order[r] = gi;
+      }
+      __syncthreads();
+      g = order[g];
+    }
+    b = g / a.n_pairs;
+    pair = g % a.n_pairs;
+  }
+  TRACE_VAL(25, static_cast<unsigned long long>(b));
+  TRACE_VAL(26, static_cast<unsigned long long>(pair));
+
+  // Keys are split by the host bound on the chunk count, so a split knows
+  // its first chunks before reading ctx and N: the loads of Q and of the
+  // first two K/V chunks go out at once (extra ones past this sequence's end
+  // are drained and ignored).
+  const int cs = split * a.nch_h / S, ce = (split + 1) * a.nch_h / S;
+  const int kvrow = b * a.hkv + kvh;
+  const int row0 = pair * kRows;
+  const bool has_b_h = row0 + kBM < a.n_max * a.G;  // tile b may hold rows
+  int nk_issued[2] = {0, 0}, nv_issued[2] = {0, 0}, n_issued = 0;
+  bool q_issued = false;
+  auto issue_k = [&](int j) {
+    const int st = j & 1;
+    tc::mbar_expect_tx(bar(KFULL + st), kTile);
+    for (int h = 0; h < 2; ++h)
+      tc::tma_load_3d(base + kOffK + st * kTile + h * kHalf, &tk, bar(KFULL + st), h * 64,
+                      (cs + j) * kBN, kvrow);
+    ++nk_issued[st];
+  };
+  auto issue_v = [&](int j) {
+    const int st = j & 1;
+    tc::mbar_expect_tx(bar(VFULL + st), kTile);
+    for (int h = 0; h < 2; ++h)
+      tc::tma_load_3d(base + kOffV + st * kTile + h * kHalf, &tv, bar(VFULL + st), h * 64,
+                      (cs + j) * kBN, kvrow);
+    ++nv_issued[st];
+  };
+  auto issue_first = [&]() {
+    tc::mbar_expect_tx(bar(QFULL), has_b_h ? 2 * kTile : kTile);
+    for (int t = 0; t < (has_b_h ? 2 : 1); ++t) {
+      const int qrow = b * a.n_max + (row0 + t * kBM) / a.G;
+      for (int h = 0; h < 2; ++h)
+        tc::tma_load_3d(base + kOffQ + t * kTile + h * kHalf, &tq, bar(QFULL), h * 64, kvh * a.G,
+                        qrow);
+    }
+    q_issued = true;
+    TRACE(20);
+    for (; n_issued < min(ce - cs, 2); ++n_issued) {
+      issue_k(n_issued);
+      issue_v(n_issued);
+    }
+    TRACE(17);
+  };
+  // every load a CTA issued lands before it leaves or reuses shared memory
+  auto drain = [&]() {
+    if (q_issued) tc::mbar_wait(bar(QFULL), 0);
+    for (int st = 0; st < 2; ++st) {
+      if (nk_issued[st] > 0) tc::mbar_wait(bar(KFULL + st), (nk_issued[st] - 1) & 1);
+      if (nv_issued[st] > 0) tc::mbar_wait(bar(VFULL + st), (nv_issued[st] - 1) & 1);
+    }
+  };
+  if (tid == 0 && !a.lpt) issue_first();
+
+  // Everything a CTA returns early on is shared by all splits of its unit.
+  const int ctx = a.ctx[b];
+  const int N = a.n_verify[b];
+  const int M = N * a.G;
+  if (tid == 0) TRACE(21);
+  if (!seq_ok(a, ctx, N) || row0 >= M) {
+    if (tid == 0) {
+      if (!seq_ok(a, ctx, N) && split == 0 && pair == 0 && kvh == 0)
+        flag_error(a.err, (N < 1 || N > a.n_max) ? LTD_DEVERR_NVERIFY : LTD_DEVERR_CTX);
+      drain();
+    }
+    return;
+  }
+  const bool has_b = row0 + kBM < M;
+  const int nk = ctx + N;
+  const int nch = (nk + kBN - 1) / kBN;
+  const int nc = max(0, min(ce, nch) - cs);
+  const int key_lo = cs * kBN, key_hi = min(ce * kBN, nk);
+  if (tid == 0) TRACE_VAL(24, static_cast<unsigned long long>(nc));
+  if (tid == 0 && a.lpt) issue_first();
   if (warp == 1) {
     tc::tmem_alloc(tc::smem_u32(holder), kTmemCols);
     tc::tmem_relinquish();
   }
-  // softmax threads: tile x, TMEM lane rr % 128, staging row rr
+  // softmax threads: tile x, TMEM lane rr % 128, row rr of the unit
   const int rr = tid - 128;
   const int x = rr >> 7;
   const int R = row0 + rr;
   const bool row_ok = tid >= 128 && R < M;
   if (tid >= 128) {
-    const int slot = row_ok ? R / a.G : 0;
+    const int slot = R / a.G;
+    const bool in = slot < a.n_max;
     for (int w = 0; w < a.W32; ++w)
       mask_s[rr * kMaxW32 + w] =
-          row_ok ? a.mask[(static_cast<int64_t>(b) * a.n_max + slot) * a.W32 + w] : 0u;
+          in ? a.mask[(static_cast<int64_t>(b) * a.n_max + slot) * a.W32 + w] : 0u;
   }
   tc::fence_before_sync();
   __syncthreads();
   tc::fence_after_sync();
-  const uint32_t tmem = *holder;
+  const uint32_t tmem = holder[0];
   if (tid == 0) TRACE(1);
   bool ok = true;
   const bool tile_active = tid >= 128 && (x == 0 || has_b) && nc > 0;
@@ -196,43 +319,17 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
-    if (lane == 0 && nc > 0) {
-      int nk_issued[2] = {0, 0}, nv_issued[2] = {0, 0};
-      tc::tma_prefetch(&tq);
-      tc::tma_prefetch(&tk);
-      tc::tma_prefetch(&tv);
-      tc::mbar_expect_tx(bar(QFULL), has_b ? 2 * kTile : kTile);
-      for (int t = 0; t < (has_b ? 2 : 1); ++t) {
-        const int qrow = b * a.n_max + (row0 + t * kBM) / a.G;
-        for (int h = 0; h < 2; ++h)
-          tc::tma_load_3d(base + kOffQ + t * kTile + h * kHalf, &tq, bar(QFULL), h * 64, kvh * a.G,
-                          qrow);
-      }
-      const int kvrow = b * a.hkv + kvh;
-      for (int j = 0; j < nc && ok; ++j) {
+    if (lane == 0) {
+      for (int j = n_issued; j < nc && ok; ++j) {
         const int st = j & 1;
-        const int key0 = key_lo + j * kBN;
-        if (j >= 2) ok = tc::mbar_wait(bar(KEMPTY + st), ((j >> 1) - 1) & 1);
+        ok = tc::mbar_wait(bar(KEMPTY + st), ((j >> 1) - 1) & 1);
         if (!ok) break;
-        tc::mbar_expect_tx(bar(KFULL + st), kTile);
-        for (int h = 0; h < 2; ++h)
-          tc::tma_load_3d(base + kOffK + st * kTile + h * kHalf, &tk, bar(KFULL + st), h * 64, key0,
-                          kvrow);
-        ++nk_issued[st];
-        if (j >= 2) ok = tc::mbar_wait(bar(VEMPTY + st), ((j >> 1) - 1) & 1);
+        issue_k(j);
+        ok = tc::mbar_wait(bar(VEMPTY + st), ((j >> 1) - 1) & 1);
         if (!ok) break;
-        tc::mbar_expect_tx(bar(VFULL + st), kTile);
-        for (int h = 0; h < 2; ++h)
-          tc::tma_load_3d(base + kOffV + st * kTile + h * kHalf, &tv, bar(VFULL + st), h * 64, key0,
-                          kvrow);
-        ++nv_issued[st];
+        issue_v(j);
       }
-      // drain: every load this CTA issued has landed before shared memory is reused
-      tc::mbar_wait(bar(QFULL), 0);
-      for (int st = 0; st < 2; ++st) {
-        if (nk_issued[st] > 0) tc::mbar_wait(bar(KFULL + st), (nk_issued[st] - 1) & 1);
-        if (nv_issued[st] > 0) tc::mbar_wait(bar(VFULL + st), (nv_issued[st] - 1) & 1);
-      }
+      drain();
       if (!ok) flag_error(a.err, LTD_DEVERR_TIMEOUT);
     }
   } else if (warp == 1) {
@@ -260,6 +357,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       ok = tc::mbar_wait(bar(QFULL), 0);
       TRACE(2);
       if (ok) ok = tc::mbar_wait(bar(KFULL + 0), 0);
+      TRACE(3);
       if (ok) {
         tc::fence_after_sync();
         for (int t = 0; t < ntile; ++t) {
@@ -301,250 +399,374 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int vis_all_below = min(ctx, key_hi);  // keys below this are all visible
     const float sl2 = a.scale_log2;
     const int w32 = a.W32;
+    const bool tr = (tid & 127) == 0;
     for (int j = 0; j < nc; ++j) {
+      if (has_b && (x == 1 || j > 0)) {
+        // tile a waits for b's previous chunk, tile b for a's current one;
+        // strict alternation keeps each barrier at most one phase ahead
+        const bool turn = x == 0 ? tc::mbar_wait(bar(BDONE), (j - 1) & 1)
+                                 : tc::mbar_wait(bar(ADONE), j & 1);
+        ok = __all_sync(0xFFFFFFFFu, turn);
+        if (!ok) break;
+      }
       ok = tc::mbar_wait(bar(SFULL + x), j & 1);
       ok = __all_sync(0xFFFFFFFFu, ok);
-      if (tid == 128 && j == 0) TRACE(11);
-
+      if (tr && j < 2) TRACE(4 + 4 * x + 2 * j);
       if (!ok) break;
       tc::fence_after_sync();
       const int kbase = key_lo + j * kBN;
-      const bool all_vis = kbase + kBN <= vis_all_below;
-      auto vis_of = [=](int q) {
-        return !row_ok ? 0u
-                       : (all_vis ? 0xFFFFFFFFu
-                                  : visible32(kbase + 32 * q, ctx, key_hi, w32, mbits));
-      };
-      // pass 1: the chunk's row max, 32 columns at a time, without branches
-      // per element; on fully visible fragments the max is taken on the raw
-      // scores (the scale is positive) and scaled once
-      float cm[4] = {-CUDART_INF_F, -CUDART_INF_F, -CUDART_INF_F, -CUDART_INF_F};
-#pragma unroll 1
-      for (int q = 0; q < 4; ++q) {
-        tc::Frag32 f;
-        tc::tmem_ld32(t_s + 32 * q, f);
-        const uint32_t vq = vis_of(q);
-        tc::tmem_wait_ld(f);
-        if (tid == 128 && j == 0 && q < 2) TRACE(3 + 2 * q);
-        if (vq == 0xFFFFFFFFu) {
-          float r[4] = {-CUDART_INF_F, -CUDART_INF_F, -CUDART_INF_F, -CUDART_INF_F};
+      const bool all_vis = row_ok && kbase + kBN <= vis_all_below;
+      tc::Frag128 f;
+      tc::tmem_ld128(t_s, f);
+      uint32_t vq[4] = {0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu};
+      if (!all_vis) {
 #pragma unroll
-          for (int c = 0; c < 32; ++c) r[c & 3] = fmaxf(r[c & 3], __uint_as_float(f.r[c]));
-#pragma unroll
-          for (int u = 0; u < 4; ++u) cm[u] = fmaxf(cm[u], r[u] * sl2);
-        } else {
-#pragma unroll
-          for (int c = 0; c < 32; ++c) {
-            const float t = ((vq >> c) & 1u) ? __uint_as_float(f.r[c]) * sl2 : -CUDART_INF_F;
-            cm[c & 3] = fmaxf(cm[c & 3], t);
-          }
-        }
-        if (tid == 128 && j == 0 && q < 2) TRACE(4 + 2 * q);
+        for (int q = 0; q < 4; ++q)
+          vq[q] = row_ok ? visible32(kbase + 32 * q, ctx, key_hi, w32, mbits) : 0u;
       }
-      const float cmax = fmaxf(fmaxf(cm[0], cm[1]), fmaxf(cm[2], cm[3]));
-      if (tid == 128 && j == 0) TRACE(14);
+      tc::tmem_wait_ld128(f);
+      if (!all_vis) {
+#pragma unroll
+        for (int c = 0; c < 128; ++c)
+          f.r[c] = ((vq[c >> 5] >> (c & 31)) & 1u) ? f.r[c] : 0xFF800000u;  // -inf if hidden
+      }
+      // the chunk's row max on the raw scores (the scale is positive)
+      float r8[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) r8[u] = __uint_as_float(f.r[u]);
+#pragma unroll
+      for (int c = 8; c < 128; c += 16) {
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+          r8[u] = tc::fmax3(r8[u], __uint_as_float(f.r[c + 2 * u]), __uint_as_float(f.r[c + 2 * u + 1]));
+      }
+      const float raw_max = fmaxf(tc::fmax3(r8[0], r8[1], r8[2]),
+                                  fmaxf(tc::fmax3(r8[3], r8[4], r8[5]), fmaxf(r8[6], r8[7])));
+      const float cmax = raw_max * sl2;
       // S(j) complete implies P_x(j-1) V finished, so O_x is stable here
       float mnew = m;
       if (cmax > m + kRescaleThreshold || (m == -CUDART_INF_F && cmax > -CUDART_INF_F)) mnew = cmax;
       const bool need = (mnew != m) && (m != -CUDART_INF_F) && (j >= 1);
-      if (__any_sync(0xFFFFFFFFu, need)) {
-        const float alpha = need ? tc::ex2(m - mnew) : 1.f;
-        l *= alpha;
-#pragma unroll 1
-        for (int q = 0; q < 4; ++q) {
-          tc::Frag32 f;
-          tc::tmem_ld32(t_o + 32 * q, f);
-          tc::tmem_wait_ld(f);
-#pragma unroll
-          for (int c = 0; c < 32; ++c) f.r[c] = __float_as_uint(__uint_as_float(f.r[c]) * alpha);
-          tc::tmem_st32(t_o + 32 * q, f);
-        }
-      }
+      const float alpha = need ? tc::ex2(m - mnew) : 1.f;
       m = mnew;
-      // pass 2: P = 2^(score - m) as bf16 pairs; fragment q (columns
-      // 32q..32q+31) becomes P columns 16q..16q+15, all already read
-      float2 ls2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+      // P = 2^(score - m) as bf16 pairs over S's first 64 columns
       const float mz = (m == -CUDART_INF_F) ? 0.f : m;  // m = -inf only if all are hidden
       const float2 sl22 = make_float2(sl2, sl2), nm2 = make_float2(-mz, -mz);
+      float2 ls2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+      tc::Frag64 pf;
+#pragma unroll
+      for (int c = 0; c < 64; ++c) {
+        const float2 t = __ffma2_rn(
+            make_float2(__uint_as_float(f.r[2 * c]), __uint_as_float(f.r[2 * c + 1])), sl22, nm2);
+        const float2 pp = make_float2(tc::ex2(t.x), tc::ex2(t.y));
+        ls2[c & 1] = __fadd2_rn(ls2[c & 1], pp);
+        pf.r[c] = pack_bf16(pp.x, pp.y);
+      }
+      tc::tmem_st64(t_s, pf);
+      if (__any_sync(0xFFFFFFFFu, need)) {
 #pragma unroll 1
-      for (int q = 0; q < 4; ++q) {
-        tc::Frag32 f;
-        tc::tmem_ld32(t_s + 32 * q, f);
-        const uint32_t vq = vis_of(q);
-        tc::tmem_wait_ld(f);
-        tc::Frag16 pf;
-        if (vq == 0xFFFFFFFFu) {
+        for (int q = 0; q < 4; ++q) {
+          tc::Frag32 o;
+          tc::tmem_ld32(t_o + 32 * q, o);
+          tc::tmem_wait_ld(o);
 #pragma unroll
-          for (int c = 0; c < 16; ++c) {
-            const float2 t = __ffma2_rn(
-                make_float2(__uint_as_float(f.r[2 * c]), __uint_as_float(f.r[2 * c + 1])), sl22, nm2);
-            const float2 pp = make_float2(tc::ex2(t.x), tc::ex2(t.y));
-            ls2[c & 1] = __fadd2_rn(ls2[c & 1], pp);
-            pf.r[c] = pack_bf16(pp.x, pp.y);
-          }
-        } else {
-#pragma unroll
-          for (int c = 0; c < 16; ++c) {
-            const float t0 =
-                ((vq >> (2 * c)) & 1u) ? __uint_as_float(f.r[2 * c]) * sl2 : -CUDART_INF_F;
-            const float t1 =
-                ((vq >> (2 * c + 1)) & 1u) ? __uint_as_float(f.r[2 * c + 1]) * sl2 : -CUDART_INF_F;
-            const float2 pp = make_float2(tc::ex2(t0 - mz), tc::ex2(t1 - mz));
-            ls2[c & 1] = __fadd2_rn(ls2[c & 1], pp);
-            pf.r[c] = pack_bf16(pp.x, pp.y);
-          }
+          for (int c = 0; c < 32; ++c) o.r[c] = __float_as_uint(__uint_as_float(o.r[c]) * alpha);
+          tc::tmem_st32(t_o + 32 * q, o);
         }
-        tc::tmem_st16(t_s + 16 * q, pf);
       }
       const float2 lsum = __fadd2_rn(ls2[0], ls2[1]);
-      l += lsum.x + lsum.y;
-      if (tid == 128 && j == 0) TRACE(15);
+      l = l * alpha + (lsum.x + lsum.y);
+      if (x == 0 && kbase + kBN > key_hi) {
+        // Keys from key_hi on may hold anything in the cache, even NaN: P is
+        // 0 there, but 0 * NaN is not, so tile a's threads clear those V rows
+        // (both 64-dim halves) before either tile's PV reads this stage.
+        const int st = j & 1;
+        // (a failed wait is flagged; the MMA thread times out on the same stage)
+        if (!__all_sync(0xFFFFFFFFu, tc::mbar_wait(bar(VFULL + st), (j >> 1) & 1)) && lane == 0)
+          flag_error(a.err, LTD_DEVERR_TIMEOUT);
+        const int z0 = key_hi - kbase;  // 1 .. 127
+        uint4* vs = reinterpret_cast<uint4*>(gbase + kOffV + st * kTile);
+        for (int idx = rr; idx < (kBN - z0) * 16; idx += kBM) {
+          const int row = z0 + (idx >> 4), piece = idx & 15;
+          vs[((piece >> 3) * kHalf + row * 128) / 16 + (piece & 7)] = make_uint4(0u, 0u, 0u, 0u);
+        }
+        tc::fence_smem_async();
+      }
       tc::tmem_wait_st();
       tc::fence_before_sync();
       tc::mbar_arrive(bar(PFULL + x));
-      if (tid == 128 && j == 0) TRACE(12);
+      if (has_b && (x == 0 || j + 1 < nc)) tc::mbar_arrive(bar(x == 0 ? ADONE : BDONE));
+      if (tr && j < 2) TRACE(5 + 4 * x + 2 * j);
     }
-    if (tid == 128) TRACE(13);
     if (ok) {
       ok = tc::mbar_wait(bar(FIN), 0);
       ok = __all_sync(0xFFFFFFFFu, ok);
     }
+    if (tr) TRACE(12 + x);
     if (!ok && lane == 0) flag_error(a.err, LTD_DEVERR_TIMEOUT);
   }
 
-  // --------------------- exchange partials with the cluster (bulk DSMEM)
+  // --------------------------------------------------------- epilogue
+  // O / l of every row (bf16; zero where a row has nothing) and its
+  // log2-sum-exp are staged in shared memory over Q and over the mask (both
+  // free once the last MMA has completed): row r's 16-byte chunk c sits at
+  // ((c ^ (r & 15)) << 4), so the row-per-thread stores of a warp spread
+  // over the banks.  One split: all threads copy the rows to the output,
+  // coalesced.  Several: the partial layout below.
+  const int unit = (b * a.hkv + kvh) * a.n_pairs + pair;
+  const int Mv = min(kRows, M - row0);
+  uint8_t* stg = gbase + kOffQ;
+  float* stg_l = reinterpret_cast<float*>(gbase + kOffMask);
+  // tcgen05.ld is warp-collective: the O load is taken by whole warps
+  // (tile_active and ok are uniform within a warp), the writes per row.
+  const bool loaded = tile_active && ok;
+  tc::Frag128 o;
+  if (loaded) {
+    tc::fence_after_sync();
+    tc::tmem_ld128(tmem + 2 * kBN + x * kD + ((32u * (warp & 3)) << 16), o);
+    tc::tmem_wait_ld128(o);
+  }
+  if (row_ok) {
+    const bool have = loaded && l > 0.f;
+    const float inv = have ? 1.f / l : 0.f;
+    uint8_t* srow = stg + rr * kRowBytes;
+#pragma unroll
+    for (int c = 0; c < 16; ++c) {
+      uint4 w = make_uint4(0u, 0u, 0u, 0u);
+      if (have) {
+        w.x = pack_bf16(__uint_as_float(o.r[8 * c]) * inv, __uint_as_float(o.r[8 * c + 1]) * inv);
+        w.y = pack_bf16(__uint_as_float(o.r[8 * c + 2]) * inv, __uint_as_float(o.r[8 * c + 3]) * inv);
+        w.z = pack_bf16(__uint_as_float(o.r[8 * c + 4]) * inv, __uint_as_float(o.r[8 * c + 5]) * inv);
+        w.w = pack_bf16(__uint_as_float(o.r[8 * c + 6]) * inv, __uint_as_float(o.r[8 * c + 7]) * inv);
+      }
+      *reinterpret_cast<uint4*>(srow + ((c ^ (rr & 15)) << 4)) = w;
+    }
+    stg_l[rr] = have ? m + __log2f(l) : -CUDART_INF_F;
+  }
+  tc::fence_smem_async();  // the staging is read by bulk copies
   tc::fence_before_sync();
   __syncthreads();
-  if (tid == 0) TRACE(16);
-  const int S = a.splits;
-  const int rank = static_cast<int>(tc::cluster_rank());
-  const int R4 = (((kRows + S - 1) / S) + 3) & ~3;
-  const int n_own = max(0, min(R4, kRows - rank * R4));
-  if (tid == 0) tc::mbar_expect_tx(bar(RECV), static_cast<uint32_t>(S * n_own) * (kRowBytes + 4));
-  // stage this split's rows: O / l in bf16 and lse = m + log2(l)
-  if (tid >= 128) {
-    float lse = -CUDART_INF_F;
-    uint8_t* srow = gbase + kOffStgO + rr * kRowBytes;
-    if (tile_active && ok) {
-      tc::fence_after_sync();
-      const uint32_t t_o = tmem + 2 * kBN + x * kD + ((32u * (warp & 3)) << 16);
-      const float inv = l > 0.f ? 1.f / l : 0.f;
-#pragma unroll 1
-      for (int q = 0; q < 4; ++q) {
-        tc::Frag32 f;
-        tc::tmem_ld32(t_o + 32 * q, f);
-        tc::tmem_wait_ld(f);
-#pragma unroll
-        for (int c16 = 0; c16 < 4; ++c16) {
-          const int c = 4 * q + c16;  // 16-byte chunk (8 values) of the row
-          uint4 w;
-          w.x = pack_bf16(__uint_as_float(f.r[8 * c16]) * inv, __uint_as_float(f.r[8 * c16 + 1]) * inv);
-          w.y = pack_bf16(__uint_as_float(f.r[8 * c16 + 2]) * inv, __uint_as_float(f.r[8 * c16 + 3]) * inv);
-          w.z = pack_bf16(__uint_as_float(f.r[8 * c16 + 4]) * inv, __uint_as_float(f.r[8 * c16 + 5]) * inv);
-          w.w = pack_bf16(__uint_as_float(f.r[8 * c16 + 6]) * inv, __uint_as_float(f.r[8 * c16 + 7]) * inv);
-          *reinterpret_cast<uint4*>(srow + ((c ^ (rr & 15)) << 4)) = w;
-        }
-      }
-      if (row_ok && l > 0.f) lse = m + __log2f(l);
-    }
-    reinterpret_cast<float*>(gbase + kOffStgL)[rr] = lse;
-    tc::fence_smem_async();  // staging becomes visible to the bulk copies
-  }
-  __syncthreads();
-  // every CTA has registered its receive count and is past its last MMA and
-  // TMA load, so its ring buffers can now be written by peers
-  tc::cluster_sync();
-  if (tid == 0) TRACE(7);
-  if (tid == 0) {
-    for (int r = 0; r < S; ++r) {
-      const int n = max(0, min(R4, kRows - r * R4));
-      if (n == 0) continue;
-      const uint32_t pbar = tc::mapa(bar(RECV), r);
-      tc::bulk_s2cluster(tc::mapa(base + kOffRecvO + (rank * R4) * kRowBytes, r),
-                         base + kOffStgO + (r * R4) * kRowBytes, n * kRowBytes, pbar);
-      tc::bulk_s2cluster(tc::mapa(base + kOffRecvL + (rank * R4) * 4, r),
-                         base + kOffStgL + (r * R4) * 4, n * 4, pbar);
-    }
-    tc::bulk_commit();
-  }
-  const bool got = tc::mbar_wait(bar(RECV), 0);
-  if (!got && tid == 0) flag_error(a.err, LTD_DEVERR_TIMEOUT);
-  if (tid == 0) TRACE(8);
-
-  // ------------------------- combine the splits of this CTA's rows (local)
-  if (got) {
-    const uint8_t* recv_o = gbase + kOffRecvO;
-    const float* recv_l = reinterpret_cast<const float*>(gbase + kOffRecvL);
-    const int ch = lane >> 1, half = lane & 1;  // lane owns output dims 4 lane .. 4 lane + 3
-    for (int lr = warp; lr < n_own; lr += kWarps) {
-      const int r = rank * R4 + lr;
-      const int Rr = row0 + r;
-      if (Rr >= M) continue;
-      const uint32_t coff = (((ch ^ (r & 15)) << 4) + half * 8);
-      float lp[kMaxCluster];
-      uint2 vp[kMaxCluster];
-#pragma unroll
-      for (int p = 0; p < kMaxCluster; ++p) {
-        if (p < S) {
-          lp[p] = recv_l[p * R4 + lr];
-          vp[p] = *reinterpret_cast<const uint2*>(recv_o + (p * R4 + lr) * kRowBytes + coff);
-        }
-      }
-      float mx = -CUDART_INF_F;
-#pragma unroll
-      for (int p = 0; p < kMaxCluster; ++p)
-        if (p < S) mx = fmaxf(mx, lp[p]);
-      float acc[4] = {0.f, 0.f, 0.f, 0.f};
-      float L = 0.f;
-#pragma unroll
-      for (int p = 0; p < kMaxCluster; ++p) {
-        if (p < S && lp[p] > -CUDART_INF_F) {
-          const float w = tc::ex2(lp[p] - mx);
-          L += w;
-          acc[0] += w * __uint_as_float(vp[p].x << 16);
-          acc[1] += w * __uint_as_float(vp[p].x & 0xFFFF0000u);
-          acc[2] += w * __uint_as_float(vp[p].y << 16);
-          acc[3] += w * __uint_as_float(vp[p].y & 0xFFFF0000u);
-        }
-      }
-      const float inv = L > 0.f ? 1.f / L : 0.f;
-      const int slot = Rr / a.G, g = Rr % a.G;
-      __nv_bfloat16* dst = a.out +
-                           ((static_cast<int64_t>(b) * a.n_max + slot) * a.hq + kvh * a.G + g) * kD +
-                           4 * lane;
-      uint2 w2;
-      w2.x = pack_bf16(acc[0] * inv, acc[1] * inv);
-      w2.y = pack_bf16(acc[2] * inv, acc[3] * inv);
-      *reinterpret_cast<uint2*>(dst) = w2;
-    }
-  }
-  if (tid == 0) TRACE(9);
-  // the sources of this CTA's outgoing copies stay valid until read
-  if (tid == 0) tc::bulk_wait_read();
-  __syncthreads();
+  if (tid == 0) TRACE(14);
   if (warp == 1) {
     __syncwarp();
     tc::fence_after_sync();
     tc::tmem_dealloc(tmem, kTmemCols);
   }
+  if (S == 1) {
+    for (int idx = tid; idx < Mv * 16; idx += kThreads) {
+      const int r = idx >> 4, c = idx & 15;
+      const int Rr = row0 + r, slot = Rr / a.G, g = Rr % a.G;
+      const uint4 v = *reinterpret_cast<const uint4*>(stg + r * kRowBytes + ((c ^ (r & 15)) << 4));
+      reinterpret_cast<uint4*>(a.out + ((static_cast<int64_t>(b) * a.n_max + slot) * a.hq +
+                                        kvh * a.G + g) * kD)[c] = v;
+    }
+    return;
+  }
+
+  // ------------------------------------- combine the splits (S > 1 only)
+  // Rows [o rs, o rs + rs) of a unit are combined by its split o ("owner").
+  // Partials are laid out owner-major, [unit][owner][split][rs][256 B], so
+  // every split writes its rows with coalesced stores and an owner reads all
+  // of its inputs with one bulk copy.
+  const int Rs = a.rs;
+  {
+    uint8_t* po = a.part_o + static_cast<int64_t>(unit) * S * S * Rs * kRowBytes;
+    float* pl = a.part_l + static_cast<int64_t>(unit) * S * S * Rs;
+    for (int idx = tid; idx < Mv * 16; idx += kThreads) {
+      const int r = idx >> 4, c = idx & 15;
+      const int o = r / Rs, rl = r - o * Rs;
+      const uint4 v = *reinterpret_cast<const uint4*>(stg + r * kRowBytes + ((c ^ (r & 15)) << 4));
+      reinterpret_cast<uint4*>(po + ((static_cast<int64_t>(o) * S + split) * Rs + rl) * kRowBytes)[c] = v;
+    }
+    for (int r = tid; r < Mv; r += kThreads) {
+      const int o = r / Rs, rl = r - o * Rs;
+      pl[(static_cast<int64_t>(o) * S + split) * Rs + rl] = stg_l[r];
+    }
+  }
+  __syncthreads();
+  uint32_t* arrive = a.sync + 2 * unit;
+  uint32_t* depart = arrive + 1;
+  if (tid == 0) {
+    __threadfence();  // with the barrier above: every thread's partial stores
+    tc::red_add_release_gpu(arrive, 1u);
+    bool got = tc::ld_acquire_gpu(arrive) >= static_cast<uint32_t>(S);
+    if (!got) {
+      const uint64_t t0 = tc::globaltimer();
+      while (!got) {
+        __nanosleep(32);
+        got = tc::ld_acquire_gpu(arrive) >= static_cast<uint32_t>(S);
+        if (!got && tc::globaltimer() - t0 > tc::kWaitLimitNs) break;
+      }
+    }
+    __threadfence();
+    if (!got) flag_error(a.err, LTD_DEVERR_TIMEOUT);
+    holder[1] = got ? 1u : 0u;
+    TRACE(15);
+  }
+  __syncthreads();
+  const int r_lo = split * Rs;
+  const int nrows = max(0, min(Mv, r_lo + Rs) - r_lo);
+  if (holder[1] != 0u && nrows > 0) {
+    if (tid == 0) {
+      // partial writes by other CTAs (generic proxy) are read by the bulk copy
+      tc::fence_proxy_async_global();
+      const int64_t ob = static_cast<int64_t>(unit) * S + split;
+      tc::mbar_expect_tx(bar(CBAR), static_cast<uint32_t>(S * Rs) * (kRowBytes + 4));
+      tc::bulk_g2s(base + kOffK, a.part_o + ob * S * Rs * kRowBytes, S * Rs * kRowBytes, bar(CBAR));
+      tc::bulk_g2s(base + kOffMask, a.part_l + ob * S * Rs, S * Rs * 4, bar(CBAR));
+    }
+    // CTA-uniform, as a barrier follows under it
+    const bool in = __syncthreads_and(tc::mbar_wait(bar(CBAR), 0)) != 0;
+    if (tid == 0) TRACE(18);
+    if (!in) {
+      if (tid == 0) flag_error(a.err, LTD_DEVERR_TIMEOUT);
+    } else {
+      const uint8_t* cin = gbase + kOffK;
+      const float* lin = reinterpret_cast<const float*>(gbase + kOffMask);
+      // A half-warp per row, a lane per 16-byte chunk: the lanes first hold
+      // the splits' log2-sum-exps (split p on lane p % 16), reduce them to
+      // weights 2^(lse_p - max) / sum, then broadcast weight p while every
+      // lane sums its chunk over the splits.  Loop bounds are warp-uniform
+      // (the shuffles need whole warps); lanes past the last row only idle.
+      const int nwork = (nrows * 16 + 31) & ~31;
+      for (int idx = tid; idx < nwork; idx += kThreads) {
+        const int rw = idx >> 4, c = idx & 15;
+        const bool live = rw < nrows;
+        const int r = live ? rw : nrows - 1;
+        float lpk[kMaxSplits / 16];
+        float mx = -CUDART_INF_F;
+#pragma unroll
+        for (int k = 0; k < kMaxSplits / 16; ++k) {
+          const int p = c + 16 * k;
+          lpk[k] = p < S ? lin[p * Rs + r] : -CUDART_INF_F;
+          mx = fmaxf(mx, lpk[k]);
+        }
+#pragma unroll
+        for (int o = 8; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xFFFFFFFFu, mx, o));
+        float L = 0.f;
+#pragma unroll
+        for (int k = 0; k < kMaxSplits / 16; ++k) {
+          lpk[k] = (lpk[k] > -CUDART_INF_F) ? tc::ex2(lpk[k] - mx) : 0.f;
+          L += lpk[k];
+        }
+#pragma unroll
+        for (int o = 8; o > 0; o >>= 1) L += __shfl_xor_sync(0xFFFFFFFFu, L, o);
+        const float inv = L > 0.f ? 1.f / L : 0.f;
+        float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        const int half = lane & 16;
+#pragma unroll
+        for (int k = 0; k < kMaxSplits / 16; ++k) {
+          if (16 * k >= S) break;  // uniform
+#pragma unroll 4
+          for (int q = 0; q < 16; ++q) {
+            const int p = 16 * k + q;
+            const float w = __shfl_sync(0xFFFFFFFFu, lpk[k], half | q);
+            if (p < S) {
+              const uint4 v =
+                  *reinterpret_cast<const uint4*>(cin + (p * Rs + r) * kRowBytes + c * 16);
+              const uint32_t e[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+              for (int t = 0; t < 4; ++t) {
+                acc[2 * t] = fmaf(w, __uint_as_float(e[t] << 16), acc[2 * t]);
+                acc[2 * t + 1] = fmaf(w, __uint_as_float(e[t] & 0xFFFF0000u), acc[2 * t + 1]);
+              }
+            }
+          }
+        }
+        if (live) {
+          const int Rr = row0 + r_lo + r;
+          const int slot = Rr / a.G, g = Rr % a.G;
+          uint4 w;
+          w.x = pack_bf16(acc[0] * inv, acc[1] * inv);
+          w.y = pack_bf16(acc[2] * inv, acc[3] * inv);
+          w.z = pack_bf16(acc[4] * inv, acc[5] * inv);
+          w.w = pack_bf16(acc[6] * inv, acc[7] * inv);
+          reinterpret_cast<uint4*>(a.out + ((static_cast<int64_t>(b) * a.n_max + slot) * a.hq +
+                                            kvh * a.G + g) * kD)[c] = w;
+        }
+      }
+      if (tid == 0) TRACE(23);
+    }
+  }
+  __syncthreads();
+  if (tid == 0) {
+    TRACE(16);
+    // every split of this unit has passed its spin once all have departed
+    const uint32_t d = atomicAdd(depart, 1u);
+    if (d == static_cast<uint32_t>(S) - 1u) {
+      atomicExch(arrive, 0u);
+      atomicExch(depart, 0u);
+    }
+  }
 }
 
 struct Plan {
-  int n_pairs, splits;
+  int n_pairs, splits, units, lpt, nch, rs;
 };
 
+// Streaming multiprocessors of the current device (152 if it cannot be asked).
+int device_sms() {
+  static std::mutex mu;
+  static int known[128] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 128) {
+    (void)cudaGetLastError();
+    return 152;
+  }
+  std::lock_guard<std::mutex> lock(mu);
+  if (known[dev] == 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1) {
+      (void)cudaGetLastError();
+      n = 152;
+    }
+    known[dev] = n;
+  }
+  return known[dev];
+}
+
+// Units = (sequence, KV head, tile pair).  With fewer units than SMs each
+// unit's keys are cut into the fewest splits that give the shortest longest
+// split, at most SMs / units of them, so all CTAs fit one wave.
 Plan plan(int32_t batch, int32_t hq, int32_t hkv, int32_t n_max, int32_t max_ctx) {
   const int G = hq / hkv;
   Plan p{};
   p.n_pairs = (n_max * G + kRows - 1) / kRows;
   const int64_t units = static_cast<int64_t>(batch) * hkv * p.n_pairs;
+  p.units = static_cast<int>(units);
   const int nch = (max_ctx + n_max + kBN - 1) / kBN;
-  constexpr int64_t kSMs = 152;
-  int s = units >= kSMs ? 1 : static_cast<int>(kSMs / units);
-  s = s > kMaxCluster ? kMaxCluster : s;
-  s = s > nch ? nch : s;
-  p.splits = s < 1 ? 1 : s;
+  const int sms = device_sms();
+  p.splits = 1;
+  if (units < sms) {
+    int smax = static_cast<int>(sms / units);
+    smax = smax < nch ? smax : nch;
+    smax = smax < kMaxSplits ? smax : kMaxSplits;
+    if (smax > 1) {
+      const int maxc = (nch + smax - 1) / smax;
+      p.splits = (nch + maxc - 1) / maxc;
+    }
+  }
+  p.lpt = (p.splits == 1 && static_cast<int64_t>(batch) * p.n_pairs <= kMaxGroups) ? 1 : 0;
+  p.nch = nch;
+  p.rs = (((kRows + p.splits - 1) / p.splits) + 3) & ~3;
   return p;
+}
+
+size_t align256(size_t n) { return (n + 255) / 256 * 256; }
+
+struct WsLayout {
+  size_t part_o, part_l, sync, total;
+};
+WsLayout ws_layout(const Plan& pl) {
+  WsLayout w{};
+  if (pl.splits <= 1) return w;
+  // [unit][owner][split][rs] rows: splits * rs <= 256 + 4 * splits
+  const size_t rows = static_cast<size_t>(pl.units) * pl.splits * pl.splits * pl.rs;
+  w.part_o = 0;
+  w.part_l = align256(rows * kRowBytes);
+  w.sync = w.part_l + align256(rows * sizeof(float));
+  w.total = w.sync + align256(static_cast<size_t>(pl.units) * 2 * sizeof(uint32_t));
+  return w;
 }
 
 using EncodeFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
@@ -565,52 +787,6 @@ EncodeFn encode_fn() {
       fn = reinterpret_cast<EncodeFn>(p);
   }
   return fn;
-}
-
-// Cluster size for `units` independent clusters: the largest s <= want for
-// which the device can keep all of them resident at once (one wave), else
-// the largest s it can run at all.  Asked once per device and size.
-int max_active_clusters(int s) {
-  static std::mutex mu;
-  static int known[128][kMaxCluster + 1];
-  static bool init = false;
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 128) return 0;
-  std::lock_guard<std::mutex> lock(mu);
-  if (!init) {
-    for (auto& row : known)
-      for (int& v : row) v = -1;
-    init = true;
-  }
-  if (known[dev][s] < 0) {
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(s, 1, 1);
-    cfg.blockDim = dim3(kThreads);
-    cfg.dynamicSmemBytes = kSmemBytes;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = s;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    int n = 0;
-    const cudaError_t e = cudaOccupancyMaxActiveClusters(&n, attn_tc_kernel, &cfg);
-    if (e != cudaSuccess) {
-      (void)cudaGetLastError();
-      n = 0;
-    }
-    known[dev][s] = n;
-  }
-  return known[dev][s];
-}
-
-int fit_splits(int want, int64_t units) {
-  for (int s = want; s > 1; --s)
-    if (max_active_clusters(s) >= units) return s;
-  for (int s = want; s > 1; --s)
-    if (max_active_clusters(s) > 0) return s;
-  return 1;
 }
 
 }  // namespace
@@ -634,12 +810,18 @@ bool attn_tc_supported(const AttnParams& p, ltd_dtype dtype) {
   return G >= 1 && G <= kBM && kBM % G == 0 && p.n_max <= LTD_MAX_N;
 }
 
-size_t attn_tc_workspace(int32_t, int32_t, int32_t, int32_t, int32_t, int32_t) { return 0; }
+
+size_t attn_tc_workspace(int32_t batch, int32_t hq, int32_t hkv, int32_t, int32_t n_max,
+                         int32_t max_ctx) {
+  return ws_layout(plan(batch, hq, hkv, n_max, max_ctx)).total;
+}
 
 int32_t attn_tc_launches(int32_t, int32_t, int32_t, int32_t, int32_t) { return 1; }
 
 cudaError_t launch_attn_tc(const AttnParams& p, cudaStream_t s) {
   const Plan pl = plan(p.batch, p.hq, p.hkv, p.n_max, p.max_ctx);
+  const WsLayout wl = ws_layout(pl);
+  if (p.ws_bytes < wl.total || (wl.total > 0 && p.ws == nullptr)) return cudaErrorInvalidValue;
   TcArgs a{};
   a.batch = p.batch;
   a.hq = p.hq;
@@ -651,11 +833,18 @@ cudaError_t launch_attn_tc(const AttnParams& p, cudaStream_t s) {
   a.W32 = (p.n_max + 31) / 32;
   a.splits = pl.splits;
   a.n_pairs = pl.n_pairs;
+  a.lpt = pl.lpt;
+  a.nch_h = pl.nch;
+  a.rs = pl.rs;
   a.ctx = p.ctx;
   a.n_verify = p.n_verify;
   a.mask = p.mask;
   a.scale_log2 = p.scale * 1.4426950408889634f;
   a.out = static_cast<__nv_bfloat16*>(p.out);
+  uint8_t* ws = static_cast<uint8_t*>(p.ws);
+  a.part_o = pl.splits > 1 ? ws + wl.part_o : nullptr;
+  a.part_l = pl.splits > 1 ? reinterpret_cast<float*>(ws + wl.part_l) : nullptr;
+  a.sync = pl.splits > 1 ? reinterpret_cast<uint32_t*>(ws + wl.sync) : nullptr;
   a.err = p.err;
 
   CUtensorMap tq, tk, tv;
@@ -672,24 +861,22 @@ cudaError_t launch_attn_tc(const AttnParams& p, cudaStream_t s) {
   cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(kSmemBytes));
   if (e != cudaSuccess) return e;
-  e = cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-  if (e != cudaSuccess) return e;
 
-  const int splits =
-      fit_splits(pl.splits, static_cast<int64_t>(p.batch) * p.hkv * pl.n_pairs);
-  a.splits = splits;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(splits, pl.n_pairs, p.batch * p.hkv);
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = kSmemBytes;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = splits;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  if (pl.splits > 1) {
+    // all splits of a unit wait for one another: they must be resident together
+    cfg.gridDim = dim3(pl.splits, pl.n_pairs, p.batch * p.hkv);
+    attr[0].id = cudaLaunchAttributeCooperative;
+    attr[0].val.cooperative = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+  } else {
+    cfg.gridDim = dim3(pl.units);
+  }
   return cudaLaunchKernelEx(&cfg, attn_tc_kernel, tq, tk, tv, a);
 }
 

@@ -186,8 +186,9 @@ def test_compaction_race_pattern_and_untouched_rows():
 
 
 # ---------------------------------------------------------------------- attention
-def _attention_case(name, seed, heads=None, seqs=None):
-    cfg = wl.config(name)
+def _attention_case(name, seed, heads=None, seqs=None, poison=False, workspace=None,
+                    bad_seq=None, **overrides):
+    cfg = wl.config(name, **overrides)
     ci = wl.draw_cycle(cfg, seed, draft_rows=False)
     rng = np.random.default_rng(seed + 5)
     masks = []
@@ -209,9 +210,24 @@ def _attention_case(name, seed, heads=None, seqs=None):
         w = oracle.mask_words(masks[b])
         mw[b, :w.shape[0], :w.shape[1]] = w
     qd, kd, vd = H.dev(q, cfg.dtype), H.dev(k, cfg.dtype), H.dev(v, cfg.dtype)
-    out = ltd.ltd_tree_attention(qd, kd, vd, H.i32(ci.ctx), cfg.max_ctx, H.i32(ci.n_verify),
-                                 torch.from_numpy(mw.view(np.int32)).cuda())
-    assert ltd.ltd_check() == 0
+    if poison:
+        # the API reads no q row past N_b and no cache row past ctx_b + N_b
+        for b in range(cfg.batch):
+            N, c = int(ci.n_verify[b]), int(ci.ctx[b])
+            qd[b, N:] = float("nan")
+            kd[b, :, c + N:] = float("nan")
+            vd[b, :, c + N:] = float("nan")
+    ctx_arg = ci.ctx.copy()
+    if bad_seq is not None:
+        ctx_arg[bad_seq] = cfg.max_ctx + 1  # out of range: flagged, the sequence skipped
+    out = ltd.ltd_tree_attention(qd, kd, vd, H.i32(ctx_arg), cfg.max_ctx, H.i32(ci.n_verify),
+                                 torch.from_numpy(mw.view(np.int32)).cuda(), workspace=workspace)
+    if bad_seq is None:
+        assert ltd.ltd_check() == 0
+    else:
+        assert ltd.ltd_check(raise_on_error=False) == 0x4
+        assert not out[bad_seq].float().abs().sum().item()
+        seqs = [b for b in (seqs if seqs is not None else range(cfg.batch)) if b != bad_seq]
     got = out.float().cpu().numpy()
     G = cfg.hq // cfg.hkv
     scale = 1.0 / math.sqrt(cfg.head_dim)
@@ -250,6 +266,38 @@ def test_attention_32b_sampled_heads():
 
 def test_attention_70b_sampled():
     _attention_case("70b", 0, heads=[3], seqs=[0, 5, 11, 15])
+
+
+def test_attention_ignores_rows_past_the_tree():
+    """NaN in q rows past N_b and in cache rows past ctx_b + N_b (a ctx that
+    ends mid-chunk) must not reach the output."""
+    _attention_case("8b", 4, poison=True, ctx_range=(1000, 1000), n_choices=(37,))
+    _attention_case("13b", 5, poison=True, ctx_range=(333, 333), n_choices=(48,))
+
+
+def test_attention_ragged_split_batch():
+    """Few units, so every unit's keys are split; short sequences leave some
+    splits without keys."""
+    _attention_case("8b", 6, batch=3, ctx_range=(20, 3000), n_choices=(7, 33, 60))
+
+
+def test_attention_flags_bad_sequence():
+    """A sequence with ctx past max_ctx is flagged and left untouched, in
+    both launch shapes (split keys; one split per unit, longest first), and
+    the other sequences are still right."""
+    _attention_case("8b", 10, bad_seq=1, batch=3, ctx_range=(500, 3000), n_choices=(20, 60))
+    _attention_case("70b", 11, bad_seq=4, heads=[0, 5], seqs=[0, 4, 9, 15])
+    assert ltd.ltd_check() == 0
+
+
+def test_attention_workspace_reuse():
+    """Back-to-back calls on one workspace: the split counters are left at
+    zero by each call, so every call combines correctly."""
+    cfg = wl.config("8b")
+    ws = ltd.attention_workspace(cfg.batch, cfg.hq, cfg.hkv, cfg.head_dim, cfg.max_n,
+                                 cfg.max_ctx, torch.bfloat16)
+    for seed in (7, 8, 9):
+        _attention_case("8b", seed, workspace=ws)
 
 
 def test_attention_all_ones_mask_equals_unmasked():

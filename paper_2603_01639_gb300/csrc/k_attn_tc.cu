@@ -11,13 +11,16 @@
 //               O_x += P_x V with P_x read from tensor memory; the order
 //               PV_a(j), S_a(j+1), PV_b(j), S_b(j+1) lets one tile's
 //               softmax run while the tensor core works on the other;
-//   warps 4-7   softmax of tile a, warps 8-11 of tile b, one thread per row
-//               (= tensor-memory lane): one 128-column load of S, the prefix
-//               + ancestor mask, a running max that rescales O only when it
-//               grows by more than 2^8, P written as bf16 over S's columns.
-//               The two tiles take turns chunk by chunk (a(j), b(j),
-//               a(j+1), ...), so one tile's softmax has the SM's exp and FMA
-//               pipes while the tensor core runs the other tile's MMAs.
+//   warps 2-9   softmax of tile a, warps 10-17 of tile b: two threads per
+//               row (= tensor-memory lane), one per 64-column half, each
+//               with one 64-column load of S, the prefix + ancestor mask and
+//               a partial row max; the halves swap maxima through shared
+//               memory at a named barrier, keep one running max that
+//               rescales O only when it grows by more than 2^8, and write P
+//               as bf16 over S's columns.  The two tiles take turns chunk
+//               by chunk (a(j), b(j), a(j+1), ...), so one tile's softmax has
+//               the SM's exp and FMA pipes while the tensor core runs the
+//               other tile's MMAs.
 // Tensor memory (512 columns): S_a | S_b | O_a | O_b.
 //
 // Two launch shapes:
@@ -48,7 +51,7 @@ constexpr int kBM = 128;  // rows per tile = TMEM lanes
 constexpr int kBN = 128;  // keys per chunk
 constexpr int kD = 128;
 constexpr int kRows = 2 * kBM;
-constexpr int kThreads = 384;
+constexpr int kThreads = 576;  // TMA warp, MMA warp, 16 softmax warps
 constexpr int kMaxW32 = LTD_MAX_N / 32;
 constexpr int kMaxSplits = 64;
 constexpr int kMaxGroups = 1024;  // (sequence, tile pair) groups ranked on the device
@@ -60,7 +63,9 @@ constexpr uint32_t kOffV = kOffK + 2 * kTile;                  // two stages
 constexpr uint32_t kOffMask = kOffV + 2 * kTile;               // [256][8] words
 constexpr uint32_t kOffCost = kOffMask + kRows * kMaxW32 * 4;  // [kMaxGroups] int
 constexpr uint32_t kOffOrder = kOffCost + kMaxGroups * 4;      // [kMaxGroups] int
-constexpr uint32_t kOffBar = kOffOrder + kMaxGroups * 4;
+constexpr uint32_t kOffXred = kOffOrder + kMaxGroups * 4;      // [2 buf][2 tile][2 half][128] f32
+constexpr uint32_t kOffLred = kOffXred + 2 * 2 * 2 * kBM * 4;     // [2 tile][2 half][128] f32
+constexpr uint32_t kOffBar = kOffLred + 2 * 2 * kBM * 4;
 constexpr uint32_t kOffHolder = kOffBar + 24 * 8;
 constexpr uint32_t kSmemBytes = kOffHolder + 16 + 1024;  // + alignment slack
 constexpr uint32_t kTmemCols = 512;
@@ -162,11 +167,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::mbar_init(bar(KEMPTY + s), 1);
       tc::mbar_init(bar(VEMPTY + s), 1);
       tc::mbar_init(bar(SFULL + s), 1);
-      tc::mbar_init(bar(PFULL + s), 128);
+      tc::mbar_init(bar(PFULL + s), 256);
     }
     tc::mbar_init(bar(FIN), 1);
-    tc::mbar_init(bar(ADONE), 128);
-    tc::mbar_init(bar(BDONE), 128);
+    tc::mbar_init(bar(ADONE), 256);
+    tc::mbar_init(bar(BDONE), 256);
     tc::mbar_init(bar(CBAR), 1);
     tc::mbar_init_fence();
     TRACE(19);
@@ -217,8 +222,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     b = g / a.n_pairs;
     pair = g % a.n_pairs;
   }
-  TRACE_VAL(25, static_cast<unsigned long long>(b));
-  TRACE_VAL(26, static_cast<unsigned long long>(pair));
+  if (tid == 0) TRACE_VAL(25, static_cast<unsigned long long>(clock64()));
+  if (tid == 0) TRACE(26);
 
   // Keys are split by the host bound on the chunk count, so a split knows
   // its first chunks before reading ctx and N: the loads of Q and of the
@@ -290,18 +295,22 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int nch = (nk + kBN - 1) / kBN;
   const int nc = max(0, min(ce, nch) - cs);
   const int key_lo = cs * kBN, key_hi = min(ce * kBN, nk);
-  if (tid == 0) TRACE_VAL(24, static_cast<unsigned long long>(nc));
+
   if (tid == 0 && a.lpt) issue_first();
   if (warp == 1) {
     tc::tmem_alloc(tc::smem_u32(holder), kTmemCols);
     tc::tmem_relinquish();
   }
-  // softmax threads: tile x, TMEM lane rr % 128, row rr of the unit
-  const int rr = tid - 128;
-  const int x = rr >> 7;
+  // softmax threads (warps 2-17): tile x, column half h, TMEM lane lrow,
+  // row rr of the unit
+  const bool smx = warp >= 2;
+  const int sw = warp - 2;
+  const int x = sw >> 3, h = (sw >> 2) & 1;
+  const int lrow = 32 * (warp & 3) + lane;
+  const int rr = kBM * x + lrow;
   const int R = row0 + rr;
-  const bool row_ok = tid >= 128 && R < M;
-  if (tid >= 128) {
+  const bool row_ok = smx && R < M;
+  if (smx && h == 0) {
     const int slot = R / a.G;
     const bool in = slot < a.n_max;
     for (int w = 0; w < a.W32; ++w)
@@ -314,7 +323,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = holder[0];
   if (tid == 0) TRACE(1);
   bool ok = true;
-  const bool tile_active = tid >= 128 && (x == 0 || has_b) && nc > 0;
+  const bool tile_active = smx && (x == 0 || has_b) && nc > 0;
   float m = -CUDART_INF_F, l = 0.f;
 
   if (warp == 0) {
@@ -390,93 +399,101 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::mbar_wait(bar(FIN), 0);
       if (!ok) flag_error(a.err, LTD_DEVERR_TIMEOUT);
     }
-  } else if (warp >= 4 && tile_active) {
+  } else if (tile_active) {
     // ------------------------------------------------------------- softmax
     const uint32_t lane_off = (32u * (warp & 3)) << 16;
     const uint32_t t_s = tmem + x * kBN + lane_off;
     const uint32_t t_o = tmem + 2 * kBN + x * kD + lane_off;
     const uint32_t* mbits = mask_s + rr * kMaxW32;
+    float* xred = reinterpret_cast<float*>(gbase + kOffXred);
     const int vis_all_below = min(ctx, key_hi);  // keys below this are all visible
     const float sl2 = a.scale_log2;
     const int w32 = a.W32;
-    const bool tr = (tid & 127) == 0;
+    const bool tr = (sw & 7) == 0 && lane == 0;
     for (int j = 0; j < nc; ++j) {
+      bool w_ok = true;
       if (has_b && (x == 1 || j > 0)) {
         // tile a waits for b's previous chunk, tile b for a's current one;
         // strict alternation keeps each barrier at most one phase ahead
-        const bool turn = x == 0 ? tc::mbar_wait(bar(BDONE), (j - 1) & 1)
-                                 : tc::mbar_wait(bar(ADONE), j & 1);
-        ok = __all_sync(0xFFFFFFFFu, turn);
-        if (!ok) break;
+        w_ok = x == 0 ? tc::mbar_wait(bar(BDONE), (j - 1) & 1) : tc::mbar_wait(bar(ADONE), j & 1);
       }
-      ok = tc::mbar_wait(bar(SFULL + x), j & 1);
-      ok = __all_sync(0xFFFFFFFFu, ok);
+      w_ok = tc::mbar_wait(bar(SFULL + x), j & 1) && w_ok;
       if (tr && j < 2) TRACE(4 + 4 * x + 2 * j);
-      if (!ok) break;
       tc::fence_after_sync();
-      const int kbase = key_lo + j * kBN;
-      const bool all_vis = row_ok && kbase + kBN <= vis_all_below;
-      tc::Frag128 f;
-      tc::tmem_ld128(t_s, f);
-      uint32_t vq[4] = {0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu};
+      const int kbase = key_lo + j * kBN + 64 * h;  // this half's first key
+      const bool all_vis = row_ok && kbase + 64 <= vis_all_below;
+      tc::Frag64 f;
+      tc::tmem_ld64(t_s + 64 * h, f);
+      uint32_t vq[2] = {0xFFFFFFFFu, 0xFFFFFFFFu};
       if (!all_vis) {
 #pragma unroll
-        for (int q = 0; q < 4; ++q)
+        for (int q = 0; q < 2; ++q)
           vq[q] = row_ok ? visible32(kbase + 32 * q, ctx, key_hi, w32, mbits) : 0u;
       }
-      tc::tmem_wait_ld128(f);
+      tc::tmem_wait_ld64(f);
+      if (tr && j == 0 && x == 0) TRACE(27);
       if (!all_vis) {
 #pragma unroll
-        for (int c = 0; c < 128; ++c)
+        for (int c = 0; c < 64; ++c)
           f.r[c] = ((vq[c >> 5] >> (c & 31)) & 1u) ? f.r[c] : 0xFF800000u;  // -inf if hidden
       }
-      // the chunk's row max on the raw scores (the scale is positive)
+      // this half's row max on the raw scores (the scale is positive)
       float r8[8];
 #pragma unroll
       for (int u = 0; u < 8; ++u) r8[u] = __uint_as_float(f.r[u]);
 #pragma unroll
-      for (int c = 8; c < 128; c += 16) {
+      for (int c = 8; c < 64; c += 16) {
 #pragma unroll
         for (int u = 0; u < 8; ++u)
           r8[u] = tc::fmax3(r8[u], __uint_as_float(f.r[c + 2 * u]), __uint_as_float(f.r[c + 2 * u + 1]));
       }
-      const float raw_max = fmaxf(tc::fmax3(r8[0], r8[1], r8[2]),
-                                  fmaxf(tc::fmax3(r8[3], r8[4], r8[5]), fmaxf(r8[6], r8[7])));
-      const float cmax = raw_max * sl2;
+      const float pmax = fmaxf(tc::fmax3(r8[0], r8[1], r8[2]),
+                               fmaxf(tc::fmax3(r8[3], r8[4], r8[5]), fmaxf(r8[6], r8[7])));
+      float* xr = xred + ((j & 1) * 2 + x) * (2 * kBM);
+      xr[h * kBM + lrow] = pmax;
+      // both halves of the tile meet here: the partner's max is readable, both
+      // have read S (so P may overwrite it), and the waits' outcome is shared
+      ok = tc::bar_red_and(1 + x, 2 * kBM, w_ok);
+      if (tr && j == 0 && x == 0) TRACE(28);
+      if (!ok) break;
+      const float cmax = fmaxf(pmax, xr[(1 - h) * kBM + lrow]) * sl2;
       // S(j) complete implies P_x(j-1) V finished, so O_x is stable here
       float mnew = m;
       if (cmax > m + kRescaleThreshold || (m == -CUDART_INF_F && cmax > -CUDART_INF_F)) mnew = cmax;
       const bool need = (mnew != m) && (m != -CUDART_INF_F) && (j >= 1);
       const float alpha = need ? tc::ex2(m - mnew) : 1.f;
       m = mnew;
-      // P = 2^(score - m) as bf16 pairs over S's first 64 columns
+      // P = 2^(score - m) as bf16 pairs: this half's 64 keys are P columns
+      // 32 h .. 32 h + 31
       const float mz = (m == -CUDART_INF_F) ? 0.f : m;  // m = -inf only if all are hidden
       const float2 sl22 = make_float2(sl2, sl2), nm2 = make_float2(-mz, -mz);
       float2 ls2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
-      tc::Frag64 pf;
+      tc::Frag32 pf;
 #pragma unroll
-      for (int c = 0; c < 64; ++c) {
+      for (int c = 0; c < 32; ++c) {
         const float2 t = __ffma2_rn(
             make_float2(__uint_as_float(f.r[2 * c]), __uint_as_float(f.r[2 * c + 1])), sl22, nm2);
         const float2 pp = make_float2(tc::ex2(t.x), tc::ex2(t.y));
         ls2[c & 1] = __fadd2_rn(ls2[c & 1], pp);
         pf.r[c] = pack_bf16(pp.x, pp.y);
       }
-      tc::tmem_st64(t_s, pf);
+      tc::tmem_st32(t_s + 32 * h, pf);
+      if (tr && j == 0 && x == 0) TRACE(29);
       if (__any_sync(0xFFFFFFFFu, need)) {
 #pragma unroll 1
-        for (int q = 0; q < 4; ++q) {
+        for (int q = 0; q < 2; ++q) {
           tc::Frag32 o;
-          tc::tmem_ld32(t_o + 32 * q, o);
+          tc::tmem_ld32(t_o + 64 * h + 32 * q, o);
           tc::tmem_wait_ld(o);
 #pragma unroll
           for (int c = 0; c < 32; ++c) o.r[c] = __float_as_uint(__uint_as_float(o.r[c]) * alpha);
-          tc::tmem_st32(t_o + 32 * q, o);
+          tc::tmem_st32(t_o + 64 * h + 32 * q, o);
         }
       }
       const float2 lsum = __fadd2_rn(ls2[0], ls2[1]);
       l = l * alpha + (lsum.x + lsum.y);
-      if (x == 0 && kbase + kBN > key_hi) {
+      const int kchunk = key_lo + j * kBN;
+      if (x == 0 && kchunk + kBN > key_hi) {
         // Keys from key_hi on may hold anything in the cache, even NaN: P is
         // 0 there, but 0 * NaN is not, so tile a's threads clear those V rows
         // (both 64-dim halves) before either tile's PV reads this stage.
@@ -484,24 +501,22 @@ __global__ void __launch_bounds__(kThreads, 1)
         // (a failed wait is flagged; the MMA thread times out on the same stage)
         if (!__all_sync(0xFFFFFFFFu, tc::mbar_wait(bar(VFULL + st), (j >> 1) & 1)) && lane == 0)
           flag_error(a.err, LTD_DEVERR_TIMEOUT);
-        const int z0 = key_hi - kbase;  // 1 .. 127
+        const int z0 = key_hi - kchunk;  // 1 .. 127
         uint4* vs = reinterpret_cast<uint4*>(gbase + kOffV + st * kTile);
-        for (int idx = rr; idx < (kBN - z0) * 16; idx += kBM) {
+        for (int idx = h * kBM + lrow; idx < (kBN - z0) * 16; idx += 2 * kBM) {
           const int row = z0 + (idx >> 4), piece = idx & 15;
           vs[((piece >> 3) * kHalf + row * 128) / 16 + (piece & 7)] = make_uint4(0u, 0u, 0u, 0u);
         }
         tc::fence_smem_async();
       }
       tc::tmem_wait_st();
+      if (tr && j == 0 && x == 0) TRACE(30);
       tc::fence_before_sync();
       tc::mbar_arrive(bar(PFULL + x));
       if (has_b && (x == 0 || j + 1 < nc)) tc::mbar_arrive(bar(x == 0 ? ADONE : BDONE));
       if (tr && j < 2) TRACE(5 + 4 * x + 2 * j);
     }
-    if (ok) {
-      ok = tc::mbar_wait(bar(FIN), 0);
-      ok = __all_sync(0xFFFFFFFFu, ok);
-    }
+    if (ok) ok = tc::mbar_wait(bar(FIN), 0);
     if (tr) TRACE(12 + x);
     if (!ok && lane == 0) flag_error(a.err, LTD_DEVERR_TIMEOUT);
   }
@@ -517,31 +532,37 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int Mv = min(kRows, M - row0);
   uint8_t* stg = gbase + kOffQ;
   float* stg_l = reinterpret_cast<float*>(gbase + kOffMask);
-  // tcgen05.ld is warp-collective: the O load is taken by whole warps
-  // (tile_active and ok are uniform within a warp), the writes per row.
-  const bool loaded = tile_active && ok;
-  tc::Frag128 o;
+  float* lred = reinterpret_cast<float*>(gbase + kOffLred);
+  if (tile_active) lred[(2 * x + h) * kBM + lrow] = l;
+  // CTA-uniform (a barrier): every active thread finished without a timeout;
+  // tcgen05.ld is warp-collective, so the O load goes by this and by the
+  // tile, never by row
+  const bool all_ok = __syncthreads_and(!tile_active || ok) != 0;
+  const bool loaded = tile_active && all_ok;
+  tc::Frag64 o;
   if (loaded) {
     tc::fence_after_sync();
-    tc::tmem_ld128(tmem + 2 * kBN + x * kD + ((32u * (warp & 3)) << 16), o);
-    tc::tmem_wait_ld128(o);
+    tc::tmem_ld64(tmem + 2 * kBN + x * kD + 64 * h + ((32u * (warp & 3)) << 16), o);
+    tc::tmem_wait_ld64(o);
   }
   if (row_ok) {
-    const bool have = loaded && l > 0.f;
-    const float inv = have ? 1.f / l : 0.f;
+    const float lt = loaded ? lred[(2 * x) * kBM + lrow] + lred[(2 * x + 1) * kBM + lrow] : 0.f;
+    const bool have = loaded && lt > 0.f;
+    const float inv = have ? 1.f / lt : 0.f;
     uint8_t* srow = stg + rr * kRowBytes;
 #pragma unroll
-    for (int c = 0; c < 16; ++c) {
+    for (int cc = 0; cc < 8; ++cc) {
+      const int c = 8 * h + cc;  // 16-byte chunk (8 values) of the row
       uint4 w = make_uint4(0u, 0u, 0u, 0u);
       if (have) {
-        w.x = pack_bf16(__uint_as_float(o.r[8 * c]) * inv, __uint_as_float(o.r[8 * c + 1]) * inv);
-        w.y = pack_bf16(__uint_as_float(o.r[8 * c + 2]) * inv, __uint_as_float(o.r[8 * c + 3]) * inv);
-        w.z = pack_bf16(__uint_as_float(o.r[8 * c + 4]) * inv, __uint_as_float(o.r[8 * c + 5]) * inv);
-        w.w = pack_bf16(__uint_as_float(o.r[8 * c + 6]) * inv, __uint_as_float(o.r[8 * c + 7]) * inv);
+        w.x = pack_bf16(__uint_as_float(o.r[8 * cc]) * inv, __uint_as_float(o.r[8 * cc + 1]) * inv);
+        w.y = pack_bf16(__uint_as_float(o.r[8 * cc + 2]) * inv, __uint_as_float(o.r[8 * cc + 3]) * inv);
+        w.z = pack_bf16(__uint_as_float(o.r[8 * cc + 4]) * inv, __uint_as_float(o.r[8 * cc + 5]) * inv);
+        w.w = pack_bf16(__uint_as_float(o.r[8 * cc + 6]) * inv, __uint_as_float(o.r[8 * cc + 7]) * inv);
       }
       *reinterpret_cast<uint4*>(srow + ((c ^ (rr & 15)) << 4)) = w;
     }
-    stg_l[rr] = have ? m + __log2f(l) : -CUDART_INF_F;
+    if (h == 0) stg_l[rr] = have ? m + __log2f(lt) : -CUDART_INF_F;
   }
   tc::fence_smem_async();  // the staging is read by bulk copies
   tc::fence_before_sync();
@@ -652,27 +673,37 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int o = 8; o > 0; o >>= 1) L += __shfl_xor_sync(0xFFFFFFFFu, L, o);
         const float inv = L > 0.f ? 1.f / L : 0.f;
+        if (tid == 0) TRACE(22);
         float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
         const int half = lane & 16;
+        // four splits per step: their weights (shuffles) and rows (shared
+        // loads) are fetched together before the FMAs use them
+        for (int p0 = 0; p0 < S; p0 += 4) {  // S is uniform
+          float w4[4];
+          uint4 v4[4];
 #pragma unroll
-        for (int k = 0; k < kMaxSplits / 16; ++k) {
-          if (16 * k >= S) break;  // uniform
-#pragma unroll 4
-          for (int q = 0; q < 16; ++q) {
-            const int p = 16 * k + q;
-            const float w = __shfl_sync(0xFFFFFFFFu, lpk[k], half | q);
-            if (p < S) {
-              const uint4 v =
-                  *reinterpret_cast<const uint4*>(cin + (p * Rs + r) * kRowBytes + c * 16);
-              const uint32_t e[4] = {v.x, v.y, v.z, v.w};
+          for (int u = 0; u < 4; ++u) {
+            const int p = p0 + u;
+            const int k = p >> 4;
+            // lpk[k] with k < kMaxSplits / 16 picked without dynamic indexing
+            const float src = k == 0 ? lpk[0] : (k == 1 ? lpk[1] : (k == 2 ? lpk[2] : lpk[3]));
+            w4[u] = __shfl_sync(0xFFFFFFFFu, src, half | (p & 15));
+            const int pc = p < S ? p : S - 1;  // in range; its weight is dropped below
+            v4[u] = *reinterpret_cast<const uint4*>(cin + (pc * Rs + r) * kRowBytes + c * 16);
+            if (p >= S) w4[u] = 0.f;
+          }
 #pragma unroll
-              for (int t = 0; t < 4; ++t) {
-                acc[2 * t] = fmaf(w, __uint_as_float(e[t] << 16), acc[2 * t]);
-                acc[2 * t + 1] = fmaf(w, __uint_as_float(e[t] & 0xFFFF0000u), acc[2 * t + 1]);
-              }
+          for (int u = 0; u < 4; ++u) {
+            const uint32_t e[4] = {v4[u].x, v4[u].y, v4[u].z, v4[u].w};
+#pragma unroll
+            for (int t = 0; t < 4; ++t) {
+              acc[2 * t] = fmaf(w4[u], __uint_as_float(e[t] << 16), acc[2 * t]);
+              acc[2 * t + 1] = fmaf(w4[u], __uint_as_float(e[t] & 0xFFFF0000u), acc[2 * t + 1]);
             }
           }
         }
+        if (tid == 0) TRACE(31);
+        if (tid == 0) TRACE_VAL(24, static_cast<unsigned long long>(clock64()));
         if (live) {
           const int Rr = row0 + r_lo + r;
           const int slot = Rr / a.G, g = Rr % a.G;

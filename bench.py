@@ -37,7 +37,7 @@ N_LAYERS = {"tiny": 1, "8b": 32, "13b": 40, "32b": 64, "70b": 80}
 def _args():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--config", default="8b", choices=list(N_LAYERS))
@@ -98,6 +98,80 @@ class ClockSampler:
         reasons = sorted({names[i] for r in rows for i in range(4) if r[4 + i].strip() == "Active"})
         return {"sm_mhz": statistics.median(sm) if sm else None,
                 "sm_max_mhz": max(mx) if mx else None, "reasons": reasons, "samples": len(rows)}
+
+
+class NvmlClockSampler:
+    """SM clock, power and clock-event reasons polled every millisecond by a
+    thread through the driver's NVML library (read-only queries), so that a
+    timed region of a few milliseconds still gets samples."""
+
+    REASONS = {0x8: "hw_slowdown", 0x40: "hw_thermal_slowdown", 0x20: "sw_thermal_slowdown",
+               0x4: "sw_power_cap", 0x80: "hw_power_brake_slowdown"}
+
+    def __init__(self, index: int):
+        import ctypes
+        import threading
+        self.ok = False
+        try:
+            self.lib = ctypes.CDLL("libnvidia-ml.so.1")
+        except OSError:
+            return
+        L = self.lib
+        if L.nvmlInit_v2() != 0:
+            return
+        count = ctypes.c_uint(0)
+        if L.nvmlDeviceGetCount_v2(ctypes.byref(count)) != 0 or count.value == 0:
+            return
+        self.h = ctypes.c_void_p()
+        idx = index if index < count.value else 0
+        if L.nvmlDeviceGetHandleByIndex_v2(idx, ctypes.byref(self.h)) != 0:
+            return
+        self.reasons_fn = getattr(L, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+            getattr(L, "nvmlDeviceGetCurrentClocksThrottleReasons", None)
+        mx = ctypes.c_uint(0)
+        self.max_mhz = float(mx.value) if L.nvmlDeviceGetMaxClockInfo(self.h, 1, ctypes.byref(mx)) == 0 \
+            else None
+        if self.max_mhz is not None:
+            self.max_mhz = float(mx.value)
+        self.samples = []
+        self.stop_flag = threading.Event()
+        self.ctypes = ctypes
+        self.thread = threading.Thread(target=self._run, daemon=True)
+        self.ok = True
+        self.thread.start()
+
+    def _run(self):
+        c = self.ctypes
+        mhz, bits, mw = c.c_uint(0), c.c_ulonglong(0), c.c_uint(0)
+        while not self.stop_flag.is_set():
+            if self.lib.nvmlDeviceGetClockInfo(self.h, 1, c.byref(mhz)) == 0:
+                r = self.reasons_fn(self.h, c.byref(bits)) if self.reasons_fn else 1
+                p = self.lib.nvmlDeviceGetPowerUsage(self.h, c.byref(mw))
+                self.samples.append((mhz.value, bits.value if r == 0 else 0, mw.value if p == 0 else 0))
+            time.sleep(0.001)
+
+    def stop(self):
+        if not self.ok:
+            return None
+        self.stop_flag.set()
+        self.thread.join(timeout=2)
+        try:
+            self.lib.nvmlShutdown()
+        except Exception:
+            pass
+        if not self.samples:
+            return None
+        reasons = sorted({name for _, b, _ in self.samples for bit, name in self.REASONS.items()
+                          if b & bit})
+        return {"sm_mhz": statistics.median(s[0] for s in self.samples), "sm_max_mhz": self.max_mhz,
+                "reasons": reasons, "samples": len(self.samples),
+                "power_w_max": round(max(s[2] for s in self.samples) / 1000.0, 1),
+                "source": "nvml, 1 ms"}
+
+
+def clock_sampler(index: int):
+    s = NvmlClockSampler(index)
+    return s if s.ok else ClockSampler(index)
 
 
 # ---------------------------------------------------------- the GPU cycle
@@ -378,7 +452,7 @@ def run_ours(args):
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize(device)
-    clocks = ClockSampler(local)
+    clocks = clock_sampler(local)
     stream = torch.cuda.current_stream()
     for i in range(K):
         ev[i][0].record(stream)

@@ -11,16 +11,14 @@
 //               O_x += P_x V with P_x read from tensor memory; the order
 //               PV_a(j), S_a(j+1), PV_b(j), S_b(j+1) lets one tile's
 //               softmax run while the tensor core works on the other;
-//   warps 2-9   softmax of tile a, warps 10-17 of tile b: two threads per
-//               row (= tensor-memory lane), one per 64-column half, each
-//               with one 64-column load of S, the prefix + ancestor mask and
-//               a partial row max; the halves swap maxima through shared
-//               memory at a named barrier, keep one running max that
-//               rescales O only when it grows by more than 2^8, and write P
-//               as bf16 over S's columns.  The two tiles take turns chunk
-//               by chunk (a(j), b(j), a(j+1), ...), so one tile's softmax has
-//               the SM's exp and FMA pipes while the tensor core runs the
-//               other tile's MMAs.
+//   warps 4-7   softmax of tile a, warps 8-11 of tile b, one thread per row
+//               (= tensor-memory lane) with the row's 128 scores in
+//               registers: the prefix + ancestor mask, then P = 2^(s - m)
+//               against the row's running max m, computed before the
+//               chunk's own max is known and redone only for a warp in which
+//               some row's max grew by more than 2^8 (S is still in tensor
+//               memory then); O is rescaled only in that case.  P is written
+//               as bf16 over S's columns.  Both tiles' softmaxes run at once.
 // Tensor memory (512 columns): S_a | S_b | O_a | O_b.
 //
 // Two launch shapes:
@@ -51,7 +49,7 @@ constexpr int kBM = 128;  // rows per tile = TMEM lanes
 constexpr int kBN = 128;  // keys per chunk
 constexpr int kD = 128;
 constexpr int kRows = 2 * kBM;
-constexpr int kThreads = 576;  // TMA warp, MMA warp, 16 softmax warps
+constexpr int kThreads = 384;  // TMA warp, MMA warp, 2 idle, 8 softmax warps
 constexpr int kMaxW32 = LTD_MAX_N / 32;
 constexpr int kMaxSplits = 64;
 constexpr int kMaxGroups = 1024;  // (sequence, tile pair) groups ranked on the device
@@ -63,19 +61,15 @@ constexpr uint32_t kOffV = kOffK + 2 * kTile;                  // two stages
 constexpr uint32_t kOffMask = kOffV + 2 * kTile;               // [256][8] words
 constexpr uint32_t kOffCost = kOffMask + kRows * kMaxW32 * 4;  // [kMaxGroups] int
 constexpr uint32_t kOffOrder = kOffCost + kMaxGroups * 4;      // [kMaxGroups] int
-constexpr uint32_t kOffXred = kOffOrder + kMaxGroups * 4;      // [2 buf][2 tile][2 half][128] f32
-constexpr uint32_t kOffLred = kOffXred + 2 * 2 * 2 * kBM * 4;     // [2 tile][2 half][128] f32
-constexpr uint32_t kOffBar = kOffLred + 2 * 2 * kBM * 4;
+constexpr uint32_t kOffBar = kOffOrder + kMaxGroups * 4;
 constexpr uint32_t kOffHolder = kOffBar + 24 * 8;
 constexpr uint32_t kSmemBytes = kOffHolder + 16 + 1024;  // + alignment slack
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kRowBytes = kD * 2;     // one bf16 output / partial row
-constexpr float kRescaleThreshold = 8.f;  // log2 units
+// P may grow to 2^8 before a row's running max is raised: bf16 bits of 2^8
+constexpr uint32_t kPMaxBits = 0x4380u;
 
-enum Bar {
-  QFULL = 0, KFULL = 1, VFULL = 3, KEMPTY = 5, VEMPTY = 7, SFULL = 9, PFULL = 11, FIN = 13,
-  ADONE = 14, BDONE = 15, CBAR = 16
-};
+enum Bar { QFULL = 0, KFULL = 1, VFULL = 3, KEMPTY = 5, VEMPTY = 7, SFULL = 9, PFULL = 11, FIN = 13, CBAR = 14 };
 
 // Optional phase timestamps for performance work (off in normal builds).
 #ifdef LTD_TRACE
@@ -167,11 +161,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::mbar_init(bar(KEMPTY + s), 1);
       tc::mbar_init(bar(VEMPTY + s), 1);
       tc::mbar_init(bar(SFULL + s), 1);
-      tc::mbar_init(bar(PFULL + s), 256);
+      tc::mbar_init(bar(PFULL + s), 128);
     }
     tc::mbar_init(bar(FIN), 1);
-    tc::mbar_init(bar(ADONE), 256);
-    tc::mbar_init(bar(BDONE), 256);
     tc::mbar_init(bar(CBAR), 1);
     tc::mbar_init_fence();
     TRACE(19);
@@ -301,16 +293,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc::tmem_alloc(tc::smem_u32(holder), kTmemCols);
     tc::tmem_relinquish();
   }
-  // softmax threads (warps 2-17): tile x, column half h, TMEM lane lrow,
-  // row rr of the unit
-  const bool smx = warp >= 2;
-  const int sw = warp - 2;
-  const int x = sw >> 3, h = (sw >> 2) & 1;
+  // softmax threads (warps 4-11): tile x, TMEM lane lrow, row rr of the unit
+  const bool smx = warp >= 4;
+  const int x = (warp - 4) >> 2;
   const int lrow = 32 * (warp & 3) + lane;
   const int rr = kBM * x + lrow;
   const int R = row0 + rr;
   const bool row_ok = smx && R < M;
-  if (smx && h == 0) {
+  if (smx) {
     const int slot = R / a.G;
     const bool in = slot < a.n_max;
     for (int w = 0; w < a.W32; ++w)
@@ -324,7 +314,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (tid == 0) TRACE(1);
   bool ok = true;
   const bool tile_active = smx && (x == 0 || has_b) && nc > 0;
-  float m = -CUDART_INF_F, l = 0.f;
+  float m = -CUDART_INF_F, l = 0.f;  // the row's running max (log2 units) and sum
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
@@ -405,95 +395,132 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t t_s = tmem + x * kBN + lane_off;
     const uint32_t t_o = tmem + 2 * kBN + x * kD + lane_off;
     const uint32_t* mbits = mask_s + rr * kMaxW32;
-    float* xred = reinterpret_cast<float*>(gbase + kOffXred);
     const int vis_all_below = min(ctx, key_hi);  // keys below this are all visible
     const float sl2 = a.scale_log2;
     const int w32 = a.W32;
-    const bool tr = (sw & 7) == 0 && lane == 0;
+    const bool tr = (tid & 127) == 0;
     for (int j = 0; j < nc; ++j) {
-      bool w_ok = true;
-      if (has_b && (x == 1 || j > 0)) {
-        // tile a waits for b's previous chunk, tile b for a's current one;
-        // strict alternation keeps each barrier at most one phase ahead
-        w_ok = x == 0 ? tc::mbar_wait(bar(BDONE), (j - 1) & 1) : tc::mbar_wait(bar(ADONE), j & 1);
-      }
-      w_ok = tc::mbar_wait(bar(SFULL + x), j & 1) && w_ok;
+      ok = tc::mbar_wait(bar(SFULL + x), j & 1);
+      ok = __all_sync(0xFFFFFFFFu, ok);
       if (tr && j < 2) TRACE(4 + 4 * x + 2 * j);
+      if (!ok) break;
       tc::fence_after_sync();
-      const int kbase = key_lo + j * kBN + 64 * h;  // this half's first key
-      const bool all_vis = row_ok && kbase + 64 <= vis_all_below;
-      tc::Frag64 f;
-      tc::tmem_ld64(t_s + 64 * h, f);
-      uint32_t vq[2] = {0xFFFFFFFFu, 0xFFFFFFFFu};
+      const int kbase = key_lo + j * kBN;
+      const bool all_vis = row_ok && kbase + kBN <= vis_all_below;
+      // P against the row's running max m (a row without one yet first takes
+      // this chunk's max); the chunk's own max is tracked on the way and, if
+      // it exceeds the reference by more than 2^8 in some row of the warp,
+      // the warp re-derives P from S, still intact in tensor memory, 32
+      // columns at a time.
+      tc::Frag128 f;
+      float mref = m;
+      float2 ls2 = make_float2(0.f, 0.f);
+      tc::tmem_ld128(t_s, f);
+      uint32_t vq[4] = {0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu};
       if (!all_vis) {
 #pragma unroll
-        for (int q = 0; q < 2; ++q)
-          vq[q] = row_ok ? visible32(kbase + 32 * q, ctx, key_hi, w32, mbits) : 0u;
+        for (int qq = 0; qq < 4; ++qq)
+          vq[qq] = row_ok ? visible32(kbase + 32 * qq, ctx, key_hi, w32, mbits) : 0u;
       }
-      tc::tmem_wait_ld64(f);
+      tc::tmem_wait_ld128(f);
       if (tr && j == 0 && x == 0) TRACE(27);
       if (!all_vis) {
 #pragma unroll
-        for (int c = 0; c < 64; ++c)
+        for (int c = 0; c < 128; ++c)
           f.r[c] = ((vq[c >> 5] >> (c & 31)) & 1u) ? f.r[c] : 0xFF800000u;  // -inf if hidden
       }
-      // this half's row max on the raw scores (the scale is positive)
-      float r8[8];
+      if (__any_sync(0xFFFFFFFFu, mref == -CUDART_INF_F)) {
+        float r8[8];
 #pragma unroll
-      for (int u = 0; u < 8; ++u) r8[u] = __uint_as_float(f.r[u]);
+        for (int u = 0; u < 8; ++u) r8[u] = __uint_as_float(f.r[u]);
 #pragma unroll
-      for (int c = 8; c < 64; c += 16) {
+        for (int c = 8; c < 128; c += 16) {
 #pragma unroll
-        for (int u = 0; u < 8; ++u)
-          r8[u] = tc::fmax3(r8[u], __uint_as_float(f.r[c + 2 * u]), __uint_as_float(f.r[c + 2 * u + 1]));
+          for (int u = 0; u < 8; ++u)
+            r8[u] = tc::fmax3(r8[u], __uint_as_float(f.r[c + 2 * u]), __uint_as_float(f.r[c + 2 * u + 1]));
+        }
+        const float cm = fmaxf(tc::fmax3(r8[0], r8[1], r8[2]),
+                               fmaxf(tc::fmax3(r8[3], r8[4], r8[5]), fmaxf(r8[6], r8[7]))) * sl2;
+        if (mref == -CUDART_INF_F) mref = cm;
       }
-      const float pmax = fmaxf(tc::fmax3(r8[0], r8[1], r8[2]),
-                               fmaxf(tc::fmax3(r8[3], r8[4], r8[5]), fmaxf(r8[6], r8[7])));
-      float* xr = xred + ((j & 1) * 2 + x) * (2 * kBM);
-      xr[h * kBM + lrow] = pmax;
-      // both halves of the tile meet here: the partner's max is readable, both
-      // have read S (so P may overwrite it), and the waits' outcome is shared
-      ok = tc::bar_red_and(1 + x, 2 * kBM, w_ok);
+      // bf16 of P >= 0 orders like an unsigned integer, so the largest P
+      // is the largest 16-bit half of the packed registers
+      uint32_t pmax2 = 0u;
+      {
+        const float mz = (mref == -CUDART_INF_F) ? 0.f : mref;  // -inf only if all are hidden
+        const float2 sl22 = make_float2(sl2, sl2), nm2 = make_float2(-mz, -mz);
+        // P packed in place: pair c is read from registers 2c, 2c+1 and
+        // written to register c (c <= 2c, so nothing unread is overwritten)
+#pragma unroll
+        for (int c = 0; c < 64; ++c) {
+          const float2 t = __ffma2_rn(
+              make_float2(__uint_as_float(f.r[2 * c]), __uint_as_float(f.r[2 * c + 1])), sl22, nm2);
+          const float2 pp = make_float2(tc::ex2(t.x), tc::ex2(t.y));
+          ls2 = __fadd2_rn(ls2, pp);
+          f.r[c] = pack_bf16(pp.x, pp.y);
+          pmax2 = __vmaxu2(pmax2, f.r[c]);
+        }
+      }
+      // P above 2^8 means the chunk max passed m + 8
+      const bool over = max(pmax2 & 0xFFFFu, pmax2 >> 16) > kPMaxBits;
+      if (!__any_sync(0xFFFFFFFFu, over)) {
+        tc::tmem_st64_lo(t_s, f);
+      } else {
+        // S is still intact in tensor memory: take the chunk's max, then
+        // derive P again, 32 columns at a time (P columns 16 qq .. 16 qq + 15
+        // overlie S columns already read)
+        float cm = -CUDART_INF_F;
+#pragma unroll 1
+        for (int qq = 0; qq < 4; ++qq) {
+          tc::Frag32 g;
+          tc::tmem_ld32(t_s + 32 * qq, g);
+          tc::tmem_wait_ld(g);
+          const uint32_t v = qq == 0 ? vq[0] : (qq == 1 ? vq[1] : (qq == 2 ? vq[2] : vq[3]));
+#pragma unroll
+          for (int c = 0; c < 32; ++c)
+            if ((v >> c) & 1u) cm = fmaxf(cm, __uint_as_float(g.r[c]));
+        }
+        if (over) mref = cm * sl2;
+        const float mz = (mref == -CUDART_INF_F) ? 0.f : mref;
+        const float2 sl22 = make_float2(sl2, sl2), nm2 = make_float2(-mz, -mz);
+        ls2 = make_float2(0.f, 0.f);
+#pragma unroll 1
+        for (int qq = 0; qq < 4; ++qq) {
+          tc::Frag32 g;
+          tc::tmem_ld32(t_s + 32 * qq, g);
+          tc::tmem_wait_ld(g);
+          const uint32_t v = qq == 0 ? vq[0] : (qq == 1 ? vq[1] : (qq == 2 ? vq[2] : vq[3]));
+          tc::Frag16 pf;
+#pragma unroll
+          for (int c = 0; c < 16; ++c) {
+            const float s0 = ((v >> (2 * c)) & 1u) ? __uint_as_float(g.r[2 * c]) : -CUDART_INF_F;
+            const float s1 = ((v >> (2 * c + 1)) & 1u) ? __uint_as_float(g.r[2 * c + 1]) : -CUDART_INF_F;
+            const float2 t = __ffma2_rn(make_float2(s0, s1), sl22, nm2);
+            const float2 pp = make_float2(tc::ex2(t.x), tc::ex2(t.y));
+            ls2 = __fadd2_rn(ls2, pp);
+            pf.r[c] = pack_bf16(pp.x, pp.y);
+          }
+          tc::tmem_st16(t_s + 16 * qq, pf);
+        }
+      }
       if (tr && j == 0 && x == 0) TRACE(28);
-      if (!ok) break;
-      const float cmax = fmaxf(pmax, xr[(1 - h) * kBM + lrow]) * sl2;
       // S(j) complete implies P_x(j-1) V finished, so O_x is stable here
-      float mnew = m;
-      if (cmax > m + kRescaleThreshold || (m == -CUDART_INF_F && cmax > -CUDART_INF_F)) mnew = cmax;
-      const bool need = (mnew != m) && (m != -CUDART_INF_F) && (j >= 1);
-      const float alpha = need ? tc::ex2(m - mnew) : 1.f;
-      m = mnew;
-      // P = 2^(score - m) as bf16 pairs: this half's 64 keys are P columns
-      // 32 h .. 32 h + 31
-      const float mz = (m == -CUDART_INF_F) ? 0.f : m;  // m = -inf only if all are hidden
-      const float2 sl22 = make_float2(sl2, sl2), nm2 = make_float2(-mz, -mz);
-      float2 ls2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
-      tc::Frag32 pf;
-#pragma unroll
-      for (int c = 0; c < 32; ++c) {
-        const float2 t = __ffma2_rn(
-            make_float2(__uint_as_float(f.r[2 * c]), __uint_as_float(f.r[2 * c + 1])), sl22, nm2);
-        const float2 pp = make_float2(tc::ex2(t.x), tc::ex2(t.y));
-        ls2[c & 1] = __fadd2_rn(ls2[c & 1], pp);
-        pf.r[c] = pack_bf16(pp.x, pp.y);
-      }
-      tc::tmem_st32(t_s + 32 * h, pf);
-      if (tr && j == 0 && x == 0) TRACE(29);
+      const bool need = (mref != m) && (m != -CUDART_INF_F);
+      const float alpha = need ? tc::ex2(m - mref) : 1.f;
       if (__any_sync(0xFFFFFFFFu, need)) {
 #pragma unroll 1
-        for (int q = 0; q < 2; ++q) {
+        for (int qq = 0; qq < 4; ++qq) {
           tc::Frag32 o;
-          tc::tmem_ld32(t_o + 64 * h + 32 * q, o);
+          tc::tmem_ld32(t_o + 32 * qq, o);
           tc::tmem_wait_ld(o);
 #pragma unroll
           for (int c = 0; c < 32; ++c) o.r[c] = __float_as_uint(__uint_as_float(o.r[c]) * alpha);
-          tc::tmem_st32(t_o + 64 * h + 32 * q, o);
+          tc::tmem_st32(t_o + 32 * qq, o);
         }
       }
-      const float2 lsum = __fadd2_rn(ls2[0], ls2[1]);
-      l = l * alpha + (lsum.x + lsum.y);
-      const int kchunk = key_lo + j * kBN;
-      if (x == 0 && kchunk + kBN > key_hi) {
+      m = mref;
+      l = l * alpha + (ls2.x + ls2.y);
+      if (x == 0 && kbase + kBN > key_hi) {
         // Keys from key_hi on may hold anything in the cache, even NaN: P is
         // 0 there, but 0 * NaN is not, so tile a's threads clear those V rows
         // (both 64-dim halves) before either tile's PV reads this stage.
@@ -501,9 +528,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         // (a failed wait is flagged; the MMA thread times out on the same stage)
         if (!__all_sync(0xFFFFFFFFu, tc::mbar_wait(bar(VFULL + st), (j >> 1) & 1)) && lane == 0)
           flag_error(a.err, LTD_DEVERR_TIMEOUT);
-        const int z0 = key_hi - kchunk;  // 1 .. 127
+        const int z0 = key_hi - kbase;  // 1 .. 127
         uint4* vs = reinterpret_cast<uint4*>(gbase + kOffV + st * kTile);
-        for (int idx = h * kBM + lrow; idx < (kBN - z0) * 16; idx += 2 * kBM) {
+        for (int idx = lrow; idx < (kBN - z0) * 16; idx += kBM) {
           const int row = z0 + (idx >> 4), piece = idx & 15;
           vs[((piece >> 3) * kHalf + row * 128) / 16 + (piece & 7)] = make_uint4(0u, 0u, 0u, 0u);
         }
@@ -513,10 +540,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (tr && j == 0 && x == 0) TRACE(30);
       tc::fence_before_sync();
       tc::mbar_arrive(bar(PFULL + x));
-      if (has_b && (x == 0 || j + 1 < nc)) tc::mbar_arrive(bar(x == 0 ? ADONE : BDONE));
       if (tr && j < 2) TRACE(5 + 4 * x + 2 * j);
     }
-    if (ok) ok = tc::mbar_wait(bar(FIN), 0);
+    if (ok) {
+      ok = tc::mbar_wait(bar(FIN), 0);
+      ok = __all_sync(0xFFFFFFFFu, ok);
+    }
     if (tr) TRACE(12 + x);
     if (!ok && lane == 0) flag_error(a.err, LTD_DEVERR_TIMEOUT);
   }
@@ -532,37 +561,31 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int Mv = min(kRows, M - row0);
   uint8_t* stg = gbase + kOffQ;
   float* stg_l = reinterpret_cast<float*>(gbase + kOffMask);
-  float* lred = reinterpret_cast<float*>(gbase + kOffLred);
-  if (tile_active) lred[(2 * x + h) * kBM + lrow] = l;
-  // CTA-uniform (a barrier): every active thread finished without a timeout;
-  // tcgen05.ld is warp-collective, so the O load goes by this and by the
-  // tile, never by row
-  const bool all_ok = __syncthreads_and(!tile_active || ok) != 0;
-  const bool loaded = tile_active && all_ok;
-  tc::Frag64 o;
+  // tcgen05.ld is warp-collective: the O load is taken by whole warps
+  // (tile_active and ok are uniform within a warp), the writes per row.
+  const bool loaded = tile_active && ok;
+  tc::Frag128 o;
   if (loaded) {
     tc::fence_after_sync();
-    tc::tmem_ld64(tmem + 2 * kBN + x * kD + 64 * h + ((32u * (warp & 3)) << 16), o);
-    tc::tmem_wait_ld64(o);
+    tc::tmem_ld128(tmem + 2 * kBN + x * kD + ((32u * (warp & 3)) << 16), o);
+    tc::tmem_wait_ld128(o);
   }
   if (row_ok) {
-    const float lt = loaded ? lred[(2 * x) * kBM + lrow] + lred[(2 * x + 1) * kBM + lrow] : 0.f;
-    const bool have = loaded && lt > 0.f;
-    const float inv = have ? 1.f / lt : 0.f;
+    const bool have = loaded && l > 0.f;
+    const float inv = have ? 1.f / l : 0.f;
     uint8_t* srow = stg + rr * kRowBytes;
 #pragma unroll
-    for (int cc = 0; cc < 8; ++cc) {
-      const int c = 8 * h + cc;  // 16-byte chunk (8 values) of the row
+    for (int c = 0; c < 16; ++c) {
       uint4 w = make_uint4(0u, 0u, 0u, 0u);
       if (have) {
-        w.x = pack_bf16(__uint_as_float(o.r[8 * cc]) * inv, __uint_as_float(o.r[8 * cc + 1]) * inv);
-        w.y = pack_bf16(__uint_as_float(o.r[8 * cc + 2]) * inv, __uint_as_float(o.r[8 * cc + 3]) * inv);
-        w.z = pack_bf16(__uint_as_float(o.r[8 * cc + 4]) * inv, __uint_as_float(o.r[8 * cc + 5]) * inv);
-        w.w = pack_bf16(__uint_as_float(o.r[8 * cc + 6]) * inv, __uint_as_float(o.r[8 * cc + 7]) * inv);
+        w.x = pack_bf16(__uint_as_float(o.r[8 * c]) * inv, __uint_as_float(o.r[8 * c + 1]) * inv);
+        w.y = pack_bf16(__uint_as_float(o.r[8 * c + 2]) * inv, __uint_as_float(o.r[8 * c + 3]) * inv);
+        w.z = pack_bf16(__uint_as_float(o.r[8 * c + 4]) * inv, __uint_as_float(o.r[8 * c + 5]) * inv);
+        w.w = pack_bf16(__uint_as_float(o.r[8 * c + 6]) * inv, __uint_as_float(o.r[8 * c + 7]) * inv);
       }
       *reinterpret_cast<uint4*>(srow + ((c ^ (rr & 15)) << 4)) = w;
     }
-    if (h == 0) stg_l[rr] = have ? m + __log2f(lt) : -CUDART_INF_F;
+    stg_l[rr] = have ? m + __log2f(l) : -CUDART_INF_F;
   }
   tc::fence_smem_async();  // the staging is read by bulk copies
   tc::fence_before_sync();

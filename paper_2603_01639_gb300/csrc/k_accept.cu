@@ -37,6 +37,8 @@ __global__ void __launch_bounds__(kNT) accept_rows_kernel(const AcceptParams p) 
   constexpr int U = 2;
   __shared__ float red[2 * kNW];
   __shared__ uint64_t redk[kNW];
+  grid_wait();
+  trigger_dependents();
 
   const int ch = blockIdx.x, i = blockIdx.y, b = blockIdx.z, tid = threadIdx.x;
   const int N = p.n_verify[b];
@@ -143,6 +145,8 @@ __global__ void __launch_bounds__(kNT) accept_walk_kernel(const AcceptParams p, 
                                                           int64_t slice) {
   extern __shared__ float dyn[];
   __shared__ WalkShared sh;
+  grid_wait();
+  trigger_dependents();
   float* ps = dyn;
   float* qs = dyn + slice;
   const int rank = blockIdx.x, b = blockIdx.y, tid = threadIdx.x;
@@ -313,6 +317,8 @@ constexpr int kCompactMaxRowBytes = 512;
 
 __global__ void __launch_bounds__(kCompactNT) kv_compact_kernel(const CompactParams p) {
   __shared__ uint4 buf[(LTD_MAX_DEPTH + 1) * kCompactMaxRowBytes / 16];
+  grid_wait();
+  trigger_dependents();
   const int h = blockIdx.x, layer = blockIdx.y >> 1, which = blockIdx.y & 1, b = blockIdx.z;
   const int a = p.accept_len[b];
   if (a < 0) return;
@@ -354,8 +360,8 @@ size_t accept_workspace(int32_t batch, int32_t n_max, int64_t vocab) {
 
 template <typename T>
 cudaError_t launch_accept_t(const AcceptParams& p, int32_t batch, cudaStream_t s) {
-  accept_rows_kernel<T><<<dim3(p.chunks, p.n_max, batch), kNT, 0, s>>>(p);
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e = launch(accept_rows_kernel<T>, dim3(p.chunks, p.n_max, batch), dim3(kNT), 0, s,
+                         nullptr, 0, p);
   if (e != cudaSuccess) return e;
   // walk cluster: enough CTAs that a vocabulary slice of p and q fits shared memory
   int C = static_cast<int>((p.vocab + 4095) / 4096);
@@ -371,19 +377,12 @@ cudaError_t launch_accept_t(const AcceptParams& p, int32_t batch, cudaStream_t s
   if (e != cudaSuccess) return e;
   e = cudaFuncSetAttribute(accept_walk_kernel<T>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   if (e != cudaSuccess) return e;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(C, batch, 1);
-  cfg.blockDim = dim3(kNT);
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = s;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = C;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, accept_walk_kernel<T>, p, C, slice);
+  return launch(accept_walk_kernel<T>, dim3(C, batch, 1), dim3(kNT), smem, s, attr, 1, p, C, slice);
 }
 
 cudaError_t launch_accept(const AcceptParams& p, int32_t batch, ltd_dtype dtype, cudaStream_t s) {
@@ -394,8 +393,7 @@ cudaError_t launch_accept(const AcceptParams& p, int32_t batch, ltd_dtype dtype,
 cudaError_t launch_compact(const CompactParams& p, int32_t batch, cudaStream_t s) {
   if (p.row_bytes > kCompactMaxRowBytes || p.row_bytes % 16 != 0) return cudaErrorInvalidValue;
   const dim3 grid(p.hkv, p.n_layers * 2, batch);
-  kv_compact_kernel<<<grid, kCompactNT, 0, s>>>(p);
-  return cudaGetLastError();
+  return launch(kv_compact_kernel, grid, dim3(kCompactNT), 0, s, nullptr, 0, p);
 }
 
 }  // namespace ltd

@@ -27,6 +27,8 @@ __global__ void __launch_bounds__(kWarps * kWarp) attn_simt_kernel(const AttnPar
   __shared__ float Qs[kRows][D];
   __shared__ float Ks[kKeys][D + 1];
   __shared__ float Vs[kKeys][D];
+  grid_wait();
+  trigger_dependents();
 
   const int tile = blockIdx.x, kvh = blockIdx.y, b = blockIdx.z;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -146,12 +148,11 @@ cudaError_t launch_t(const AttnParams& p, cudaStream_t s) {
   const dim3 grid(tiles, p.hkv, p.batch);
   const dim3 block(kWarps * kWarp);
   switch (p.d) {
-    case 32: attn_simt_kernel<T, 32><<<grid, block, 0, s>>>(p); break;
-    case 64: attn_simt_kernel<T, 64><<<grid, block, 0, s>>>(p); break;
-    case 96: attn_simt_kernel<T, 96><<<grid, block, 0, s>>>(p); break;
-    default: attn_simt_kernel<T, 128><<<grid, block, 0, s>>>(p); break;
+    case 32: return launch(attn_simt_kernel<T, 32>, grid, block, 0, s, nullptr, 0, p);
+    case 64: return launch(attn_simt_kernel<T, 64>, grid, block, 0, s, nullptr, 0, p);
+    case 96: return launch(attn_simt_kernel<T, 96>, grid, block, 0, s, nullptr, 0, p);
+    default: return launch(attn_simt_kernel<T, 128>, grid, block, 0, s, nullptr, 0, p);
   }
-  return cudaGetLastError();
 }
 
 }  // namespace

@@ -168,6 +168,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc::mbar_init_fence();
     TRACE(19);
   }
+  // everything above touches only shared memory and this launch's
+  // parameters; what follows may read another kernel's output
+  grid_wait();
+  trigger_dependents();
 
   // ------------------------------------------------------ which unit
   int split = 0, pair, b, kvh;
@@ -916,22 +920,16 @@ cudaError_t launch_attn_tc(const AttnParams& p, cudaStream_t s) {
                                        static_cast<int>(kSmemBytes));
   if (e != cudaSuccess) return e;
 
-  cudaLaunchConfig_t cfg = {};
-  cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = kSmemBytes;
-  cfg.stream = s;
-  cudaLaunchAttribute attr[1];
   if (pl.splits > 1) {
     // all splits of a unit wait for one another: they must be resident together
-    cfg.gridDim = dim3(pl.splits, pl.n_pairs, p.batch * p.hkv);
+    cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeCooperative;
     attr[0].val.cooperative = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-  } else {
-    cfg.gridDim = dim3(pl.units);
+    return launch(attn_tc_kernel, dim3(pl.splits, pl.n_pairs, p.batch * p.hkv), dim3(kThreads),
+                  kSmemBytes, s, attr, 1, tq, tk, tv, a);
   }
-  return cudaLaunchKernelEx(&cfg, attn_tc_kernel, tq, tk, tv, a);
+  return launch(attn_tc_kernel, dim3(pl.units), dim3(kThreads), kSmemBytes, s, nullptr, 0, tq, tk, tv,
+                a);
 }
 
 }  // namespace ltd

@@ -52,6 +52,8 @@ __device__ unsigned long long g_expand_trace[4096][8];
 
 __global__ void tree_reset_kernel(ltd_tree t, const int32_t* __restrict__ roots,
                                   uint32_t* seq_ticket) {
+  grid_wait();
+  trigger_dependents();
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= t.batch) return;
   const int64_t nb = static_cast<int64_t>(b) * t.max_nodes;
@@ -130,6 +132,8 @@ template <typename T, int U>
 __global__ void __launch_bounds__(kNT) expand_kernel(const ExpandParams p) {
   constexpr int VEC = 16 / sizeof(T);
   __shared__ ExpandShared sh;
+  grid_wait();
+  trigger_dependents();
   const int ch = blockIdx.x, f = blockIdx.y, b = blockIdx.z, tid = threadIdx.x;
   const int lane = tid & 31, warp = tid >> 5;
   if (tid == 0) TRACE(0);
@@ -310,19 +314,12 @@ __global__ void __launch_bounds__(kNT) expand_kernel(const ExpandParams p) {
 
 template <typename T, int U>
 cudaError_t launch_u(const ExpandParams& p, int32_t batch, cudaStream_t s) {
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(p.chunks, p.F, batch);
-  cfg.blockDim = dim3(kNT);
-  cfg.dynamicSmemBytes = 0;
-  cfg.stream = s;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = p.chunks;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, expand_kernel<T, U>, p);
+  return launch(expand_kernel<T, U>, dim3(p.chunks, p.F, batch), dim3(kNT), 0, s, attr, 1, p);
 }
 
 template <typename T>
@@ -383,8 +380,8 @@ ExpandRecordLayout expand_layout(int32_t batch, int32_t k, int64_t max_vocab) {
 cudaError_t launch_tree_reset(const ltd_tree* t, const int32_t* roots, cudaStream_t s) {
   uint32_t* seq_ticket = static_cast<uint32_t*>(t->scratch);
   const int threads = 128;
-  tree_reset_kernel<<<(t->batch + threads - 1) / threads, threads, 0, s>>>(*t, roots, seq_ticket);
-  return cudaGetLastError();
+  return launch(tree_reset_kernel, dim3((t->batch + threads - 1) / threads), dim3(threads), 0, s,
+                nullptr, 0, *t, roots, seq_ticket);
 }
 
 cudaError_t launch_expand(const ExpandParams& p, int32_t batch, ltd_dtype dtype, cudaStream_t s) {

@@ -27,6 +27,8 @@ __global__ void __launch_bounds__(kNT) select_kernel(const SelectParams p) {
   uint32_t* words = reinterpret_cast<uint32_t*>(par_s + p.max_nodes);         // [n_max][W32]
   __shared__ int32_t warp_tot[kNT / kWarp];
 
+  grid_wait();
+  trigger_dependents();
   const int b = blockIdx.x, tid = threadIdx.x;
   const int64_t nb = static_cast<int64_t>(b) * p.max_nodes;
   const int n = p.n_nodes[b];
@@ -146,8 +148,7 @@ cudaError_t launch_select(const SelectParams& p, int32_t batch, cudaStream_t s) 
   cudaError_t e = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  select_kernel<<<batch, kNT, smem, s>>>(p);
-  return cudaGetLastError();
+  return launch(select_kernel, dim3(batch), dim3(kNT), smem, s, nullptr, 0, p);
 }
 
 }  // namespace ltd

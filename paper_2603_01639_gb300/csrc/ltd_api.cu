@@ -3,6 +3,7 @@
 // memory; the per-device error word is a file-scope __device__ variable.
 #include <cuda_runtime.h>
 
+#include <cstdlib>
 #include <mutex>
 
 #include "ltd.h"
@@ -24,6 +25,14 @@ uint32_t* device_error_word() {
     ptrs[dev] = static_cast<uint32_t*>(p);
   }
   return ptrs[dev];
+}
+
+bool pdl_enabled() {
+  static const bool on = [] {
+    const char* v = std::getenv("LTD_NO_PDL");
+    return !(v != nullptr && v[0] == '1');
+  }();
+  return on;
 }
 
 namespace {

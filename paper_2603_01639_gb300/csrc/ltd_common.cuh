@@ -288,4 +288,15 @@ __device__ __forceinline__ void flag_error(uint32_t* err, uint32_t bits) {
   if (err) atomicOr(err, bits);
 }
 
+// Programmatic dependent launch.  Every kernel of this library is launched
+// so that it may start while the previous kernel on the stream finishes;
+// grid_wait() returns once that kernel has completed and its writes are
+// visible (at once when there is none), and must come before any read of
+// data another kernel wrote.  trigger_dependents() lets the next kernel on
+// the stream start its own prologue.
+__device__ __forceinline__ void grid_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void trigger_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 }  // namespace ltd

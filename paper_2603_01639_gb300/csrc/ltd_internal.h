@@ -13,6 +13,42 @@ namespace ltd {
 // Address of this device's error word (lives in ltd_api.cu).
 uint32_t* device_error_word();
 
+// Whether launches carry the programmatic-dependent-launch attribute (on
+// unless the environment sets LTD_NO_PDL=1; read once).
+bool pdl_enabled();
+
+// Launch `kernel` with up to three extra launch attributes plus, when
+// enabled, programmatic stream serialization (the kernel calls grid_wait()
+// before reading another kernel's output).  If the runtime refuses the
+// combination, the launch is repeated without it.
+template <typename... KArgs, typename... Args>
+cudaError_t launch(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                   const cudaLaunchAttribute* extra, int n_extra, Args&&... args) {
+  cudaLaunchAttribute attr[4];
+  int n = 0;
+  for (int i = 0; i < n_extra && i < 3; ++i) attr[n++] = extra[i];
+  const int base_n = n;
+  if (pdl_enabled()) {
+    attr[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[n].val.programmaticStreamSerializationAllowed = 1;
+    ++n;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = n;
+  cudaError_t e = cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
+  if (e != cudaSuccess && n != base_n) {
+    (void)cudaGetLastError();
+    cfg.numAttrs = base_n;
+    e = cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
+  }
+  return e;
+}
+
 // Work split of a vocabulary scan: `chunks` CTAs per row, each covering
 // `chunk_elems` elements (a multiple of 8, so chunk starts stay 16-byte
 // aligned for both dtypes).

@@ -563,6 +563,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   // coalesced.  Several: the partial layout below.
   const int unit = (b * a.hkv + kvh) * a.n_pairs + pair;
   const int Mv = min(kRows, M - row0);
+  // the producer has drained every load (Q included) and the MMAs are done
+  // before the staging below overwrites Q
+  tc::fence_before_sync();
+  __syncthreads();
   uint8_t* stg = gbase + kOffQ;
   float* stg_l = reinterpret_cast<float*>(gbase + kOffMask);
   // tcgen05.ld is warp-collective: the O load is taken by whole warps
@@ -671,77 +675,44 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else {
       const uint8_t* cin = gbase + kOffK;
       const float* lin = reinterpret_cast<const float*>(gbase + kOffMask);
-      // A half-warp per row, a lane per 16-byte chunk: the lanes first hold
-      // the splits' log2-sum-exps (split p on lane p % 16), reduce them to
-      // weights 2^(lse_p - max) / sum, then broadcast weight p while every
-      // lane sums its chunk over the splits.  Loop bounds are warp-uniform
-      // (the shuffles need whole warps); lanes past the last row only idle.
-      const int nwork = (nrows * 16 + 31) & ~31;
-      for (int idx = tid; idx < nwork; idx += kThreads) {
-        const int rw = idx >> 4, c = idx & 15;
-        const bool live = rw < nrows;
-        const int r = live ? rw : nrows - 1;
-        float lpk[kMaxSplits / 16];
+      // A thread per (row, 16-byte chunk): the splits' log2-sum-exps give
+      // the row's max, then each split's weight 2^(lse_p - max) and its chunk
+      // are fetched with independent shared loads (four splits in flight)
+      // and accumulated; every split wrote every row below Mv (zeros where
+      // it had no keys).
+      for (int idx = tid; idx < nrows * 16; idx += kThreads) {
+        const int r = idx >> 4, c = idx & 15;
+        const float* lr = lin + r;
         float mx = -CUDART_INF_F;
-#pragma unroll
-        for (int k = 0; k < kMaxSplits / 16; ++k) {
-          const int p = c + 16 * k;
-          lpk[k] = p < S ? lin[p * Rs + r] : -CUDART_INF_F;
-          mx = fmaxf(mx, lpk[k]);
-        }
-#pragma unroll
-        for (int o = 8; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xFFFFFFFFu, mx, o));
-        float L = 0.f;
-#pragma unroll
-        for (int k = 0; k < kMaxSplits / 16; ++k) {
-          lpk[k] = (lpk[k] > -CUDART_INF_F) ? tc::ex2(lpk[k] - mx) : 0.f;
-          L += lpk[k];
-        }
-#pragma unroll
-        for (int o = 8; o > 0; o >>= 1) L += __shfl_xor_sync(0xFFFFFFFFu, L, o);
-        const float inv = L > 0.f ? 1.f / L : 0.f;
-        if (tid == 0) TRACE(22);
+#pragma unroll 4
+        for (int p = 0; p < S; ++p) mx = fmaxf(mx, lr[p * Rs]);
         float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-        const int half = lane & 16;
-        // four splits per step: their weights (shuffles) and rows (shared
-        // loads) are fetched together before the FMAs use them
-        for (int p0 = 0; p0 < S; p0 += 4) {  // S is uniform
-          float w4[4];
-          uint4 v4[4];
-#pragma unroll
-          for (int u = 0; u < 4; ++u) {
-            const int p = p0 + u;
-            const int k = p >> 4;
-            // lpk[k] with k < kMaxSplits / 16 picked without dynamic indexing
-            const float src = k == 0 ? lpk[0] : (k == 1 ? lpk[1] : (k == 2 ? lpk[2] : lpk[3]));
-            w4[u] = __shfl_sync(0xFFFFFFFFu, src, half | (p & 15));
-            const int pc = p < S ? p : S - 1;  // in range; its weight is dropped below
-            v4[u] = *reinterpret_cast<const uint4*>(cin + (pc * Rs + r) * kRowBytes + c * 16);
-            if (p >= S) w4[u] = 0.f;
-          }
-#pragma unroll
-          for (int u = 0; u < 4; ++u) {
-            const uint32_t e[4] = {v4[u].x, v4[u].y, v4[u].z, v4[u].w};
+        float L = 0.f;
+        if (mx > -CUDART_INF_F) {
+          const uint8_t* cr = cin + r * kRowBytes + c * 16;
+#pragma unroll 4
+          for (int p = 0; p < S; ++p) {
+            const float w = tc::ex2(lr[p * Rs] - mx);  // 0 for a split without keys
+            const uint4 v = *reinterpret_cast<const uint4*>(cr + p * Rs * kRowBytes);
+            L += w;
+            const uint32_t e[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
             for (int t = 0; t < 4; ++t) {
-              acc[2 * t] = fmaf(w4[u], __uint_as_float(e[t] << 16), acc[2 * t]);
-              acc[2 * t + 1] = fmaf(w4[u], __uint_as_float(e[t] & 0xFFFF0000u), acc[2 * t + 1]);
+              acc[2 * t] = fmaf(w, __uint_as_float(e[t] << 16), acc[2 * t]);
+              acc[2 * t + 1] = fmaf(w, __uint_as_float(e[t] & 0xFFFF0000u), acc[2 * t + 1]);
             }
           }
         }
-        if (tid == 0) TRACE(31);
-        if (tid == 0) TRACE_VAL(24, static_cast<unsigned long long>(clock64()));
-        if (live) {
-          const int Rr = row0 + r_lo + r;
-          const int slot = Rr / a.G, g = Rr % a.G;
-          uint4 w;
-          w.x = pack_bf16(acc[0] * inv, acc[1] * inv);
-          w.y = pack_bf16(acc[2] * inv, acc[3] * inv);
-          w.z = pack_bf16(acc[4] * inv, acc[5] * inv);
-          w.w = pack_bf16(acc[6] * inv, acc[7] * inv);
-          reinterpret_cast<uint4*>(a.out + ((static_cast<int64_t>(b) * a.n_max + slot) * a.hq +
-                                            kvh * a.G + g) * kD)[c] = w;
-        }
+        const float inv = L > 0.f ? 1.f / L : 0.f;
+        const int Rr = row0 + r_lo + r;
+        const int slot = Rr / a.G, g = Rr % a.G;
+        uint4 w;
+        w.x = pack_bf16(acc[0] * inv, acc[1] * inv);
+        w.y = pack_bf16(acc[2] * inv, acc[3] * inv);
+        w.z = pack_bf16(acc[4] * inv, acc[5] * inv);
+        w.w = pack_bf16(acc[6] * inv, acc[7] * inv);
+        reinterpret_cast<uint4*>(a.out + ((static_cast<int64_t>(b) * a.n_max + slot) * a.hq +
+                                          kvh * a.G + g) * kD)[c] = w;
       }
       if (tid == 0) TRACE(23);
     }

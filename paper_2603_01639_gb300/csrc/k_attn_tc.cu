@@ -99,8 +99,8 @@ struct TcArgs {
   const uint32_t* mask;
   float scale_log2;
   __nv_bfloat16* out;
-  uint8_t* part_o;  // [unit][owner][split][rs][256 B] O / l, bf16 (splits > 1)
-  float* part_l;    // [unit][owner][split][rs] log2-sum-exp
+  uint8_t* part_o;  // [unit][split][256 rows][256 B] O / l, bf16, chunks swizzled (splits > 1)
+  float* part_l;    // [unit][split][256] log2-sum-exp
   uint32_t* sync;   // [unit][2] arrive, depart
   uint32_t* err;
 };
@@ -616,30 +616,20 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 
   // ------------------------------------- combine the splits (S > 1 only)
-  // Rows [o rs, o rs + rs) of a unit are combined by its split o ("owner").
-  // Partials are laid out owner-major, [unit][owner][split][rs][256 B], so
-  // every split writes its rows with coalesced stores and an owner reads all
-  // of its inputs with one bulk copy.
+  // Each split stores its staged rows and sums with one bulk copy each
+  // (split-major: [unit][split][row]); rows [o rs, o rs + rs) of a unit are
+  // combined by its split o ("owner"), which pulls that block of every
+  // split with one bulk copy per split.
   const int Rs = a.rs;
-  {
-    uint8_t* po = a.part_o + static_cast<int64_t>(unit) * S * S * Rs * kRowBytes;
-    float* pl = a.part_l + static_cast<int64_t>(unit) * S * S * Rs;
-    for (int idx = tid; idx < Mv * 16; idx += kThreads) {
-      const int r = idx >> 4, c = idx & 15;
-      const int o = r / Rs, rl = r - o * Rs;
-      const uint4 v = *reinterpret_cast<const uint4*>(stg + r * kRowBytes + ((c ^ (r & 15)) << 4));
-      reinterpret_cast<uint4*>(po + ((static_cast<int64_t>(o) * S + split) * Rs + rl) * kRowBytes)[c] = v;
-    }
-    for (int r = tid; r < Mv; r += kThreads) {
-      const int o = r / Rs, rl = r - o * Rs;
-      pl[(static_cast<int64_t>(o) * S + split) * Rs + rl] = stg_l[r];
-    }
-  }
-  __syncthreads();
   uint32_t* arrive = a.sync + 2 * unit;
   uint32_t* depart = arrive + 1;
   if (tid == 0) {
-    __threadfence();  // with the barrier above: every thread's partial stores
+    const int64_t pb = static_cast<int64_t>(unit) * S + split;
+    tc::bulk_s2g(a.part_o + pb * kRows * kRowBytes, base + kOffQ, Mv * kRowBytes);
+    tc::bulk_s2g(a.part_l + pb * kRows, base + kOffMask, ((Mv + 3) & ~3) * 4);
+    tc::bulk_commit();
+    tc::bulk_wait_all();
+    tc::fence_proxy_async_global();
     tc::red_add_release_gpu(arrive, 1u);
     bool got = tc::ld_acquire_gpu(arrive) >= static_cast<uint32_t>(S);
     if (!got) {
@@ -650,7 +640,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!got && tc::globaltimer() - t0 > tc::kWaitLimitNs) break;
       }
     }
-    __threadfence();
     if (!got) flag_error(a.err, LTD_DEVERR_TIMEOUT);
     holder[1] = got ? 1u : 0u;
     TRACE(15);
@@ -660,12 +649,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int nrows = max(0, min(Mv, r_lo + Rs) - r_lo);
   if (holder[1] != 0u && nrows > 0) {
     if (tid == 0) {
-      // partial writes by other CTAs (generic proxy) are read by the bulk copy
+      // the acquire above orders the other splits' stores before these reads
       tc::fence_proxy_async_global();
-      const int64_t ob = static_cast<int64_t>(unit) * S + split;
-      tc::mbar_expect_tx(bar(CBAR), static_cast<uint32_t>(S * Rs) * (kRowBytes + 4));
-      tc::bulk_g2s(base + kOffK, a.part_o + ob * S * Rs * kRowBytes, S * Rs * kRowBytes, bar(CBAR));
-      tc::bulk_g2s(base + kOffMask, a.part_l + ob * S * Rs, S * Rs * 4, bar(CBAR));
+      const int nl = min(Rs, kRows - r_lo);  // a multiple of 4
+      tc::mbar_expect_tx(bar(CBAR), static_cast<uint32_t>(S) * (nrows * kRowBytes + nl * 4));
+      for (int p = 0; p < S; ++p) {
+        const int64_t pb = static_cast<int64_t>(unit) * S + p;
+        tc::bulk_g2s(base + kOffK + p * Rs * kRowBytes, a.part_o + (pb * kRows + r_lo) * kRowBytes,
+                     nrows * kRowBytes, bar(CBAR));
+        tc::bulk_g2s(base + kOffMask + p * Rs * 4, a.part_l + pb * kRows + r_lo, nl * 4, bar(CBAR));
+      }
     }
     // CTA-uniform, as a barrier follows under it
     const bool in = __syncthreads_and(tc::mbar_wait(bar(CBAR), 0)) != 0;
@@ -689,7 +682,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
         float L = 0.f;
         if (mx > -CUDART_INF_F) {
-          const uint8_t* cr = cin + r * kRowBytes + c * 16;
+          // rows keep the staging's chunk swizzle (by row within the unit)
+          const uint8_t* cr = cin + r * kRowBytes + ((c ^ ((r_lo + r) & 15)) << 4);
 #pragma unroll 4
           for (int p = 0; p < S; ++p) {
             const float w = tc::ex2(lr[p * Rs] - mx);  // 0 for a split without keys
@@ -789,8 +783,8 @@ struct WsLayout {
 WsLayout ws_layout(const Plan& pl) {
   WsLayout w{};
   if (pl.splits <= 1) return w;
-  // [unit][owner][split][rs] rows: splits * rs <= 256 + 4 * splits
-  const size_t rows = static_cast<size_t>(pl.units) * pl.splits * pl.splits * pl.rs;
+  // [unit][split][256] rows
+  const size_t rows = static_cast<size_t>(pl.units) * pl.splits * kRows;
   w.part_o = 0;
   w.part_l = align256(rows * kRowBytes);
   w.sync = w.part_l + align256(rows * sizeof(float));

@@ -107,6 +107,7 @@ struct SelectParams {
   const float* cum;
   const int32_t* n_nodes;
   int32_t max_nodes;
+  int32_t sort_len;  // power of two >= max_nodes (set by launch_select)
   const int32_t* n_verify;
   int32_t n_max;
   const int32_t* ctx;

@@ -124,6 +124,7 @@ struct ExpandShared {
   // gathered by rank 0
   uint64_t peer_top[kMaxChunks][kWarp];
   float2 peer_ms[kMaxChunks];
+  float thr;
   int n_cand;
   int last;
 };
@@ -178,12 +179,20 @@ __global__ void __launch_bounds__(kNT) expand_kernel(const ExpandParams p) {
   float m = tmax, s = tsum;
   block_ms<kNT>(m, s, sh.red);
 
-  // ---- stage 2: T = k-th largest per-thread max (a lower bound of the
-  // chunk's k-th largest logit)
-  sh.fstage[warp * kWarp + lane] = warp_sort_desc_f(tmax);
+  // ---- stage 2: T = k-th largest of the 32 half-warp maxima, a lower bound
+  // of the chunk's k-th largest logit (k half-warps hold an element >= T)
+  float hm = tmax;
+#pragma unroll
+  for (int o = 8; o > 0; o >>= 1) hm = fmaxf(hm, __shfl_xor_sync(0xFFFFFFFFu, hm, o));
+  if ((lane & 15) == 0) sh.fstage[warp * 2 + (lane >> 4)] = hm;
   if (tid == 0) sh.n_cand = 0;
-  tree_merge<float, warp_merge_desc_f>(sh.fstage);
-  const float thr = sh.fstage[k - 1];
+  __syncthreads();
+  if (warp == 0) {
+    const float v = warp_sort_desc_f(sh.fstage[lane]);  // 2 * kNW = 32 half-warps
+    if (lane == k - 1) sh.thr = v;
+  }
+  __syncthreads();
+  const float thr = sh.thr;
 
   // ---- stage 3: the candidates >= T, ranked exactly by (logit desc, token asc)
   if (tmax >= thr) {
@@ -200,15 +209,21 @@ __global__ void __launch_bounds__(kNT) expand_kernel(const ExpandParams p) {
   }
   __syncthreads();
   const int nc = sh.n_cand;
-  WarpTopK wt;
-  wt.init();
   if (nc <= kCand) {
-    for (int c0 = warp * kWarp; c0 < nc; c0 += kNT) {
-      const int c = c0 + lane;
-      wt.offer(c < nc ? sh.cand[c] : 0ull, k);
+    // typically a few dozen: one warp ranks them
+    if (warp == 0) {
+      WarpTopK wt;
+      wt.init();
+      for (int c0 = 0; c0 < nc; c0 += kWarp) {
+        const int c = c0 + lane;
+        wt.offer(c < nc ? sh.cand[c] : 0ull, k);
+      }
+      sh.top[lane] = wt.v;
     }
   } else {
-    // exact fallback: every element of the chunk is offered
+    // exact fallback (huge tie sets): every element of the chunk is offered
+    WarpTopK wt;
+    wt.init();
 #pragma unroll
     for (int u = 0; u < U; ++u)
 #pragma unroll
@@ -216,40 +231,44 @@ __global__ void __launch_bounds__(kNT) expand_kernel(const ExpandParams p) {
         const int64_t i = lo + (static_cast<int64_t>(u) * kNT + tid) * VEC + j;
         wt.offer(i < hi ? make_key(xv[u][j], static_cast<uint32_t>(i)) : 0ull, k);
       }
+    sh.stage[warp * kWarp + lane] = wt.v;
+    tree_merge<uint64_t, warp_merge_desc>(sh.stage);
+    if (tid < kWarp) sh.top[tid] = sh.stage[tid];
   }
-  sh.stage[warp * kWarp + lane] = wt.v;
-  tree_merge<uint64_t, warp_merge_desc>(sh.stage);
-  if (tid < kWarp) sh.top[tid] = sh.stage[tid];
   if (tid == 0) {
     sh.ms = make_float2(m, s);
     TRACE(2);
   }
 
-  // ---- row: rank 0 gathers the chunk results of its cluster
+  // ---- row: rank 0 gathers the chunk results of its cluster (warp 0 reads
+  // every peer's list into registers; the merges follow once the peers
+  // may leave)
   const int C = p.chunks;
   tc::cluster_sync();
-  if (ch == 0) {
-    if (tid < C * kWarp) {
-      const int peer = tid / kWarp, e = tid % kWarp;
-      const uint32_t a = tc::mapa(tc::smem_u32(&sh.top[e]), peer);
-      uint64_t v;
-      asm volatile("ld.shared::cluster.u64 %0, [%1];" : "=l"(v) : "r"(a) : "memory");
-      sh.peer_top[peer][e] = v;
-    }
-    if (tid < C) sh.peer_ms[tid] = tc::ld_cluster_f2(tc::mapa(tc::smem_u32(&sh.ms), tid));
+  uint64_t lists[kMaxChunks];
+  if (ch == 0 && warp == 0) {
+#pragma unroll
+    for (int c = 0; c < kMaxChunks; ++c)
+      lists[c] = c < C ? tc::ld_cluster_u64(tc::mapa(tc::smem_u32(&sh.top[lane]), c)) : 0ull;
+    if (lane < C) sh.peer_ms[lane] = tc::ld_cluster_f2(tc::mapa(tc::smem_u32(&sh.ms), lane));
   }
   // no CTA leaves while rank 0 may still read its shared memory
   tc::cluster_sync();
   if (ch != 0) return;
   if (tid == 0) TRACE(3);
-
-  if (tid == 0) {
-    float M = -CUDART_INF_F, S = 0.f;
-    for (int c = 0; c < C; ++c) ms_merge(M, S, sh.peer_ms[c].x, sh.peer_ms[c].y);
-    sh.red[0] = M + logf(S);
+  if (warp == 0) {
+    uint64_t v = lists[0];
+#pragma unroll
+    for (int c = 1; c < kMaxChunks; ++c)
+      if (c < C) v = warp_merge_desc(v, lists[c]);
+    sh.stage[lane] = v;
+    if (lane == 0) {
+      float M = -CUDART_INF_F, S = 0.f;
+      for (int c = 0; c < C; ++c) ms_merge(M, S, sh.peer_ms[c].x, sh.peer_ms[c].y);
+      sh.red[0] = M + logf(S);
+    }
   }
-  sh.stage[warp * kWarp + lane] = (warp < C) ? sh.peer_top[warp][lane] : 0ull;
-  tree_merge<uint64_t, warp_merge_desc>(sh.stage);
+  __syncthreads();
   const float lse = sh.red[0];
 
   const int64_t nb = static_cast<int64_t>(b) * p.max_nodes;
@@ -291,19 +310,31 @@ __global__ void __launch_bounds__(kNT) expand_kernel(const ExpandParams p) {
   if (!sh.last) return;
   __threadfence();
   if (tid == 0) TRACE(5);
-  {
+  const int pool = k * k;
+  if (pool <= 4 * kWarp) {
+    // a small pool: one warp, no block barriers
+    if (warp == 0) {
+      WarpTopK pt;
+      pt.init();
+      for (int j0 = 0; j0 < pool; j0 += kWarp) {
+        const int j = j0 + lane;
+        const int id = base + j;
+        pt.offer(j < pool ? make_key(__ldcg(&p.cum[nb + id]), static_cast<uint32_t>(id)) : 0ull, k);
+      }
+      if (lane < k) p.frontier[b * k + lane] = static_cast<int32_t>(key_index(pt.v));
+    }
+  } else {
     WarpTopK pt;
     pt.init();
-    const int pool = k * k;
     for (int j0 = warp * kWarp; j0 < pool; j0 += kNT) {
       const int j = j0 + lane;
       const int id = base + j;
       pt.offer(j < pool ? make_key(__ldcg(&p.cum[nb + id]), static_cast<uint32_t>(id)) : 0ull, k);
     }
     sh.stage[warp * kWarp + lane] = pt.v;
+    tree_merge<uint64_t, warp_merge_desc>(sh.stage);
+    if (tid < k) p.frontier[b * k + tid] = static_cast<int32_t>(key_index(sh.stage[tid]));
   }
-  tree_merge<uint64_t, warp_merge_desc>(sh.stage);
-  if (tid < k) p.frontier[b * k + tid] = static_cast<int32_t>(key_index(sh.stage[tid]));
   if (tid == 0) {
     p.n_nodes[b] = base + p.F * k;
     p.n_levels[b] = p.level;

@@ -181,6 +181,24 @@ ltd_status ltd_tree_attention(const void* d_q, const void* d_k, const void* d_v,
                               const uint32_t* d_mask, float scale, void* d_workspace,
                               size_t workspace_bytes, ltd_stream_t stream);
 
+/* ltd_tree_attention, and in addition a hint for the next call: once this
+ * call has loaded its own keys and values, the tensor-core kernel asks L2 to
+ * fetch the rows it just used from d_next_k / d_next_v (the next layer's
+ * cache, same layout and sizes; the same ctx and N), so that the next call's
+ * loads find them in L2 instead of HBM.  Results are identical to
+ * ltd_tree_attention; the hint is skipped when one layer's keys and values
+ * exceed 64 MB (they would crowd L2) and by the CUDA-core kernel.  The
+ * paper has no counterpart: it is a deployment convenience for consecutive
+ * layers.  d_next_k and d_next_v must both be valid 16-byte aligned device
+ * pointers or both NULL (then this is ltd_tree_attention). */
+ltd_status ltd_tree_attention_next(const void* d_q, const void* d_k, const void* d_v, void* d_out,
+                                   ltd_dtype dtype, int32_t batch, int32_t hq, int32_t hkv,
+                                   int32_t head_dim, int32_t s_cap, const int32_t* d_ctx,
+                                   int32_t max_ctx, const int32_t* d_n_verify, int32_t n_max,
+                                   const uint32_t* d_mask, float scale, void* d_workspace,
+                                   size_t workspace_bytes, const void* d_next_k,
+                                   const void* d_next_v, ltd_stream_t stream);
+
 /* Which kernel ltd_tree_attention runs for these sizes: returns 1 for the
  * tcgen05 tensor-core kernel, 0 for the CUDA-core kernel, -1 if the sizes are
  * unsupported.  *launches (if not NULL) receives the number of kernel

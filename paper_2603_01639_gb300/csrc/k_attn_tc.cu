@@ -102,6 +102,8 @@ struct TcArgs {
   uint8_t* part_o;  // [unit][split][256 rows][256 B] O / l, bf16, chunks swizzled (splits > 1)
   float* part_l;    // [unit][split][256] log2-sum-exp
   uint32_t* sync;   // [unit][2] arrive, depart
+  const uint8_t* next_k;  // the next call's caches: L2 prefetch targets (or null)
+  const uint8_t* next_v;
   uint32_t* err;
 };
 
@@ -334,6 +336,17 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       drain();
       if (!ok) flag_error(a.err, LTD_DEVERR_TIMEOUT);
+      if (a.next_k != nullptr && nc > 0) {
+        // this CTA's loads have landed: ask L2 for the same rows of the next
+        // call's caches, 128 rows (32 KB) per request
+        const int r_end = min(key_hi, key_lo + nc * kBN);
+        for (int r = key_lo; r < r_end; r += kBN) {
+          const uint32_t bytes = static_cast<uint32_t>(min(kBN, r_end - r)) * kRowBytes;
+          const int64_t off = (static_cast<int64_t>(kvrow) * a.s_cap + r) * kRowBytes;
+          tc::prefetch_l2(a.next_k + off, bytes);
+          tc::prefetch_l2(a.next_v + off, bytes);
+        }
+      }
     }
   } else if (warp == 1) {
     // ----------------------------------------------------------------- MMA
@@ -869,6 +882,13 @@ cudaError_t launch_attn_tc(const AttnParams& p, cudaStream_t s) {
   a.part_l = pl.splits > 1 ? reinterpret_cast<float*>(ws + wl.part_l) : nullptr;
   a.sync = pl.splits > 1 ? reinterpret_cast<uint32_t*>(ws + wl.sync) : nullptr;
   a.err = p.err;
+  // the hint only while one layer's keys and values fit well inside L2
+  const uint64_t layer_kv = static_cast<uint64_t>(p.batch) * p.hkv *
+                            (static_cast<uint64_t>(p.max_ctx) + p.n_max) * kRowBytes * 2;
+  if (p.next_k != nullptr && p.next_v != nullptr && layer_kv <= (64ull << 20)) {
+    a.next_k = static_cast<const uint8_t*>(p.next_k);
+    a.next_v = static_cast<const uint8_t*>(p.next_v);
+  }
 
   CUtensorMap tq, tk, tv;
   const uint64_t row = kD * 2;

@@ -216,12 +216,13 @@ size_t ltd_attention_workspace_bytes(int32_t batch, int32_t hq, int32_t hkv, int
   return ws;
 }
 
-ltd_status ltd_tree_attention(const void* d_q, const void* d_k, const void* d_v, void* d_out,
-                              ltd_dtype dtype, int32_t batch, int32_t hq, int32_t hkv,
-                              int32_t head_dim, int32_t s_cap, const int32_t* d_ctx,
-                              int32_t max_ctx, const int32_t* d_n_verify, int32_t n_max,
-                              const uint32_t* d_mask, float scale, void* d_workspace,
-                              size_t workspace_bytes, ltd_stream_t stream) {
+namespace {
+ltd_status tree_attention(const void* d_q, const void* d_k, const void* d_v, void* d_out,
+                          ltd_dtype dtype, int32_t batch, int32_t hq, int32_t hkv, int32_t head_dim,
+                          int32_t s_cap, const int32_t* d_ctx, int32_t max_ctx,
+                          const int32_t* d_n_verify, int32_t n_max, const uint32_t* d_mask,
+                          float scale, void* d_workspace, size_t workspace_bytes,
+                          const void* d_next_k, const void* d_next_v, ltd_stream_t stream) {
   if (!d_q || !d_k || !d_v || !d_out || !d_ctx || !d_n_verify || !d_mask || !dtype_ok(dtype))
     return LTD_ERR_INVALID_ARG;
   if (batch < 1 || hq < 1 || hkv < 1 || hq % hkv != 0 || n_max < 1 || n_max > LTD_MAX_N ||
@@ -232,6 +233,8 @@ ltd_status ltd_tree_attention(const void* d_q, const void* d_k, const void* d_v,
   if (!(scale > 0.f)) return LTD_ERR_INVALID_ARG;
   if (!aligned16(d_q) || !aligned16(d_k) || !aligned16(d_v) || !aligned16(d_out))
     return LTD_ERR_SHAPE;
+  if ((d_next_k == nullptr) != (d_next_v == nullptr)) return LTD_ERR_INVALID_ARG;
+  if (!aligned16(d_next_k) || !aligned16(d_next_v)) return LTD_ERR_SHAPE;
   const size_t need =
       ltd_attention_workspace_bytes(batch, hq, hkv, head_dim, n_max, max_ctx, dtype);
   if (d_workspace == nullptr || workspace_bytes < need) return LTD_ERR_SHAPE;
@@ -255,10 +258,36 @@ ltd_status ltd_tree_attention(const void* d_q, const void* d_k, const void* d_v,
   p.scale = scale;
   p.ws = d_workspace;
   p.ws_bytes = workspace_bytes;
+  p.next_k = d_next_k;
+  p.next_v = d_next_v;
   p.err = err;
   const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (attn_tc_supported(p, dtype)) return from_cuda(launch_attn_tc(p, s));
   return from_cuda(launch_attn_simt(p, dtype, s));
+}
+}  // namespace
+
+ltd_status ltd_tree_attention(const void* d_q, const void* d_k, const void* d_v, void* d_out,
+                              ltd_dtype dtype, int32_t batch, int32_t hq, int32_t hkv,
+                              int32_t head_dim, int32_t s_cap, const int32_t* d_ctx,
+                              int32_t max_ctx, const int32_t* d_n_verify, int32_t n_max,
+                              const uint32_t* d_mask, float scale, void* d_workspace,
+                              size_t workspace_bytes, ltd_stream_t stream) {
+  return tree_attention(d_q, d_k, d_v, d_out, dtype, batch, hq, hkv, head_dim, s_cap, d_ctx, max_ctx,
+                        d_n_verify, n_max, d_mask, scale, d_workspace, workspace_bytes, nullptr,
+                        nullptr, stream);
+}
+
+ltd_status ltd_tree_attention_next(const void* d_q, const void* d_k, const void* d_v, void* d_out,
+                                   ltd_dtype dtype, int32_t batch, int32_t hq, int32_t hkv,
+                                   int32_t head_dim, int32_t s_cap, const int32_t* d_ctx,
+                                   int32_t max_ctx, const int32_t* d_n_verify, int32_t n_max,
+                                   const uint32_t* d_mask, float scale, void* d_workspace,
+                                   size_t workspace_bytes, const void* d_next_k,
+                                   const void* d_next_v, ltd_stream_t stream) {
+  return tree_attention(d_q, d_k, d_v, d_out, dtype, batch, hq, hkv, head_dim, s_cap, d_ctx, max_ctx,
+                        d_n_verify, n_max, d_mask, scale, d_workspace, workspace_bytes, d_next_k,
+                        d_next_v, stream);
 }
 
 int32_t ltd_attention_kernel(ltd_dtype dtype, int32_t batch, int32_t hq, int32_t hkv,

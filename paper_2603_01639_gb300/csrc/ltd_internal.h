@@ -133,6 +133,8 @@ struct AttnParams {
   float scale;
   void* ws;
   size_t ws_bytes;
+  const void* next_k;  // L2 prefetch hint for the next call (may be null)
+  const void* next_v;
   uint32_t* err;
 };
 size_t attn_simt_workspace(const AttnParams& p);

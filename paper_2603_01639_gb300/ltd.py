@@ -29,7 +29,7 @@ EXPORTS = [
     "ltd_tree_bytes", "ltd_tree_init", "ltd_tree_reset", "ltd_expand_tree", "ltd_select_verify",
     "ltd_attention_workspace_bytes", "ltd_tree_attention", "ltd_accept_workspace_bytes",
     "ltd_accept", "ltd_kv_compact", "ltd_check", "ltd_status_string", "ltd_version",
-    "ltd_attention_kernel", "ltd_selftest_umma", "ltd_accept_noalloc",
+    "ltd_attention_kernel", "ltd_selftest_umma", "ltd_accept_noalloc", "ltd_tree_attention_next",
 ]
 LTD_ACCEPT_NOALLOC_SCRATCH_BYTES = 1 << 20
 
@@ -73,6 +73,9 @@ def lib():
                 "ltd_attention_workspace_bytes": (sz, [i32, i32, i32, i32, i32, i32, C.c_int]),
                 "ltd_tree_attention": (C.c_int, [vp, vp, vp, vp, C.c_int, i32, i32, i32, i32, i32,
                                                  vp, i32, vp, i32, vp, C.c_float, vp, sz, vp]),
+                "ltd_tree_attention_next": (C.c_int, [vp, vp, vp, vp, C.c_int, i32, i32, i32, i32,
+                                                      i32, vp, i32, vp, i32, vp, C.c_float, vp, sz,
+                                                      vp, vp, vp]),
                 "ltd_accept_workspace_bytes": (sz, [i32, i32, i64]),
                 "ltd_accept": (C.c_int, [tp, vp, vp, C.c_int, i64, i64, vp, vp, i32, vp, u64, u64,
                                          vp, vp, vp, vp, vp, C.POINTER(ltd_kv_cache), vp, sz, vp]),
@@ -223,8 +226,9 @@ def attention_workspace(batch, hq, hkv, head_dim, n_max, max_ctx, dtype, device=
 
 
 def ltd_tree_attention(q, k_cache, v_cache, ctx, max_ctx, n_verify, mask, scale=None,
-                       out=None, workspace=None, stream=None):
-    """q [B][n_max][hq][d]; k/v [B][hkv][s_cap][d]; returns out like q."""
+                       out=None, workspace=None, stream=None, next_k=None, next_v=None):
+    """q [B][n_max][hq][d]; k/v [B][hkv][s_cap][d]; returns out like q.  next_k/next_v:
+    the next call's caches (same shapes), for ltd_tree_attention_next's L2 hint."""
     for t, n in ((q, "q"), (k_cache, "k_cache"), (v_cache, "v_cache")):
         _need(t, n, q.dtype)
     _need(ctx, "ctx", torch.int32)
@@ -238,10 +242,23 @@ def ltd_tree_attention(q, k_cache, v_cache, ctx, max_ctx, n_verify, mask, scale=
         out = torch.zeros_like(q)
     if workspace is None:
         workspace = attention_workspace(B, hq, hkv, d, n_max, max_ctx, q.dtype, q.device)
-    _ok(lib().ltd_tree_attention(_ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(out), _dtype(q), B,
-                                 hq, hkv, d, s_cap, _ptr(ctx), max_ctx, _ptr(n_verify), n_max,
-                                 _ptr(mask), float(scale), _ptr(workspace), workspace.numel(),
-                                 _stream(stream)), "ltd_tree_attention")
+    if next_k is None and next_v is None:
+        _ok(lib().ltd_tree_attention(_ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(out), _dtype(q),
+                                     B, hq, hkv, d, s_cap, _ptr(ctx), max_ctx, _ptr(n_verify),
+                                     n_max, _ptr(mask), float(scale), _ptr(workspace),
+                                     workspace.numel(), _stream(stream)), "ltd_tree_attention")
+        return out
+    if (next_k is None) != (next_v is None):
+        raise LtdError("next_k and next_v go together")
+    for t, n in ((next_k, "next_k"), (next_v, "next_v")):
+        _need(t, n, q.dtype)
+        if t.shape != k_cache.shape:
+            raise LtdError(f"{n} must have the shape of k_cache")
+    _ok(lib().ltd_tree_attention_next(_ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(out), _dtype(q),
+                                      B, hq, hkv, d, s_cap, _ptr(ctx), max_ctx, _ptr(n_verify),
+                                      n_max, _ptr(mask), float(scale), _ptr(workspace),
+                                      workspace.numel(), _ptr(next_k), _ptr(next_v),
+                                      _stream(stream)), "ltd_tree_attention_next")
     return out
 
 

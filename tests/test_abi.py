@@ -93,6 +93,13 @@ def test_entry_points_reject_bad_arguments_before_launch(L):
     assert L.ltd_tree_attention(*bad) == 2
     bad = list(args); bad[15] = 0.0
     assert L.ltd_tree_attention(*bad) == 1
+    nxt = args[:18] + [fake, fake, s]                                               # the hint
+    bad = list(nxt); bad[19] = None                                                # one of two
+    assert L.ltd_tree_attention_next(*bad) == 1
+    bad = list(nxt); bad[18] = C.c_void_p((1 << 24) + 8)                          # misaligned
+    assert L.ltd_tree_attention_next(*bad) == 2
+    bad = list(nxt); bad[8] = 80
+    assert L.ltd_tree_attention_next(*bad) == 3
     assert L.ltd_accept_workspace_bytes(1, 8, 1000) > 0
     assert L.ltd_accept_workspace_bytes(1, 300, 1000) == 0
     kv = ltd.ltd_kv_cache(fake, fake, 1, 1, 70, 256, 1)                            # 140-byte rows

@@ -290,6 +290,25 @@ def test_attention_flags_bad_sequence():
     assert ltd.ltd_check() == 0
 
 
+def test_attention_next_layer_hint_changes_nothing():
+    """ltd_tree_attention_next (L2 hint for the next layer's caches) returns
+    the bytes ltd_tree_attention returns."""
+    for name in ("8b", "13b"):
+        cfg = wl.config(name)
+        ci = wl.draw_cycle(cfg, 12, draft_rows=False)
+        q, k, v = wl.draw_attention(cfg, 12, ci.ctx, ci.n_verify)
+        qd, kd, vd = H.dev(q, cfg.dtype), H.dev(k, cfg.dtype), H.dev(v, cfg.dtype)
+        k2, v2 = torch.roll(kd, 1, dims=2), torch.roll(vd, 1, dims=2)
+        W32 = (cfg.max_n + 31) // 32
+        mw = torch.zeros(cfg.batch, cfg.max_n, W32, dtype=torch.int32, device="cuda")
+        mw[..., 0] = 1
+        c, n = H.i32(ci.ctx), H.i32(ci.n_verify)
+        a = ltd.ltd_tree_attention(qd, kd, vd, c, cfg.max_ctx, n, mw)
+        b = ltd.ltd_tree_attention(qd, kd, vd, c, cfg.max_ctx, n, mw, next_k=k2, next_v=v2)
+        assert ltd.ltd_check() == 0
+        assert torch.equal(a, b)
+
+
 def test_attention_workspace_reuse():
     """Back-to-back calls on one workspace: the split counters are left at
     zero by each call, so every call combines correctly."""

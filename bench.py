@@ -45,6 +45,9 @@ def _args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-sample-s", type=float, default=15.0)
+    ap.add_argument("--no-next-hint", action="store_true",
+                    help="run the cycle without the next-layer L2 hint (for profiling one layer's "
+                         "own traffic)")
     return ap.parse_args()
 
 
@@ -439,9 +442,11 @@ def run_ours(args):
     layers = N_LAYERS[args.config]
     cyc = Cycle(cfg, layers, replica_seed(args.seed, rank), device)
 
+    verify = cyc.verify_phase_plain if args.no_next_hint else cyc.verify_phase
+
     def full():
         cyc.draft_phase()
-        cyc.verify_phase()
+        verify()
         cyc.accept_phase()
 
     for _ in range(max(args.warmup, 3)):
@@ -449,7 +454,7 @@ def run_ours(args):
     torch.cuda.synchronize(device)
     ltd.ltd_check()
     g_draft = _graph(torch, cyc.draft_phase)
-    g_verify = _graph(torch, cyc.verify_phase)
+    g_verify = _graph(torch, verify)
     g_plain = _graph(torch, cyc.verify_phase_plain)
     g_accept = _graph(torch, cyc.accept_phase)
     for _ in range(2):

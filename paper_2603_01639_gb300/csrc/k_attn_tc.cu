@@ -73,11 +73,11 @@ enum Bar { QFULL = 0, KFULL = 1, VFULL = 3, KEMPTY = 5, VEMPTY = 7, SFULL = 9, P
 
 // Optional phase timestamps for performance work (off in normal builds).
 #ifdef LTD_TRACE
-__device__ unsigned long long g_attn_trace[2048][32];
+__device__ unsigned long long g_attn_trace[4096][48];
 #define TRACE_VAL(slot, v)                                                                    \
   do {                                                                                        \
     const int cta_ = blockIdx.x + gridDim.x * (blockIdx.y + gridDim.y * blockIdx.z);          \
-    if (cta_ < 2048) g_attn_trace[cta_][slot] = (v);                                          \
+    if (cta_ < 4096) g_attn_trace[cta_][slot] = (v);                                          \
   } while (0)
 #define TRACE(slot) TRACE_VAL(slot, tc::globaltimer())
 #else
@@ -325,15 +325,25 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
+#ifdef LTD_TRACE
+      unsigned long long w_empty = 0, t_e = 0;
+#endif
       for (int j = n_issued; j < nc && ok; ++j) {
         const int st = j & 1;
+#ifdef LTD_TRACE
+        t_e = tc::globaltimer();
+#endif
         ok = tc::mbar_wait(bar(KEMPTY + st), ((j >> 1) - 1) & 1);
         if (!ok) break;
         issue_k(j);
         ok = tc::mbar_wait(bar(VEMPTY + st), ((j >> 1) - 1) & 1);
         if (!ok) break;
         issue_v(j);
+#ifdef LTD_TRACE
+        w_empty += tc::globaltimer() - t_e;
+#endif
       }
+      TRACE_VAL(32, w_empty);
       drain();
       if (!ok) flag_error(a.err, LTD_DEVERR_TIMEOUT);
       if (a.next_k != nullptr && nc > 0) {
@@ -354,53 +364,94 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t id_s = tc::idesc_bf16(kBM, kBN, false);
       const uint32_t id_o = tc::idesc_bf16(kBM, kD, true);
       const int ntile = has_b ? 2 : 1;
+      // Every shared-memory descriptor is computed once, so the issue loop
+      // below is MMA instructions only (the thread shares its scheduler with
+      // two softmax warps, and each MMA lasts just 64 cycles).
+      uint64_t dq[2][8], dk[2][8], dv[2][8];
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+#pragma unroll
+        for (int ks = 0; ks < 8; ++ks) {
+          dq[u][ks] = tc::sdesc_sw128(base + kOffQ + u * kTile + (ks >> 2) * kHalf + (ks & 3) * 32, 16, 1024);
+          dk[u][ks] = tc::sdesc_sw128(base + kOffK + u * kTile + (ks >> 2) * kHalf + (ks & 3) * 32, 16, 1024);
+          dv[u][ks] = tc::sdesc_sw128(base + kOffV + u * kTile + ks * 2048, kHalf, 1024);
+        }
+      }
+      // (t and st are compile-time constants at every call)
       auto issue_s = [&](int t, int st) {
-        for (int ks = 0; ks < 8; ++ks) {
-          const uint64_t da =
-              tc::sdesc_sw128(base + kOffQ + t * kTile + (ks >> 2) * kHalf + (ks & 3) * 32, 16, 1024);
-          const uint64_t db =
-              tc::sdesc_sw128(base + kOffK + st * kTile + (ks >> 2) * kHalf + (ks & 3) * 32, 16, 1024);
-          tc::mma_bf16(tmem + t * kBN, da, db, id_s, ks > 0 ? 1u : 0u);
-        }
+#pragma unroll
+        for (int ks = 0; ks < 8; ++ks)
+          tc::mma_bf16(tmem + t * kBN, dq[t][ks], dk[st][ks], id_s, ks > 0 ? 1u : 0u);
       };
-      auto issue_pv = [&](int t, int st, bool acc) {
-        for (int ks = 0; ks < 8; ++ks) {
-          const uint64_t db = tc::sdesc_sw128(base + kOffV + st * kTile + ks * 2048, kHalf, 1024);
-          tc::mma_bf16_ts(tmem + 2 * kBN + t * kD, tmem + t * kBN + 8 * ks, db, id_o,
-                          (acc || ks > 0) ? 1u : 0u);
-        }
+      auto issue_pv = [&](int t, int st, uint32_t acc) {
+#pragma unroll
+        for (int ks = 0; ks < 8; ++ks)
+          tc::mma_bf16_ts(tmem + 2 * kBN + t * kD, tmem + t * kBN + 8 * ks, dv[st][ks], id_o,
+                          ks > 0 ? 1u : acc);
       };
+#ifdef LTD_TRACE
+      unsigned long long w_load = 0, w_p = 0, t_w;
+#define TW_BEGIN() t_w = tc::globaltimer()
+#define TW_END(acc) acc += tc::globaltimer() - t_w
+#else
+#define TW_BEGIN() \
+  do {             \
+  } while (0)
+#define TW_END(acc) \
+  do {              \
+  } while (0)
+#endif
       ok = tc::mbar_wait(bar(QFULL), 0);
       TRACE(2);
       if (ok) ok = tc::mbar_wait(bar(KFULL + 0), 0);
       TRACE(3);
       if (ok) {
         tc::fence_after_sync();
-        for (int t = 0; t < ntile; ++t) {
-          issue_s(t, 0);
-          tc::mma_commit(bar(SFULL + t));
+        issue_s(0, 0);
+        tc::mma_commit(bar(SFULL + 0));
+        if (ntile > 1) {
+          issue_s(1, 0);
+          tc::mma_commit(bar(SFULL + 1));
         }
         tc::mma_commit(bar(KEMPTY + 0));
       }
-      for (int j = 0; j < nc && ok; ++j) {
-        const int st = j & 1;
+      // chunk j in stage st = j & 1: PV_x(j) and S_x(j+1) per tile
+      auto step = [&](int j, int st) -> bool {
         const bool nxt = j + 1 < nc;
-        ok = tc::mbar_wait(bar(VFULL + st), (j >> 1) & 1);
-        if (ok && nxt) ok = tc::mbar_wait(bar(KFULL + ((j + 1) & 1)), ((j + 1) >> 1) & 1);
-        for (int t = 0; t < ntile && ok; ++t) {
-          ok = tc::mbar_wait(bar(PFULL + t), j & 1);
-          if (!ok) break;
+        TW_BEGIN();
+        bool k = tc::mbar_wait(bar(VFULL + st), (j >> 1) & 1);
+        if (k && nxt) k = tc::mbar_wait(bar(KFULL + (st ^ 1)), ((j + 1) >> 1) & 1);
+        TW_END(w_load);
+        const uint32_t acc = j > 0 ? 1u : 0u;
+#pragma unroll
+        for (int t = 0; t < 2; ++t) {
+          if (!k || t >= ntile) break;
+          TW_BEGIN();
+          k = tc::mbar_wait(bar(PFULL + t), j & 1);
+          TW_END(w_p);
+          if (!k) break;
           tc::fence_after_sync();
-          issue_pv(t, st, j > 0);
+          issue_pv(t, st, acc);
           if (nxt) {
-            issue_s(t, (j + 1) & 1);
+            issue_s(t, st ^ 1);
             tc::mma_commit(bar(SFULL + t));
           }
         }
-        if (!ok) break;
-        if (nxt) tc::mma_commit(bar(KEMPTY + ((j + 1) & 1)));
+        if (!k) return false;
+        if (nxt) tc::mma_commit(bar(KEMPTY + (st ^ 1)));
         tc::mma_commit(bar(VEMPTY + st));
+        return true;
+      };
+      for (int j = 0; j < nc && ok; j += 2) {
+        ok = step(j, 0);
+        if (ok && j + 1 < nc) ok = step(j + 1, 1);
       }
+      TRACE_VAL(22, w_load);
+      TRACE_VAL(24, w_p);
+      TRACE_VAL(29, static_cast<unsigned long long>(nc));
+      TRACE(31);
+#undef TW_BEGIN
+#undef TW_END
       // every MMA of this CTA completes before tensor memory is read or freed
       tc::mma_commit(bar(FIN));
       tc::mbar_wait(bar(FIN), 0);
@@ -416,8 +467,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     const float sl2 = a.scale_log2;
     const int w32 = a.W32;
     const bool tr = (tid & 127) == 0;
+#ifdef LTD_TRACE
+    unsigned long long w_s = 0, t_s0 = 0;
+#endif
     for (int j = 0; j < nc; ++j) {
+#ifdef LTD_TRACE
+      t_s0 = tc::globaltimer();
+#endif
       ok = tc::mbar_wait(bar(SFULL + x), j & 1);
+#ifdef LTD_TRACE
+      w_s += tc::globaltimer() - t_s0;
+#endif
       ok = __all_sync(0xFFFFFFFFu, ok);
       if (tr && j < 2) TRACE(4 + 4 * x + 2 * j);
       if (!ok) break;
@@ -564,6 +624,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       ok = __all_sync(0xFFFFFFFFu, ok);
     }
     if (tr) TRACE(12 + x);
+    if (tr) TRACE_VAL(33 + x, w_s);
     if (!ok && lane == 0) flag_error(a.err, LTD_DEVERR_TIMEOUT);
   }
 

@@ -499,6 +499,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int qq = 0; qq < 4; ++qq)
           vq[qq] = row_ok ? visible32(kbase + 32 * qq, ctx, key_hi, w32, mbits) : 0u;
       }
+      __syncwarp();  // the wait below is warp-collective; the branch above is per row
       tc::tmem_wait_ld128(f);
       if (tr && j == 0 && x == 0) TRACE(27);
       if (!all_vis) {
@@ -613,6 +614,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tc::fence_smem_async();
       }
+      __syncwarp();  // the zeroing loop above runs per thread; the wait is warp-collective
       tc::tmem_wait_st();
       if (tr && j == 0 && x == 0) TRACE(30);
       tc::fence_before_sync();

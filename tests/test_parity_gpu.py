@@ -187,7 +187,7 @@ def test_compaction_race_pattern_and_untouched_rows():
 
 # ---------------------------------------------------------------------- attention
 def _attention_case(name, seed, heads=None, seqs=None, poison=False, workspace=None,
-                    bad_seq=None, **overrides):
+                    bad_seq=None, key_ramp=None, **overrides):
     cfg = wl.config(name, **overrides)
     ci = wl.draw_cycle(cfg, seed, draft_rows=False)
     rng = np.random.default_rng(seed + 5)
@@ -204,6 +204,11 @@ def _attention_case(name, seed, heads=None, seqs=None, poison=False, workspace=N
                 a = par[a]
         masks.append(m)
     q, k, v = wl.draw_attention(cfg, seed, ci.ctx, ci.n_verify)
+    if key_ramp is not None:
+        # key j scaled by 1 + key_ramp * j / S_cap: a row's scores grow (or,
+        # for a negative ramp, shrink) along the cache
+        ramp = 1.0 + key_ramp * np.arange(cfg.s_cap, dtype=np.float32) / cfg.s_cap
+        k = wl.round_to(k * ramp[None, None, :, None], cfg.dtype)
     W32 = (cfg.max_n + 31) // 32
     mw = np.zeros((cfg.batch, cfg.max_n, W32), np.uint32)
     for b in range(cfg.batch):
@@ -266,6 +271,14 @@ def test_attention_32b_sampled_heads():
 
 def test_attention_70b_sampled():
     _attention_case("70b", 0, heads=[3], seqs=[0, 5, 11, 15])
+
+
+def test_attention_scores_growing_along_the_cache():
+    # later chunks pass a row's running max by far more than its P may grow
+    # unchecked: those chunks re-derive P from the chunk's max and rescale O
+    _attention_case("8b", 6, ctx_range=(1500, 1500), n_choices=(40,), key_ramp=40.0)
+    _attention_case("13b", 7, ctx_range=(900, 900), n_choices=(64,), key_ramp=60.0)
+    _attention_case("13b", 8, ctx_range=(900, 900), n_choices=(64,), key_ramp=-0.9)
 
 
 def test_attention_ignores_rows_past_the_tree():

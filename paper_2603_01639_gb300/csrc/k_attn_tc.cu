@@ -105,6 +105,9 @@ struct TcArgs {
   const uint8_t* next_k;  // the next call's caches: L2 prefetch targets (or null)
   const uint8_t* next_v;
   uint32_t* err;
+  // K and V through one tensor map when both caches fit one 4-D map (the
+  // fourth coordinate picks the cache), else one map each
+  int32_t kv_one, kv_wk, kv_wv;
 };
 
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
@@ -155,7 +158,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (tid == 0) {
     tc::tma_prefetch(&tq);
     tc::tma_prefetch(&tk);
-    tc::tma_prefetch(&tv);
+    if (!a.kv_one) tc::tma_prefetch(&tv);
+    TRACE(42);
     tc::mbar_init(bar(QFULL), 1);
     for (int s = 0; s < 2; ++s) {
       tc::mbar_init(bar(KFULL + s), 1);
@@ -174,6 +178,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   // parameters; what follows may read another kernel's output
   grid_wait();
   trigger_dependents();
+  if (tid == 0) TRACE(43);
 
   // ------------------------------------------------------ which unit
   int split = 0, pair, b, kvh;
@@ -237,16 +242,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int st = j & 1;
     tc::mbar_expect_tx(bar(KFULL + st), kTile);
     for (int h = 0; h < 2; ++h)
-      tc::tma_load_3d(base + kOffK + st * kTile + h * kHalf, &tk, bar(KFULL + st), h * 64,
-                      (cs + j) * kBN, kvrow);
+      tc::tma_load_4d(base + kOffK + st * kTile + h * kHalf, &tk, bar(KFULL + st), h * 64,
+                      (cs + j) * kBN, kvrow, a.kv_wk);
     ++nk_issued[st];
   };
   auto issue_v = [&](int j) {
     const int st = j & 1;
     tc::mbar_expect_tx(bar(VFULL + st), kTile);
     for (int h = 0; h < 2; ++h)
-      tc::tma_load_3d(base + kOffV + st * kTile + h * kHalf, &tv, bar(VFULL + st), h * 64,
-                      (cs + j) * kBN, kvrow);
+      tc::tma_load_4d(base + kOffV + st * kTile + h * kHalf, a.kv_one ? &tk : &tv, bar(VFULL + st),
+                      h * 64, (cs + j) * kBN, kvrow, a.kv_wv);
     ++nv_issued[st];
   };
   auto issue_first = [&]() {
@@ -261,7 +266,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     TRACE(20);
     for (; n_issued < min(ce - cs, 2); ++n_issued) {
       issue_k(n_issued);
+      if (n_issued == 0) TRACE(44);
       issue_v(n_issued);
+      if (n_issued == 0) TRACE(45);
     }
     TRACE(17);
   };
@@ -903,6 +910,22 @@ bool encode_tmap_bf16_3d(CUtensorMap* map, const void* base, uint64_t d0, uint64
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+namespace {
+bool encode_tmap_bf16_4d(CUtensorMap* map, const void* base, uint64_t d0, uint64_t d1, uint64_t d2,
+                         uint64_t d3, uint64_t stride1, uint64_t stride2, uint64_t stride3, uint32_t b0,
+                         uint32_t b1, uint32_t b2, uint32_t b3) {
+  EncodeFn fn = encode_fn();
+  if (fn == nullptr) return false;
+  const cuuint64_t dims[4] = {d0, d1, d2, d3};
+  const cuuint64_t strides[3] = {stride1, stride2, stride3};
+  const cuuint32_t box[4] = {b0, b1, b2, b3};
+  const cuuint32_t estr[4] = {1, 1, 1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+}  // namespace
+
 bool attn_tc_supported(const AttnParams& p, ltd_dtype dtype) {
   if (dtype != LTD_BF16 || p.d != kD || p.hkv < 1 || p.hq % p.hkv != 0) return false;
   const int G = p.hq / p.hkv;
@@ -958,12 +981,25 @@ cudaError_t launch_attn_tc(const AttnParams& p, cudaStream_t s) {
   if (!encode_tmap_bf16_3d(&tq, p.q, kD, p.hq, static_cast<uint64_t>(p.batch) * p.n_max, row,
                            row * p.hq, 64, a.G, kBM / a.G))
     return cudaErrorInvalidValue;
-  if (!encode_tmap_bf16_3d(&tk, p.k, kD, p.s_cap, static_cast<uint64_t>(p.batch) * p.hkv, row,
-                           row * p.s_cap, 64, kBN, 1))
-    return cudaErrorInvalidValue;
-  if (!encode_tmap_bf16_3d(&tv, p.v, kD, p.s_cap, static_cast<uint64_t>(p.batch) * p.hkv, row,
-                           row * p.s_cap, 64, kBN, 1))
-    return cudaErrorInvalidValue;
+  // One map for both caches saves the kernel a descriptor fetch, which a
+  // launch otherwise waits for behind its own first loads.
+  const uint64_t rows_kv = static_cast<uint64_t>(p.batch) * p.hkv;
+  const uint64_t ka = reinterpret_cast<uint64_t>(p.k), va = reinterpret_cast<uint64_t>(p.v);
+  const uint64_t lo = ka < va ? ka : va, gap = ka < va ? va - ka : ka - va;
+  a.kv_one = gap > 0 && gap % 16 == 0 && gap < (1ull << 40) &&
+             encode_tmap_bf16_4d(&tk, reinterpret_cast<const void*>(lo), kD, p.s_cap, rows_kv, 2, row,
+                                 row * p.s_cap, gap, 64, kBN, 1, 1);
+  if (a.kv_one) {
+    a.kv_wk = ka < va ? 0 : 1;
+    a.kv_wv = 1 - a.kv_wk;
+    tv = tk;
+  } else {
+    const uint64_t whole = row * p.s_cap * rows_kv;
+    a.kv_wk = a.kv_wv = 0;
+    if (!encode_tmap_bf16_4d(&tk, p.k, kD, p.s_cap, rows_kv, 1, row, row * p.s_cap, whole, 64, kBN, 1, 1) ||
+        !encode_tmap_bf16_4d(&tv, p.v, kD, p.s_cap, rows_kv, 1, row, row * p.s_cap, whole, 64, kBN, 1, 1))
+      return cudaErrorInvalidValue;
+  }
   cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(kSmemBytes));
   if (e != cudaSuccess) return e;

@@ -36,7 +36,7 @@ constexpr int kMaxVec = 8;   // 16-byte vectors per thread
 
 // Optional phase timestamps for performance work (off in normal builds).
 #ifdef LTD_TRACE
-__device__ unsigned long long g_expand_trace[4096][8];
+__device__ unsigned long long g_expand_trace[4096][16];
 #define TRACE(slot)                                                                  \
   do {                                                                               \
     const int cta_ = blockIdx.x + gridDim.x * (blockIdx.y + gridDim.y * blockIdx.z); \
@@ -83,19 +83,6 @@ __device__ __forceinline__ float warp_sort_desc_f(float v) {
   }
   return v;
 }
-// The 32 largest of two descending lane-sorted float lists, descending.
-__device__ __forceinline__ float warp_merge_desc_f(float a, float b) {
-  const int lane = threadIdx.x & 31;
-  const float br = __shfl_sync(0xFFFFFFFFu, b, 31 - lane);
-  float v = fmaxf(a, br);
-#pragma unroll
-  for (int stride = 16; stride > 0; stride >>= 1) {
-    const float o = __shfl_xor_sync(0xFFFFFFFFu, v, stride);
-    v = ((lane & stride) == 0) ? fmaxf(v, o) : fminf(v, o);
-  }
-  return v;
-}
-
 // Tree merge of one descending 32-entry list per warp (stage[w][lane]) into
 // stage[0][0..32).  All threads call; returns after a barrier.
 template <typename V, V (*Merge)(V, V)>
@@ -113,11 +100,54 @@ __device__ __forceinline__ void tree_merge(V* stage) {
   __syncthreads();
 }
 
+// Element j of a 16-byte vector of T, as float (j a compile-time constant).
+template <typename T>
+__device__ __forceinline__ float elem(const uint4& r, int j);
+template <>
+__device__ __forceinline__ float elem<float>(const uint4& r, int j) {
+  const uint32_t w = j == 0 ? r.x : (j == 1 ? r.y : (j == 2 ? r.z : r.w));
+  return __uint_as_float(w);
+}
+template <>
+__device__ __forceinline__ float elem<__nv_bfloat16>(const uint4& r, int j) {
+  const int q = j >> 1;
+  const uint32_t w = q == 0 ? r.x : (q == 1 ? r.y : (q == 2 ? r.z : r.w));
+  return __uint_as_float((j & 1) ? (w & 0xFFFF0000u) : (w << 16));
+}
+// Raw bits of element i of x, or of -inf past the end.
+__device__ __forceinline__ uint32_t raw_or_ninf(const float* x, int64_t i, int64_t hi) {
+  return i < hi ? __float_as_uint(x[i]) : 0xFF800000u;
+}
+__device__ __forceinline__ uint32_t raw_or_ninf(const __nv_bfloat16* x, int64_t i, int64_t hi) {
+  return i < hi ? static_cast<uint32_t>(__bfloat16_as_ushort(x[i])) : 0xFF80u;
+}
+template <typename T>
+__device__ __forceinline__ uint4 load_tail(const T* x, int64_t i, int64_t hi) {
+  uint32_t w[4];
+  if constexpr (sizeof(T) == 4) {
+#pragma unroll
+    for (int q = 0; q < 4; ++q) w[q] = raw_or_ninf(x, i + q, hi);
+  } else {
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      w[q] = raw_or_ninf(x, i + 2 * q, hi) | (raw_or_ninf(x, i + 2 * q + 1, hi) << 16);
+  }
+  return make_uint4(w[0], w[1], w[2], w[3]);
+}
+// A streaming 16-byte load that the compiler may neither repeat nor move.
+__device__ __forceinline__ uint4 ld_stream16_once(const void* p) {
+  uint4 r;
+  asm volatile("ld.global.cs.v4.u32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+               : "l"(p));
+  return r;
+}
+
 struct ExpandShared {
   uint64_t stage[kNW * kWarp];
   float fstage[kNW * kWarp];
   uint64_t cand[kCand];
-  float red[2 * kNW];
+  float red[2 * kNW + 1];
   // published to the cluster: the chunk's sorted top list and (max, sum exp)
   uint64_t top[kWarp];
   float2 ms;
@@ -126,6 +156,7 @@ struct ExpandShared {
   float2 peer_ms[kMaxChunks];
   float thr;
   int n_cand;
+  int wcnt[kNW];
   int last;
 };
 
@@ -152,62 +183,100 @@ __global__ void __launch_bounds__(kNT) expand_kernel(const ExpandParams p) {
                (static_cast<int64_t>(b) * p.rows_per_seq + row) * p.vocab;
   const int64_t lo = static_cast<int64_t>(ch) * p.chunk_elems;
   const int64_t hi = min(lo + p.chunk_elems, p.vocab);
-  float xv[U][VEC];
+  // the chunk stays in registers as loaded (16 bytes per vector) and is
+  // unpacked where it is used
+  uint4 raw[U];
 #pragma unroll
   for (int u = 0; u < U; ++u) {
     const int64_t i = lo + (static_cast<int64_t>(u) * kNT + tid) * VEC;
-    if (i + VEC <= hi) {
-      unpack16(ld_stream16(x + i), xv[u], static_cast<const T*>(nullptr));
-    } else {
-#pragma unroll
-      for (int j = 0; j < VEC; ++j) xv[u][j] = (i + j < hi) ? to_f<T>(x[i + j]) : -CUDART_INF_F;
-    }
+    raw[u] = (i + VEC <= hi) ? ld_stream16_once(x + i) : load_tail(x, i, hi);
   }
   float tmax = -CUDART_INF_F;
 #pragma unroll
   for (int u = 0; u < U; ++u)
 #pragma unroll
-    for (int j = 0; j < VEC; ++j) tmax = fmaxf(tmax, xv[u][j]);
+    for (int j = 0; j < VEC; ++j) tmax = fmaxf(tmax, elem<T>(raw[u], j));
   float tsum = 0.f;
   if (tmax > -CUDART_INF_F) {
 #pragma unroll
     for (int u = 0; u < U; ++u)
 #pragma unroll
-      for (int j = 0; j < VEC; ++j) tsum += __expf(xv[u][j] - tmax);
+      for (int j = 0; j < VEC; ++j) tsum += __expf(elem<T>(raw[u], j) - tmax);
   }
   if (tid == 0) TRACE(1);
-  float m = tmax, s = tsum;
-  block_ms<kNT>(m, s, sh.red);
-
   // ---- stage 2: T = k-th largest of the 32 half-warp maxima, a lower bound
-  // of the chunk's k-th largest logit (k half-warps hold an element >= T)
+  // of the chunk's k-th largest logit (k half-warps hold an element >= T);
+  // the largest of them is the chunk's max M
   float hm = tmax;
 #pragma unroll
   for (int o = 8; o > 0; o >>= 1) hm = fmaxf(hm, __shfl_xor_sync(0xFFFFFFFFu, hm, o));
   if ((lane & 15) == 0) sh.fstage[warp * 2 + (lane >> 4)] = hm;
-  if (tid == 0) sh.n_cand = 0;
   __syncthreads();
   if (warp == 0) {
     const float v = warp_sort_desc_f(sh.fstage[lane]);  // 2 * kNW = 32 half-warps
     if (lane == k - 1) sh.thr = v;
+    if (lane == 0) sh.red[2 * kNW] = v;  // the chunk max
   }
+  if (tid == 0) TRACE(10);
   __syncthreads();
+  if (tid == 0) TRACE(11);
   const float thr = sh.thr;
+  const float cmax = sh.red[2 * kNW];
+  // the chunk's sum of exp(x - cmax): one rescale per thread, then a warp sum
+  {
+    float e = (tmax > -CUDART_INF_F) ? tsum * __expf(tmax - cmax) : 0.f;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) e += __shfl_xor_sync(0xFFFFFFFFu, e, o);
+    if (lane == 0) sh.red[warp] = e;
+  }
 
-  // ---- stage 3: the candidates >= T, ranked exactly by (logit desc, token asc)
+  // ---- stage 3: the candidates >= T, ranked exactly by (logit desc, token asc);
+  // each thread marks its elements >= T, the warps' counts give every
+  // thread its slots (no atomics)
+  uint64_t cmask = 0ull;
   if (tmax >= thr) {
 #pragma unroll
     for (int u = 0; u < U; ++u)
 #pragma unroll
       for (int j = 0; j < VEC; ++j) {
         const int64_t i = lo + (static_cast<int64_t>(u) * kNT + tid) * VEC + j;
-        if (xv[u][j] >= thr && i < hi) {
-          const int slot = atomicAdd(&sh.n_cand, 1);
-          if (slot < kCand) sh.cand[slot] = make_key(xv[u][j], static_cast<uint32_t>(i));
-        }
+        if (elem<T>(raw[u], j) >= thr && i < hi) cmask |= 1ull << (u * VEC + j);
       }
   }
+  const int cnt = __popcll(cmask);
+  int incl = cnt;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+    if (lane >= o) incl += y;
+  }
+  if (lane == 31) sh.wcnt[warp] = incl;
   __syncthreads();
+  {
+    int below = (lane < warp) ? sh.wcnt[lane] : 0;  // kNW <= 32 warps
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) below += __shfl_xor_sync(0xFFFFFFFFu, below, o);
+    int slot = below + incl - cnt;
+    if (cmask != 0ull) {
+#pragma unroll
+      for (int u = 0; u < U; ++u)
+#pragma unroll
+        for (int j = 0; j < VEC; ++j)
+          if ((cmask >> (u * VEC + j)) & 1ull) {
+            const int64_t i = lo + (static_cast<int64_t>(u) * kNT + tid) * VEC + j;
+            if (slot < kCand) sh.cand[slot] = make_key(elem<T>(raw[u], j), static_cast<uint32_t>(i));
+            ++slot;
+          }
+    }
+  }
+  if (tid < kWarp) {
+    int t = tid < kNW ? sh.wcnt[tid] : 0;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xFFFFFFFFu, t, o);
+    if (tid == 0) sh.n_cand = t;
+  }
+  __syncthreads();
+  if (tid == 0) TRACE(12);
   const int nc = sh.n_cand;
   if (nc <= kCand) {
     // typically a few dozen: one warp ranks them
@@ -229,51 +298,60 @@ __global__ void __launch_bounds__(kNT) expand_kernel(const ExpandParams p) {
 #pragma unroll
       for (int j = 0; j < VEC; ++j) {
         const int64_t i = lo + (static_cast<int64_t>(u) * kNT + tid) * VEC + j;
-        wt.offer(i < hi ? make_key(xv[u][j], static_cast<uint32_t>(i)) : 0ull, k);
+        wt.offer(i < hi ? make_key(elem<T>(raw[u], j), static_cast<uint32_t>(i)) : 0ull, k);
       }
     sh.stage[warp * kWarp + lane] = wt.v;
     tree_merge<uint64_t, warp_merge_desc>(sh.stage);
     if (tid < kWarp) sh.top[tid] = sh.stage[tid];
   }
-  if (tid == 0) {
-    sh.ms = make_float2(m, s);
-    TRACE(2);
+  if (warp == 1) {
+    // (max, sum exp) of the chunk from the warps' sums
+    float csum = lane < kNW ? sh.red[lane] : 0.f;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) csum += __shfl_xor_sync(0xFFFFFFFFu, csum, o);
+    if (lane == 0) sh.ms = make_float2(cmax, csum);
   }
+  if (tid == 0) TRACE(2);
 
   // ---- row: rank 0 gathers the chunk results of its cluster (warp 0 reads
-  // every peer's list into registers; the merges follow once the peers
-  // may leave)
+  // every peer's list and merges them) before the barrier that lets the
+  // peers leave
   const int C = p.chunks;
   tc::cluster_sync();
-  uint64_t lists[kMaxChunks];
   if (ch == 0 && warp == 0) {
+    uint64_t lists[kMaxChunks];
 #pragma unroll
     for (int c = 0; c < kMaxChunks; ++c)
       lists[c] = c < C ? tc::ld_cluster_u64(tc::mapa(tc::smem_u32(&sh.top[lane]), c)) : 0ull;
-    if (lane < C) sh.peer_ms[lane] = tc::ld_cluster_f2(tc::mapa(tc::smem_u32(&sh.ms), lane));
-  }
-  // no CTA leaves while rank 0 may still read its shared memory
-  tc::cluster_sync();
-  if (ch != 0) return;
-  if (tid == 0) TRACE(3);
-  if (warp == 0) {
+    const float2 pm = lane < C ? tc::ld_cluster_f2(tc::mapa(tc::smem_u32(&sh.ms), lane))
+                               : make_float2(-CUDART_INF_F, 0.f);
     uint64_t v = lists[0];
 #pragma unroll
     for (int c = 1; c < kMaxChunks; ++c)
       if (c < C) v = warp_merge_desc(v, lists[c]);
     sh.stage[lane] = v;
-    if (lane == 0) {
-      float M = -CUDART_INF_F, S = 0.f;
-      for (int c = 0; c < C; ++c) ms_merge(M, S, sh.peer_ms[c].x, sh.peer_ms[c].y);
-      sh.red[0] = M + logf(S);
+    // (max, sum exp) of the row from the lanes' chunk pairs
+    float M = pm.x, S = pm.y;
+#pragma unroll
+    for (int o = 1; o < kMaxChunks; o <<= 1) {
+      const float M2 = __shfl_xor_sync(0xFFFFFFFFu, M, o), S2 = __shfl_xor_sync(0xFFFFFFFFu, S, o);
+      ms_merge(M, S, M2, S2);
     }
+    if (lane == 0) sh.red[0] = M + logf(S);
   }
-  __syncthreads();
+  // no CTA leaves while rank 0 may still read its shared memory; the
+  // barrier also publishes warp 0's results to the rest of rank 0
+  tc::cluster_sync();
+  if (ch != 0) return;
+  if (tid == 0) TRACE(3);
+  if (tid == 0) TRACE(7);
   const float lse = sh.red[0];
 
   const int64_t nb = static_cast<int64_t>(b) * p.max_nodes;
   const int parent = (p.level == 1) ? 0 : __ldcg(&p.frontier[b * k + f]);
+  if (tid == 0) TRACE(8);
   const float cum_p = (p.level == 1) ? 0.f : __ldcg(&p.cum[nb + parent]);
+  if (tid == 0) TRACE(9);
   const int base = (p.level == 1) ? 1 : 1 + k + (p.level - 2) * k * k;
   if (tid < k) {
     const uint64_t key = sh.stage[tid];
@@ -314,13 +392,18 @@ __global__ void __launch_bounds__(kNT) expand_kernel(const ExpandParams p) {
   if (pool <= 4 * kWarp) {
     // a small pool: one warp, no block barriers
     if (warp == 0) {
+      // all of the pool's loads go out before the first is needed
+      uint64_t keys[4];
+#pragma unroll
+      for (int r = 0; r < 4; ++r) {
+        const int j = r * kWarp + lane;
+        keys[r] = j < pool ? make_key(__ldcg(&p.cum[nb + base + j]), static_cast<uint32_t>(base + j)) : 0ull;
+      }
       WarpTopK pt;
       pt.init();
-      for (int j0 = 0; j0 < pool; j0 += kWarp) {
-        const int j = j0 + lane;
-        const int id = base + j;
-        pt.offer(j < pool ? make_key(__ldcg(&p.cum[nb + id]), static_cast<uint32_t>(id)) : 0ull, k);
-      }
+#pragma unroll
+      for (int r = 0; r < 4; ++r)
+        if (r * kWarp < pool) pt.offer(keys[r], k);
       if (lane < k) p.frontier[b * k + lane] = static_cast<int32_t>(key_index(pt.v));
     }
   } else {
@@ -426,7 +509,7 @@ extern "C" int ltd_expand_trace_read(unsigned long long* host, int n) {
              : 1;
 }
 extern "C" int ltd_expand_trace_clear() {
-  static unsigned long long zeros[4096 * 8];
+  static unsigned long long zeros[4096 * 16];
   return cudaMemcpyToSymbol(g_expand_trace, zeros, sizeof(zeros)) == cudaSuccess ? 0 : 1;
 }
 #endif

@@ -499,15 +499,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::Frag128 f;
       float mref = m;
       float2 ls2 = make_float2(0.f, 0.f);
-      tc::tmem_ld128(t_s, f);
       uint32_t vq[4] = {0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu};
       if (!all_vis) {
 #pragma unroll
         for (int qq = 0; qq < 4; ++qq)
           vq[qq] = row_ok ? visible32(kbase + 32 * qq, ctx, key_hi, w32, mbits) : 0u;
       }
-      __syncwarp();  // the wait below is warp-collective; the branch above is per row
-      tc::tmem_wait_ld128(f);
+      __syncwarp();  // the load below is warp-collective; the branch above is per row
+      tc::tmem_ld128_sync(t_s, f);
       if (tr && j == 0 && x == 0) TRACE(27);
       if (!all_vis) {
 #pragma unroll
@@ -558,8 +557,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll 1
         for (int qq = 0; qq < 4; ++qq) {
           tc::Frag32 g;
-          tc::tmem_ld32(t_s + 32 * qq, g);
-          tc::tmem_wait_ld(g);
+          tc::tmem_ld32_sync(t_s + 32 * qq, g);
           const uint32_t v = qq == 0 ? vq[0] : (qq == 1 ? vq[1] : (qq == 2 ? vq[2] : vq[3]));
 #pragma unroll
           for (int c = 0; c < 32; ++c)
@@ -572,8 +570,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll 1
         for (int qq = 0; qq < 4; ++qq) {
           tc::Frag32 g;
-          tc::tmem_ld32(t_s + 32 * qq, g);
-          tc::tmem_wait_ld(g);
+          tc::tmem_ld32_sync(t_s + 32 * qq, g);
           const uint32_t v = qq == 0 ? vq[0] : (qq == 1 ? vq[1] : (qq == 2 ? vq[2] : vq[3]));
           tc::Frag16 pf;
 #pragma unroll
@@ -596,8 +593,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll 1
         for (int qq = 0; qq < 4; ++qq) {
           tc::Frag32 o;
-          tc::tmem_ld32(t_o + 32 * qq, o);
-          tc::tmem_wait_ld(o);
+          tc::tmem_ld32_sync(t_o + 32 * qq, o);
 #pragma unroll
           for (int c = 0; c < 32; ++c) o.r[c] = __float_as_uint(__uint_as_float(o.r[c]) * alpha);
           tc::tmem_st32(t_o + 32 * qq, o);
@@ -658,8 +654,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc::Frag128 o;
   if (loaded) {
     tc::fence_after_sync();
-    tc::tmem_ld128(tmem + 2 * kBN + x * kD + ((32u * (warp & 3)) << 16), o);
-    tc::tmem_wait_ld128(o);
+    tc::tmem_ld128_sync(tmem + 2 * kBN + x * kD + ((32u * (warp & 3)) << 16), o);
   }
   if (row_ok) {
     const bool have = loaded && l > 0.f;

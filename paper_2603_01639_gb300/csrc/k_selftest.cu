@@ -71,8 +71,7 @@ __global__ void __launch_bounds__(128) umma_selftest_kernel(const __grid_constan
   const int row = tid;
   for (int q = 0; q < 4; ++q) {
     tc::Frag32 f;
-    tc::tmem_ld32(tmem + ((32u * warp) << 16) + 32u * q, f);
-    tc::tmem_wait_ld(f);
+    tc::tmem_ld32_sync(tmem + ((32u * warp) << 16) + 32u * q, f);
     for (int j = 0; j < 32; ++j) C[row * 128 + 32 * q + j] = ok ? __uint_as_float(f.r[j]) : 0.f;
   }
   tc::fence_before_sync();

@@ -548,7 +548,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // P above 2^8 means the chunk max passed m + 8
       const bool over = max(pmax2 & 0xFFFFu, pmax2 >> 16) > kPMaxBits;
       if (!__any_sync(0xFFFFFFFFu, over)) {
-        tc::tmem_st64_lo(t_s, f);
+        tc::tmem_st64_lo_sync(t_s, f);
       } else {
         // S is still intact in tensor memory: take the chunk's max, then
         // derive P again, 32 columns at a time (P columns 16 qq .. 16 qq + 15
@@ -582,7 +582,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             ls2 = __fadd2_rn(ls2, pp);
             pf.r[c] = pack_bf16(pp.x, pp.y);
           }
-          tc::tmem_st16(t_s + 16 * qq, pf);
+          tc::tmem_st16_sync(t_s + 16 * qq, pf);
         }
       }
       if (tr && j == 0 && x == 0) TRACE(28);
@@ -596,7 +596,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc::tmem_ld32_sync(t_o + 32 * qq, o);
 #pragma unroll
           for (int c = 0; c < 32; ++c) o.r[c] = __float_as_uint(__uint_as_float(o.r[c]) * alpha);
-          tc::tmem_st32(t_o + 32 * qq, o);
+          tc::tmem_st32_sync(t_o + 32 * qq, o);
         }
       }
       m = mref;

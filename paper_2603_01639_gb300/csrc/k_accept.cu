@@ -9,11 +9,14 @@
 //    marks from slot 0; the argmax at the end is the bonus token;
 //  - stochastic (T = 1): SpecInfer-style multi-candidate speculative
 //    sampling.  Each CTA holds one vocabulary slice of p (target) and q
-//    (draft) in shared memory.  Child i of the current slot is accepted if
+//    (draft) in its threads' registers.  Child i of the current slot is accepted if
 //    r_i q(x_i) < p(x_i) -- every CTA evaluates that test identically --
 //    else p <- max(p - q, 0) / Z, with Z summed over the cluster through
-//    distributed shared memory (partials added in rank order, so every CTA
-//    holds the same Z).  With no child accepted the bonus is a Gumbel-max
+//    distributed shared memory (every warp adds all warp partials of the
+//    cluster in one fixed order, so every CTA holds the same Z).  The
+//    children's p(x), q(x) are loaded with the slice; a rejection costs one
+//    cluster barrier and one pass over the slice, which also takes the next
+//    rejection's partial sum.  With no child accepted the bonus is a Gumbel-max
 //    draw from p, reduced over the cluster the same way.
 // kv_compact_kernel: grid (KV heads, layers x {K, V}, batch); each CTA stages
 // the accepted rows in shared memory, then writes them to ctx+t, so a row
@@ -30,6 +33,7 @@ constexpr int kNT = 512;
 constexpr int kNW = kNT / kWarp;
 constexpr int64_t kSliceMax = 16384;  // vocabulary elements per walk CTA
 constexpr int kMaxWalkCluster = static_cast<int>(kAcceptMaxVocab / kSliceMax);
+static_assert(LTD_MAX_N <= kNT, "one verified slot per walk thread");
 
 template <typename T>
 __global__ void __launch_bounds__(kNT) accept_rows_kernel(const AcceptParams p) {
@@ -89,15 +93,69 @@ __global__ void __launch_bounds__(kNT) accept_rows_kernel(const AcceptParams p) 
       }
     }
   }
-  block_ms<kNT>(m, s, red);
-  best = block_max_u64<kNT>(best, redk);
+  // the chunk's max first (no exponentials), then each thread's sum rescaled
+  // to it once; only thread 0 needs the results
+  const int lane = tid & 31, warp = tid >> 5;
+  float wm = m;
+  uint64_t wb = best;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    wm = fmaxf(wm, __shfl_xor_sync(0xFFFFFFFFu, wm, o));
+    const uint64_t ob = __shfl_xor_sync(0xFFFFFFFFu, wb, o);
+    wb = ob > wb ? ob : wb;
+  }
+  if (lane == 0) {
+    red[warp] = wm;
+    redk[warp] = wb;
+  }
+  __syncthreads();
+  float M = red[0];
+#pragma unroll
+  for (int w = 1; w < kNW; ++w) M = fmaxf(M, red[w]);
+  float e = (m > -CUDART_INF_F) ? s * __expf(m - M) : 0.f;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) e += __shfl_xor_sync(0xFFFFFFFFu, e, o);
+  __syncthreads();  // every thread has read the maxima
+  if (lane == 0) red[warp] = e;
+  __syncthreads();
   if (tid == 0) {
+    float S = 0.f;
+    uint64_t B = 0ull;
+    for (int w = 0; w < kNW; ++w) {
+      S += red[w];
+      B = redk[w] > B ? redk[w] : B;
+    }
+    m = M;
+    s = S;
+    best = B;
     AcceptRecord* r = p.rec + (static_cast<int64_t>(b) * p.n_max + i) * p.chunks + ch;
     r->m = m;
     r->s = s;
     r->key = best;
   }
 }
+
+// Optional walk timeline for performance work (off in normal builds):
+// per sequence, (event, globaltimer) pairs from rank 0's thread 0.
+#ifdef LTD_TRACE
+__device__ unsigned long long g_walk_trace[64][128];
+__device__ int g_walk_trace_n[64];
+#define WTRACE(ev)                                                              \
+  do {                                                                          \
+    if (rank == 0 && tid == 0 && b < 64) {                                      \
+      const int i_ = g_walk_trace_n[b];                                         \
+      if (i_ < 64) {                                                            \
+        g_walk_trace[b][2 * i_] = (ev);                                         \
+        g_walk_trace[b][2 * i_ + 1] = tc::globaltimer();                        \
+        g_walk_trace_n[b] = i_ + 1;                                             \
+      }                                                                         \
+    }                                                                           \
+  } while (0)
+#else
+#define WTRACE(ev) \
+  do {             \
+  } while (0)
+#endif
 
 struct WalkShared {
   int32_t node[LTD_MAX_N];
@@ -110,19 +168,33 @@ struct WalkShared {
   int32_t path[LTD_MAX_DEPTH + 1];
   float red[2 * kNW];
   uint64_t redk[kNW];
-  float cell_z[2];          // cluster exchange cells, double-buffered by round
+  float kp[LTD_MAX_N];      // p and q of the current slot's children
+  float kq[LTD_MAX_N];
+  float wpart[2][kMaxWalkCluster][kNW];  // every CTA's warp sums, by round parity
+  int wcnt[kNW];
   uint64_t cell_key[2];
   float2 cell_ms;
   int n_kids;
 };
 
-// Sum of every cluster CTA's `v` (rank order, so all CTAs get the same bits).
-__device__ __forceinline__ float cluster_sum(float v, float* cells, int& round, int C) {
+// Sum over the cluster of every thread's `v`: every warp pushes its sum into
+// every CTA's table ([round parity][rank][warp]) before the cluster barrier,
+// then every warp adds its own CTA's table in one fixed order, so every
+// thread of every CTA holds the same bits.  One cluster barrier, no remote
+// reads after it.
+__device__ __forceinline__ float cluster_sum_warps(float v, float (*wpart)[kMaxWalkCluster][kNW],
+                                                  int& round, int C) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int c = round & 1;
-  if (threadIdx.x == 0) cells[c] = v;
+  const uint32_t rank = tc::cluster_rank();
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
+  if (lane < C) tc::st_cluster_f1(tc::mapa(tc::smem_u32(&wpart[c][rank][warp]), lane), v);
   tc::cluster_sync();
   float t = 0.f;
-  for (int r = 0; r < C; ++r) t += tc::ld_cluster_f1(tc::mapa(tc::smem_u32(&cells[c]), r));
+  for (int e = lane; e < C * kNW; e += kWarp) t += wpart[c][e / kNW][e % kNW];
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xFFFFFFFFu, t, o);
   ++round;
   return t;
 }
@@ -142,13 +214,10 @@ __device__ __forceinline__ uint64_t cluster_max_u64(uint64_t v, uint64_t* cells,
 
 template <typename T>
 __global__ void __launch_bounds__(kNT) accept_walk_kernel(const AcceptParams p, int C,
-                                                          int64_t slice) {
-  extern __shared__ float dyn[];
+                                                          int64_t slice, int vec_ok) {
   __shared__ WalkShared sh;
   grid_wait();
   trigger_dependents();
-  float* ps = dyn;
-  float* qs = dyn + slice;
   const int rank = blockIdx.x, b = blockIdx.y, tid = threadIdx.x;
   const int N = p.n_verify[b];
   const int mode = p.mode[b];
@@ -230,19 +299,43 @@ __global__ void __launch_bounds__(kNT) accept_walk_kernel(const AcceptParams p, 
   const T* draft = reinterpret_cast<const T*>(p.draft);
   const int64_t lo = static_cast<int64_t>(rank) * slice;
   const int64_t hi = min(lo + slice, V);
+  // The slice lives in registers: KG groups of VEC elements per thread.
+  // With 16-byte-aligned rows (vec_ok) group k of a thread is the VEC
+  // consecutive elements at lo + (k kNT + tid) VEC, loaded with one 16-byte
+  // load; otherwise element (k, j) is lo + (k VEC + j) kNT + tid.
+  constexpr int VEC = 16 / static_cast<int>(sizeof(T));
+  constexpr int KG = static_cast<int>(kSliceMax) / (VEC * kNT);
+  static_assert(KG * VEC * kNT == kSliceMax, "slices split evenly over the threads");
+  auto el = [&](int k, int j) -> int64_t {
+    return vec_ok ? lo + (static_cast<int64_t>(k) * kNT + tid) * VEC + j
+                  : lo + (static_cast<int64_t>(k) * VEC + j) * kNT + tid;
+  };
+  float pr[KG][VEC], qr[KG][VEC];
   int round = 0, cur = 0, len = 0, bonus = -1;
   if (tid == 0) sh.path[0] = 0;
+  const int lane = tid & 31, warp = tid >> 5;
+  WTRACE(0);
   for (int step = 0; step <= p.max_depth; ++step) {
     const int u = sh.node[cur];
     const float lse_t = row_lse(cur);
-    if (tid == 0) {
-      int nk = 0;
-      for (int j = cur + 1; j < N; ++j)
-        if (sh.pslot[j] == cur) sh.kids[nk++] = j;
-      sh.n_kids = nk;
+    WTRACE(1);
+    // the current slot's children, in slot order (one slot per thread)
+    {
+      const bool kid = tid < N && tid > cur && sh.pslot[tid] == cur;
+      const unsigned bal = __ballot_sync(0xFFFFFFFFu, kid);
+      if (lane == 0) sh.wcnt[warp] = __popc(bal);
+      __syncthreads();
+      int before = 0, total = 0;
+      for (int w = 0; w < kNW; ++w) {
+        before += (w < warp) ? sh.wcnt[w] : 0;
+        total += sh.wcnt[w];
+      }
+      if (kid) sh.kids[before + __popc(bal & ((1u << lane) - 1u))] = tid;
+      if (tid == 0) sh.n_kids = total;
     }
     __syncthreads();
     const int nk = sh.n_kids;
+    WTRACE(2 + 100 * nk);
     const T* trow = target + (static_cast<int64_t>(b) * p.n_max + cur) * V;
     const T* qrow = nullptr;
     float lse_q = 0.f;
@@ -250,35 +343,83 @@ __global__ void __launch_bounds__(kNT) accept_walk_kernel(const AcceptParams p, 
       qrow = draft + (static_cast<int64_t>(b) * p.rows_per_seq + p.xrow[nb + u]) * V;
       lse_q = p.xlse[nb + u];
     }
-    for (int64_t v = lo + tid; v < hi; v += kNT) {
-      ps[v - lo] = __expf(to_f<T>(trow[v]) - lse_t);
-      if (nk > 0) qs[v - lo] = __expf(to_f<T>(qrow[v]) - lse_q);
+    // the children's p(x), q(x) and this CTA's slice, all loads at once; the
+    // slice pass also takes this thread's share of the first residual sum.
+    // The slice goes 16 bytes of logits per thread-step where the rows allow
+    // it (groups of VEC elements), the rest one element at a time.
+    if (tid < nk) {
+      const int x = sh.tok[sh.kids[tid]];
+      sh.kp[tid] = __expf(to_f<T>(trow[x]) - lse_t);
+      sh.kq[tid] = __expf(to_f<T>(qrow[x]) - lse_q);
+    }
+    float part = 0.f;
+    {
+      uint4 rt[KG], rq[KG];
+#pragma unroll
+      for (int k = 0; k < KG; ++k) {
+        // every load of the slice is issued before the first is used
+        rt[k] = make_uint4(0u, 0u, 0u, 0u);
+        rq[k] = make_uint4(0u, 0u, 0u, 0u);
+        if (vec_ok && el(k, 0) < hi) {
+          rt[k] = ld_stream16_once(trow + el(k, 0));
+          if (nk > 0) rq[k] = ld_stream16_once(qrow + el(k, 0));
+        }
+      }
+#pragma unroll
+      for (int k = 0; k < KG; ++k)
+#pragma unroll
+        for (int j = 0; j < VEC; ++j) {
+          const int64_t v = el(k, j);
+          const bool in = v < hi;
+          float tv = 0.f, dv = 0.f;
+          if (vec_ok) {
+            tv = elem<T>(rt[k], j);
+            dv = elem<T>(rq[k], j);
+          } else if (in) {
+            tv = to_f<T>(trow[v]);
+            if (nk > 0) dv = to_f<T>(qrow[v]);
+          }
+          pr[k][j] = 0.f;
+          qr[k][j] = 0.f;
+          if (in) {
+            pr[k][j] = __expf(tv - lse_t);
+            if (nk > 0) qr[k][j] = __expf(dv - lse_q);
+          }
+          part += fmaxf(pr[k][j] - qr[k][j], 0.f);
+        }
     }
     __syncthreads();
+    WTRACE(3);
     int accepted = -1, nz = 0;
     const uint64_t pre = hash_prefix(p.seed, b, p.cycle, kStreamRatio, cur);
     for (int c = 0; c < nk; ++c) {
-      const int x = sh.tok[sh.kids[c]];
       // p(x) after nz rejections, by the same arithmetic as the slice update
-      float px = __expf(to_f<T>(trow[x]) - lse_t);
-      const float qx = __expf(to_f<T>(qrow[x]) - lse_q);
+      // (sh.Z holds 1 / Z, or 0 where the residual was empty)
+      float px = sh.kp[c];
+      const float qx = sh.kq[c];
       for (int jz = 0; jz < nz; ++jz)
-        if (sh.Z[jz] > 0.f) px = fmaxf(px - qx, 0.f) / sh.Z[jz];
+        if (sh.Z[jz] > 0.f) px = fmaxf(px - qx, 0.f) * sh.Z[jz];
       if (uniform_ratio(pre, static_cast<uint64_t>(c)) * qx < px) {
         accepted = sh.kids[c];
         break;
       }
-      float part = 0.f;
-      for (int64_t v = lo + tid; v < hi; v += kNT) part += fmaxf(ps[v - lo] - qs[v - lo], 0.f);
-      part = block_sum<kNT>(part, sh.red);
-      const float z = cluster_sum(part, sh.cell_z, round, C);
-      if (z > 0.f)
-        for (int64_t v = lo + tid; v < hi; v += kNT)
-          ps[v - lo] = fmaxf(ps[v - lo] - qs[v - lo], 0.f) / z;
-      __syncthreads();
-      if (tid == 0) sh.Z[nz] = z;
+      const float z = cluster_sum_warps(part, sh.wpart, round, C);
+      WTRACE(4);
+      const float zi = z > 0.f ? __frcp_rn(z) : 0.f;
+      // the residual update, with this thread's share of the next sum
+      part = 0.f;
+#pragma unroll
+      for (int k = 0; k < KG; ++k)
+#pragma unroll
+        for (int j = 0; j < VEC; ++j) {
+          if (zi > 0.f) pr[k][j] = fmaxf(pr[k][j] - qr[k][j], 0.f) * zi;
+          part += fmaxf(pr[k][j] - qr[k][j], 0.f);
+        }
+      // every thread records the same value, so no barrier is needed before
+      // any thread reads it back
+      sh.Z[nz] = zi;
       ++nz;
-      __syncthreads();
+      WTRACE(5);
     }
     if (accepted >= 0) {
       cur = accepted;
@@ -288,20 +429,43 @@ __global__ void __launch_bounds__(kNT) accept_walk_kernel(const AcceptParams p, 
       continue;
     }
     const uint64_t preb = hash_prefix(p.seed, b, p.cycle, kStreamBonus, cur);
+    // Gumbel-max: the largest log p(v) + G_v, with G_v = -log(-log u_v),
+    // ranked as p(v) / (-log u_v) (the same order)
     uint64_t bestk = 0ull;
-    for (int64_t v = lo + tid; v < hi; v += kNT) {
-      const float pv = ps[v - lo];
+    auto offer = [&](float pv, int64_t v) {
       if (pv > 0.f) {
-        const float g = uniform_gumbel(preb, static_cast<uint64_t>(v));
-        const uint64_t key = make_key(logf(pv) - logf(-logf(g)), static_cast<uint32_t>(v));
+        const float e = -__logf(uniform_gumbel(preb, static_cast<uint64_t>(v)));
+        const uint64_t key = make_key(__fdividef(pv, e), static_cast<uint32_t>(v));
         bestk = key > bestk ? key : bestk;
       }
+    };
+    // (a loop the size of one group, run KG times: this code runs once per
+    // sequence, so its instruction fetch, not its arithmetic, would dominate
+    // if it were unrolled over the whole slice)
+#pragma unroll 1
+    for (int k = 0; k < KG; ++k) {
+      if (el(k, 0) >= hi) continue;
+      float pk[VEC];
+#pragma unroll
+      for (int j = 0; j < VEC; ++j) {
+        float x = pr[0][j];
+#pragma unroll
+        for (int kk = 1; kk < KG; ++kk) x = (k == kk) ? pr[kk][j] : x;
+        pk[j] = x;
+      }
+#pragma unroll
+      for (int j = 0; j < VEC; ++j)
+        if (el(k, j) < hi) offer(pk[j], el(k, j));
     }
+    WTRACE(8);
     bestk = block_max_u64<kNT>(bestk, sh.redk);
+    WTRACE(9);
     bestk = cluster_max_u64(bestk, sh.cell_key, round, C);
     bonus = static_cast<int>(key_index(bestk));
+    WTRACE(6);
     break;
   }
+  WTRACE(7);
   if (rank == 0 && tid == 0) {
     for (int t = 0; t <= p.max_depth; ++t) path_out[t] = (t <= len) ? sh.path[t] : -1;
     p.accept_len[b] = len;
@@ -363,18 +527,18 @@ cudaError_t launch_accept_t(const AcceptParams& p, int32_t batch, cudaStream_t s
   cudaError_t e = launch(accept_rows_kernel<T>, dim3(p.chunks, p.n_max, batch), dim3(kNT), 0, s,
                          nullptr, 0, p);
   if (e != cudaSuccess) return e;
-  // walk cluster: enough CTAs that a vocabulary slice of p and q fits shared memory
+  // walk cluster: enough CTAs that a vocabulary slice of p and q fits the
+  // threads' registers (kSliceMax elements per CTA)
   int C = static_cast<int>((p.vocab + 4095) / 4096);
   if (C > 8) C = 8;
   const int need = static_cast<int>((p.vocab + kSliceMax - 1) / kSliceMax);
   if (C < need) C = need;
   if (C < 1) C = 1;
   if (C > kMaxWalkCluster) return cudaErrorInvalidValue;
-  const int64_t slice = (p.vocab + C - 1) / C;
-  const size_t smem = static_cast<size_t>(2 * slice) * sizeof(float);
-  e = cudaFuncSetAttribute(accept_walk_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           static_cast<int>(smem));
-  if (e != cudaSuccess) return e;
+  const int64_t slice = ((p.vocab + C - 1) / C + 7) / 8 * 8;  // whole 16-byte groups
+  constexpr int kVec = 16 / static_cast<int>(sizeof(T));
+  const int vec_ok = (p.vocab % kVec == 0) && (reinterpret_cast<uintptr_t>(p.target) % 16 == 0) &&
+                     (reinterpret_cast<uintptr_t>(p.draft) % 16 == 0);
   e = cudaFuncSetAttribute(accept_walk_kernel<T>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   if (e != cudaSuccess) return e;
   cudaLaunchAttribute attr[1];
@@ -382,7 +546,8 @@ cudaError_t launch_accept_t(const AcceptParams& p, int32_t batch, cudaStream_t s
   attr[0].val.clusterDim.x = C;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
-  return launch(accept_walk_kernel<T>, dim3(C, batch, 1), dim3(kNT), smem, s, attr, 1, p, C, slice);
+  return launch(accept_walk_kernel<T>, dim3(C, batch, 1), dim3(kNT), 0, s, attr, 1, p, C, slice,
+                vec_ok);
 }
 
 cudaError_t launch_accept(const AcceptParams& p, int32_t batch, ltd_dtype dtype, cudaStream_t s) {
@@ -395,5 +560,17 @@ cudaError_t launch_compact(const CompactParams& p, int32_t batch, cudaStream_t s
   const dim3 grid(p.hkv, p.n_layers * 2, batch);
   return launch(kv_compact_kernel, grid, dim3(kCompactNT), 0, s, nullptr, 0, p);
 }
+
+#ifdef LTD_TRACE
+extern "C" int ltd_walk_trace_read(unsigned long long* host, int* counts) {
+  if (cudaMemcpyFromSymbol(host, g_walk_trace, sizeof(g_walk_trace)) != cudaSuccess) return 1;
+  return cudaMemcpyFromSymbol(counts, g_walk_trace_n, sizeof(g_walk_trace_n)) == cudaSuccess ? 0 : 1;
+}
+extern "C" int ltd_walk_trace_clear() {
+  void* p = nullptr;
+  if (cudaGetSymbolAddress(&p, g_walk_trace_n) != cudaSuccess) return 1;
+  return cudaMemset(p, 0, sizeof(g_walk_trace_n)) == cudaSuccess ? 0 : 1;
+}
+#endif
 
 }  // namespace ltd

@@ -100,20 +100,6 @@ __device__ __forceinline__ void tree_merge(V* stage) {
   __syncthreads();
 }
 
-// Element j of a 16-byte vector of T, as float (j a compile-time constant).
-template <typename T>
-__device__ __forceinline__ float elem(const uint4& r, int j);
-template <>
-__device__ __forceinline__ float elem<float>(const uint4& r, int j) {
-  const uint32_t w = j == 0 ? r.x : (j == 1 ? r.y : (j == 2 ? r.z : r.w));
-  return __uint_as_float(w);
-}
-template <>
-__device__ __forceinline__ float elem<__nv_bfloat16>(const uint4& r, int j) {
-  const int q = j >> 1;
-  const uint32_t w = q == 0 ? r.x : (q == 1 ? r.y : (q == 2 ? r.z : r.w));
-  return __uint_as_float((j & 1) ? (w & 0xFFFF0000u) : (w << 16));
-}
 // Raw bits of element i of x, or of -inf past the end.
 __device__ __forceinline__ uint32_t raw_or_ninf(const float* x, int64_t i, int64_t hi) {
   return i < hi ? __float_as_uint(x[i]) : 0xFF800000u;
@@ -134,15 +120,6 @@ __device__ __forceinline__ uint4 load_tail(const T* x, int64_t i, int64_t hi) {
   }
   return make_uint4(w[0], w[1], w[2], w[3]);
 }
-// A streaming 16-byte load that the compiler may neither repeat nor move.
-__device__ __forceinline__ uint4 ld_stream16_once(const void* p) {
-  uint4 r;
-  asm volatile("ld.global.cs.v4.u32 {%0, %1, %2, %3}, [%4];"
-               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
-               : "l"(p));
-  return r;
-}
-
 struct ExpandShared {
   uint64_t stage[kNW * kWarp];
   float fstage[kNW * kWarp];

@@ -284,6 +284,29 @@ __device__ __forceinline__ uint4 ld_stream16(const void* p) {
   return __ldcs(reinterpret_cast<const uint4*>(p));
 }
 
+// Element j of a 16-byte vector of T, as float (j a compile-time constant).
+template <typename T>
+__device__ __forceinline__ float elem(const uint4& r, int j);
+template <>
+__device__ __forceinline__ float elem<float>(const uint4& r, int j) {
+  const uint32_t w = j == 0 ? r.x : (j == 1 ? r.y : (j == 2 ? r.z : r.w));
+  return __uint_as_float(w);
+}
+template <>
+__device__ __forceinline__ float elem<__nv_bfloat16>(const uint4& r, int j) {
+  const int q = j >> 1;
+  const uint32_t w = q == 0 ? r.x : (q == 1 ? r.y : (q == 2 ? r.z : r.w));
+  return __uint_as_float((j & 1) ? (w & 0xFFFF0000u) : (w << 16));
+}
+// A streaming 16-byte load that the compiler may neither repeat nor move.
+__device__ __forceinline__ uint4 ld_stream16_once(const void* p) {
+  uint4 r;
+  asm volatile("ld.global.cs.v4.u32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+               : "l"(p));
+  return r;
+}
+
 __device__ __forceinline__ void flag_error(uint32_t* err, uint32_t bits) {
   if (err) atomicOr(err, bits);
 }

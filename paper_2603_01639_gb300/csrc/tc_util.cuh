@@ -389,6 +389,9 @@ __device__ __forceinline__ void st_cluster_f4(uint32_t caddr, float4 v) {
                "f"(v.z), "f"(v.w)
                : "memory");
 }
+__device__ __forceinline__ void st_cluster_f1(uint32_t caddr, float v) {
+  asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(caddr), "f"(v) : "memory");
+}
 __device__ __forceinline__ void st_cluster_f2(uint32_t caddr, float2 v) {
   asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(caddr), "f"(v.x), "f"(v.y)
                : "memory");

@@ -277,6 +277,9 @@ def test_attention_scores_growing_along_the_cache():
     # later chunks pass a row's running max by far more than its P may grow
     # unchecked: those chunks re-derive P from the chunk's max and rescale O
     _attention_case("8b", 6, ctx_range=(1500, 1500), n_choices=(40,), key_ramp=40.0)
+    # full-length 8B layer: two chunks per split, both in one softmax round
+    # (a max that grows between them rescales the first chunk's P)
+    _attention_case("8b", 9, key_ramp=40.0)
     _attention_case("13b", 7, ctx_range=(900, 900), n_choices=(64,), key_ramp=60.0)
     _attention_case("13b", 8, ctx_range=(900, 900), n_choices=(64,), key_ramp=-0.9)
 

@@ -558,32 +558,66 @@ def run_ours(args):
 def run_e2e(cyc, args, device):
     """The same cycle through the public binding: per step, copy the draft
     logits, every layer's q and new K/V rows and the target logits from pinned
-    host memory, run the cycle, read back path / accept length / bonus / ctx."""
+    host memory, run the cycle, read back path / accept length / bonus / ctx.
+    The step's inputs sit in one pinned buffer and go over in one copy into
+    one device buffer that holds the draft and target logits and every q in
+    place; each layer's new K/V rows are then placed into its cache on the
+    device (a host copy straight into the cache's strided rows ran at a few
+    GB/s)."""
     import torch
     ltd, cfg = cyc.ltd, cyc.cfg
-    pin = lambda t: t.cpu().pin_memory()  # noqa: E731
-    h_draft, h_target = pin(cyc.draft), pin(cyc.target)
-    h_q = [pin(q) for q in cyc.q]
     c0 = int(cyc.ci.ctx.min())
     N = cfg.max_n
-    h_knew = [pin(k[:, :, c0:c0 + N]) for k in cyc.k]
-    h_vnew = [pin(v[:, :, c0:c0 + N]) for v in cyc.v]
+    # buffer order: draft logits | every q, new K, new V | target logits | root
+    parts = ([cyc.draft] + list(cyc.q) + [k[:, :, c0:c0 + N] for k in cyc.k]
+             + [v[:, :, c0:c0 + N] for v in cyc.v] + [cyc.target, cyc.root])
+    offs, total = [], 0
+    for t in parts:
+        offs.append(total)
+        total += (t.numel() * t.element_size() + 255) // 256 * 256
+    h_buf = torch.empty(total, dtype=torch.uint8).pin_memory()
+    d_buf = torch.empty(total, dtype=torch.uint8, device=device)
+    views = []
+    for t, o in zip(parts, offs):
+        nbytes = t.numel() * t.element_size()
+        h_buf[o:o + nbytes].view(t.dtype).view(t.shape).copy_(t.cpu().contiguous())
+        views.append(d_buf[o:o + nbytes].view(t.dtype).view(t.shape))
+    L = cyc.layers
+    cyc.draft = views[0]
+    cyc.q = views[1:1 + L]
+    d_knew, d_vnew = views[1 + L:1 + 2 * L], views[1 + 2 * L:1 + 3 * L]
+    cyc.target, cyc.root = views[-2], views[-1]
+    # three spans of the buffer: what the draft phase needs, what attention
+    # needs, what acceptance needs (then the root)
+    a0, a1, a2 = offs[1], offs[-2], offs[-1]
     outs = {k: torch.empty(v.shape, dtype=v.dtype).pin_memory() for k, v in cyc.acc.items()}
-    h2d = (h_draft.numel() * h_draft.element_size() + h_target.numel() * h_target.element_size()
-           + sum(t.numel() * t.element_size() for t in h_q + h_knew + h_vnew) + 4 * cfg.batch)
+    h2d = sum(t.numel() * t.element_size() for t in parts)
     d2h = sum(v.numel() * v.element_size() for v in outs.values())
-    h_root = cyc.root.cpu().pin_memory()
+    side = torch.cuda.Stream(device)
+    ev_kv, ev_tgt = torch.cuda.Event(), torch.cuda.Event()
 
     def step():
-        cyc.root.copy_(h_root, non_blocking=True)
-        cyc.draft.copy_(h_draft, non_blocking=True)
-        for l in range(cyc.layers):
-            cyc.q[l].copy_(h_q[l], non_blocking=True)
-            cyc.k[l][:, :, c0:c0 + N].copy_(h_knew[l], non_blocking=True)
-            cyc.v[l][:, :, c0:c0 + N].copy_(h_vnew[l], non_blocking=True)
-        cyc.target.copy_(h_target, non_blocking=True)
+        # side stream: attention's inputs (and their placement into the
+        # caches), then acceptance's, while the main stream copies the draft
+        # logits and drafts.  (Finer steps -- the draft rows level by level,
+        # each layer's inputs behind its own event -- measured slower: the
+        # cross-stream waits break the chain of programmatic launches.)
+        main = torch.cuda.current_stream(device)
+        side.wait_stream(main)
+        d_buf[a2:].copy_(h_buf[a2:], non_blocking=True)  # root
+        d_buf[:a0].copy_(h_buf[:a0], non_blocking=True)
+        with torch.cuda.stream(side):
+            d_buf[a0:a1].copy_(h_buf[a0:a1], non_blocking=True)
+            for l in range(L):
+                cyc.k[l][:, :, c0:c0 + N].copy_(d_knew[l])
+                cyc.v[l][:, :, c0:c0 + N].copy_(d_vnew[l])
+            ev_kv.record(side)
+            d_buf[a1:a2].copy_(h_buf[a1:a2], non_blocking=True)
+            ev_tgt.record(side)
         cyc.draft_phase()
+        main.wait_event(ev_kv)
         cyc.verify_phase()
+        main.wait_event(ev_tgt)
         cyc.accept_phase()
         for k in outs:
             outs[k].copy_(cyc.acc[k], non_blocking=True)
@@ -591,15 +625,26 @@ def run_e2e(cyc, args, device):
     for _ in range(max(3, args.warmup)):
         step()
     torch.cuda.synchronize(device)
+    # the whole step (copies in, the three phases, copies out) as one CUDA
+    # graph, as a serving loop would replay it
+    try:
+        g = _graph(torch, step)
+        run, how = g.replay, "one CUDA graph per step: h2d copies from pinned memory (attention and acceptance inputs on a second stream, overlapping the draft phase), phases, d2h copies"
+    except RuntimeError as exc:  # capture refused: time the eager calls
+        torch.cuda.synchronize(device)
+        run, how = step, f"eager calls (graph capture failed: {str(exc)[:80]})"
+    for _ in range(max(3, args.warmup)):
+        run()
+    torch.cuda.synchronize(device)
     s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     s.record()
     for _ in range(args.steps):
-        step()
+        run()
     e.record()
     torch.cuda.synchronize(device)
     us = s.elapsed_time(e) * 1e3 / args.steps / cfg.batch
     return {"value": round(us, 2), "unit": "us", "h2d_bytes_per_step": int(h2d),
-            "d2h_bytes_per_step": int(d2h)}
+            "d2h_bytes_per_step": int(d2h), "how": how}
 
 
 def main():

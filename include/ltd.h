@@ -154,6 +154,25 @@ ltd_status ltd_select_verify(const ltd_tree* tree, const int32_t* d_n_verify, in
                              const int32_t* d_ctx, int32_t* d_node_ids, int32_t* d_pos,
                              uint32_t* d_mask, ltd_stream_t stream);
 
+/* Observations of the learned policies (section 3.1 and Appendix A,
+ * "Observation Space"), gathered on the device for a host-side policy.
+ * Depth policy, after an expansion:
+ *  d_out  [batch][k*k + 2] float: the cum_logprob of the candidate tokens of
+ *         the last level built (its k^2 nodes in id order; k at level 1),
+ *         padded with LTD_POLICY_PAD to k^2, then the draft depth D (levels
+ *         built) and the sequence length L = ctx[b].
+ * Size policy, after the draft:
+ *  v_pad  >= the tree's max_nodes (1 + k + (max_depth-1) k^2)
+ *  d_out  [batch][v_pad + 2] float: the cum_logprob of every node in id
+ *         order (root = 0), padded with LTD_POLICY_PAD, then D and L.
+ *  d_ctx  [batch] context length.
+ * Both only read the tree; the buffers are the caller's. */
+#define LTD_POLICY_PAD (-100.0f)
+ltd_status ltd_depth_observation(const ltd_tree* tree, const int32_t* d_ctx, float* d_out,
+                                 ltd_stream_t stream);
+ltd_status ltd_size_observation(const ltd_tree* tree, const int32_t* d_ctx, int32_t v_pad,
+                                float* d_out, ltd_stream_t stream);
+
 /* Tree attention of the verified tokens against the KV cache (section 3.2
  * "Draft Tree Verification"; tree attention as in SpecInfer, section 2.1).
  * For slot i < N_b and query head h, KV head g = h / (hq/hkv):

@@ -173,6 +173,20 @@ ltd_status ltd_expand_tree(const ltd_tree* tree, int32_t level, const void* d_dr
   return from_cuda(launch_expand(p, tree->batch, dtype, reinterpret_cast<cudaStream_t>(stream)));
 }
 
+ltd_status ltd_depth_observation(const ltd_tree* tree, const int32_t* d_ctx, float* d_out,
+                                 ltd_stream_t stream) {
+  if (!tree_ok(tree) || d_ctx == nullptr || d_out == nullptr) return LTD_ERR_INVALID_ARG;
+  return from_cuda(launch_depth_obs(tree, d_ctx, d_out, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+ltd_status ltd_size_observation(const ltd_tree* tree, const int32_t* d_ctx, int32_t v_pad,
+                                float* d_out, ltd_stream_t stream) {
+  if (!tree_ok(tree) || d_ctx == nullptr || d_out == nullptr) return LTD_ERR_INVALID_ARG;
+  if (v_pad < tree->max_nodes) return LTD_ERR_SHAPE;
+  return from_cuda(
+      launch_size_obs(tree, d_ctx, v_pad, d_out, reinterpret_cast<cudaStream_t>(stream)));
+}
+
 ltd_status ltd_select_verify(const ltd_tree* tree, const int32_t* d_n_verify, int32_t n_max,
                              const int32_t* d_ctx, int32_t* d_node_ids, int32_t* d_pos,
                              uint32_t* d_mask, ltd_stream_t stream) {

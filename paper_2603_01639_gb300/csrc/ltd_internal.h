@@ -187,6 +187,12 @@ struct AcceptParams {
   uint32_t* err;
 };
 size_t accept_workspace(int32_t batch, int32_t n_max, int64_t vocab);
+
+// Policy observations (k_policy.cu); entries past the tree hold kPolicyPad.
+constexpr float kPolicyPad = LTD_POLICY_PAD;
+cudaError_t launch_depth_obs(const ltd_tree* t, const int32_t* ctx, float* out, cudaStream_t s);
+cudaError_t launch_size_obs(const ltd_tree* t, const int32_t* ctx, int32_t v_pad, float* out,
+                            cudaStream_t s);
 cudaError_t launch_accept(const AcceptParams& p, int32_t batch, ltd_dtype dtype, cudaStream_t s);
 
 struct CompactParams {

@@ -30,7 +30,9 @@ EXPORTS = [
     "ltd_attention_workspace_bytes", "ltd_tree_attention", "ltd_accept_workspace_bytes",
     "ltd_accept", "ltd_kv_compact", "ltd_check", "ltd_status_string", "ltd_version",
     "ltd_attention_kernel", "ltd_selftest_umma", "ltd_accept_noalloc", "ltd_tree_attention_next",
+    "ltd_depth_observation", "ltd_size_observation",
 ]
+LTD_POLICY_PAD = -100.0
 LTD_ACCEPT_NOALLOC_SCRATCH_BYTES = 1 << 20
 
 
@@ -70,6 +72,8 @@ def lib():
                 "ltd_tree_reset": (C.c_int, [tp, vp, vp]),
                 "ltd_expand_tree": (C.c_int, [tp, i32, vp, C.c_int, i64, i64, vp, vp]),
                 "ltd_select_verify": (C.c_int, [tp, vp, i32, vp, vp, vp, vp, vp]),
+                "ltd_depth_observation": (C.c_int, [tp, vp, vp, vp]),
+                "ltd_size_observation": (C.c_int, [tp, vp, i32, vp, vp]),
                 "ltd_attention_workspace_bytes": (sz, [i32, i32, i32, i32, i32, i32, C.c_int]),
                 "ltd_tree_attention": (C.c_int, [vp, vp, vp, vp, C.c_int, i32, i32, i32, i32, i32,
                                                  vp, i32, vp, i32, vp, C.c_float, vp, sz, vp]),
@@ -215,6 +219,31 @@ def ltd_select_verify(tree: Tree, n_verify: torch.Tensor, n_max: int, ctx: torch
     _ok(lib().ltd_select_verify(C.byref(tree.s), _ptr(n_verify), n_max, _ptr(ctx), _ptr(ids),
                                 _ptr(pos), _ptr(mask), _stream(stream)), "ltd_select_verify")
     return ids, pos, mask
+
+
+def ltd_depth_observation(tree: Tree, ctx: torch.Tensor, out=None, stream=None):
+    """Depth-policy observation [B][k*k + 2] (float32): the last level's
+    candidate cum log-probs (padded with LTD_POLICY_PAD), then D and L."""
+    _need(ctx, "ctx", torch.int32)
+    kk = tree.k * tree.k
+    if out is None:
+        out = torch.empty(tree.batch, kk + 2, dtype=torch.float32, device=ctx.device)
+    _ok(lib().ltd_depth_observation(C.byref(tree.s), _ptr(ctx), _ptr(out), _stream(stream)),
+        "ltd_depth_observation")
+    return out
+
+
+def ltd_size_observation(tree: Tree, ctx: torch.Tensor, v_pad=None, out=None, stream=None):
+    """Size-policy observation [B][v_pad + 2] (float32): every node's cum
+    log-prob in id order (padded with LTD_POLICY_PAD), then D and L;
+    v_pad defaults to the tree's max_nodes."""
+    _need(ctx, "ctx", torch.int32)
+    v_pad = tree.max_nodes if v_pad is None else v_pad
+    if out is None:
+        out = torch.empty(tree.batch, v_pad + 2, dtype=torch.float32, device=ctx.device)
+    _ok(lib().ltd_size_observation(C.byref(tree.s), _ptr(ctx), v_pad, _ptr(out), _stream(stream)),
+        "ltd_size_observation")
+    return out
 
 
 def attention_workspace(batch, hq, hkv, head_dim, n_max, max_ctx, dtype, device="cuda"):

@@ -1,0 +1,67 @@
+"""Host-side policies of LTD (section 3.1; Appendix A and B): lightweight MLPs
+that read the device-gathered observations and choose the draft depth (the
+depth policy, one continue/stop decision per level) and the verify size N
+(the size policy, N in [20, 240]).
+
+Architectures follow the paper: the depth policy has one hidden layer of
+1024 ReLU units and two actions; the size policy has hidden layers of 1024
+and 256 ReLU units and one action per size in [20, 240].  No trained weights
+exist here: the weights are seeded random (He-normal), which fixes the
+shapes and the cost of a decision, not its quality.  Inference is numpy
+fp32 on the host, as the policies are not on the device hot path.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+N_MIN, N_MAX = 20, 240
+
+
+def _dense(rng: np.random.Generator, n_in: int, n_out: int):
+    w = rng.standard_normal((n_in, n_out), dtype=np.float32) * np.float32(np.sqrt(2.0 / n_in))
+    return w, np.zeros(n_out, np.float32)
+
+
+class MLP:
+    """ReLU MLP with seeded random weights; forward(x [B][n_in]) -> logits."""
+
+    def __init__(self, n_in: int, hidden: tuple, n_out: int, seed: int):
+        rng = np.random.default_rng(seed)
+        dims = (n_in,) + tuple(hidden) + (n_out,)
+        self.layers = [_dense(rng, a, b) for a, b in zip(dims[:-1], dims[1:])]
+
+    def forward(self, x: np.ndarray) -> np.ndarray:
+        h = np.asarray(x, np.float32)
+        for i, (w, b) in enumerate(self.layers):
+            h = h @ w + b
+            if i + 1 < len(self.layers):
+                h = np.maximum(h, 0.0)
+        return h
+
+
+def _normalise(obs: np.ndarray) -> np.ndarray:
+    """Scores as they are; D and L (the last two entries) scaled to O(1)."""
+    x = np.array(obs, np.float32, copy=True)
+    x[:, -2] *= np.float32(1.0 / 16.0)
+    x[:, -1] *= np.float32(1.0 / 8192.0)
+    return x
+
+
+class DepthPolicy:
+    """pi_D: observation [B][k*k + 2] -> continue drafting (bool [B])."""
+
+    def __init__(self, k: int, seed: int = 0):
+        self.net = MLP(k * k + 2, (1024,), 2, seed)
+
+    def decide(self, obs: np.ndarray) -> np.ndarray:
+        return np.argmax(self.net.forward(_normalise(obs)), axis=1) == 1
+
+
+class SizePolicy:
+    """pi_V: observation [B][v_pad + 2] -> verify size N in [20, 240] ([B])."""
+
+    def __init__(self, v_pad: int, seed: int = 1):
+        self.net = MLP(v_pad + 2, (1024, 256), N_MAX - N_MIN + 1, seed)
+
+    def decide(self, obs: np.ndarray) -> np.ndarray:
+        return N_MIN + np.argmax(self.net.forward(_normalise(obs)), axis=1).astype(np.int32)

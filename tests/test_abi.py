@@ -81,6 +81,10 @@ def test_entry_points_reject_bad_arguments_before_launch(L):
     assert L.ltd_expand_tree(C.byref(t), 1, fake, 1, 996, 9, None, s) == 2        # bf16 row not 16B
     assert L.ltd_select_verify(C.byref(t), fake, 257, fake, fake, fake, fake, s) == 2
     assert L.ltd_select_verify(C.byref(t), None, 8, fake, fake, fake, fake, s) == 1
+    assert L.ltd_depth_observation(None, fake, fake, s) == 1
+    assert L.ltd_depth_observation(C.byref(t), None, fake, s) == 1
+    assert L.ltd_size_observation(C.byref(t), fake, t.max_nodes - 1, fake, s) == 2  # v_pad short
+    assert L.ltd_size_observation(C.byref(t), fake, t.max_nodes, None, s) == 1
     ws = L.ltd_attention_workspace_bytes(1, 4, 1, 64, 8, 128, 0)
     assert ws > 0
     assert L.ltd_attention_workspace_bytes(1, 5, 2, 64, 8, 128, 0) == 0          # hq % hkv

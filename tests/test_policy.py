@@ -1,0 +1,38 @@
+"""Host policies (section 3.1, Appendix A/B): shapes of the paper's MLPs, the
+action ranges, and seeded determinism.  No GPU."""
+import numpy as np
+
+from paper_2603_01639_gb300 import policy
+
+
+def test_depth_policy_shapes_and_actions():
+    k = 10
+    p = policy.DepthPolicy(k, seed=3)
+    dims = [w.shape for w, _ in p.net.layers]
+    assert dims == [(k * k + 2, 1024), (1024, 2)]          # one hidden layer of 1024
+    rng = np.random.default_rng(0)
+    obs = np.concatenate([rng.normal(-5, 2, (4, k * k)), [[3, 4096]] * 4], axis=1)
+    a = p.decide(obs)
+    assert a.shape == (4,) and a.dtype == bool
+    assert np.array_equal(a, policy.DepthPolicy(k, seed=3).decide(obs))
+
+
+def test_size_policy_shapes_and_range():
+    v_pad = 1 + 10 + 5 * 100
+    p = policy.SizePolicy(v_pad, seed=4)
+    dims = [w.shape for w, _ in p.net.layers]
+    assert dims == [(v_pad + 2, 1024), (1024, 256), (256, 221)]  # [1024, 256] hidden, N in 20..240
+    rng = np.random.default_rng(1)
+    obs = np.concatenate([rng.normal(-8, 3, (5, v_pad)), [[6, 2048]] * 5], axis=1)
+    n = p.decide(obs)
+    assert n.dtype == np.int32 and n.shape == (5,)
+    assert ((n >= 20) & (n <= 240)).all()
+    assert np.array_equal(n, policy.SizePolicy(v_pad, seed=4).decide(obs))
+
+
+def test_mlp_is_the_plain_relu_network():
+    net = policy.MLP(3, (4,), 2, seed=0)
+    x = np.array([[1.0, -2.0, 0.5]], np.float32)
+    (w1, b1), (w2, b2) = net.layers
+    ref = np.maximum(x @ w1 + b1, 0) @ w2 + b2
+    assert np.allclose(net.forward(x), ref)

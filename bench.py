@@ -43,6 +43,7 @@ def _args():
     ap.add_argument("--config", default="8b", choices=list(N_LAYERS))
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-policy", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-sample-s", type=float, default=15.0)
     ap.add_argument("--no-next-hint", action="store_true",
@@ -531,6 +532,10 @@ def run_ours(args):
                 "tflops": round(att_flops / (att_launch_ms * 1e-3) / 1e12, 1),
                 "frac_of_8tbs": round(achieved / 8000.0, 4)}
 
+    pol = None
+    if not args.no_policy:
+        pol = time_policies(cyc, verify, K, device)
+
     e2e = None
     if not args.no_e2e:
         e2e = run_e2e(cyc, args, device)
@@ -556,13 +561,82 @@ def run_ours(args):
             "phases_us": {"draft_select": round(draft_ms * 1e3, 2),
                           "attention_all_layers": round(verify_ms * 1e3, 2),
                           "accept_compact": round(accept_ms * 1e3, 2)},
-            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "policy": pol,
             "gpu_launches": cyc.launches_per_step() * K, "clocks": clk,
         }
         print(json.dumps(line), flush=True)
     if world > 1:
         torch.distributed.destroy_process_group()
     return 0
+
+
+def time_policies(cyc, verify, steps, device):
+    """The cycle with both learned policies in the loop (section 3.1): after
+    every level the depth observation is gathered on the device, read back
+    and fed to the depth policy; after the draft the size observation goes
+    to the size policy.  Each decision needs the host, so this cycle runs as
+    eager calls with one stream sync per decision.  The policies' weights are
+    seeded random and their decisions are computed but not applied (depth
+    and N stay the workload's), so the device work equals the timed cycle's;
+    the same eager cycle without the policies is timed beside it."""
+    import torch
+    from paper_2603_01639_gb300 import policy
+    ltd, cfg, tree = cyc.ltd, cyc.cfg, cyc.tree
+    B, kk, v_pad = cfg.batch, cfg.W * cfg.W, tree.max_nodes
+    pi_d, pi_v = policy.DepthPolicy(cfg.W, seed=0), policy.SizePolicy(v_pad, seed=1)
+    d_obs = torch.empty(B, kk + 2, dtype=torch.float32, device=device)
+    s_obs = torch.empty(B, v_pad + 2, dtype=torch.float32, device=device)
+    h_d = torch.empty(B, kk + 2, dtype=torch.float32).pin_memory()
+    h_s = torch.empty(B, v_pad + 2, dtype=torch.float32).pin_memory()
+    stream = torch.cuda.current_stream(device)
+    mlp_s = {"depth": [], "size": []}
+
+    def decide(net, d_src, h_dst, key):
+        h_dst.copy_(d_src, non_blocking=True)
+        stream.synchronize()
+        t0 = time.perf_counter()
+        net.decide(h_dst.numpy())
+        mlp_s[key].append(time.perf_counter() - t0)
+
+    def adaptive():
+        ltd.ltd_tree_reset(tree, cyc.root)
+        for level in range(1, cyc.max_depth + 1):
+            ltd.ltd_expand_tree(tree, level, cyc.draft, active=cyc.actives[level])
+            ltd.ltd_depth_observation(tree, cyc.ctx, out=d_obs)
+            decide(pi_d, d_obs, h_d, "depth")
+        ltd.ltd_size_observation(tree, cyc.ctx, v_pad, out=s_obs)
+        decide(pi_v, s_obs, h_s, "size")
+        ltd.ltd_select_verify(tree, cyc.n_verify, cfg.max_n, cyc.ctx, out=cyc.sel)
+        verify()
+        cyc.accept_phase()
+
+    def fixed():
+        cyc.draft_phase()
+        verify()
+        cyc.accept_phase()
+
+    res = {}
+    for name, fn in (("eager_fixed", fixed), ("eager_with_policies", adaptive)):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize(device)
+        for v in mlp_s.values():
+            v.clear()
+        t0 = time.perf_counter()
+        for _ in range(steps):
+            fn()
+        torch.cuda.synchronize(device)
+        res[name] = (time.perf_counter() - t0) / steps * 1e6
+    over = res["eager_with_policies"] - res["eager_fixed"]
+    return {"cycle_us_eager_with_policies": round(res["eager_with_policies"], 1),
+            "cycle_us_eager_fixed": round(res["eager_fixed"], 1),
+            "overhead_us": round(over, 1),
+            "overhead_frac": round(over / res["eager_with_policies"], 4),
+            "depth_decisions_per_cycle": cyc.max_depth,
+            "depth_mlp_us": round(statistics.median(mlp_s["depth"]) * 1e6, 1),
+            "size_mlp_us": round(statistics.median(mlp_s["size"]) * 1e6, 1),
+            "mlp": "numpy fp32 on the host, seeded random weights, batch " + str(B),
+            "how": "host wall clock over K eager cycles; decisions computed, not applied"}
 
 
 def run_e2e(cyc, args, device):

@@ -8,18 +8,20 @@ through the seeded inputs of ``paper_2603_01639_gb300.workload``.
 
 Every function follows the paper (Zhang et al., "Learning To Draft: Adaptive
 Speculative Decoding with Reinforcement Learning", §3.2 "Draft-and-Verify
-Cycle") or, where the paper is silent, the reading stated in its docstring.
-All pins are in ``tests/test_oracle_pins.py``; no function here is left
-"parity unpinned".
+Cycle"; Appendix A.2 for the policies' observations) or, where the paper is
+silent, the reading stated in its docstring.  All pins are in
+``tests/test_oracle_pins.py``; no function here is left "parity unpinned".
 """
 
 from .ltd_oracle import (  # noqa: F401
     GAMMA,
+    POLICY_PAD,
     OracleTree,
     accept_greedy,
     accept_stochastic,
     compact_kv,
     cycle,
+    depth_observation,
     expand_level,
     grow_tree,
     log_softmax,
@@ -27,6 +29,7 @@ from .ltd_oracle import (  # noqa: F401
     mix64,
     rank_by_logit,
     select_verify,
+    size_observation,
     splitmix64_stream,
     tree_attention,
     uniform_gumbel,

@@ -391,6 +391,41 @@ def compact_kv(cache: np.ndarray, ctx: int, path) -> np.ndarray:
     return out
 
 
+# --------------------------------------------------------- policy observations
+POLICY_PAD = -100.0   # fill of unused observation slots (the paper only says "padded")
+
+
+def depth_observation(tree: OracleTree, ctx: int) -> np.ndarray:
+    """Observation of the depth policy after the last built level (Appendix
+    A.2, "Depth Policy", observation space): the cumulative log-probabilities
+    of the candidates that level produced, W^2 of them (W at level 1, padded
+    to W^2 with POLICY_PAD), in node-id order, then the draft depth D (levels
+    built) and the sequence length L = ctx.  Returned in fp64."""
+    W, lvl = tree.W, tree.levels
+    out = np.full(W * W + 2, POLICY_PAD, np.float64)
+    if lvl >= 1:
+        first = 1 if lvl == 1 else 1 + W + (lvl - 2) * W * W
+        count = W if lvl == 1 else W * W
+        out[:count] = tree.cum[first:first + count]
+    out[W * W] = lvl
+    out[W * W + 1] = ctx
+    return out
+
+
+def size_observation(tree: OracleTree, ctx: int, v_pad: int) -> np.ndarray:
+    """Observation of the size policy after drafting (Appendix A.2, "Size
+    Policy", observation space): the cumulative log-probabilities of all
+    1 + W + (L-1) W^2 tree nodes, root included, in node-id order, padded to
+    ``v_pad`` with POLICY_PAD, then D (levels built) and L = ctx."""
+    n = tree.n_nodes
+    assert v_pad >= n
+    out = np.full(v_pad + 2, POLICY_PAD, np.float64)
+    out[:n] = tree.cum
+    out[v_pad] = tree.levels
+    out[v_pad + 1] = ctx
+    return out
+
+
 # ------------------------------------------------------------- whole cycle
 def cycle(root_token, draft_rows, W, L, N, ctx, target_rows, mode="greedy",
           seed=0, b=0, cycle_no=0):

@@ -1,11 +1,12 @@
 """Host-side policies of LTD (section 3.1; Appendix A and B): lightweight MLPs
 that read the device-gathered observations and choose the draft depth (the
 depth policy, one continue/stop decision per level) and the verify size N
-(the size policy, N in [20, 240]).
+(the size policy, N in [20, 240] in 12 steps).
 
 Architectures follow the paper: the depth policy has one hidden layer of
 1024 ReLU units and two actions; the size policy has hidden layers of 1024
-and 256 ReLU units and one action per size in [20, 240].  No trained weights
+and 256 ReLU units and 12 actions mapped linearly onto N = 20, 40, ..., 240
+(Appendix A.2, "Size Policy", action space).  No trained weights
 exist here: the weights are seeded random (He-normal), which fixes the
 shapes and the cost of a decision, not its quality.  Inference is numpy
 fp32 on the host, as the policies are not on the device hot path.
@@ -14,7 +15,8 @@ from __future__ import annotations
 
 import numpy as np
 
-N_MIN, N_MAX = 20, 240
+N_MIN, N_MAX, N_ACTIONS = 20, 240, 12
+N_STEP = (N_MAX - N_MIN) // (N_ACTIONS - 1)   # 20
 
 
 def _dense(rng: np.random.Generator, n_in: int, n_out: int):
@@ -58,10 +60,11 @@ class DepthPolicy:
 
 
 class SizePolicy:
-    """pi_V: observation [B][v_pad + 2] -> verify size N in [20, 240] ([B])."""
+    """pi_V: observation [B][v_pad + 2] -> verify size N in {20, 40, ..., 240} ([B])."""
 
     def __init__(self, v_pad: int, seed: int = 1):
-        self.net = MLP(v_pad + 2, (1024, 256), N_MAX - N_MIN + 1, seed)
+        self.net = MLP(v_pad + 2, (1024, 256), N_ACTIONS, seed)
 
     def decide(self, obs: np.ndarray) -> np.ndarray:
-        return N_MIN + np.argmax(self.net.forward(_normalise(obs)), axis=1).astype(np.int32)
+        a = np.argmax(self.net.forward(_normalise(obs)), axis=1).astype(np.int32)
+        return (N_MIN + N_STEP * a).astype(np.int32)

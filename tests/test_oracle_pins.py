@@ -450,6 +450,63 @@ def _mutant_log_softmax_dropped_lse(x):
     return x - x.max(), float(x.max())  # mistake: drops log sum exp(x - m)
 
 
+# ------------------------------------------------------ policy observation pins
+def test_worked_example_observations():
+    """Depth and size observations of the hand-worked tree: the exact cums of
+    the worked nodes (as fractions), selected by their depth, not by id."""
+    g = _worked()
+    rows = _rows_from_weights(g["draft_row_weights"])
+    W, ctx = g["W"], g["ctx"]
+    by_depth = {}
+    for node in sorted(g["expected_nodes"], key=lambda n: n["id"]):
+        by_depth.setdefault(node["depth"], []).append(math.log(Fraction(node["cum"])))
+    for L in (1, 2, 3):
+        tree = oracle.grow_tree(g["root_token"], rows, W, L)
+        obs = O.depth_observation(tree, ctx)
+        want = by_depth[L]
+        assert len(obs) == W * W + 2
+        assert obs[:len(want)] == pytest.approx(want, abs=1e-12)
+        assert (obs[len(want):W * W] == O.POLICY_PAD).all()
+        assert obs[W * W] == L and obs[W * W + 1] == ctx
+    tree = oracle.grow_tree(g["root_token"], rows, W, g["L"])
+    v_pad = 40
+    obs = O.size_observation(tree, ctx, v_pad)
+    allc = [math.log(Fraction(n["cum"])) if n["id"] else 0.0
+            for n in sorted(g["expected_nodes"], key=lambda n: n["id"])]
+    assert obs[:len(allc)] == pytest.approx(allc, abs=1e-12)
+    assert (obs[len(allc):v_pad] == O.POLICY_PAD).all()
+    assert obs[v_pad] == g["L"] and obs[v_pad + 1] == ctx
+
+
+@pytest.mark.parametrize("W,L", [(1, 3), (2, 1), (3, 4), (4, 2), (10, 3)])
+def test_observations_against_depth_and_path_sums(W, L):
+    """The depth observation holds exactly the level's candidates (the nodes
+    whose depth is L: W at level 1, the whole W^2 pool after), and the size
+    observation every node's path sum of scipy log-probs; the count of real
+    entries is the paper's 1 + W + (D-2) W^2 with D = L + 1."""
+    tree, rows, _ = _random_tree(W * 31 + L, W, L, vocab=40)
+    ctx = 777 + L
+    d = O.depth_observation(tree, ctx)
+    level = [tree.cum[i] for i in range(tree.n_nodes) if tree.depth[i] == L]
+    assert len(level) == (W if L == 1 else W * W)
+    np.testing.assert_array_equal(d[:len(level)], level)
+    assert (d[len(level):W * W] == O.POLICY_PAD).all()
+    assert list(d[W * W:]) == [L, ctx]
+    v_pad = 1 + W + (L - 1) * W * W + 7
+    s = O.size_observation(tree, ctx, v_pad)
+    D = L + 1
+    n_real = 1 + W + (D - 2) * W * W
+    for c in range(n_real):
+        total, a = 0.0, c
+        while tree.parent[a] >= 0:
+            p = tree.parent[a]
+            total += scipy.special.log_softmax(rows[tree.xrow[p]])[tree.token[a]]
+            a = p
+        assert s[c] == pytest.approx(total, abs=1e-12)
+    assert (s[n_real:v_pad] == O.POLICY_PAD).all()
+    assert list(s[v_pad:]) == [L, ctx]
+
+
 def test_planted_mistake_in_log_softmax_is_caught(monkeypatch):
     monkeypatch.setattr(O, "log_softmax", _mutant_log_softmax_dropped_lse)
     with pytest.raises(AssertionError):
@@ -524,3 +581,17 @@ def test_brute_force_enumeration_is_exhaustive():
     target[3, 2] = 1
     best, bonus = _brute_force_greedy(t, ids, target)
     assert best == [0, 1, 3] and bonus == 2
+
+
+def test_planted_mistake_in_depth_observation_is_caught(monkeypatch):
+    def shifted(tree, ctx):   # mistake: the level's first id off by one
+        out = np.full(tree.W * tree.W + 2, O.POLICY_PAD)
+        lvl, W = tree.levels, tree.W
+        first = 1 if lvl == 1 else W + (lvl - 2) * W * W
+        cnt = W if lvl == 1 else W * W
+        out[:cnt] = tree.cum[first:first + cnt]
+        out[-2:] = (lvl, ctx)
+        return out
+    monkeypatch.setattr(O, "depth_observation", shifted)
+    with pytest.raises(AssertionError):
+        test_observations_against_depth_and_path_sums(3, 4)

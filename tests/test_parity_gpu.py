@@ -80,6 +80,61 @@ def test_70b_batched_ragged_mixed():
     assert len(set(ci.depth.tolist())) > 1 and len(set(ci.ctx.tolist())) > 1
 
 
+# ------------------------------------------------------- policy observations
+def _check_obs(got, ref, dev_cum, ids, n_real, tail_at):
+    """Real slots: the device tree's cums bit for bit and the oracle's within
+    CUM_TOL; pad slots: exactly LTD_POLICY_PAD; D and L exact."""
+    np.testing.assert_array_equal(got[:n_real], dev_cum[ids])
+    err = np.abs(got[:n_real] - ref[:n_real]) / np.maximum(1.0, np.abs(ref[:n_real]))
+    assert n_real == 0 or err.max() <= H.CUM_TOL, err.max()
+    assert (got[n_real:tail_at] == np.float32(ltd.LTD_POLICY_PAD)).all()
+    assert oracle.POLICY_PAD == ltd.LTD_POLICY_PAD
+    assert got[tail_at] == ref[tail_at] and got[tail_at + 1] == ref[tail_at + 1]
+
+
+@pytest.mark.parametrize("name,seed", [("tiny", 0), ("8b", 0), ("70b", 0)])
+def test_policy_observations(name, seed):
+    """Depth observation after every level (ragged depths: a finished
+    sequence keeps reporting its last level) and the size observation of the
+    finished tree, padded beyond max_nodes."""
+    cfg = wl.config(name)
+    ci = wl.draw_cycle(cfg, seed)
+    B, W = cfg.batch, cfg.W
+    kk = W * W
+    draft = H.dev(ci.draft_rows, cfg.dtype)
+    ctx = H.i32(ci.ctx)
+    depth = np.asarray(ci.depth)
+    tree = ltd.Tree(B, cfg.max_depth, W, cfg.vocab)
+    ltd.ltd_tree_reset(tree, H.i32(ci.root))
+    otrees = [oracle.OracleTree.rooted(int(ci.root[b]), W) for b in range(B)]
+    for level in range(1, int(depth.max()) + 1):
+        act = depth >= level
+        ltd.ltd_expand_tree(tree, level, draft, active=None if act.all() else H.i32(act.astype(np.int32)))
+        r0 = 0 if level == 1 else 1 + (level - 2) * W
+        r1 = 1 if level == 1 else r0 + W
+        for b in np.flatnonzero(act):
+            oracle.expand_level(otrees[b], ci.draft_rows[b][r0:r1])
+        got = ltd.ltd_depth_observation(tree, ctx).cpu().numpy()
+        cum = tree.view()["cum_logprob"].cpu().numpy()
+        assert ltd.ltd_check() == 0
+        for b in range(B):
+            t = otrees[b]
+            lv = t.levels
+            first = 1 if lv == 1 else 1 + W + (lv - 2) * kk
+            count = W if lv == 1 else kk
+            ref = oracle.depth_observation(t, int(ci.ctx[b]))
+            _check_obs(got[b], ref, cum[b], np.arange(first, first + count), count, kk)
+    assert min(H.tree_margin(t, W) for t in otrees) > H.CUT_MARGIN
+    v_pad = tree.max_nodes + 13
+    got = ltd.ltd_size_observation(tree, ctx, v_pad).cpu().numpy()
+    cum = tree.view()["cum_logprob"].cpu().numpy()
+    assert ltd.ltd_check() == 0
+    for b in range(B):
+        ref = oracle.size_observation(otrees[b], int(ci.ctx[b]), v_pad)
+        n = otrees[b].n_nodes
+        _check_obs(got[b], ref, cum[b], np.arange(n), n, v_pad)
+
+
 def test_determinism_and_reuse_of_scratch():
     """Same inputs twice through the same tree and workspace: identical bits
     (tickets and scratch are left ready for reuse)."""

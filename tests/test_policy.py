@@ -21,12 +21,12 @@ def test_size_policy_shapes_and_range():
     v_pad = 1 + 10 + 5 * 100
     p = policy.SizePolicy(v_pad, seed=4)
     dims = [w.shape for w, _ in p.net.layers]
-    assert dims == [(v_pad + 2, 1024), (1024, 256), (256, 221)]  # [1024, 256] hidden, N in 20..240
+    assert dims == [(v_pad + 2, 1024), (1024, 256), (256, 12)]   # [1024, 256] hidden, 12 actions
     rng = np.random.default_rng(1)
     obs = np.concatenate([rng.normal(-8, 3, (5, v_pad)), [[6, 2048]] * 5], axis=1)
     n = p.decide(obs)
     assert n.dtype == np.int32 and n.shape == (5,)
-    assert ((n >= 20) & (n <= 240)).all()
+    assert ((n >= 20) & (n <= 240) & (n % 20 == 0)).all()
     assert np.array_equal(n, policy.SizePolicy(v_pad, seed=4).decide(obs))
 
 
@@ -36,3 +36,16 @@ def test_mlp_is_the_plain_relu_network():
     (w1, b1), (w2, b2) = net.layers
     ref = np.maximum(x @ w1 + b1, 0) @ w2 + b2
     assert np.allclose(net.forward(x), ref)
+
+
+def test_size_actions_map_linearly_onto_20_to_240():
+    p = policy.SizePolicy(8, seed=0)
+    w, b = p.net.layers[-1]
+    obs = np.zeros((1, 10), np.float32)
+    got = []
+    for a in range(12):                 # force each action through the output bias
+        b[:] = 0.0
+        w[:] = 0.0
+        b[a] = 1.0
+        got.append(int(p.decide(obs)[0]))
+    assert got == list(range(20, 241, 20))

@@ -578,7 +578,9 @@ def time_policies(cyc, verify, steps, device):
     eager calls with one stream sync per decision.  The policies' weights are
     seeded random and their decisions are computed but not applied (depth
     and N stay the workload's), so the device work equals the timed cycle's;
-    the same eager cycle without the policies is timed beside it."""
+    the same eager cycle without the policies is timed beside it.  Then the
+    same networks run on the device (ltd_depth_policy / ltd_size_policy), the
+    cycle captured as one CUDA graph with and without them."""
     import torch
     from paper_2603_01639_gb300 import policy
     ltd, cfg, tree = cyc.ltd, cyc.cfg, cyc.tree
@@ -615,6 +617,46 @@ def time_policies(cyc, verify, steps, device):
         verify()
         cyc.accept_phase()
 
+    # the same policies on the device: each decision is written where the
+    # next launch reads it, and the whole cycle stays one CUDA graph
+    dnet, snet = pi_d.net.device(device), pi_v.net.device(device)
+    act_scr = torch.empty(B, dtype=torch.int32, device=device)
+    n_scr = torch.empty(B, dtype=torch.int32, device=device)
+
+    def device_adaptive():
+        ltd.ltd_tree_reset(tree, cyc.root)
+        for level in range(1, cyc.max_depth + 1):
+            ltd.ltd_expand_tree(tree, level, cyc.draft, active=cyc.actives[level])
+            ltd.ltd_depth_policy(tree, cyc.ctx, dnet, active_in=cyc.actives[level],
+                                 active_out=act_scr)
+        ltd.ltd_size_policy(tree, cyc.ctx, snet, cfg.max_n, v_pad=v_pad, n_verify=n_scr)
+        ltd.ltd_select_verify(tree, cyc.n_verify, cfg.max_n, cyc.ctx, out=cyc.sel)
+        verify()
+        cyc.accept_phase()
+
+    def depth_only():
+        ltd.ltd_depth_policy(tree, cyc.ctx, dnet, active_in=None, active_out=act_scr)
+
+    def size_only():
+        ltd.ltd_size_policy(tree, cyc.ctx, snet, cfg.max_n, v_pad=v_pad, n_verify=n_scr)
+
+    dev = {}
+    for name, fn in (("graph_fixed", fixed), ("graph_with_device_policies", device_adaptive),
+                     ("depth_policy_launch", depth_only), ("size_policy_launch", size_only)):
+        fn()
+        torch.cuda.synchronize(device)
+        g = _graph(torch, fn)
+        for _ in range(3):
+            g.replay()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(steps):
+            g.replay()
+        e1.record(stream)
+        torch.cuda.synchronize(device)
+        dev[name] = e0.elapsed_time(e1) / steps * 1e3
+    cyc.ltd.ltd_check()
+
     res = {}
     for name, fn in (("eager_fixed", fixed), ("eager_with_policies", adaptive)):
         for _ in range(3):
@@ -636,7 +678,17 @@ def time_policies(cyc, verify, steps, device):
             "depth_mlp_us": round(statistics.median(mlp_s["depth"]) * 1e6, 1),
             "size_mlp_us": round(statistics.median(mlp_s["size"]) * 1e6, 1),
             "mlp": "numpy fp32 on the host, seeded random weights, batch " + str(B),
-            "how": "host wall clock over K eager cycles; decisions computed, not applied"}
+            "how": "host wall clock over K eager cycles; decisions computed, not applied",
+            "device": {
+                "cycle_us_graph_with_device_policies": round(dev["graph_with_device_policies"], 2),
+                "cycle_us_graph_fixed": round(dev["graph_fixed"], 2),
+                "overhead_us": round(dev["graph_with_device_policies"] - dev["graph_fixed"], 2),
+                "overhead_frac": round(1 - dev["graph_fixed"] / dev["graph_with_device_policies"], 4),
+                "depth_policy_us": round(dev["depth_policy_launch"], 2),
+                "size_policy_us": round(dev["size_policy_launch"], 2),
+                "how": "the same networks in mlp_policy_kernel, decisions written to device "
+                       "buffers (not applied), each cycle one CUDA graph; CUDA events over K "
+                       "replays; the policy launches timed alone as graphs of one launch"}}
 
 
 def run_e2e(cyc, args, device):

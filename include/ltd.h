@@ -173,6 +173,82 @@ ltd_status ltd_depth_observation(const ltd_tree* tree, const int32_t* d_ctx, flo
 ltd_status ltd_size_observation(const ltd_tree* tree, const int32_t* d_ctx, int32_t v_pad,
                                 float* d_out, ltd_stream_t stream);
 
+/* The two policies evaluated on the device, so that a decision needs no
+ * round trip to the host and the whole adaptive cycle stays one stream of
+ * launches (capturable in one CUDA graph).  A policy is a ReLU MLP (section
+ * 3.1; Appendix A.2: the depth policy one hidden layer of 1024 units and two
+ * actions STOP = 0 / CONTINUE = 1, the size policy hidden layers of 1024 and
+ * 256 units and 12 actions mapped to V = 20, 40, ..., 240):
+ *   h_0 = observation (the vectors ltd_depth_observation /
+ *         ltd_size_observation write), h_{l+1} = relu(h_l W_l + b_l),
+ *   logits = h_{n-1} W_{n-1} + b_{n-1}, action = argmax (ties to the lower
+ *   action), all in fp32 (accumulation order fixed, run to run identical).
+ * ltd_mlp describes the network; every pointer is device memory owned by
+ * the caller and only read:
+ *   n_layers   1..LTD_MLP_MAX_LAYERS weight matrices
+ *   layout     LTD_MLP_ROW_MAJOR, or LTD_MLP_PACKED for a network that
+ *              ltd_mlp_pack() rearranged (the policies then stream each
+ *              CTA's weight slice with a few large bulk copies; row-major
+ *              weights are read with plain loads, correct but slower)
+ *   dims       dims[0] inputs (k^2 + 2 for the depth policy, v_pad + 2 for
+ *              the size policy, v_pad <= 8192), dims[n_layers] actions,
+ *              hidden widths dims[1..n_layers-1]; every width after dims[0]
+ *              in 1..LTD_MLP_MAX_WIDTH
+ *   w[l]       [dims[l]][dims[l+1]] float, row-major (h_l W_l), 16-byte
+ *              aligned
+ *   b[l]       [dims[l+1]] float
+ * ltd_depth_policy, after level D of the draft:
+ *   d_active_in   [batch] int32, nonzero = the sequence is still drafting
+ *                 (NULL = all); d_active_out [batch] int32 (may equal
+ *                 d_active_in): 1 where the sequence was active, the policy
+ *                 chose CONTINUE and the tree has a level left, else 0.
+ *                 Pass d_active_out as the next ltd_expand_tree's d_active.
+ *   d_logits      optional [batch][2] float (NULL = not written); rows of
+ *                 inactive sequences are written too.
+ *   dims[n_layers] must be 2.
+ * ltd_size_policy, after the draft:
+ *   n_cap         the verify-buffer capacity (n_max of ltd_select_verify)
+ *   d_n_verify    [batch] int32 out: N = min(1 + V, n_cap, nodes in the
+ *                 tree), V = 20 + 20 a for action a (N counts the root).
+ *   d_logits      optional [batch][dims[n_layers]] float.
+ *   dims[n_layers] in 1..LTD_MLP_MAX_WIDTH (12 for the paper's policy).
+ * Errors: LTD_ERR_INVALID_ARG for NULL tree / d_ctx / net / outputs,
+ * n_layers or layout out of range, or weights not 16-byte aligned; LTD_ERR_SHAPE when dims[0] does not match the
+ * observation length, a width is out of range, the depth policy does not
+ * have 2 actions, or (size policy) v_pad is below the tree's max_nodes or
+ * above 8192 or n_cap < 1. */
+#define LTD_MLP_MAX_LAYERS 4
+#define LTD_MLP_MAX_WIDTH 2048
+#define LTD_MLP_ROW_MAJOR 0
+#define LTD_MLP_PACKED 1
+typedef struct ltd_mlp {
+  int32_t n_layers;
+  int32_t layout;
+  int32_t dims[LTD_MLP_MAX_LAYERS + 1];
+  const float* w[LTD_MLP_MAX_LAYERS];
+  const float* b[LTD_MLP_MAX_LAYERS];
+} ltd_mlp;
+/* Rearrange a row-major network for the device policies: each weight
+ * matrix is stored as the column slices the policy kernel's CTAs own, each
+ * slice [dims[l]][slice width] contiguous and zero-padded to a multiple of
+ * four columns.  The layout is private to this library build.
+ *  ltd_mlp_packed_bytes  bytes of device memory the packed weights need
+ *                        (0 for a network the policies would reject)
+ *  ltd_mlp_pack          reads net (LTD_MLP_ROW_MAJOR) on the stream and
+ *                        writes the packed weights into d_mem (256-byte
+ *                        aligned, >= ltd_mlp_packed_bytes); fills *packed
+ *                        with pointers into d_mem, the same dims, the same
+ *                        bias pointers and layout LTD_MLP_PACKED. */
+size_t ltd_mlp_packed_bytes(const ltd_mlp* net);
+ltd_status ltd_mlp_pack(const ltd_mlp* net, void* d_mem, size_t bytes, ltd_mlp* packed,
+                        ltd_stream_t stream);
+ltd_status ltd_depth_policy(const ltd_tree* tree, const int32_t* d_ctx, const ltd_mlp* net,
+                            const int32_t* d_active_in, int32_t* d_active_out, float* d_logits,
+                            ltd_stream_t stream);
+ltd_status ltd_size_policy(const ltd_tree* tree, const int32_t* d_ctx, int32_t v_pad,
+                           const ltd_mlp* net, int32_t n_cap, int32_t* d_n_verify,
+                           float* d_logits, ltd_stream_t stream);
+
 /* Tree attention of the verified tokens against the KV cache (section 3.2
  * "Draft Tree Verification"; tree attention as in SpecInfer, section 2.1).
  * For slot i < N_b and query head h, KV head g = h / (hq/hkv):

@@ -22,14 +22,18 @@ from .ltd_oracle import (  # noqa: F401
     compact_kv,
     cycle,
     depth_observation,
+    depth_policy_step,
     expand_level,
+    first_argmax,
     grow_tree,
     log_softmax,
     mask_words,
+    mlp_forward,
     mix64,
     rank_by_logit,
     select_verify,
     size_observation,
+    size_policy_step,
     splitmix64_stream,
     tree_attention,
     uniform_gumbel,

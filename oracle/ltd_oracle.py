@@ -426,6 +426,47 @@ def size_observation(tree: OracleTree, ctx: int, v_pad: int) -> np.ndarray:
     return out
 
 
+def mlp_forward(x: np.ndarray, layers) -> np.ndarray:
+    """The policies' network (section 3.1; App. A.2 "Architecture"): a
+    feed-forward ReLU network, h <- relu(h W + b) for every hidden layer and
+    logits = h W + b for the last, with W stored [n_in][n_out].  fp64."""
+    h = np.asarray(x, dtype=np.float64)
+    for i, (w, b) in enumerate(layers):
+        h = h @ np.asarray(w, np.float64) + np.asarray(b, np.float64)
+        if i + 1 < len(layers):
+            h = np.maximum(h, 0.0)
+    return h
+
+
+def first_argmax(z) -> int:
+    """Index of the largest entry, ties to the lower index."""
+    z = list(z)
+    best = 0
+    for j in range(1, len(z)):
+        if z[j] > z[best]:
+            best = j
+    return best
+
+
+def depth_policy_step(tree: OracleTree, ctx: int, layers, active: bool, max_depth: int):
+    """One decision of the depth policy after the last built level (App. A.2
+    "Depth Policy": a binary STOP / CONTINUE action per level).  Action 1 is
+    CONTINUE; a sequence keeps drafting if it was active, the policy says
+    CONTINUE and a level is left.  Returns (keep drafting, logits)."""
+    z = mlp_forward(depth_observation(tree, ctx)[None, :], layers)[0]
+    return bool(active and first_argmax(z) == 1 and tree.levels < max_depth), z
+
+
+def size_policy_step(tree: OracleTree, ctx: int, v_pad: int, layers, n_cap: int):
+    """The size policy's decision after the draft (App. A.2 "Size Policy":
+    discrete actions mapped linearly onto V = 20, 40, ..., 240).  V counts
+    candidate tokens, N = V + 1 counts the root too; N is capped by the verify
+    buffer (n_cap) and by the tree's node count.  Returns (N, logits)."""
+    z = mlp_forward(size_observation(tree, ctx, v_pad)[None, :], layers)[0]
+    v = 20 + 20 * first_argmax(z)
+    return min(1 + v, n_cap, tree.n_nodes), z
+
+
 # ------------------------------------------------------------- whole cycle
 def cycle(root_token, draft_rows, W, L, N, ctx, target_rows, mode="greedy",
           seed=0, b=0, cycle_no=0):

@@ -187,6 +187,62 @@ ltd_status ltd_size_observation(const ltd_tree* tree, const int32_t* d_ctx, int3
       launch_size_obs(tree, d_ctx, v_pad, d_out, reinterpret_cast<cudaStream_t>(stream)));
 }
 
+// Common checks of a policy network; n_in is the observation length.
+static ltd_status mlp_ok(const ltd_mlp* net, int32_t n_in) {
+  if (net == nullptr || net->n_layers < 1 || net->n_layers > LTD_MLP_MAX_LAYERS)
+    return LTD_ERR_INVALID_ARG;
+  if (net->layout != LTD_MLP_ROW_MAJOR && net->layout != LTD_MLP_PACKED) return LTD_ERR_INVALID_ARG;
+  for (int l = 0; l < net->n_layers; ++l)
+    if (net->w[l] == nullptr || net->b[l] == nullptr ||
+        reinterpret_cast<uintptr_t>(net->w[l]) % 16 != 0)
+      return LTD_ERR_INVALID_ARG;
+  if (n_in >= 0 && net->dims[0] != n_in) return LTD_ERR_SHAPE;
+  if (net->dims[0] < 1) return LTD_ERR_SHAPE;
+  for (int l = 1; l <= net->n_layers; ++l)
+    if (net->dims[l] < 1 || net->dims[l] > LTD_MLP_MAX_WIDTH) return LTD_ERR_SHAPE;
+  return LTD_OK;
+}
+
+size_t ltd_mlp_packed_bytes(const ltd_mlp* net) {
+  if (mlp_ok(net, -1) != LTD_OK) return 0;
+  size_t off[LTD_MLP_MAX_LAYERS];
+  return mlp_packed_floats(net, off) * sizeof(float);
+}
+
+ltd_status ltd_mlp_pack(const ltd_mlp* net, void* d_mem, size_t bytes, ltd_mlp* packed,
+                        ltd_stream_t stream) {
+  if (packed == nullptr || d_mem == nullptr || reinterpret_cast<uintptr_t>(d_mem) % 256 != 0)
+    return LTD_ERR_INVALID_ARG;
+  const ltd_status st = mlp_ok(net, -1);
+  if (st != LTD_OK) return st;
+  if (net->layout != LTD_MLP_ROW_MAJOR) return LTD_ERR_INVALID_ARG;
+  if (bytes < ltd_mlp_packed_bytes(net)) return LTD_ERR_SHAPE;
+  return from_cuda(launch_mlp_pack(net, static_cast<float*>(d_mem), packed,
+                                   reinterpret_cast<cudaStream_t>(stream)));
+}
+
+ltd_status ltd_depth_policy(const ltd_tree* tree, const int32_t* d_ctx, const ltd_mlp* net,
+                            const int32_t* d_active_in, int32_t* d_active_out, float* d_logits,
+                            ltd_stream_t stream) {
+  if (!tree_ok(tree) || d_ctx == nullptr || d_active_out == nullptr) return LTD_ERR_INVALID_ARG;
+  const ltd_status st = mlp_ok(net, tree->k * tree->k + 2);
+  if (st != LTD_OK) return st;
+  if (net->dims[net->n_layers] != 2) return LTD_ERR_SHAPE;
+  return from_cuda(launch_mlp_policy(tree, d_ctx, net, 0, 0, d_active_in, d_active_out, 0,
+                                     nullptr, d_logits, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+ltd_status ltd_size_policy(const ltd_tree* tree, const int32_t* d_ctx, int32_t v_pad,
+                           const ltd_mlp* net, int32_t n_cap, int32_t* d_n_verify,
+                           float* d_logits, ltd_stream_t stream) {
+  if (!tree_ok(tree) || d_ctx == nullptr || d_n_verify == nullptr) return LTD_ERR_INVALID_ARG;
+  if (v_pad < tree->max_nodes || v_pad > 8192 || n_cap < 1) return LTD_ERR_SHAPE;
+  const ltd_status st = mlp_ok(net, v_pad + 2);
+  if (st != LTD_OK) return st;
+  return from_cuda(launch_mlp_policy(tree, d_ctx, net, 1, v_pad, nullptr, nullptr, n_cap,
+                                     d_n_verify, d_logits, reinterpret_cast<cudaStream_t>(stream)));
+}
+
 ltd_status ltd_select_verify(const ltd_tree* tree, const int32_t* d_n_verify, int32_t n_max,
                              const int32_t* d_ctx, int32_t* d_node_ids, int32_t* d_pos,
                              uint32_t* d_mask, ltd_stream_t stream) {

@@ -193,6 +193,16 @@ constexpr float kPolicyPad = LTD_POLICY_PAD;
 cudaError_t launch_depth_obs(const ltd_tree* t, const int32_t* ctx, float* out, cudaStream_t s);
 cudaError_t launch_size_obs(const ltd_tree* t, const int32_t* ctx, int32_t v_pad, float* out,
                             cudaStream_t s);
+// Packed policy weights (k_policy.cu): units of a layer's column slice per
+// CTA, the packed float count (and each matrix's offset), and the packing.
+int mlp_packed_units(int n_out);
+size_t mlp_packed_floats(const ltd_mlp* net, size_t offsets[LTD_MLP_MAX_LAYERS]);
+cudaError_t launch_mlp_pack(const ltd_mlp* net, float* base, ltd_mlp* packed, cudaStream_t s);
+// Depth (size_policy 0) or size (1) policy MLP on the device (k_policy.cu).
+cudaError_t launch_mlp_policy(const ltd_tree* t, const int32_t* ctx, const ltd_mlp* net,
+                              int32_t size_policy, int32_t v_pad, const int32_t* active_in,
+                              int32_t* active_out, int32_t n_cap, int32_t* n_verify,
+                              float* logits, cudaStream_t s);
 cudaError_t launch_accept(const AcceptParams& p, int32_t batch, ltd_dtype dtype, cudaStream_t s);
 
 struct CompactParams {

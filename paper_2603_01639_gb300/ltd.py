@@ -30,9 +30,12 @@ EXPORTS = [
     "ltd_attention_workspace_bytes", "ltd_tree_attention", "ltd_accept_workspace_bytes",
     "ltd_accept", "ltd_kv_compact", "ltd_check", "ltd_status_string", "ltd_version",
     "ltd_attention_kernel", "ltd_selftest_umma", "ltd_accept_noalloc", "ltd_tree_attention_next",
-    "ltd_depth_observation", "ltd_size_observation",
+    "ltd_depth_observation", "ltd_size_observation", "ltd_depth_policy", "ltd_size_policy",
+    "ltd_mlp_packed_bytes", "ltd_mlp_pack",
 ]
 LTD_POLICY_PAD = -100.0
+LTD_MLP_MAX_LAYERS, LTD_MLP_MAX_WIDTH = 4, 2048
+LTD_MLP_ROW_MAJOR, LTD_MLP_PACKED = 0, 1
 LTD_ACCEPT_NOALLOC_SCRATCH_BYTES = 1 << 20
 
 
@@ -55,6 +58,12 @@ class ltd_kv_cache(C.Structure):
                 ("s_cap", C.c_int32), ("dtype", C.c_int32)]
 
 
+class ltd_mlp(C.Structure):
+    _fields_ = [("n_layers", C.c_int32), ("layout", C.c_int32),
+                ("dims", C.c_int32 * (LTD_MLP_MAX_LAYERS + 1)),
+                ("w", C.c_void_p * LTD_MLP_MAX_LAYERS), ("b", C.c_void_p * LTD_MLP_MAX_LAYERS)]
+
+
 def lib():
     """Load libltd.so once; raise if it is not built."""
     global _lib
@@ -74,6 +83,10 @@ def lib():
                 "ltd_select_verify": (C.c_int, [tp, vp, i32, vp, vp, vp, vp, vp]),
                 "ltd_depth_observation": (C.c_int, [tp, vp, vp, vp]),
                 "ltd_size_observation": (C.c_int, [tp, vp, i32, vp, vp]),
+                "ltd_mlp_packed_bytes": (sz, [C.POINTER(ltd_mlp)]),
+                "ltd_mlp_pack": (C.c_int, [C.POINTER(ltd_mlp), vp, sz, C.POINTER(ltd_mlp), vp]),
+                "ltd_depth_policy": (C.c_int, [tp, vp, C.POINTER(ltd_mlp), vp, vp, vp, vp]),
+                "ltd_size_policy": (C.c_int, [tp, vp, i32, C.POINTER(ltd_mlp), i32, vp, vp, vp]),
                 "ltd_attention_workspace_bytes": (sz, [i32, i32, i32, i32, i32, i32, C.c_int]),
                 "ltd_tree_attention": (C.c_int, [vp, vp, vp, vp, C.c_int, i32, i32, i32, i32, i32,
                                                  vp, i32, vp, i32, vp, C.c_float, vp, sz, vp]),
@@ -244,6 +257,74 @@ def ltd_size_observation(tree: Tree, ctx: torch.Tensor, v_pad=None, out=None, st
     _ok(lib().ltd_size_observation(C.byref(tree.s), _ptr(ctx), v_pad, _ptr(out), _stream(stream)),
         "ltd_size_observation")
     return out
+
+
+class MlpNet:
+    """A policy MLP's weights on the device ([n_in][n_out] fp32 matrices and
+    biases) and the ltd_mlp struct that points at them; with ``packed`` the
+    struct points at the library's packed copy (ltd_mlp_pack), which the
+    device policies stream with bulk copies."""
+
+    def __init__(self, layers, device="cuda", packed=True, stream=None):
+        if not 1 <= len(layers) <= LTD_MLP_MAX_LAYERS:
+            raise LtdError(f"an MLP has 1..{LTD_MLP_MAX_LAYERS} layers")
+        self.w = [torch.as_tensor(w, dtype=torch.float32).to(device).contiguous() for w, _ in layers]
+        self.b = [torch.as_tensor(b, dtype=torch.float32).to(device).contiguous() for _, b in layers]
+        self.s = ltd_mlp()
+        self.s.n_layers = len(layers)
+        self.s.dims[0] = self.w[0].shape[0]
+        for i, (w, b) in enumerate(zip(self.w, self.b)):
+            if w.dim() != 2 or b.shape != (w.shape[1],) or (i and w.shape[0] != self.w[i - 1].shape[1]):
+                raise LtdError("MLP layer shapes do not chain")
+            self.s.dims[i + 1] = w.shape[1]
+            self.s.w[i] = w.data_ptr()
+            self.s.b[i] = b.data_ptr()
+        self.row_major = self.s
+        if packed:
+            n = lib().ltd_mlp_packed_bytes(C.byref(self.s))
+            if n == 0:
+                raise LtdError("ltd_mlp_packed_bytes: the policies would reject this network")
+            self.pbuf = torch.empty(n + 256, dtype=torch.uint8, device=device)
+            off = (-self.pbuf.data_ptr()) % 256
+            p = ltd_mlp()
+            _ok(lib().ltd_mlp_pack(C.byref(self.s), C.c_void_p(self.pbuf.data_ptr() + off), n,
+                                   C.byref(p), _stream(stream)), "ltd_mlp_pack")
+            self.s = p
+
+    @property
+    def n_in(self):
+        return self.s.dims[0]
+
+    @property
+    def n_out(self):
+        return self.s.dims[self.s.n_layers]
+
+
+def ltd_depth_policy(tree: Tree, ctx: torch.Tensor, net: MlpNet, active_in=None, active_out=None,
+                     logits=None, stream=None):
+    """Depth policy on the device after the last built level: returns the
+    next level's active mask [B] int32 (1 = keep drafting)."""
+    _need(ctx, "ctx", torch.int32)
+    if active_out is None:
+        active_out = torch.empty(tree.batch, dtype=torch.int32, device=ctx.device)
+    _ok(lib().ltd_depth_policy(C.byref(tree.s), _ptr(ctx), C.byref(net.s), _ptr(active_in),
+                               _ptr(active_out), _ptr(logits), _stream(stream)),
+        "ltd_depth_policy")
+    return active_out
+
+
+def ltd_size_policy(tree: Tree, ctx: torch.Tensor, net: MlpNet, n_cap: int, v_pad=None,
+                    n_verify=None, logits=None, stream=None):
+    """Size policy on the device after the draft: returns N per sequence
+    ([B] int32, root included, at most n_cap and the tree's node count)."""
+    _need(ctx, "ctx", torch.int32)
+    v_pad = tree.max_nodes if v_pad is None else v_pad
+    if n_verify is None:
+        n_verify = torch.empty(tree.batch, dtype=torch.int32, device=ctx.device)
+    _ok(lib().ltd_size_policy(C.byref(tree.s), _ptr(ctx), v_pad, C.byref(net.s), n_cap,
+                              _ptr(n_verify), _ptr(logits), _stream(stream)),
+        "ltd_size_policy")
+    return n_verify
 
 
 def attention_workspace(batch, hq, hkv, head_dim, n_max, max_ctx, dtype, device="cuda"):

@@ -85,6 +85,48 @@ def test_entry_points_reject_bad_arguments_before_launch(L):
     assert L.ltd_depth_observation(C.byref(t), None, fake, s) == 1
     assert L.ltd_size_observation(C.byref(t), fake, t.max_nodes - 1, fake, s) == 2  # v_pad short
     assert L.ltd_size_observation(C.byref(t), fake, t.max_nodes, None, s) == 1
+    net = ltd.ltd_mlp()
+    net.n_layers = 2
+    net.dims[0], net.dims[1], net.dims[2] = 4 * 4 + 2, 1024, 2
+    for i in range(2):
+        net.w[i] = 1 << 24
+        net.b[i] = 1 << 24
+    P = C.byref(net)
+    assert L.ltd_depth_policy(C.byref(t), fake, None, None, fake, None, s) == 1
+    assert L.ltd_depth_policy(C.byref(t), fake, P, None, None, None, s) == 1        # no output
+    net.dims[0] = 17
+    assert L.ltd_depth_policy(C.byref(t), fake, P, None, fake, None, s) == 2        # obs length
+    net.dims[0], net.dims[2] = 18, 3
+    assert L.ltd_depth_policy(C.byref(t), fake, P, None, fake, None, s) == 2        # 3 actions
+    net.dims[2] = 2
+    net.w[1] = None
+    assert L.ltd_depth_policy(C.byref(t), fake, P, None, fake, None, s) == 1        # null weight
+    net.w[1] = 1 << 24
+    net.n_layers = 5
+    assert L.ltd_depth_policy(C.byref(t), fake, P, None, fake, None, s) == 1        # > max layers
+    net.n_layers = 2
+    net.dims[0], net.dims[2] = t.max_nodes + 2, 12
+    assert L.ltd_size_policy(C.byref(t), fake, t.max_nodes - 1, P, 64, fake, None, s) == 2
+    assert L.ltd_size_policy(C.byref(t), fake, t.max_nodes, P, 0, fake, None, s) == 2
+    assert L.ltd_size_policy(C.byref(t), fake, t.max_nodes, P, 64, None, None, s) == 1
+    net.dims[1] = ltd.LTD_MLP_MAX_WIDTH + 1
+    assert L.ltd_size_policy(C.byref(t), fake, t.max_nodes, P, 64, fake, None, s) == 2  # width
+    net.dims[1] = 1024
+    net.layout = 2
+    assert L.ltd_size_policy(C.byref(t), fake, t.max_nodes, P, 64, fake, None, s) == 1  # layout
+    assert L.ltd_mlp_packed_bytes(P) == 0
+    net.layout = ltd.LTD_MLP_ROW_MAJOR
+    net.w[0] = (1 << 24) + 4
+    assert L.ltd_size_policy(C.byref(t), fake, t.max_nodes, P, 64, fake, None, s) == 1  # misaligned
+    assert L.ltd_mlp_packed_bytes(P) == 0
+    net.w[0] = 1 << 24
+    # packed size: every weight plus column padding, whole 256-byte blocks
+    n = L.ltd_mlp_packed_bytes(P)
+    assert n >= 4 * ((t.max_nodes + 2) * 1024 + 1024 * 12) and n % 256 == 0
+    out = ltd.ltd_mlp()
+    assert L.ltd_mlp_pack(P, fake, n, None, s) == 1
+    assert L.ltd_mlp_pack(P, C.c_void_p((1 << 24) + 16), n, C.byref(out), s) == 1   # d_mem align
+    assert L.ltd_mlp_pack(P, fake, n - 4, C.byref(out), s) == 2
     ws = L.ltd_attention_workspace_bytes(1, 4, 1, 64, 8, 128, 0)
     assert ws > 0
     assert L.ltd_attention_workspace_bytes(1, 5, 2, 64, 8, 128, 0) == 0          # hq % hkv

@@ -507,6 +507,72 @@ def test_observations_against_depth_and_path_sums(W, L):
     assert list(s[v_pad:]) == [L, ctx]
 
 
+# ----------------------------------------------------------- policy MLP pins
+def test_mlp_hand_worked():
+    """x = (1, 2); hidden = relu(x W1 + b1) = relu(3.5, -7) = (3.5, 0);
+    logits = (3.5*2, 3.5*(-1) + 1) = (7, -2.5), worked by hand."""
+    w1, b1 = [[1.0, -1.0], [1.0, -3.0]], [0.5, 0.0]
+    w2, b2 = [[2.0, -1.0], [5.0, 7.0]], [0.0, 1.0]
+    z = O.mlp_forward(np.array([[1.0, 2.0]]), [(w1, b1), (w2, b2)])
+    assert z.tolist() == [[7.0, -2.5]]
+    assert O.first_argmax(z[0]) == 0
+
+
+def test_mlp_against_torch_linear_layers():
+    """torch.nn.Linear holds W as [out][in] and computes x W^T + b; the
+    oracle's [in][out] matrices transposed into it give the same network
+    (n_in, hidden and n_out all differ, so a transposed operand cannot pass)."""
+    rng = np.random.default_rng(5)
+    dims = [7, 11, 5, 3]
+    layers = [(rng.standard_normal((a, b)), rng.standard_normal(b)) for a, b in zip(dims[:-1], dims[1:])]
+    mods = []
+    for i, (w, b) in enumerate(layers):
+        lin = torch.nn.Linear(w.shape[0], w.shape[1], dtype=torch.float64)
+        with torch.no_grad():
+            lin.weight.copy_(torch.from_numpy(w.T))
+            lin.bias.copy_(torch.from_numpy(b))
+        mods.append(lin)
+        if i + 1 < len(layers):
+            mods.append(torch.nn.ReLU())
+    x = rng.standard_normal((4, dims[0]))
+    ref = torch.nn.Sequential(*mods)(torch.from_numpy(x)).detach().numpy()
+    np.testing.assert_allclose(O.mlp_forward(x, layers), ref, rtol=1e-13, atol=1e-13)
+
+
+def test_argmax_ties_to_the_lower_action():
+    assert O.first_argmax([1.0, 3.0, 3.0, 2.0]) == 1
+    assert O.first_argmax([0.0, 0.0]) == 0
+
+
+def _bias_only(n_in, n_out, action):
+    w = np.zeros((n_in, n_out))
+    b = np.zeros(n_out)
+    b[action] = 1.0
+    return [(w, b)]
+
+
+def test_size_policy_maps_actions_to_20_through_240():
+    """12 actions map linearly onto V = 20..240 (App. A.2); N = V + 1 counts
+    the root and is capped by the verify buffer and the tree size."""
+    big, _, _ = _random_tree(3, 10, 3, vocab=50)     # 211 nodes
+    v_pad = big.n_nodes
+    got = [O.size_policy_step(big, 100, v_pad, _bias_only(v_pad + 2, 12, a), 256)[0]
+           for a in range(12)]
+    assert got == [21, 41, 61, 81, 101, 121, 141, 161, 181, 201, 211, 211]
+    assert O.size_policy_step(big, 100, v_pad, _bias_only(v_pad + 2, 12, 11), 64)[0] == 64
+    small, _, _ = _random_tree(4, 2, 2, vocab=9)     # 7 nodes
+    assert O.size_policy_step(small, 5, 7, _bias_only(9, 12, 0), 256)[0] == 7
+
+
+def test_depth_policy_continue_stop_and_limits():
+    tree, _, _ = _random_tree(6, 3, 2, vocab=20)
+    cont, stop = _bias_only(11, 2, 1), _bias_only(11, 2, 0)
+    assert O.depth_policy_step(tree, 9, cont, True, 4)[0] is True
+    assert O.depth_policy_step(tree, 9, stop, True, 4)[0] is False
+    assert O.depth_policy_step(tree, 9, cont, False, 4)[0] is False    # already stopped
+    assert O.depth_policy_step(tree, 9, cont, True, 2)[0] is False     # no level left
+
+
 def test_planted_mistake_in_log_softmax_is_caught(monkeypatch):
     monkeypatch.setattr(O, "log_softmax", _mutant_log_softmax_dropped_lse)
     with pytest.raises(AssertionError):
@@ -595,3 +661,14 @@ def test_planted_mistake_in_depth_observation_is_caught(monkeypatch):
     monkeypatch.setattr(O, "depth_observation", shifted)
     with pytest.raises(AssertionError):
         test_observations_against_depth_and_path_sums(3, 4)
+
+
+def test_planted_mistake_in_mlp_is_caught(monkeypatch):
+    def no_relu(x, layers):   # mistake: the hidden ReLU dropped
+        h = np.asarray(x, np.float64)
+        for w, b in layers:
+            h = h @ np.asarray(w, np.float64) + np.asarray(b, np.float64)
+        return h
+    monkeypatch.setattr(O, "mlp_forward", no_relu)
+    with pytest.raises(AssertionError):
+        test_mlp_hand_worked()

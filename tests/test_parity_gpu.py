@@ -135,6 +135,134 @@ def test_policy_observations(name, seed):
         _check_obs(got[b], ref, cum[b], np.arange(n), n, v_pad)
 
 
+# ------------------------------------------------------- policies on device
+def _abs_bound(x, layers):
+    """Forward of |x| through |W|, |b| without the ReLU's cut: bounds every
+    partial sum, so fp32 rounding stays below ~n eps times it."""
+    h = np.abs(np.asarray(x, np.float64))
+    for w, b in layers:
+        h = h @ np.abs(np.asarray(w, np.float64)) + np.abs(np.asarray(b, np.float64))
+    return h
+
+
+@pytest.mark.parametrize("name,seed,packed", [("8b", 0, True), ("8b", 0, False), ("70b", 0, True),
+                                              ("70b", 2, False)])
+def test_device_policies_match_the_oracle_network(name, seed, packed):
+    """The paper-size networks (seeded random weights), packed for the
+    streaming kernel and row-major: logits against the fp64 oracle network
+    fed the same observation, decisions where the fp64 top-two gap is clear
+    of the fp32 error."""
+    from paper_2603_01639_gb300 import policy
+    cfg = wl.config(name)
+    ci = wl.draw_cycle(cfg, seed)
+    B, W = cfg.batch, cfg.W
+    draft = H.dev(ci.draft_rows, cfg.dtype)
+    ctx = H.i32(ci.ctx)
+    tree = ltd.Tree(B, cfg.max_depth, W, cfg.vocab)
+    dp = policy.DepthPolicy(W, seed=3)
+    sp = policy.SizePolicy(tree.max_nodes, seed=4)
+    dnet, snet = dp.net.device(packed=packed), sp.net.device(packed=packed)
+    ltd.ltd_tree_reset(tree, H.i32(ci.root))
+    depth = np.asarray(ci.depth)
+
+    def check(obs, logits, layers):
+        ref = oracle.mlp_forward(obs.astype(np.float64), layers)
+        tol = 2e-5 * _abs_bound(obs, layers) + 1e-6
+        assert (np.abs(logits - ref) <= tol).all(), np.abs(logits - ref).max()
+        return ref, tol
+
+    for level in range(1, int(depth.max()) + 1):
+        act = H.i32((depth >= level).astype(np.int32))
+        ltd.ltd_expand_tree(tree, level, draft, active=act)
+        logits = torch.empty(B, 2, dtype=torch.float32, device="cuda")
+        out = ltd.ltd_depth_policy(tree, ctx, dnet, active_in=act, logits=logits)
+        obs = ltd.ltd_depth_observation(tree, ctx).cpu().numpy()
+        assert ltd.ltd_check() == 0
+        ref, tol = check(obs, logits.cpu().numpy(), dp.net.layers)
+        want = (ref[:, 1] > ref[:, 0]) & (depth >= level) & (level < cfg.max_depth)
+        clear = np.abs(ref[:, 1] - ref[:, 0]) > 2 * tol.max(axis=1)
+        assert clear.all(), "near-tie in a depth decision; pick another seed"
+        np.testing.assert_array_equal(out.cpu().numpy(), want.astype(np.int32))
+    logits = torch.empty(B, 12, dtype=torch.float32, device="cuda")
+    n = ltd.ltd_size_policy(tree, ctx, snet, cfg.max_n, logits=logits).cpu().numpy()
+    obs = ltd.ltd_size_observation(tree, ctx).cpu().numpy()
+    assert ltd.ltd_check() == 0
+    ref, tol = check(obs, logits.cpu().numpy(), sp.net.layers)
+    nodes = tree.view()["n_nodes"].cpu().numpy()
+    for b in range(B):
+        top2 = np.sort(ref[b])[-2:]
+        assert top2[1] - top2[0] > 2 * tol[b].max(), "near-tie in a size decision"
+        a = int(np.argmax(ref[b]))
+        assert n[b] == min(21 + 20 * a, cfg.max_n, int(nodes[b]))
+
+
+def _designed_nets(kk, v_pad):
+    """Networks whose decisions read off the observation exactly (powers of
+    two and small integers, so fp32 and fp64 agree bit for bit):
+    depth: STOP logit D, CONTINUE logit L/2048 + 1.75 -> keep drafting while
+    D < L/2048 + 1.75; size: logit_j = j D - j^2/2 -> action D, V = 20 + 20 D."""
+    w1 = np.zeros((kk + 2, 2), np.float32)
+    w1[kk, 0] = 1.0
+    w1[kk + 1, 1] = 1.0 / 2048
+    depth = [(w1, np.zeros(2, np.float32)), (np.eye(2, dtype=np.float32), np.array([0, 1.75], np.float32))]
+    s1 = np.zeros((v_pad + 2, 1), np.float32)
+    s1[v_pad, 0] = 1.0
+    j = np.arange(12, dtype=np.float32)
+    size = [(s1, np.zeros(1, np.float32)), (j[None, :], -0.5 * j * j)]
+    return depth, size
+
+
+@pytest.mark.parametrize("name,seed", [("tiny", 0), ("70b", 0), ("70b", 3)])
+def test_adaptive_draft_driven_by_device_policies(name, seed):
+    """The depth policy's decisions drive the draft on the device (each
+    level's active mask is the previous decision), the size policy's N feeds
+    the selection; the oracle follows its own decisions.  Levels, trees, N
+    and the selection must agree exactly."""
+    cfg = wl.config(name)
+    ci = wl.draw_cycle(cfg, seed)
+    B, W = cfg.batch, cfg.W
+    draft = H.dev(ci.draft_rows, cfg.dtype)
+    ctx = H.i32(ci.ctx)
+    tree = ltd.Tree(B, cfg.max_depth, W, cfg.vocab)
+    dl, sl = _designed_nets(W * W, tree.max_nodes)
+    dnet, snet = ltd.MlpNet(dl), ltd.MlpNet(sl)
+    # the oracle's adaptive draft
+    otrees = []
+    for b in range(B):
+        t = oracle.OracleTree.rooted(int(ci.root[b]), W)
+        keep = True
+        while keep:
+            lv = t.levels + 1
+            r0 = 0 if lv == 1 else 1 + (lv - 2) * W
+            oracle.expand_level(t, ci.draft_rows[b][r0:(1 if lv == 1 else r0 + W)])
+            keep, _ = oracle.depth_policy_step(t, int(ci.ctx[b]), dl, True, cfg.max_depth)
+        otrees.append(t)
+    # the device's: every level launched, sequences stop on the device
+    ltd.ltd_tree_reset(tree, H.i32(ci.root))
+    act = torch.ones(B, dtype=torch.int32, device="cuda")
+    for level in range(1, cfg.max_depth + 1):
+        ltd.ltd_expand_tree(tree, level, draft, active=act)
+        ltd.ltd_depth_policy(tree, ctx, dnet, active_in=act, active_out=act)
+    n_dev = ltd.ltd_size_policy(tree, ctx, snet, cfg.max_n)
+    got = ltd.ltd_select_verify(tree, n_dev, cfg.max_n, ctx)
+    assert ltd.ltd_check() == 0
+    levels = [t.levels for t in otrees]
+    if B > 1:
+        assert len(set(levels)) > 1, "the designed policy should stop sequences at different depths"
+    v = tree.view()
+    np.testing.assert_array_equal(v["n_levels"].cpu().numpy(), levels)
+    assert min(H.tree_margin(t, W) for t in otrees) > H.CUT_MARGIN
+    ci.depth = np.array(levels, np.int32)
+    H.compare_trees(cfg, ci, tree, otrees)
+    n_ref = [oracle.size_policy_step(t, int(ci.ctx[b]), tree.max_nodes, sl, cfg.max_n)[0]
+             for b, t in enumerate(otrees)]
+    np.testing.assert_array_equal(n_dev.cpu().numpy(), n_ref)
+    ci.n_verify = np.array(n_ref, np.int32)
+    sels = [oracle.select_verify(t, int(n), int(ci.ctx[b])) for b, (t, n) in enumerate(zip(otrees, n_ref))]
+    assert min(H.select_margin(t, int(n)) for t, n in zip(otrees, n_ref)) > H.CUT_MARGIN
+    H.compare_select(cfg, ci, got, sels, otrees)
+
+
 def test_determinism_and_reuse_of_scratch():
     """Same inputs twice through the same tree and workspace: identical bits
     (tickets and scratch are left ready for reuse)."""

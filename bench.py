@@ -532,6 +532,14 @@ def run_ours(args):
                 "tflops": round(att_flops / (att_launch_ms * 1e-3) / 1e12, 1),
                 "frac_of_8tbs": round(achieved / 8000.0, 4)}
 
+    # the cycle's throughput, the reward of section 3.1: tokens emitted
+    # (accepted + bonus) over the device time of the cycle
+    acc_len = cyc.acc["accept_len"].cpu().numpy()
+    reward = {"accept_len": acc_len.tolist(),
+              "tokens_per_cycle": int((acc_len + 1).sum()),
+              "tokens_per_s": round(float((acc_len + 1).sum()) / (ms_per_step * 1e-3), 1),
+              "how": "(accepted + 1) summed over the batch / device time of one cycle"}
+
     pol = None
     if not args.no_policy:
         pol = time_policies(cyc, verify, K, device)
@@ -561,7 +569,7 @@ def run_ours(args):
             "phases_us": {"draft_select": round(draft_ms * 1e3, 2),
                           "attention_all_layers": round(verify_ms * 1e3, 2),
                           "accept_compact": round(accept_ms * 1e3, 2)},
-            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "policy": pol,
+            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "policy": pol, "reward": reward,
             "gpu_launches": cyc.launches_per_step() * K, "clocks": clk,
         }
         print(json.dumps(line), flush=True)

@@ -532,6 +532,29 @@ def run_ours(args):
                 "tflops": round(att_flops / (att_launch_ms * 1e-3) / 1e12, 1),
                 "frac_of_8tbs": round(achieved / 8000.0, 4)}
 
+    # the acceptance phase under each verification rule on this cycle (all
+    # sequences on one rule; the timed cycle above keeps the workload's)
+    rules = {}
+    saved_mode = cyc.mode.clone()
+    for rname, rmode in (("greedy", ltd.LTD_GREEDY), ("stochastic", ltd.LTD_STOCHASTIC),
+                         ("point_mass", ltd.LTD_STOCHASTIC_POINT_MASS)):
+        cyc.mode.fill_(rmode)
+        g_rule = _graph(torch, cyc.accept_phase)
+        g_rule.replay()
+        torch.cuda.synchronize(device)
+        r0, r1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        r0.record(stream)
+        for _ in range(K):
+            g_rule.replay()
+        r1.record(stream)
+        torch.cuda.synchronize(device)
+        rules[rname] = round(r0.elapsed_time(r1) / K * 1e3, 2)
+    cyc.mode.copy_(saved_mode)
+    ltd.ltd_check()
+    # re-run the workload's own acceptance so the outputs below are its own
+    g_accept.replay()
+    torch.cuda.synchronize(device)
+
     # the cycle's throughput, the reward of section 3.1: tokens emitted
     # (accepted + bonus) over the device time of the cycle
     acc_len = cyc.acc["accept_len"].cpu().numpy()
@@ -569,6 +592,7 @@ def run_ours(args):
             "phases_us": {"draft_select": round(draft_ms * 1e3, 2),
                           "attention_all_layers": round(verify_ms * 1e3, 2),
                           "accept_compact": round(accept_ms * 1e3, 2)},
+            "accept_rules_us": rules,
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "policy": pol, "reward": reward,
             "gpu_launches": cyc.launches_per_step() * K, "clocks": clk,
         }

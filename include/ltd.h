@@ -54,7 +54,7 @@ typedef enum ltd_status {
 } ltd_status;
 
 typedef enum ltd_dtype { LTD_F32 = 0, LTD_BF16 = 1 } ltd_dtype;
-typedef enum ltd_mode { LTD_GREEDY = 0, LTD_STOCHASTIC = 1 } ltd_mode;
+typedef enum ltd_mode { LTD_GREEDY = 0, LTD_STOCHASTIC = 1, LTD_STOCHASTIC_POINT_MASS = 2 } ltd_mode;
 
 /* Limits of this build. */
 #define LTD_MAX_K 32          /* beam width k                              */
@@ -68,7 +68,7 @@ typedef enum ltd_mode { LTD_GREEDY = 0, LTD_STOCHASTIC = 1 } ltd_mode;
 #define LTD_DEVERR_CTX 0x4u       /* ctx < 0, ctx > max_ctx, ctx+N > s_cap */
 #define LTD_DEVERR_TREE 0x8u      /* selection not ancestor-closed        */
 #define LTD_DEVERR_TIMEOUT 0x10u  /* a bounded wait gave up               */
-#define LTD_DEVERR_MODE 0x20u     /* mode other than greedy/stochastic    */
+#define LTD_DEVERR_MODE 0x20u     /* mode not one of ltd_mode             */
 
 /* ------------------------------------------------------------------------
  * Draft tree (section 3.2, "Draft Tree Generation").
@@ -325,8 +325,15 @@ typedef struct ltd_kv_cache {
  * + w_j) over the words (b, cycle, stream, slot, i-or-token), mix64 being the
  * splitmix64 finaliser; r = (h >> 40) 2^-24 (stream 0), g = (2 (h >> 41) + 1)
  * 2^-24 (stream 1).
+ * Stochastic with point-mass proposals (LTD_STOCHASTIC_POINT_MASS, T = 1):
+ * the children are deterministic top-k proposals, so each is treated as a
+ * point mass on its token: child x_i is accepted if r_i (1 - p(R)) < p(x_i),
+ * R the children rejected so far at this slot, else x_i joins R; with no
+ * child accepted the bonus is the Gumbel-max draw over the tokens outside R.
+ * The emitted token is distributed exactly as p for any set of children;
+ * no draft row is read and a rejection costs no pass over the vocabulary.
  *  d_target_logits  [batch][n_max][vocab] (dtype), row i = target at slot i
- *  d_draft_rows     the row store given to ltd_expand_tree (stochastic only)
+ *  d_draft_rows     the row store given to ltd_expand_tree (LTD_STOCHASTIC only)
  *  d_node_ids       ltd_select_verify output
  *  d_ctx            [batch] in; d_new_ctx [batch] out = ctx + 1 + accept_len
  *  d_path           out [batch][max_depth+1] accepted slots, -1 after the end

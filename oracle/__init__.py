@@ -18,6 +18,7 @@ from .ltd_oracle import (  # noqa: F401
     POLICY_PAD,
     OracleTree,
     accept_greedy,
+    accept_point_mass,
     accept_stochastic,
     compact_kv,
     cycle,

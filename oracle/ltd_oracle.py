@@ -378,6 +378,56 @@ def accept_stochastic(tree: OracleTree, chosen, target_rows, draft_rows, seed, b
         slot = accepted
 
 
+def accept_point_mass(tree: OracleTree, chosen, target_rows, seed, b, cycle_no):
+    """Stochastic verification at T = 1 with point-mass proposals (a variant
+    of the rule above for a tree whose children are the draft's top-W tokens,
+    not samples from q: each child is a deterministic proposal, so its
+    proposal distribution is a point mass on its token).
+
+    At the current slot u: p = softmax(target row of u); the rejected set R
+    starts empty.  Child x_i (slot order) is accepted if
+    r_i (1 - p(R)) < p(x_i), i.e. r_i < p(x_i) / (1 - p(R)), the probability
+    of x_i under p restricted to the tokens not yet rejected; otherwise x_i
+    joins R.  With no child accepted the bonus is the Gumbel-max draw
+    argmax_t [log p(t) - log(-log g_t)] over the tokens outside R with
+    p(t) > 0.  Offering tokens one at a time this way and sampling the rest
+    from the restricted p emits a token distributed exactly as p, for any
+    set of children.  Returns (path, accept_len, bonus, margins) like
+    accept_stochastic."""
+    kids = _children_slots(tree, chosen)
+    slot = 0
+    path = [0]
+    margins = []
+    while True:
+        p = np.exp(log_softmax(target_rows[slot])[0])
+        accepted = None
+        rejected = []
+        removed = 0.0
+        for i, c in enumerate(kids[slot]):
+            x = tree.token[int(chosen[c])]
+            r = uniform_ratio(seed, b, cycle_no, slot, i)
+            lhs, rhs = r * (1.0 - removed), p[x]
+            margins.append(abs(lhs - rhs) / max(abs(rhs), 1e-300))
+            if lhs < rhs:
+                accepted = c
+                break
+            rejected.append(x)
+            removed += p[x]
+        if accepted is None:
+            vocab = p.size
+            g = uniform_gumbel(seed, b, cycle_no, slot, np.arange(vocab))
+            keep = p.copy()
+            keep[rejected] = 0.0
+            with np.errstate(divide="ignore"):
+                score = np.where(keep > 0, np.log(keep) - np.log(-np.log(g)), -np.inf)
+            bonus = int(np.argmax(score))
+            top2 = np.sort(score)[-2:]
+            margins.append(float(top2[1] - top2[0]) if np.isfinite(top2[0]) else float("inf"))
+            return path, len(path) - 1, bonus, margins
+        path.append(accepted)
+        slot = accepted
+
+
 # ---------------------------------------------------------------- compaction
 def compact_kv(cache: np.ndarray, ctx: int, path) -> np.ndarray:
     """KV compaction implied by "discards the remainder" (§3.2 Draft Tree

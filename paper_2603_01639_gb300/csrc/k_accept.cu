@@ -17,7 +17,11 @@
 //    children's p(x), q(x) are loaded with the slice; a rejection costs one
 //    cluster barrier and one pass over the slice, which also takes the next
 //    rejection's partial sum.  With no child accepted the bonus is a Gumbel-max
-//    draw from p, reduced over the cluster the same way.
+//    draw from p, reduced over the cluster the same way;
+//  - stochastic with point-mass proposals: child i is accepted if
+//    r_i (1 - p(rejected so far)) < p(x_i), with p(x_i) loaded with the
+//    slice as above; a rejection only adds p(x_i) to the removed mass (no
+//    pass, no barrier), and the Gumbel-max bonus skips the rejected tokens.
 // kv_compact_kernel: grid (KV heads, layers x {K, V}, batch); each CTA stages
 // the accepted rows in shared memory, then writes them to ctx+t, so a row
 // that is both a source and a destination is read before it is overwritten.
@@ -223,7 +227,8 @@ __global__ void __launch_bounds__(kNT) accept_walk_kernel(const AcceptParams p, 
   const int mode = p.mode[b];
   int32_t* path_out = p.path + static_cast<int64_t>(b) * (p.max_depth + 1);
   // everything below is uniform over the cluster (one sequence)
-  if (N < 1 || N > p.n_max || (mode != LTD_GREEDY && mode != LTD_STOCHASTIC)) {
+  if (N < 1 || N > p.n_max ||
+      (mode != LTD_GREEDY && mode != LTD_STOCHASTIC && mode != LTD_STOCHASTIC_POINT_MASS)) {
     if (rank == 0 && tid == 0) {
       flag_error(p.err, (N < 1 || N > p.n_max) ? LTD_DEVERR_NVERIFY : LTD_DEVERR_MODE);
       for (int t = 0; t <= p.max_depth; ++t) path_out[t] = -1;
@@ -295,6 +300,7 @@ __global__ void __launch_bounds__(kNT) accept_walk_kernel(const AcceptParams p, 
   }
 
   // ---------------------------------------------------------- stochastic
+  const bool pm = mode == LTD_STOCHASTIC_POINT_MASS;  // no q: children are point masses
   const T* target = reinterpret_cast<const T*>(p.target);
   const T* draft = reinterpret_cast<const T*>(p.draft);
   const int64_t lo = static_cast<int64_t>(rank) * slice;
@@ -339,7 +345,8 @@ __global__ void __launch_bounds__(kNT) accept_walk_kernel(const AcceptParams p, 
     const T* trow = target + (static_cast<int64_t>(b) * p.n_max + cur) * V;
     const T* qrow = nullptr;
     float lse_q = 0.f;
-    if (nk > 0) {
+    const bool use_q = nk > 0 && !pm;
+    if (use_q) {
       qrow = draft + (static_cast<int64_t>(b) * p.rows_per_seq + p.xrow[nb + u]) * V;
       lse_q = p.xlse[nb + u];
     }
@@ -350,7 +357,7 @@ __global__ void __launch_bounds__(kNT) accept_walk_kernel(const AcceptParams p, 
     if (tid < nk) {
       const int x = sh.tok[sh.kids[tid]];
       sh.kp[tid] = __expf(to_f<T>(trow[x]) - lse_t);
-      sh.kq[tid] = __expf(to_f<T>(qrow[x]) - lse_q);
+      sh.kq[tid] = use_q ? __expf(to_f<T>(qrow[x]) - lse_q) : 0.f;
     }
     float part = 0.f;
     {
@@ -362,7 +369,7 @@ __global__ void __launch_bounds__(kNT) accept_walk_kernel(const AcceptParams p, 
         rq[k] = make_uint4(0u, 0u, 0u, 0u);
         if (vec_ok && el(k, 0) < hi) {
           rt[k] = ld_stream16_once(trow + el(k, 0));
-          if (nk > 0) rq[k] = ld_stream16_once(qrow + el(k, 0));
+          if (use_q) rq[k] = ld_stream16_once(qrow + el(k, 0));
         }
       }
 #pragma unroll
@@ -377,13 +384,13 @@ __global__ void __launch_bounds__(kNT) accept_walk_kernel(const AcceptParams p, 
             dv = elem<T>(rq[k], j);
           } else if (in) {
             tv = to_f<T>(trow[v]);
-            if (nk > 0) dv = to_f<T>(qrow[v]);
+            if (use_q) dv = to_f<T>(qrow[v]);
           }
           pr[k][j] = 0.f;
           qr[k][j] = 0.f;
           if (in) {
             pr[k][j] = __expf(tv - lse_t);
-            if (nk > 0) qr[k][j] = __expf(dv - lse_q);
+            if (use_q) qr[k][j] = __expf(dv - lse_q);
           }
           part += fmaxf(pr[k][j] - qr[k][j], 0.f);
         }
@@ -392,7 +399,18 @@ __global__ void __launch_bounds__(kNT) accept_walk_kernel(const AcceptParams p, 
     WTRACE(3);
     int accepted = -1, nz = 0;
     const uint64_t pre = hash_prefix(p.seed, b, p.cycle, kStreamRatio, cur);
+    float removed = 0.f;  // point-mass rule: p mass of the rejected children
     for (int c = 0; c < nk; ++c) {
+      if (pm) {
+        const float px = sh.kp[c];
+        if (uniform_ratio(pre, static_cast<uint64_t>(c)) * (1.f - removed) < px) {
+          accepted = sh.kids[c];
+          break;
+        }
+        removed += px;
+        ++nz;
+        continue;
+      }
       // p(x) after nz rejections, by the same arithmetic as the slice update
       // (sh.Z holds 1 / Z, or 0 where the residual was empty)
       float px = sh.kp[c];
@@ -432,8 +450,15 @@ __global__ void __launch_bounds__(kNT) accept_walk_kernel(const AcceptParams p, 
     // Gumbel-max: the largest log p(v) + G_v, with G_v = -log(-log u_v),
     // ranked as p(v) / (-log u_v) (the same order)
     uint64_t bestk = 0ull;
+    // the point-mass rule draws the bonus from p without the rejected children
+    auto rejected = [&](int64_t v) {
+      bool r = false;
+      if (pm)
+        for (int c = 0; c < nz; ++c) r |= sh.tok[sh.kids[c]] == static_cast<int32_t>(v);
+      return r;
+    };
     auto offer = [&](float pv, int64_t v) {
-      if (pv > 0.f) {
+      if (pv > 0.f && !rejected(v)) {
         const float e = -__logf(uniform_gumbel(preb, static_cast<uint64_t>(v)));
         const uint64_t key = make_key(__fdividef(pv, e), static_cast<uint32_t>(v));
         bestk = key > bestk ? key : bestk;

@@ -62,6 +62,8 @@ def oracle_accept(cfg, ci, trees, sels, target, seed, cycle_no):
         if ci.mode[b] == 0:
             path, a, bonus = oracle.accept_greedy(trees[b], ids, rows)
             margins = []
+        elif ci.mode[b] == 2:
+            path, a, bonus, margins = oracle.accept_point_mass(trees[b], ids, rows, seed, b, cycle_no)
         else:
             path, a, bonus, margins = oracle.accept_stochastic(
                 trees[b], ids, rows, ci.draft_rows[b].astype(np.float64), seed, b, cycle_no)

@@ -410,6 +410,64 @@ def test_stochastic_zero_probability_child_rejected():
 
 
 # ------------------------------------------------------------------ RNG pins
+# ------------------------------------------------ point-mass stochastic rule
+def test_point_mass_preserves_target_distribution_for_deterministic_children():
+    """The children are a fixed top-k set (not samples from any q): the
+    first emitted token is still distributed exactly as p."""
+    vocab, k, trials = 6, 3, 30000
+    rng = np.random.default_rng(321)
+    xt = rng.standard_normal(vocab) * 1.5
+    p = scipy.special.softmax(xt)
+    kids = np.argsort(-p)[:k]                      # deterministic: the k likeliest
+    tree = _star_tree(0, kids, k)
+    ids = np.arange(k + 1)
+    counts = np.zeros(vocab)
+    for trial in range(trials):
+        target = np.vstack([xt] + [rng.standard_normal(vocab) for _ in range(k)])
+        path, a, bonus, _ = oracle.accept_point_mass(tree, ids, target, seed=11, b=0, cycle_no=trial)
+        first = tree.token[path[1]] if a >= 1 else bonus
+        counts[first] += 1
+    chi2 = ((counts - trials * p) ** 2 / (trials * p)).sum()
+    assert scipy.stats.chi2.sf(chi2, vocab - 1) > 1e-4, (counts / trials, p)
+
+
+def test_point_mass_accept_probabilities_in_closed_form():
+    """Two children x1, x2: P(x1) = p1, P(x2) = (1 - p1) p2 / (1 - p1) = p2,
+    and the bonus never repeats a rejected child."""
+    vocab, trials = 5, 20000
+    xt = np.array([1.0, 0.2, -0.5, 0.7, -1.2])
+    p = scipy.special.softmax(xt)
+    tree = _star_tree(0, [3, 0], 2)
+    hits = np.zeros(3)
+    for trial in range(trials):
+        path, a, bonus, _ = oracle.accept_point_mass(tree, np.arange(3), np.vstack([xt, xt, xt]),
+                                                     seed=2, b=0, cycle_no=trial)
+        if a == 0:
+            assert bonus not in (3, 0)
+            hits[2] += 1
+        else:
+            hits[path[1] - 1] += 1
+    expect = np.array([p[3], p[0], 1 - p[3] - p[0]]) * trials
+    chi2 = ((hits - expect) ** 2 / expect).sum()
+    assert scipy.stats.chi2.sf(chi2, 2) > 1e-4, (hits / trials, expect / trials)
+
+
+def test_point_mass_certain_and_impossible_children():
+    vocab = 4
+    sure = np.array([30.0, -30.0, -30.0, -30.0])       # p(0) ~ 1
+    tree = _star_tree(0, [0], 1)
+    for c in range(20):
+        path, a, _, _ = oracle.accept_point_mass(tree, np.arange(2), np.vstack([sure, sure]),
+                                                 seed=4, b=0, cycle_no=c)
+        assert a == 1
+    never = np.array([0.0, -1e4, 0.0, 0.0])            # p(1) = 0
+    tree = _star_tree(0, [1], 1)
+    for c in range(20):
+        path, a, bonus, _ = oracle.accept_point_mass(tree, np.arange(2), np.vstack([never, never]),
+                                                     seed=4, b=0, cycle_no=c)
+        assert a == 0 and bonus != 1
+
+
 def test_splitmix64_published_vector():
     with open(os.path.join(GOLDEN, "splitmix64_seed0.txt")) as f:
         vals = [int(line, 16) for line in f if line.strip() and not line.startswith("#")]

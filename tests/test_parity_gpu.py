@@ -263,6 +263,50 @@ def test_adaptive_draft_driven_by_device_policies(name, seed):
     H.compare_select(cfg, ci, got, sels, otrees)
 
 
+# ------------------------------------------------ point-mass stochastic rule
+def _accept_case(cfg, ci, target, acc_seed=1234, cycle_no=0):
+    trees, sels, _ = H.oracle_side(cfg, ci)
+    assert min(H.tree_margin(t, cfg.W) for t in trees) > H.CUT_MARGIN
+    ref = H.oracle_accept(cfg, ci, trees, sels, target, acc_seed, cycle_no)
+    assert H.stochastic_margins_ok(ref), "near-tie in a stochastic decision; pick another seed"
+    draft = H.dev(ci.draft_rows, cfg.dtype)
+    tree = H.gpu_draft(cfg, ci, draft)
+    got = H.gpu_select(cfg, ci, tree)
+    out = ltd.ltd_accept(tree, H.dev(target, cfg.dtype), draft, got[0], H.i32(ci.n_verify),
+                         H.i32(ci.mode), H.i32(ci.ctx), seed=acc_seed, cycle=cycle_no)
+    assert ltd.ltd_check() == 0
+    H.compare_accept(cfg, out, ref)
+    return ref
+
+
+@pytest.mark.parametrize("seed", [0, 1, 3])
+def test_point_mass_cycles_accepting(seed):
+    """Every sequence on the point-mass rule, the target rows at each
+    expanded node a sharpened copy of its draft row (so children are
+    accepted, and rejected ones leave the bonus draw)."""
+    cfg = wl.config("13b")
+    ci = wl.draw_cycle(cfg, seed)
+    ci.mode = np.full(cfg.batch, ltd.LTD_STOCHASTIC_POINT_MASS, np.int32)
+    trees, sels, target = H.oracle_side(cfg, ci)
+    for b in range(cfg.batch):
+        for sl, nid in enumerate(sels[b][0]):
+            xr = trees[b].xrow[int(nid)]
+            if xr >= 0:
+                target[b, sl] = wl.round_to(ci.draft_rows[b, xr] * 5.0, cfg.dtype)
+    ref = _accept_case(cfg, ci, target, cycle_no=seed)
+    assert ref[0]["accept_len"] >= 1
+
+
+@pytest.mark.parametrize("seed", [0, 2])
+def test_70b_batch_with_all_three_rules(seed):
+    """The ragged 70B batch with greedy, stochastic and point-mass sequences."""
+    cfg = wl.config("70b")
+    ci = wl.draw_cycle(cfg, seed)
+    ci.mode = (np.arange(cfg.batch) % 3).astype(np.int32)
+    _, _, target = H.oracle_side(cfg, ci)
+    _accept_case(cfg, ci, target, cycle_no=seed)
+
+
 def test_determinism_and_reuse_of_scratch():
     """Same inputs twice through the same tree and workspace: identical bits
     (tickets and scratch are left ready for reuse)."""

@@ -537,7 +537,8 @@ def run_ours(args):
     rules = {}
     saved_mode = cyc.mode.clone()
     for rname, rmode in (("greedy", ltd.LTD_GREEDY), ("stochastic", ltd.LTD_STOCHASTIC),
-                         ("point_mass", ltd.LTD_STOCHASTIC_POINT_MASS)):
+                         ("point_mass", ltd.LTD_STOCHASTIC_POINT_MASS),
+                         ("no_replacement", ltd.LTD_STOCHASTIC_NO_REPLACEMENT)):
         cyc.mode.fill_(rmode)
         g_rule = _graph(torch, cyc.accept_phase)
         g_rule.replay()

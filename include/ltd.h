@@ -54,7 +54,12 @@ typedef enum ltd_status {
 } ltd_status;
 
 typedef enum ltd_dtype { LTD_F32 = 0, LTD_BF16 = 1 } ltd_dtype;
-typedef enum ltd_mode { LTD_GREEDY = 0, LTD_STOCHASTIC = 1, LTD_STOCHASTIC_POINT_MASS = 2 } ltd_mode;
+typedef enum ltd_mode {
+  LTD_GREEDY = 0,
+  LTD_STOCHASTIC = 1,
+  LTD_STOCHASTIC_POINT_MASS = 2,
+  LTD_STOCHASTIC_NO_REPLACEMENT = 3
+} ltd_mode;
 
 /* Limits of this build. */
 #define LTD_MAX_K 32          /* beam width k                              */
@@ -332,8 +337,14 @@ typedef struct ltd_kv_cache {
  * child accepted the bonus is the Gumbel-max draw over the tokens outside R.
  * The emitted token is distributed exactly as p for any set of children;
  * no draft row is read and a rejection costs no pass over the vocabulary.
+ * Stochastic without replacement (LTD_STOCHASTIC_NO_REPLACEMENT, T = 1): as
+ * LTD_STOCHASTIC, for children drawn from q without replacement: child x_i
+ * is proposed by q_i = q with the rejected children removed, renormalised;
+ * accept if r_i q_i(x_i) < p_i(x_i), else p_{i+1} = max(p_i - q_i, 0) / sum
+ * and q_{i+1} = q_i without x_i, renormalised.
  *  d_target_logits  [batch][n_max][vocab] (dtype), row i = target at slot i
- *  d_draft_rows     the row store given to ltd_expand_tree (LTD_STOCHASTIC only)
+ *  d_draft_rows     the row store given to ltd_expand_tree (read by the
+ *                   LTD_STOCHASTIC and LTD_STOCHASTIC_NO_REPLACEMENT rules)
  *  d_node_ids       ltd_select_verify output
  *  d_ctx            [batch] in; d_new_ctx [batch] out = ctx + 1 + accept_len
  *  d_path           out [batch][max_depth+1] accepted slots, -1 after the end

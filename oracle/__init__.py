@@ -20,6 +20,7 @@ from .ltd_oracle import (  # noqa: F401
     accept_greedy,
     accept_point_mass,
     accept_stochastic,
+    accept_without_replacement,
     compact_kv,
     cycle,
     depth_observation,

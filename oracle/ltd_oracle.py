@@ -378,6 +378,56 @@ def accept_stochastic(tree: OracleTree, chosen, target_rows, draft_rows, seed, b
         slot = accepted
 
 
+def accept_without_replacement(tree: OracleTree, chosen, target_rows, draft_rows, seed, b,
+                               cycle_no):
+    """Stochastic verification at T = 1 for children drawn from q without
+    replacement (a variant of the rule above: recursive rejection sampling).
+    Child x_i is proposed by q_i, the draft distribution with the children
+    rejected so far removed and renormalised (q_0 = q); it is accepted if
+    r_i q_i(x_i) < p_i(x_i), else p_{i+1} = max(p_i - q_i, 0) / sum (p_i kept
+    when that sum is 0) and q_{i+1} = q_i with x_i removed, renormalised.
+    With no child accepted the bonus is the Gumbel-max draw from the last p.
+    Same uniforms and return value as accept_stochastic."""
+    kids = _children_slots(tree, chosen)
+    slot = 0
+    path = [0]
+    margins = []
+    while True:
+        u = int(chosen[slot])
+        p = np.exp(log_softmax(target_rows[slot])[0])
+        accepted = None
+        if kids[slot]:
+            q = np.exp(log_softmax(draft_rows[tree.xrow[u]])[0])
+            for i, c in enumerate(kids[slot]):
+                x = tree.token[int(chosen[c])]
+                r = uniform_ratio(seed, b, cycle_no, slot, i)
+                lhs, rhs = r * q[x], p[x]
+                margins.append(abs(lhs - rhs) / max(abs(rhs), 1e-300))
+                if lhs < rhs:
+                    accepted = c
+                    break
+                res = np.maximum(p - q, 0.0)
+                z = res.sum()
+                if z > 0:
+                    p = res / z
+                q = q.copy()
+                q[x] = 0.0
+                qs = q.sum()
+                if qs > 0:
+                    q = q / qs
+        if accepted is None:
+            vocab = p.size
+            g = uniform_gumbel(seed, b, cycle_no, slot, np.arange(vocab))
+            with np.errstate(divide="ignore"):
+                score = np.where(p > 0, np.log(p) - np.log(-np.log(g)), -np.inf)
+            bonus = int(np.argmax(score))
+            top2 = np.sort(score)[-2:]
+            margins.append(float(top2[1] - top2[0]) if np.isfinite(top2[0]) else float("inf"))
+            return path, len(path) - 1, bonus, margins
+        path.append(accepted)
+        slot = accepted
+
+
 def accept_point_mass(tree: OracleTree, chosen, target_rows, seed, b, cycle_no):
     """Stochastic verification at T = 1 with point-mass proposals (a variant
     of the rule above for a tree whose children are the draft's top-W tokens,

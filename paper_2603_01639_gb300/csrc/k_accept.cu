@@ -21,7 +21,12 @@
 //  - stochastic with point-mass proposals: child i is accepted if
 //    r_i (1 - p(rejected so far)) < p(x_i), with p(x_i) loaded with the
 //    slice as above; a rejection only adds p(x_i) to the removed mass (no
-//    pass, no barrier), and the Gumbel-max bonus skips the rejected tokens.
+//    pass, no barrier), and the Gumbel-max bonus skips the rejected tokens;
+//  - stochastic for children drawn from q without replacement: as the first
+//    stochastic rule, but after a rejection the rejected token's q is zeroed
+//    (in its owner thread's registers) and q renormalised by a scalar,
+//    1 / (1 - q-mass of the rejected children), in the same pass as the
+//    residual update.
 // kv_compact_kernel: grid (KV heads, layers x {K, V}, batch); each CTA stages
 // the accepted rows in shared memory, then writes them to ctx+t, so a row
 // that is both a source and a destination is read before it is overwritten.
@@ -169,6 +174,7 @@ struct WalkShared {
   int32_t next[LTD_MAX_N];
   int32_t kids[LTD_MAX_N];
   float Z[LTD_MAX_N];
+  float S[LTD_MAX_N];  // without-replacement rule: scale of q at each rejection
   int32_t path[LTD_MAX_DEPTH + 1];
   float red[2 * kNW];
   uint64_t redk[kNW];
@@ -228,7 +234,8 @@ __global__ void __launch_bounds__(kNT) accept_walk_kernel(const AcceptParams p, 
   int32_t* path_out = p.path + static_cast<int64_t>(b) * (p.max_depth + 1);
   // everything below is uniform over the cluster (one sequence)
   if (N < 1 || N > p.n_max ||
-      (mode != LTD_GREEDY && mode != LTD_STOCHASTIC && mode != LTD_STOCHASTIC_POINT_MASS)) {
+      (mode != LTD_GREEDY && mode != LTD_STOCHASTIC && mode != LTD_STOCHASTIC_POINT_MASS &&
+       mode != LTD_STOCHASTIC_NO_REPLACEMENT)) {
     if (rank == 0 && tid == 0) {
       flag_error(p.err, (N < 1 || N > p.n_max) ? LTD_DEVERR_NVERIFY : LTD_DEVERR_MODE);
       for (int t = 0; t <= p.max_depth; ++t) path_out[t] = -1;
@@ -300,7 +307,8 @@ __global__ void __launch_bounds__(kNT) accept_walk_kernel(const AcceptParams p, 
   }
 
   // ---------------------------------------------------------- stochastic
-  const bool pm = mode == LTD_STOCHASTIC_POINT_MASS;  // no q: children are point masses
+  const bool pm = mode == LTD_STOCHASTIC_POINT_MASS;     // no q: children are point masses
+  const bool nr = mode == LTD_STOCHASTIC_NO_REPLACEMENT;  // q loses each rejected child
   const T* target = reinterpret_cast<const T*>(p.target);
   const T* draft = reinterpret_cast<const T*>(p.draft);
   const int64_t lo = static_cast<int64_t>(rank) * slice;
@@ -400,6 +408,7 @@ __global__ void __launch_bounds__(kNT) accept_walk_kernel(const AcceptParams p, 
     int accepted = -1, nz = 0;
     const uint64_t pre = hash_prefix(p.seed, b, p.cycle, kStreamRatio, cur);
     float removed = 0.f;  // point-mass rule: p mass of the rejected children
+    float qs = 1.f, qrej = 0.f;  // without replacement: q scale, q mass rejected
     for (int c = 0; c < nk; ++c) {
       if (pm) {
         const float px = sh.kp[c];
@@ -412,30 +421,52 @@ __global__ void __launch_bounds__(kNT) accept_walk_kernel(const AcceptParams p, 
         continue;
       }
       // p(x) after nz rejections, by the same arithmetic as the slice update
-      // (sh.Z holds 1 / Z, or 0 where the residual was empty)
+      // (sh.Z holds 1 / Z, or 0 where the residual was empty; sh.S the scale
+      // of q at that rejection, 1 unless q loses its rejected children)
       float px = sh.kp[c];
       const float qx = sh.kq[c];
       for (int jz = 0; jz < nz; ++jz)
-        if (sh.Z[jz] > 0.f) px = fmaxf(px - qx, 0.f) * sh.Z[jz];
-      if (uniform_ratio(pre, static_cast<uint64_t>(c)) * qx < px) {
+        if (sh.Z[jz] > 0.f) px = fmaxf(px - qx * sh.S[jz], 0.f) * sh.Z[jz];
+      if (uniform_ratio(pre, static_cast<uint64_t>(c)) * (qx * qs) < px) {
         accepted = sh.kids[c];
         break;
       }
       const float z = cluster_sum_warps(part, sh.wpart, round, C);
       WTRACE(4);
       const float zi = z > 0.f ? __frcp_rn(z) : 0.f;
-      // the residual update, with this thread's share of the next sum
+      // without replacement: the rejected token leaves q, the rest rescales
+      const int64_t xrej = nr ? static_cast<int64_t>(sh.tok[sh.kids[c]]) : -1;
+      float qs_next = qs;
+      if (nr) {
+        qrej += qx;
+        qs_next = (1.f - qrej) > 0.f ? __frcp_rn(1.f - qrej) : 0.f;
+      }
+      // the residual update, with this thread's share of the next sum (the
+      // plain rule keeps q as it is: its own loop, without the q scaling)
       part = 0.f;
+      if (nr) {
 #pragma unroll
-      for (int k = 0; k < KG; ++k)
+        for (int k = 0; k < KG; ++k)
 #pragma unroll
-        for (int j = 0; j < VEC; ++j) {
-          if (zi > 0.f) pr[k][j] = fmaxf(pr[k][j] - qr[k][j], 0.f) * zi;
-          part += fmaxf(pr[k][j] - qr[k][j], 0.f);
-        }
-      // every thread records the same value, so no barrier is needed before
-      // any thread reads it back
+          for (int j = 0; j < VEC; ++j) {
+            if (zi > 0.f) pr[k][j] = fmaxf(pr[k][j] - qr[k][j] * qs, 0.f) * zi;
+            if (el(k, j) == xrej) qr[k][j] = 0.f;
+            part += fmaxf(pr[k][j] - qr[k][j] * qs_next, 0.f);
+          }
+      } else {
+#pragma unroll
+        for (int k = 0; k < KG; ++k)
+#pragma unroll
+          for (int j = 0; j < VEC; ++j) {
+            if (zi > 0.f) pr[k][j] = fmaxf(pr[k][j] - qr[k][j], 0.f) * zi;
+            part += fmaxf(pr[k][j] - qr[k][j], 0.f);
+          }
+      }
+      // every thread records the same values, so no barrier is needed before
+      // any thread reads them back
       sh.Z[nz] = zi;
+      sh.S[nz] = qs;
+      qs = qs_next;
       ++nz;
       WTRACE(5);
     }

@@ -21,6 +21,15 @@ namespace ltd {
 
 namespace {
 
+// Split cluster barrier: every thread arrives (relaxed: no memory ordering)
+// and later waits; between the two it may work on its own data.
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() {
+  asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
+}
+
 constexpr int kPolicyNT = 256;
 
 __global__ void __launch_bounds__(kPolicyNT) depth_obs_kernel(const ltd_tree t, const int32_t* ctx,
@@ -221,7 +230,7 @@ __global__ void __launch_bounds__(kMlpNT, 1) mlp_policy_kernel(const MlpArgs a) 
     for (int u = tid; u < u_cnt; u += kMlpNT) bias_s[l * kMlpBiasMax + u] = __ldg(a.net.b[l] + u0 + u);
   }
   // peers must have started before their shared memory is written
-  tc::cluster_arrive_relaxed();
+  cluster_arrive_relaxed();
   bool peers_known = false;
   MTRACE(1);
   grid_wait();
@@ -312,7 +321,7 @@ __global__ void __launch_bounds__(kMlpNT, 1) mlp_policy_kernel(const MlpArgs a) 
       const int n_outs = u_cnt * gn;
       const float* bl = bias_s + l * kMlpBiasMax;
       if (!peers_known) {
-        tc::cluster_wait();
+        cluster_wait();
         peers_known = true;
       }
       // a unit sum adds P partials: one thread per unit when there are many

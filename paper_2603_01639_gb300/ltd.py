@@ -20,7 +20,7 @@ _lib = None
 _lock = threading.Lock()
 
 LTD_F32, LTD_BF16 = 0, 1
-LTD_GREEDY, LTD_STOCHASTIC, LTD_STOCHASTIC_POINT_MASS = 0, 1, 2
+LTD_GREEDY, LTD_STOCHASTIC, LTD_STOCHASTIC_POINT_MASS, LTD_STOCHASTIC_NO_REPLACEMENT = 0, 1, 2, 3
 LTD_MAX_K, LTD_MAX_DEPTH, LTD_MAX_N, LTD_MAX_TREE_NODES = 32, 16, 256, 4096
 DEVERR = {0x1: "LEVEL", 0x2: "NVERIFY", 0x4: "CTX", 0x8: "TREE", 0x10: "TIMEOUT", 0x20: "MODE"}
 

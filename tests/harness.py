@@ -64,6 +64,9 @@ def oracle_accept(cfg, ci, trees, sels, target, seed, cycle_no):
             margins = []
         elif ci.mode[b] == 2:
             path, a, bonus, margins = oracle.accept_point_mass(trees[b], ids, rows, seed, b, cycle_no)
+        elif ci.mode[b] == 3:
+            path, a, bonus, margins = oracle.accept_without_replacement(
+                trees[b], ids, rows, ci.draft_rows[b].astype(np.float64), seed, b, cycle_no)
         else:
             path, a, bonus, margins = oracle.accept_stochastic(
                 trees[b], ids, rows, ci.draft_rows[b].astype(np.float64), seed, b, cycle_no)

@@ -410,6 +410,50 @@ def test_stochastic_zero_probability_child_rejected():
 
 
 # ------------------------------------------------------------------ RNG pins
+# --------------------------------------------- without-replacement rule
+def test_without_replacement_preserves_target_distribution():
+    """Children drawn from q WITHOUT replacement (distinct tokens, as a
+    top-k tree has): the first emitted token is distributed as p."""
+    vocab, k, trials = 6, 3, 30000
+    rng = np.random.default_rng(77)
+    xt = rng.standard_normal(vocab) * 1.5
+    xq = rng.standard_normal(vocab) * 1.5
+    p = scipy.special.softmax(xt)
+    q = scipy.special.softmax(xq)
+    counts = np.zeros(vocab)
+    for trial in range(trials):
+        kids = rng.choice(vocab, size=k, p=q, replace=False)   # sequential draws without replacement
+        tree = _star_tree(0, kids, k)
+        target = np.vstack([xt] + [rng.standard_normal(vocab) for _ in range(k)])
+        path, a, bonus, _ = oracle.accept_without_replacement(tree, np.arange(k + 1), target, xq[None, :],
+                                                              seed=13, b=0, cycle_no=trial)
+        first = tree.token[path[1]] if a >= 1 else bonus
+        counts[first] += 1
+    chi2 = ((counts - trials * p) ** 2 / (trials * p)).sum()
+    assert scipy.stats.chi2.sf(chi2, vocab - 1) > 1e-4, (counts / trials, p)
+
+
+def test_with_replacement_rule_is_biased_for_distinct_children():
+    """The plain rule keeps q after a rejection, which assumes i.i.d.
+    children; for distinct children it is off -- the variant above is what
+    makes the difference (guards against the two rules being the same)."""
+    vocab, k, trials = 4, 3, 20000
+    xt = np.array([2.0, 1.5, -1.0, 0.0])
+    xq = np.array([2.0, 1.8, 1.6, -3.0])
+    p = scipy.special.softmax(xt)
+    q = scipy.special.softmax(xq)
+    rng = np.random.default_rng(5)
+    counts = np.zeros(vocab)
+    for trial in range(trials):
+        kids = rng.choice(vocab, size=k, p=q, replace=False)
+        tree = _star_tree(0, kids, k)
+        path, a, bonus, _ = oracle.accept_stochastic(tree, np.arange(k + 1), np.vstack([xt] * (k + 1)),
+                                                     xq[None, :], seed=3, b=0, cycle_no=trial)
+        counts[tree.token[path[1]] if a >= 1 else bonus] += 1
+    chi2 = ((counts - trials * p) ** 2 / (trials * p)).sum()
+    assert scipy.stats.chi2.sf(chi2, vocab - 1) < 1e-6
+
+
 # ------------------------------------------------ point-mass stochastic rule
 def test_point_mass_preserves_target_distribution_for_deterministic_children():
     """The children are a fixed top-k set (not samples from any q): the

@@ -279,14 +279,16 @@ def _accept_case(cfg, ci, target, acc_seed=1234, cycle_no=0):
     return ref
 
 
+@pytest.mark.parametrize("mode", [2, 3])
 @pytest.mark.parametrize("seed", [0, 1, 3])
-def test_point_mass_cycles_accepting(seed):
-    """Every sequence on the point-mass rule, the target rows at each
-    expanded node a sharpened copy of its draft row (so children are
-    accepted, and rejected ones leave the bonus draw)."""
+def test_variant_rules_accepting(seed, mode):
+    """Every sequence on the point-mass (2) or without-replacement (3) rule,
+    the target rows at each expanded node a sharpened copy of its draft row
+    (so children are accepted, and rejected ones leave the bonus draw)."""
+    assert mode in (ltd.LTD_STOCHASTIC_POINT_MASS, ltd.LTD_STOCHASTIC_NO_REPLACEMENT)
     cfg = wl.config("13b")
     ci = wl.draw_cycle(cfg, seed)
-    ci.mode = np.full(cfg.batch, ltd.LTD_STOCHASTIC_POINT_MASS, np.int32)
+    ci.mode = np.full(cfg.batch, mode, np.int32)
     trees, sels, target = H.oracle_side(cfg, ci)
     for b in range(cfg.batch):
         for sl, nid in enumerate(sels[b][0]):
@@ -297,14 +299,40 @@ def test_point_mass_cycles_accepting(seed):
     assert ref[0]["accept_len"] >= 1
 
 
-@pytest.mark.parametrize("seed", [0, 2])
-def test_70b_batch_with_all_three_rules(seed):
-    """The ragged 70B batch with greedy, stochastic and point-mass sequences."""
+@pytest.mark.parametrize("seed", [0, 2, 3])
+def test_70b_batch_with_every_rule(seed):
+    """The ragged 70B batch with greedy, stochastic, point-mass and
+    without-replacement sequences side by side."""
     cfg = wl.config("70b")
     ci = wl.draw_cycle(cfg, seed)
-    ci.mode = (np.arange(cfg.batch) % 3).astype(np.int32)
+    ci.mode = (np.arange(cfg.batch) % 4).astype(np.int32)
     _, _, target = H.oracle_side(cfg, ci)
     _accept_case(cfg, ci, target, cycle_no=seed)
+
+
+def test_unknown_rule_is_flagged_and_the_others_still_run():
+    """A mode outside ltd_mode raises the MODE bit; that sequence's outputs
+    are -1 and the other sequences of the batch are still right."""
+    cfg = wl.config("70b")
+    ci = wl.draw_cycle(cfg, 0)
+    ci.mode = (np.arange(cfg.batch) % 4).astype(np.int32)
+    trees, sels, target = H.oracle_side(cfg, ci)
+    ref = H.oracle_accept(cfg, ci, trees, sels, target, 1234, 0)
+    draft = H.dev(ci.draft_rows, cfg.dtype)
+    tree = H.gpu_draft(cfg, ci, draft)
+    got = H.gpu_select(cfg, ci, tree)
+    bad = ci.mode.copy()
+    bad[5] = 7
+    out = ltd.ltd_accept(tree, H.dev(target, cfg.dtype), draft, got[0], H.i32(ci.n_verify),
+                         H.i32(bad), H.i32(ci.ctx), seed=1234, cycle=0)
+    bits = ltd.ltd_check(raise_on_error=False)
+    assert bits == 0x20
+    o = {k: v.cpu().numpy() for k, v in out.items()}
+    assert o["accept_len"][5] == -1 and o["bonus"][5] == -1 and (o["path"][5] == -1).all()
+    assert o["new_ctx"][5] == ci.ctx[5]
+    for b in range(cfg.batch):
+        if b != 5:
+            assert o["accept_len"][b] == ref[b]["accept_len"] and o["bonus"][b] == ref[b]["bonus"]
 
 
 def test_determinism_and_reuse_of_scratch():

@@ -730,16 +730,19 @@ def run_e2e(cyc, args, device):
     host memory, run the cycle, read back path / accept length / bonus / ctx.
     The step's inputs sit in one pinned buffer and go over in one copy into
     one device buffer that holds the draft and target logits and every q in
-    place; each layer's new K/V rows are then placed into its cache on the
-    device (a host copy straight into the cache's strided rows ran at a few
-    GB/s)."""
+    place; every layer's new K/V rows are then placed into its cache on the
+    device by one ltd_kv_append launch (a host copy straight into the
+    cache's strided rows ran at a few GB/s, one device copy per layer and
+    tensor cost a launch each)."""
     import torch
     ltd, cfg = cyc.ltd, cyc.cfg
     c0 = int(cyc.ci.ctx.min())
     N = cfg.max_n
-    # buffer order: draft logits | every q, new K, new V | target logits | root
-    parts = ([cyc.draft] + list(cyc.q) + [k[:, :, c0:c0 + N] for k in cyc.k]
-             + [v[:, :, c0:c0 + N] for v in cyc.v] + [cyc.target, cyc.root])
+    # buffer order: draft logits | every q, every layer's new K, new V |
+    # target logits | root
+    knew = torch.stack([k[:, :, c0:c0 + N] for k in cyc.k])
+    vnew = torch.stack([v[:, :, c0:c0 + N] for v in cyc.v])
+    parts = [cyc.draft] + list(cyc.q) + [knew, vnew, cyc.target, cyc.root]
     offs, total = [], 0
     for t in parts:
         offs.append(total)
@@ -754,7 +757,7 @@ def run_e2e(cyc, args, device):
     L = cyc.layers
     cyc.draft = views[0]
     cyc.q = views[1:1 + L]
-    d_knew, d_vnew = views[1 + L:1 + 2 * L], views[1 + 2 * L:1 + 3 * L]
+    d_knew, d_vnew = views[1 + L], views[2 + L]
     cyc.target, cyc.root = views[-2], views[-1]
     # three spans of the buffer: what the draft phase needs, what attention
     # needs, what acceptance needs (then the root)
@@ -777,9 +780,8 @@ def run_e2e(cyc, args, device):
         d_buf[:a0].copy_(h_buf[:a0], non_blocking=True)
         with torch.cuda.stream(side):
             d_buf[a0:a1].copy_(h_buf[a0:a1], non_blocking=True)
-            for l in range(L):
-                cyc.k[l][:, :, c0:c0 + N].copy_(d_knew[l])
-                cyc.v[l][:, :, c0:c0 + N].copy_(d_vnew[l])
+            # every layer's new rows into its cache, one launch
+            ltd.ltd_kv_append(cyc.kv, d_knew, d_vnew, cyc.ctx, cyc.n_verify)
             ev_kv.record(side)
             d_buf[a1:a2].copy_(h_buf[a1:a2], non_blocking=True)
             ev_tgt.record(side)

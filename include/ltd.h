@@ -393,6 +393,22 @@ ltd_status ltd_accept_noalloc(const ltd_tree* tree, const void* d_target_logits,
                               int32_t* d_new_ctx, int32_t* d_path, int32_t* d_accept_len,
                               int32_t* d_bonus, const ltd_kv_cache* kv, ltd_stream_t stream);
 
+/* Write the verified tokens' new keys and values into every layer's cache,
+ * at the rows tree attention reads them from (section 3.2, "Draft Tree
+ * Verification": the target forward over the V candidates):
+ *   cache_K[l][b][h][ctx_b + i] = d_new_k[l][b][h][i],  i < N_b,
+ * and the same for V, in one launch for all layers.
+ *  d_new_k, d_new_v  [n_layers][batch][hkv][n_max][head_dim] in the cache's
+ *                    dtype (rows i >= N_b are not read)
+ *  d_ctx, d_n_verify [batch]
+ * A sequence with N_b outside [1, n_max] or ctx_b + N_b > s_cap is flagged
+ * (LTD_DEVERR_NVERIFY / LTD_DEVERR_CTX) and its rows are left as they are.
+ * Rows must be whole 16-byte units (LTD_ERR_UNSUPPORTED otherwise), the
+ * arrays 16-byte aligned (LTD_ERR_INVALID_ARG otherwise). */
+ltd_status ltd_kv_append(const ltd_kv_cache* kv, int32_t batch, int32_t n_max,
+                         const void* d_new_k, const void* d_new_v, const int32_t* d_ctx,
+                         const int32_t* d_n_verify, ltd_stream_t stream);
+
 /* In-place KV compaction ("discards the remainder", section 3.2): for every
  * layer, sequence, KV head and K/V tensor, row ctx+t <- row ctx+path[t] for
  * t = 0..accept_len, every source read before any row is written.  Rows

@@ -27,6 +27,7 @@
 //    (in its owner thread's registers) and q renormalised by a scalar,
 //    1 / (1 - q-mass of the rejected children), in the same pass as the
 //    residual update.
+// kv_append_kernel: the verified tokens' new K/V rows into every layer's cache.
 // kv_compact_kernel: grid (KV heads, layers x {K, V}, batch); each CTA stages
 // the accepted rows in shared memory, then writes them to ctx+t, so a row
 // that is both a source and a destination is read before it is overwritten.
@@ -569,7 +570,36 @@ __global__ void __launch_bounds__(kCompactNT) kv_compact_kernel(const CompactPar
   }
 }
 
+// Grid (hkv, layers x {K, V}, batch): one CTA copies one head's N new rows
+// (whole 16-byte units, coalesced) to rows ctx .. ctx + N - 1.
+__global__ void __launch_bounds__(kCompactNT) kv_append_kernel(const AppendParams p) {
+  grid_wait();
+  trigger_dependents();
+  const int h = blockIdx.x, layer = blockIdx.y >> 1, which = blockIdx.y & 1, b = blockIdx.z;
+  const int ctx = p.ctx[b], N = p.n_verify[b];
+  if (N < 1 || N > p.n_max || ctx < 0 || ctx + N > p.s_cap) {
+    if (threadIdx.x == 0 && h == 0 && blockIdx.y == 0)
+      flag_error(p.err, (N < 1 || N > p.n_max) ? LTD_DEVERR_NVERIFY : LTD_DEVERR_CTX);
+    return;
+  }
+  const int64_t head = (static_cast<int64_t>(layer) * p.batch + b) * p.hkv + h;
+  const uint4* src = reinterpret_cast<const uint4*>((which ? p.new_v : p.new_k) +
+                                                    head * p.n_max * p.row_bytes);
+  uint4* dst = reinterpret_cast<uint4*>(static_cast<char*>(which ? p.v_layers[layer]
+                                                                 : p.k_layers[layer]) +
+                                        ((static_cast<int64_t>(b) * p.hkv + h) * p.s_cap + ctx) *
+                                            p.row_bytes);
+  const int n = N * (p.row_bytes / 16);
+  for (int i = threadIdx.x; i < n; i += kCompactNT) dst[i] = __ldcs(src + i);
+}
+
 }  // namespace
+
+cudaError_t launch_append(const AppendParams& p, cudaStream_t s) {
+  if (p.row_bytes % 16 != 0) return cudaErrorInvalidValue;
+  const dim3 grid(p.hkv, p.n_layers * 2, p.batch);
+  return launch(kv_append_kernel, grid, dim3(kCompactNT), 0, s, nullptr, 0, p);
+}
 
 size_t accept_workspace(int32_t batch, int32_t n_max, int64_t vocab) {
   const VocabSplit vs =

@@ -393,6 +393,39 @@ size_t ltd_accept_workspace_bytes(int32_t batch, int32_t n_max, int64_t vocab) {
   return accept_workspace(batch, n_max, vocab);
 }
 
+ltd_status ltd_kv_append(const ltd_kv_cache* kv, int32_t batch, int32_t n_max,
+                         const void* d_new_k, const void* d_new_v, const int32_t* d_ctx,
+                         const int32_t* d_n_verify, ltd_stream_t stream) {
+  if (kv == nullptr || !kv->d_k_layers || !kv->d_v_layers || !d_new_k || !d_new_v || !d_ctx ||
+      !d_n_verify || !dtype_ok(kv->dtype))
+    return LTD_ERR_INVALID_ARG;
+  if (reinterpret_cast<uintptr_t>(d_new_k) % 16 != 0 ||
+      reinterpret_cast<uintptr_t>(d_new_v) % 16 != 0)
+    return LTD_ERR_INVALID_ARG;
+  if (batch < 1 || n_max < 1 || n_max > LTD_MAX_N || kv->n_layers < 1 || kv->hkv < 1 ||
+      kv->s_cap < 1)
+    return LTD_ERR_SHAPE;
+  const int64_t row_bytes = static_cast<int64_t>(kv->head_dim) * dtype_size(kv->dtype);
+  if (kv->head_dim < 1 || row_bytes % 16 != 0 || row_bytes > 512) return LTD_ERR_UNSUPPORTED;
+  uint32_t* err = device_error_word();
+  if (err == nullptr) return LTD_ERR_CUDA;
+  AppendParams p{};
+  p.k_layers = kv->d_k_layers;
+  p.v_layers = kv->d_v_layers;
+  p.new_k = static_cast<const uint8_t*>(d_new_k);
+  p.new_v = static_cast<const uint8_t*>(d_new_v);
+  p.n_layers = kv->n_layers;
+  p.batch = batch;
+  p.hkv = kv->hkv;
+  p.s_cap = kv->s_cap;
+  p.n_max = n_max;
+  p.row_bytes = static_cast<int32_t>(row_bytes);
+  p.ctx = d_ctx;
+  p.n_verify = d_n_verify;
+  p.err = err;
+  return from_cuda(launch_append(p, reinterpret_cast<cudaStream_t>(stream)));
+}
+
 ltd_status ltd_kv_compact(const ltd_kv_cache* kv, int32_t batch, const int32_t* d_path,
                           int32_t path_stride, const int32_t* d_accept_len, const int32_t* d_ctx,
                           ltd_stream_t stream) {

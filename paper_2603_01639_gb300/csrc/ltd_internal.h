@@ -218,4 +218,18 @@ struct CompactParams {
 };
 cudaError_t launch_compact(const CompactParams& p, int32_t batch, cudaStream_t s);
 
+// The verified tokens' new K/V rows into every layer's cache (k_accept.cu).
+struct AppendParams {
+  void* const* k_layers;
+  void* const* v_layers;
+  const uint8_t* new_k;  // [n_layers][batch][hkv][n_max][row]
+  const uint8_t* new_v;
+  int32_t n_layers, batch, hkv, s_cap, n_max;
+  int32_t row_bytes;
+  const int32_t* ctx;
+  const int32_t* n_verify;
+  uint32_t* err;
+};
+cudaError_t launch_append(const AppendParams& p, cudaStream_t s);
+
 }  // namespace ltd

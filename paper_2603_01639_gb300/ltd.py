@@ -31,7 +31,7 @@ EXPORTS = [
     "ltd_accept", "ltd_kv_compact", "ltd_check", "ltd_status_string", "ltd_version",
     "ltd_attention_kernel", "ltd_selftest_umma", "ltd_accept_noalloc", "ltd_tree_attention_next",
     "ltd_depth_observation", "ltd_size_observation", "ltd_depth_policy", "ltd_size_policy",
-    "ltd_mlp_packed_bytes", "ltd_mlp_pack",
+    "ltd_mlp_packed_bytes", "ltd_mlp_pack", "ltd_kv_append",
 ]
 LTD_POLICY_PAD = -100.0
 LTD_MLP_MAX_LAYERS, LTD_MLP_MAX_WIDTH = 4, 2048
@@ -97,6 +97,7 @@ def lib():
                 "ltd_accept": (C.c_int, [tp, vp, vp, C.c_int, i64, i64, vp, vp, i32, vp, u64, u64,
                                          vp, vp, vp, vp, vp, C.POINTER(ltd_kv_cache), vp, sz, vp]),
                 "ltd_kv_compact": (C.c_int, [C.POINTER(ltd_kv_cache), i32, vp, i32, vp, vp, vp]),
+                "ltd_kv_append": (C.c_int, [C.POINTER(ltd_kv_cache), i32, i32, vp, vp, vp, vp, vp]),
                 "ltd_check": (C.c_int, [vp, C.POINTER(C.c_uint32)]),
                 "ltd_status_string": (C.c_char_p, [C.c_int]),
                 "ltd_version": (i32, []),
@@ -450,6 +451,21 @@ def ltd_kv_compact(kv: KVCache, path, accept_len, ctx, stream=None):
     _need(path, "path", torch.int32)
     _ok(lib().ltd_kv_compact(C.byref(kv.s), path.shape[0], _ptr(path), path.shape[1],
                              _ptr(accept_len), _ptr(ctx), _stream(stream)), "ltd_kv_compact")
+
+
+def ltd_kv_append(kv: KVCache, new_k, new_v, ctx, n_verify, stream=None):
+    """new_k, new_v: [n_layers][batch][hkv][n_max][head_dim] in the cache's
+    dtype; rows ctx_b .. ctx_b + N_b - 1 of every layer's cache receive them."""
+    for t, n in ((new_k, "new_k"), (new_v, "new_v")):
+        _need(t, n, kv.k_layers[0].dtype)
+        if t.dim() != 5 or t.shape[0] != len(kv.k_layers):
+            raise LtdError(f"{n} must be [n_layers][batch][hkv][n_max][head_dim]")
+    if new_k.shape != new_v.shape:
+        raise LtdError("new_k and new_v differ in shape")
+    _need(ctx, "ctx", torch.int32)
+    _need(n_verify, "n_verify", torch.int32)
+    _ok(lib().ltd_kv_append(C.byref(kv.s), new_k.shape[1], new_k.shape[3], _ptr(new_k), _ptr(new_v),
+                            _ptr(ctx), _ptr(n_verify), _stream(stream)), "ltd_kv_append")
 
 
 def ltd_check(stream=None, raise_on_error=True) -> int:

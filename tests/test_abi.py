@@ -151,3 +151,10 @@ def test_entry_points_reject_bad_arguments_before_launch(L):
     kv = ltd.ltd_kv_cache(fake, fake, 1, 1, 70, 256, 1)                            # 140-byte rows
     assert L.ltd_kv_compact(C.byref(kv), 1, fake, 4, fake, fake, s) == 3
     assert L.ltd_kv_compact(None, 1, fake, 4, fake, fake, s) == 1
+    kv_ok = ltd.ltd_kv_cache(fake, fake, 2, 1, 64, 256, 1)                          # 128-byte rows
+    assert L.ltd_kv_append(C.byref(kv), 1, 8, fake, fake, fake, fake, s) == 3        # 140-byte rows
+    assert L.ltd_kv_append(None, 1, 8, fake, fake, fake, fake, s) == 1
+    assert L.ltd_kv_append(C.byref(kv_ok), 1, 8, C.c_void_p((1 << 24) + 8), fake, fake, fake, s) == 1
+    assert L.ltd_kv_append(C.byref(kv_ok), 1, 0, fake, fake, fake, fake, s) == 2     # n_max 0
+    assert L.ltd_kv_append(C.byref(kv_ok), 0, 8, fake, fake, fake, fake, s) == 2     # batch 0
+    assert L.ltd_kv_append(C.byref(kv_ok), 1, 8, fake, None, fake, fake, s) == 1

@@ -335,6 +335,31 @@ def test_unknown_rule_is_flagged_and_the_others_still_run():
             assert o["accept_len"][b] == ref[b]["accept_len"] and o["bonus"][b] == ref[b]["bonus"]
 
 
+def test_kv_append_writes_every_layer_and_flags_bad_sequences():
+    """The new rows land at ctx_b .. ctx_b + N_b - 1 of every layer's K and V
+    (bit for bit), nothing else changes; N out of range and ctx + N past the
+    cache are flagged and leave that sequence's rows alone."""
+    g = torch.Generator(device="cuda").manual_seed(3)
+    L, B, hkv, s_cap, d, n_max = 3, 4, 2, 512, 128, 16
+    k = [torch.randn(B, hkv, s_cap, d, generator=g, device="cuda").to(torch.bfloat16) for _ in range(L)]
+    v = [torch.randn(B, hkv, s_cap, d, generator=g, device="cuda").to(torch.bfloat16) for _ in range(L)]
+    k0 = [t.clone() for t in k]
+    v0 = [t.clone() for t in v]
+    kv = ltd.KVCache(k, v)
+    nk = torch.randn(L, B, hkv, n_max, d, generator=g, device="cuda").to(torch.bfloat16)
+    nv = torch.randn(L, B, hkv, n_max, d, generator=g, device="cuda").to(torch.bfloat16)
+    ctx = np.array([100, 300, 10, 500], np.int32)
+    n = np.array([16, 5, 0, 16], np.int32)           # b=2: N = 0; b=3: 500 + 16 > 512
+    ltd.ltd_kv_append(kv, nk, nv, H.i32(ctx), H.i32(n))
+    assert ltd.ltd_check(raise_on_error=False) == 0x2 | 0x4
+    for l in range(L):
+        for cache, before, new in ((k[l], k0[l], nk[l]), (v[l], v0[l], nv[l])):
+            want = before.clone()
+            for b in (0, 1):
+                want[b, :, ctx[b]:ctx[b] + n[b]] = new[b, :, :n[b]]
+            assert torch.equal(cache, want)
+
+
 def test_determinism_and_reuse_of_scratch():
     """Same inputs twice through the same tree and workspace: identical bits
     (tickets and scratch are left ready for reuse)."""

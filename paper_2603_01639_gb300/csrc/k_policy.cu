@@ -71,17 +71,16 @@ __global__ void __launch_bounds__(kPolicyNT) size_obs_kernel(const ltd_tree t, c
 // ------------------------------------------------ policies on the device
 // One thread-block cluster of kMlpC CTAs (on the SMs of one GPC) evaluates
 // the MLP for groups of up to kMlpG sequences at a time, so every weight is
-// read once per group.
-// Each CTA owns a slice of every layer's output units; a thread owns one
-// unit and a strided share of the input rows (P threads per unit, their
-// partial sums added in a fixed order).  A layer whose rows can be copied
-// A packed network (ltd_mlp_pack: every CTA's column slice of W stored
-// contiguously) streams the slice through a ring of shared-memory stages,
-// one bulk copy of up to kMlpStageBytes per chunk issued up to kMlpStages
-// chunks ahead (also across layers), so the whole slice is in flight at
-// once; a row-major network is read with plain loads.  The layer's outputs are pushed into
-// every CTA's next-activation buffer through distributed shared memory and
-// one cluster barrier per layer publishes them.
+// read once per group.  Each CTA owns a slice of every layer's output units;
+// a thread owns a quad of four consecutive units and every P-th input row,
+// the P partial sums of a unit being added in a fixed order.  A packed
+// network (ltd_mlp_pack: every CTA's column slice of W stored contiguously)
+// streams the slice through a ring of shared-memory stages, one bulk copy
+// of up to kMlpStageBytes per stage, issued up to kMlpStages stages ahead
+// (also across layers), so the whole slice is in flight at once; a
+// row-major network is read with plain loads.  Each layer's outputs are
+// pushed into every CTA's next activation buffer through distributed shared
+// memory, and one cluster barrier per layer publishes them.
 #ifdef LTD_TRACE
 __device__ unsigned long long g_mlp_trace[16][16];
 __device__ unsigned long long g_mlp_chunk_trace[16][64];  // per chunk: issued, landed

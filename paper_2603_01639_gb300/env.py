@@ -104,6 +104,8 @@ class CycleEnv:
         next level for the sequences that continue.  Returns the depth
         observation (a stopped sequence keeps reporting its last level) and
         whether any sequence is still drafting."""
+        if self.ci is None:
+            raise RuntimeError("reset() starts an episode")
         cont = np.asarray(cont, bool).reshape(-1)
         if cont.shape[0] != self.cfg.batch:
             raise ValueError("one depth decision per sequence")
@@ -127,6 +129,8 @@ class CycleEnv:
         """Verify N_b nodes per sequence (root included) and return the reward
         [B] (tokens per second) and an info dict."""
         cfg, ci = self.cfg, self.ci
+        if ci is None:
+            raise RuntimeError("reset() starts an episode")
         view = {k: v.cpu().numpy() for k, v in self.tree.view().items()}
         n = np.asarray(n_verify, np.int64).reshape(-1)
         if n.shape[0] != cfg.batch or (n < 1).any() or (n > cfg.max_n).any() or \
@@ -160,6 +164,7 @@ class CycleEnv:
         ltd.ltd_check()
         a = acc["accept_len"].cpu().numpy()
         reward = throughput_reward(a, self.t_draft, t_verify)
+        self.ci = None  # the episode is over
         info = {"accept_len": a, "bonus": acc["bonus"].cpu().numpy(),
                 "path": acc["path"].cpu().numpy(), "levels": view["n_levels"].copy(),
                 "n_verify": n.astype(np.int32), "ids": ids,

@@ -75,7 +75,9 @@ class DepthPolicy:
 
 
 class SizePolicy:
-    """pi_V: observation [B][v_pad + 2] -> verify size N in {20, 40, ..., 240} ([B])."""
+    """pi_V: observation [B][v_pad + 2] -> candidate count V in {20, 40, ...,
+    240} ([B]); ``verify_size`` turns it into the verify size N the library
+    takes (root included), as ltd_size_policy does on the device."""
 
     def __init__(self, v_pad: int, seed: int = 1):
         self.net = MLP(v_pad + 2, (1024, 256), N_ACTIONS, seed, _obs_scale(v_pad + 2))
@@ -83,3 +85,8 @@ class SizePolicy:
     def decide(self, obs: np.ndarray) -> np.ndarray:
         a = np.argmax(self.net.forward(obs), axis=1).astype(np.int32)
         return (N_MIN + N_STEP * a).astype(np.int32)
+
+    def verify_size(self, obs: np.ndarray, n_cap: int, n_nodes) -> np.ndarray:
+        """N = min(1 + V, n_cap, nodes in the tree) per sequence."""
+        v = self.decide(obs)
+        return np.minimum(np.minimum(1 + v, n_cap), np.asarray(n_nodes)).astype(np.int32)

@@ -49,3 +49,15 @@ def test_size_actions_map_linearly_onto_20_to_240():
         b[a] = 1.0
         got.append(int(p.decide(obs)[0]))
     assert got == list(range(20, 241, 20))
+
+
+def test_verify_size_counts_the_root_and_respects_the_caps():
+    p = policy.SizePolicy(8, seed=0)
+    w, b = p.net.layers[-1]
+    w[:] = 0.0
+    b[:] = 0.0
+    b[2] = 1.0                                    # action 2: V = 60
+    obs = np.zeros((3, 10), np.float32)
+    n = p.verify_size(obs, n_cap=64, n_nodes=[511, 30, 511])
+    assert n.tolist() == [61, 30, 61]
+    assert p.verify_size(obs, n_cap=48, n_nodes=[511, 511, 511]).tolist() == [48, 48, 48]

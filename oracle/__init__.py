@@ -36,6 +36,7 @@ from .ltd_oracle import (  # noqa: F401
     select_verify,
     size_observation,
     size_policy_step,
+    softmax_t,
     splitmix64_stream,
     tree_attention,
     uniform_gumbel,

@@ -72,6 +72,13 @@ def rank_by_logit(x: np.ndarray, W: int) -> np.ndarray:
     return order[:W]
 
 
+def softmax_t(x: np.ndarray, temperature: float = 1.0) -> np.ndarray:
+    """softmax(x / T) in fp64: the distribution sampled at temperature T
+    (T = 1 is the plain softmax)."""
+    assert temperature > 0.0
+    return np.exp(log_softmax(np.asarray(x, dtype=np.float64) / temperature)[0])
+
+
 def mask_words(mask: np.ndarray) -> np.ndarray:
     """Pack a boolean [N][N'] mask into uint32 words: bit j of row i lives in
     word j // 32 at bit position j % 32."""
@@ -330,12 +337,14 @@ def accept_greedy(tree: OracleTree, chosen, target_rows):
         path.append(slot)
 
 
-def accept_stochastic(tree: OracleTree, chosen, target_rows, draft_rows, seed, b, cycle_no):
-    """Stochastic verification at T = 1 (reading: SpecInfer's multi-candidate
-    speculative sampling with the Leviathan/Chen ratio test).
+def accept_stochastic(tree: OracleTree, chosen, target_rows, draft_rows, seed, b, cycle_no,
+                      temperature: float = 1.0):
+    """Stochastic verification at temperature T (reading: SpecInfer's
+    multi-candidate speculative sampling with the Leviathan/Chen ratio test;
+    the paper's experiments use T = 1, the default).
 
-    At the current slot u: p = softmax(target row of u), q = softmax(draft row
-    that expanded u).  For each verified child x_i of u in slot order: accept
+    At the current slot u: p = softmax(target row of u / T), q =
+    softmax(draft row that expanded u / T).  For each verified child x_i of u in slot order: accept
     if r_i * q(x_i) < p(x_i) with r_i = uniform_ratio(seed, b, cycle, u, i);
     otherwise p <- max(p - q, 0) / sum (p kept when that sum is 0).  When no
     child is accepted, the bonus is argmax_t [log p(t) - log(-log g_t)] over
@@ -349,10 +358,10 @@ def accept_stochastic(tree: OracleTree, chosen, target_rows, draft_rows, seed, b
     margins = []
     while True:
         u = int(chosen[slot])
-        p = np.exp(log_softmax(target_rows[slot])[0])
+        p = softmax_t(target_rows[slot], temperature)
         accepted = None
         if kids[slot]:
-            q = np.exp(log_softmax(draft_rows[tree.xrow[u]])[0])
+            q = softmax_t(draft_rows[tree.xrow[u]], temperature)
             for i, c in enumerate(kids[slot]):
                 x = tree.token[int(chosen[c])]
                 r = uniform_ratio(seed, b, cycle_no, slot, i)
@@ -379,9 +388,9 @@ def accept_stochastic(tree: OracleTree, chosen, target_rows, draft_rows, seed, b
 
 
 def accept_without_replacement(tree: OracleTree, chosen, target_rows, draft_rows, seed, b,
-                               cycle_no):
-    """Stochastic verification at T = 1 for children drawn from q without
-    replacement (a variant of the rule above: recursive rejection sampling).
+                               cycle_no, temperature: float = 1.0):
+    """Stochastic verification at temperature T (p and q as in
+    accept_stochastic) for children drawn from q without replacement (a variant of the rule above: recursive rejection sampling).
     Child x_i is proposed by q_i, the draft distribution with the children
     rejected so far removed and renormalised (q_0 = q); it is accepted if
     r_i q_i(x_i) < p_i(x_i), else p_{i+1} = max(p_i - q_i, 0) / sum (p_i kept
@@ -394,10 +403,10 @@ def accept_without_replacement(tree: OracleTree, chosen, target_rows, draft_rows
     margins = []
     while True:
         u = int(chosen[slot])
-        p = np.exp(log_softmax(target_rows[slot])[0])
+        p = softmax_t(target_rows[slot], temperature)
         accepted = None
         if kids[slot]:
-            q = np.exp(log_softmax(draft_rows[tree.xrow[u]])[0])
+            q = softmax_t(draft_rows[tree.xrow[u]], temperature)
             for i, c in enumerate(kids[slot]):
                 x = tree.token[int(chosen[c])]
                 r = uniform_ratio(seed, b, cycle_no, slot, i)
@@ -428,8 +437,10 @@ def accept_without_replacement(tree: OracleTree, chosen, target_rows, draft_rows
         slot = accepted
 
 
-def accept_point_mass(tree: OracleTree, chosen, target_rows, seed, b, cycle_no):
-    """Stochastic verification at T = 1 with point-mass proposals (a variant
+def accept_point_mass(tree: OracleTree, chosen, target_rows, seed, b, cycle_no,
+                      temperature: float = 1.0):
+    """Stochastic verification at temperature T (p = softmax(target row / T))
+    with point-mass proposals (a variant
     of the rule above for a tree whose children are the draft's top-W tokens,
     not samples from q: each child is a deterministic proposal, so its
     proposal distribution is a point mass on its token).
@@ -449,7 +460,7 @@ def accept_point_mass(tree: OracleTree, chosen, target_rows, seed, b, cycle_no):
     path = [0]
     margins = []
     while True:
-        p = np.exp(log_softmax(target_rows[slot])[0])
+        p = softmax_t(target_rows[slot], temperature)
         accepted = None
         rejected = []
         removed = 0.0

@@ -410,6 +410,49 @@ def test_stochastic_zero_probability_child_rejected():
 
 
 # ------------------------------------------------------------------ RNG pins
+# ------------------------------------------------------------- temperature
+def test_softmax_at_temperature_is_scipy_softmax_of_scaled_logits():
+    x = np.array([0.5, -1.0, 2.0, 0.0, 3.5])
+    for T in (0.25, 1.0, 3.0):
+        np.testing.assert_allclose(O.softmax_t(x, T), scipy.special.softmax(x / T), rtol=1e-13)
+
+
+@pytest.mark.parametrize("T", [0.5, 2.0])
+def test_stochastic_rule_at_temperature_samples_the_tempered_target(T):
+    """Children i.i.d. from q_T = softmax(draft / T): the first emitted token
+    follows p_T = softmax(target / T)."""
+    vocab, k, trials = 6, 3, 20000
+    rng = np.random.default_rng(int(T * 100))
+    xt = rng.standard_normal(vocab) * 1.5
+    xq = rng.standard_normal(vocab) * 1.5
+    p = scipy.special.softmax(xt / T)
+    q = scipy.special.softmax(xq / T)
+    counts = np.zeros(vocab)
+    for trial in range(trials):
+        kids = rng.choice(vocab, size=k, p=q)
+        tree = _star_tree(0, kids, k)
+        target = np.vstack([xt] + [rng.standard_normal(vocab) for _ in range(k)])
+        path, a, bonus, _ = oracle.accept_stochastic(tree, np.arange(k + 1), target, xq[None, :],
+                                                     seed=5, b=0, cycle_no=trial, temperature=T)
+        counts[tree.token[path[1]] if a >= 1 else bonus] += 1
+    chi2 = ((counts - trials * p) ** 2 / (trials * p)).sum()
+    assert scipy.stats.chi2.sf(chi2, vocab - 1) > 1e-4, (counts / trials, p)
+
+
+def test_point_mass_at_temperature_samples_the_tempered_target():
+    vocab, k, trials, T = 6, 2, 20000, 0.5
+    xt = np.array([1.0, 0.4, -0.3, 0.9, -1.1, 0.2])
+    p = scipy.special.softmax(xt / T)
+    tree = _star_tree(0, [0, 3], k)
+    counts = np.zeros(vocab)
+    for trial in range(trials):
+        path, a, bonus, _ = oracle.accept_point_mass(tree, np.arange(k + 1), np.vstack([xt] * (k + 1)),
+                                                     seed=8, b=0, cycle_no=trial, temperature=T)
+        counts[tree.token[path[1]] if a >= 1 else bonus] += 1
+    chi2 = ((counts - trials * p) ** 2 / (trials * p)).sum()
+    assert scipy.stats.chi2.sf(chi2, vocab - 1) > 1e-4, (counts / trials, p)
+
+
 # --------------------------------------------- without-replacement rule
 def test_without_replacement_preserves_target_distribution():
     """Children drawn from q WITHOUT replacement (distinct tokens, as a

@@ -270,7 +270,9 @@ class Cycle:
                                              cfg.max_n, cfg.max_ctx)
 
     def launches_per_step(self):
-        return 1 + self.max_depth + 1 + self.layers * self.attention_kernel()[1] + 2
+        # reset, one expansion per level, selection, attention per layer,
+        # acceptance (row statistics, walk) and the compaction of every layer
+        return 1 + self.max_depth + 1 + self.layers * self.attention_kernel()[1] + 3
 
     # algorithmic bytes / flops of one attention launch
     def attention_algorithmic(self):

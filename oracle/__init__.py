@@ -28,6 +28,7 @@ from .ltd_oracle import (  # noqa: F401
     expand_level,
     first_argmax,
     grow_tree,
+    lm_head_row_stats,
     log_softmax,
     mask_words,
     mlp_forward,

@@ -502,6 +502,23 @@ def compact_kv(cache: np.ndarray, ctx: int, path) -> np.ndarray:
     return out
 
 
+# ------------------------------------------------------- target LM-head rows
+def lm_head_row_stats(hidden: np.ndarray, weight: np.ndarray):
+    """The target's verification logits and the row statistics acceptance
+    reads from them (section 3.2, "Draft Tree Verification": one target
+    forward over the verified tokens; the last layer maps each hidden state
+    to vocabulary logits).  logits[r][v] = sum_k hidden[r][k] weight[v][k]
+    in fp64; per row the max, the log-sum-exp and the argmax (ties to the
+    lower token id).  Returns (logits, row_max, row_lse, row_argmax)."""
+    h = np.asarray(hidden, dtype=np.float64)
+    w = np.asarray(weight, dtype=np.float64)
+    logits = h @ w.T
+    row_max = logits.max(axis=1)
+    row_lse = row_max + np.log(np.exp(logits - row_max[:, None]).sum(axis=1))
+    row_argmax = np.array([first_argmax(r) for r in logits], dtype=np.int64)
+    return logits, row_max, row_lse, row_argmax
+
+
 # --------------------------------------------------------- policy observations
 POLICY_PAD = -100.0   # fill of unused observation slots (the paper only says "padded")
 

@@ -410,6 +410,31 @@ def test_stochastic_zero_probability_child_rejected():
 
 
 # ------------------------------------------------------------------ RNG pins
+# ---------------------------------------------------- LM-head row statistics
+def test_lm_head_rows_against_torch_linear_and_scipy():
+    """logits = hidden W^T as torch.nn.functional.linear computes it (W held
+    [vocab][d_model]); row statistics from scipy's logsumexp and a brute-force
+    first-maximum scan."""
+    rng = np.random.default_rng(9)
+    h = rng.standard_normal((5, 12))
+    w = rng.standard_normal((37, 12))
+    logits, mx, lse, am = O.lm_head_row_stats(h, w)
+    ref = torch.nn.functional.linear(torch.from_numpy(h), torch.from_numpy(w)).numpy()
+    np.testing.assert_allclose(logits, ref, rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(lse, scipy.special.logsumexp(ref, axis=1), rtol=1e-12)
+    np.testing.assert_array_equal(mx, ref.max(axis=1))
+    for r in range(5):
+        best = max(range(37), key=lambda v: (ref[r, v], -v))
+        assert am[r] == best
+
+
+def test_lm_head_argmax_ties_to_the_lower_token():
+    h = np.array([[1.0, 0.0]])
+    w = np.array([[0.0, 1.0], [2.0, 0.0], [2.0, 5.0], [1.0, 1.0]])   # tokens 1 and 2 tie at 2
+    _, mx, _, am = O.lm_head_row_stats(h, w)
+    assert mx[0] == 2.0 and am[0] == 1
+
+
 # ------------------------------------------------------------- temperature
 def test_softmax_at_temperature_is_scipy_softmax_of_scaled_logits():
     x = np.array([0.5, -1.0, 2.0, 0.0, 3.5])

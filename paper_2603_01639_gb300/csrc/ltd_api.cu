@@ -6,6 +6,8 @@
 #include <cstdlib>
 #include <mutex>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "ltd.h"
 #include "ltd_internal.h"
 
@@ -69,6 +71,18 @@ ltd_status from_cuda(cudaError_t e) { return e == cudaSuccess ? LTD_OK : LTD_ERR
 
 using namespace ltd;
 
+namespace {
+// An NVTX range over one API call (named after it), so a profiler can
+// attribute the kernels a call launches; without a tool attached the calls
+// are no-ops.
+struct ApiRange {
+  explicit ApiRange(const char* name) { nvtxRangePushA(name); }
+  ~ApiRange() { nvtxRangePop(); }
+  ApiRange(const ApiRange&) = delete;
+  ApiRange& operator=(const ApiRange&) = delete;
+};
+}  // namespace
+
 extern "C" {
 
 int32_t ltd_version(void) { return 100; }
@@ -129,6 +143,7 @@ ltd_status ltd_tree_init(ltd_tree* tree, void* d_mem, size_t bytes, int32_t batc
 
 ltd_status ltd_tree_reset(const ltd_tree* tree, const int32_t* d_root_tokens,
                           ltd_stream_t stream) {
+  const ApiRange nvtx_range("ltd_tree_reset");
   if (!tree_ok(tree) || d_root_tokens == nullptr) return LTD_ERR_INVALID_ARG;
   return from_cuda(launch_tree_reset(tree, d_root_tokens, reinterpret_cast<cudaStream_t>(stream)));
 }
@@ -136,6 +151,7 @@ ltd_status ltd_tree_reset(const ltd_tree* tree, const int32_t* d_root_tokens,
 ltd_status ltd_expand_tree(const ltd_tree* tree, int32_t level, const void* d_draft_rows,
                            ltd_dtype dtype, int64_t vocab, int64_t rows_per_seq,
                            const int32_t* d_active, ltd_stream_t stream) {
+  const ApiRange nvtx_range("ltd_expand_tree");
   if (!tree_ok(tree) || d_draft_rows == nullptr || !dtype_ok(dtype)) return LTD_ERR_INVALID_ARG;
   if (level < 1 || level > tree->max_depth) return LTD_ERR_SHAPE;
   if (vocab < tree->k || vocab > tree->max_vocab) return LTD_ERR_SHAPE;
@@ -175,12 +191,14 @@ ltd_status ltd_expand_tree(const ltd_tree* tree, int32_t level, const void* d_dr
 
 ltd_status ltd_depth_observation(const ltd_tree* tree, const int32_t* d_ctx, float* d_out,
                                  ltd_stream_t stream) {
+  const ApiRange nvtx_range("ltd_depth_observation");
   if (!tree_ok(tree) || d_ctx == nullptr || d_out == nullptr) return LTD_ERR_INVALID_ARG;
   return from_cuda(launch_depth_obs(tree, d_ctx, d_out, reinterpret_cast<cudaStream_t>(stream)));
 }
 
 ltd_status ltd_size_observation(const ltd_tree* tree, const int32_t* d_ctx, int32_t v_pad,
                                 float* d_out, ltd_stream_t stream) {
+  const ApiRange nvtx_range("ltd_size_observation");
   if (!tree_ok(tree) || d_ctx == nullptr || d_out == nullptr) return LTD_ERR_INVALID_ARG;
   if (v_pad < tree->max_nodes) return LTD_ERR_SHAPE;
   return from_cuda(
@@ -211,6 +229,7 @@ size_t ltd_mlp_packed_bytes(const ltd_mlp* net) {
 
 ltd_status ltd_mlp_pack(const ltd_mlp* net, void* d_mem, size_t bytes, ltd_mlp* packed,
                         ltd_stream_t stream) {
+  const ApiRange nvtx_range("ltd_mlp_pack");
   if (packed == nullptr || d_mem == nullptr || reinterpret_cast<uintptr_t>(d_mem) % 256 != 0)
     return LTD_ERR_INVALID_ARG;
   const ltd_status st = mlp_ok(net, -1);
@@ -224,6 +243,7 @@ ltd_status ltd_mlp_pack(const ltd_mlp* net, void* d_mem, size_t bytes, ltd_mlp* 
 ltd_status ltd_depth_policy(const ltd_tree* tree, const int32_t* d_ctx, const ltd_mlp* net,
                             const int32_t* d_active_in, int32_t* d_active_out, float* d_logits,
                             ltd_stream_t stream) {
+  const ApiRange nvtx_range("ltd_depth_policy");
   if (!tree_ok(tree) || d_ctx == nullptr || d_active_out == nullptr) return LTD_ERR_INVALID_ARG;
   const ltd_status st = mlp_ok(net, tree->k * tree->k + 2);
   if (st != LTD_OK) return st;
@@ -235,6 +255,7 @@ ltd_status ltd_depth_policy(const ltd_tree* tree, const int32_t* d_ctx, const lt
 ltd_status ltd_size_policy(const ltd_tree* tree, const int32_t* d_ctx, int32_t v_pad,
                            const ltd_mlp* net, int32_t n_cap, int32_t* d_n_verify,
                            float* d_logits, ltd_stream_t stream) {
+  const ApiRange nvtx_range("ltd_size_policy");
   if (!tree_ok(tree) || d_ctx == nullptr || d_n_verify == nullptr) return LTD_ERR_INVALID_ARG;
   if (v_pad < tree->max_nodes || v_pad > 8192 || n_cap < 1) return LTD_ERR_SHAPE;
   const ltd_status st = mlp_ok(net, v_pad + 2);
@@ -246,6 +267,7 @@ ltd_status ltd_size_policy(const ltd_tree* tree, const int32_t* d_ctx, int32_t v
 ltd_status ltd_select_verify(const ltd_tree* tree, const int32_t* d_n_verify, int32_t n_max,
                              const int32_t* d_ctx, int32_t* d_node_ids, int32_t* d_pos,
                              uint32_t* d_mask, ltd_stream_t stream) {
+  const ApiRange nvtx_range("ltd_select_verify");
   if (!tree_ok(tree) || !d_n_verify || !d_ctx || !d_node_ids || !d_pos || !d_mask)
     return LTD_ERR_INVALID_ARG;
   if (n_max < 1 || n_max > LTD_MAX_N) return LTD_ERR_SHAPE;
@@ -343,6 +365,7 @@ ltd_status ltd_tree_attention(const void* d_q, const void* d_k, const void* d_v,
                               int32_t max_ctx, const int32_t* d_n_verify, int32_t n_max,
                               const uint32_t* d_mask, float scale, void* d_workspace,
                               size_t workspace_bytes, ltd_stream_t stream) {
+  const ApiRange nvtx_range("ltd_tree_attention");
   return tree_attention(d_q, d_k, d_v, d_out, dtype, batch, hq, hkv, head_dim, s_cap, d_ctx, max_ctx,
                         d_n_verify, n_max, d_mask, scale, d_workspace, workspace_bytes, nullptr,
                         nullptr, stream);
@@ -355,6 +378,7 @@ ltd_status ltd_tree_attention_next(const void* d_q, const void* d_k, const void*
                                    const uint32_t* d_mask, float scale, void* d_workspace,
                                    size_t workspace_bytes, const void* d_next_k,
                                    const void* d_next_v, ltd_stream_t stream) {
+  const ApiRange nvtx_range("ltd_tree_attention_next");
   return tree_attention(d_q, d_k, d_v, d_out, dtype, batch, hq, hkv, head_dim, s_cap, d_ctx, max_ctx,
                         d_n_verify, n_max, d_mask, scale, d_workspace, workspace_bytes, d_next_k,
                         d_next_v, stream);
@@ -396,6 +420,7 @@ size_t ltd_accept_workspace_bytes(int32_t batch, int32_t n_max, int64_t vocab) {
 ltd_status ltd_kv_append(const ltd_kv_cache* kv, int32_t batch, int32_t n_max,
                          const void* d_new_k, const void* d_new_v, const int32_t* d_ctx,
                          const int32_t* d_n_verify, ltd_stream_t stream) {
+  const ApiRange nvtx_range("ltd_kv_append");
   if (kv == nullptr || !kv->d_k_layers || !kv->d_v_layers || !d_new_k || !d_new_v || !d_ctx ||
       !d_n_verify || !dtype_ok(kv->dtype))
     return LTD_ERR_INVALID_ARG;
@@ -429,6 +454,7 @@ ltd_status ltd_kv_append(const ltd_kv_cache* kv, int32_t batch, int32_t n_max,
 ltd_status ltd_kv_compact(const ltd_kv_cache* kv, int32_t batch, const int32_t* d_path,
                           int32_t path_stride, const int32_t* d_accept_len, const int32_t* d_ctx,
                           ltd_stream_t stream) {
+  const ApiRange nvtx_range("ltd_kv_compact");
   if (kv == nullptr || !kv->d_k_layers || !kv->d_v_layers || !d_path || !d_accept_len || !d_ctx ||
       !dtype_ok(kv->dtype))
     return LTD_ERR_INVALID_ARG;
@@ -460,6 +486,7 @@ ltd_status ltd_accept(const ltd_tree* tree, const void* d_target_logits, const v
                       int32_t* d_new_ctx, int32_t* d_path, int32_t* d_accept_len,
                       int32_t* d_bonus, const ltd_kv_cache* kv, void* d_workspace,
                       size_t workspace_bytes, ltd_stream_t stream) {
+  const ApiRange nvtx_range("ltd_accept");
   if (!tree_ok(tree) || !d_target_logits || !d_draft_rows || !dtype_ok(dtype) || !d_node_ids ||
       !d_n_verify || !d_mode || !d_ctx || !d_new_ctx || !d_path || !d_accept_len || !d_bonus)
     return LTD_ERR_INVALID_ARG;

@@ -20,7 +20,14 @@ tie-breaking:
   Leviathan/Chen ratio test (the paper only states that the target
   distribution is preserved, §1 and §5.1 "Metrics").
 
-Readings where the paper is silent or loose (all listed in the design doc):
+Around the cycle, also written out here: the two policies' observations and
+network (Appendix A.2: depth observation, size observation, ReLU MLP,
+argmax decisions), two more stochastic verification rules for trees whose
+children are not i.i.d. draws (point-mass proposals, proposals without
+replacement), every stochastic rule at a temperature T, and the target
+LM head's logits with the row statistics acceptance reads.
+
+Readings where the paper is silent or loose:
 
 * depth: L = levels below the root, V_all = 1 + W + (L-1) W^2 (the paper's D
   is L + 1);

@@ -47,7 +47,7 @@ typedef enum ltd_status {
   LTD_OK = 0,
   LTD_ERR_INVALID_ARG = 1, /* null pointer, bad enum, non-positive size   */
   LTD_ERR_SHAPE = 2,       /* sizes inconsistent with each other/limits   */
-  LTD_ERR_UNSUPPORTED = 3, /* valid request this build does not implement */
+  LTD_ERR_UNSUPPORTED = 3, /* valid request the library does not implement */
   LTD_ERR_CUDA = 4,        /* a CUDA runtime call failed                  */
   LTD_ERR_DEVICE = 5,      /* a kernel flagged bad per-sequence data      */
   LTD_ERR_TIMEOUT = 6      /* a bounded device wait gave up               */
@@ -61,7 +61,7 @@ typedef enum ltd_mode {
   LTD_STOCHASTIC_NO_REPLACEMENT = 3
 } ltd_mode;
 
-/* Limits of this build. */
+/* Limits of the library. */
 #define LTD_MAX_K 32          /* beam width k                              */
 #define LTD_MAX_DEPTH 16      /* levels below the root                     */
 #define LTD_MAX_N 256         /* verify size, root included               */

@@ -61,3 +61,28 @@ def test_verify_size_counts_the_root_and_respects_the_caps():
     n = p.verify_size(obs, n_cap=64, n_nodes=[511, 30, 511])
     assert n.tolist() == [61, 30, 61]
     assert p.verify_size(obs, n_cap=48, n_nodes=[511, 511, 511]).tolist() == [48, 48, 48]
+
+
+def test_host_policies_match_the_oracle_network():
+    """The host (numpy fp32) policies against the oracle's fp64 network on
+    the same observations: logits within the fp32 accumulation bound,
+    decisions equal wherever the fp64 top-two gap is clear of it."""
+    import oracle
+    rng = np.random.default_rng(11)
+    k, v_pad = 10, 1 + 10 + 5 * 100
+    dp, sp = policy.DepthPolicy(k, seed=5), policy.SizePolicy(v_pad, seed=6)
+    for pol, n_in in ((dp, k * k + 2), (sp, v_pad + 2)):
+        obs = np.concatenate([rng.normal(-8, 3, (16, n_in - 2)),
+                              np.stack([rng.integers(1, 9, 16), rng.integers(512, 8192, 16)], 1)],
+                             axis=1).astype(np.float32)
+        got = pol.net.forward(obs)
+        ref = oracle.mlp_forward(obs, pol.net.layers)
+        h = np.abs(obs.astype(np.float64))
+        for w, b in pol.net.layers:
+            h = h @ np.abs(w.astype(np.float64)) + np.abs(b.astype(np.float64))
+        tol = 1e-5 * h + 1e-6
+        assert (np.abs(got - ref) <= tol).all()
+        top2 = np.sort(ref, axis=1)[:, -2:]
+        clear = (top2[:, 1] - top2[:, 0]) > 2 * tol.max(axis=1)
+        assert clear.sum() >= 8, "too many near-ties to check decisions; pick another seed"
+        np.testing.assert_array_equal(np.argmax(got, axis=1)[clear], np.argmax(ref, axis=1)[clear])

@@ -138,6 +138,13 @@ def _dtype(t: torch.Tensor) -> int:
     raise LtdError(f"unsupported dtype {t.dtype}")
 
 
+def _need_vec(t: torch.Tensor, name: str, numel: int, dtype):
+    """A contiguous CUDA tensor of ``dtype`` holding exactly ``numel`` values."""
+    _need(t, name, dtype)
+    if t.numel() != numel:
+        raise LtdError(f"{name} must hold {numel} values, got {t.numel()}")
+
+
 def _need(t: torch.Tensor, name: str, dtype=None):
     if not t.is_cuda:
         raise LtdError(f"{name} must be a CUDA tensor")
@@ -308,6 +315,11 @@ def ltd_depth_policy(tree: Tree, ctx: torch.Tensor, net: MlpNet, active_in=None,
     _need(ctx, "ctx", torch.int32)
     if active_out is None:
         active_out = torch.empty(tree.batch, dtype=torch.int32, device=ctx.device)
+    _need_vec(active_out, "active_out", tree.batch, torch.int32)
+    if active_in is not None:
+        _need_vec(active_in, "active_in", tree.batch, torch.int32)
+    if logits is not None:
+        _need_vec(logits, "logits", tree.batch * 2, torch.float32)
     _ok(lib().ltd_depth_policy(C.byref(tree.s), _ptr(ctx), C.byref(net.s), _ptr(active_in),
                                _ptr(active_out), _ptr(logits), _stream(stream)),
         "ltd_depth_policy")
@@ -322,6 +334,9 @@ def ltd_size_policy(tree: Tree, ctx: torch.Tensor, net: MlpNet, n_cap: int, v_pa
     v_pad = tree.max_nodes if v_pad is None else v_pad
     if n_verify is None:
         n_verify = torch.empty(tree.batch, dtype=torch.int32, device=ctx.device)
+    _need_vec(n_verify, "n_verify", tree.batch, torch.int32)
+    if logits is not None:
+        _need_vec(logits, "logits", tree.batch * net.n_out, torch.float32)
     _ok(lib().ltd_size_policy(C.byref(tree.s), _ptr(ctx), v_pad, C.byref(net.s), n_cap,
                               _ptr(n_verify), _ptr(logits), _stream(stream)),
         "ltd_size_policy")

@@ -86,3 +86,16 @@ def test_host_policies_match_the_oracle_network():
         clear = (top2[:, 1] - top2[:, 0]) > 2 * tol.max(axis=1)
         assert clear.sum() >= 8, "too many near-ties to check decisions; pick another seed"
         np.testing.assert_array_equal(np.argmax(got, axis=1)[clear], np.argmax(ref, axis=1)[clear])
+
+
+def test_device_policy_bindings_check_their_buffers_on_the_host():
+    """Wrong buffers are refused by the binding before any launch (CPU
+    tensors, wrong dtype or size), so no device call is made."""
+    import pytest
+    import torch
+
+    from paper_2603_01639_gb300 import ltd
+    with pytest.raises(ltd.LtdError):
+        ltd._need_vec(torch.zeros(4, dtype=torch.int32), "x", 4, torch.int32)   # not on a GPU
+    with pytest.raises(ltd.LtdError):
+        ltd._need(torch.zeros(4, dtype=torch.float32), "x", torch.int32)

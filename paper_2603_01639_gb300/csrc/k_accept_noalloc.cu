@@ -56,7 +56,13 @@ extern "C" ltd_status ltd_accept_noalloc(const ltd_tree* tree, const void* d_tar
                                          const int32_t* d_ctx, int32_t* d_new_ctx, int32_t* d_path,
                                          int32_t* d_accept_len, int32_t* d_bonus,
                                          const ltd_kv_cache* kv, ltd_stream_t stream) {
-  if (tree == nullptr || n_max < 1 || n_max > LTD_MAX_N || vocab < 1) return LTD_ERR_SHAPE;
+  // The same argument checks, in the same order, as ltd_accept: a missing or
+  // malformed tree or a missing buffer is LTD_ERR_INVALID_ARG before any
+  // size is looked at.
+  if (!tree_valid(tree) || !d_target_logits || !d_draft_rows || !d_node_ids || !d_n_verify ||
+      !d_mode || !d_ctx || !d_new_ctx || !d_path || !d_accept_len || !d_bonus)
+    return LTD_ERR_INVALID_ARG;
+  if (n_max < 1 || n_max > LTD_MAX_N || vocab < 1) return LTD_ERR_SHAPE;
   const size_t need = ltd_accept_workspace_bytes(tree->batch, n_max, vocab);
   if (need == 0 || need > LTD_ACCEPT_NOALLOC_SCRATCH_BYTES) return LTD_ERR_SHAPE;
   unsigned char* scratch = scratch_address();

@@ -67,6 +67,9 @@ bool tree_ok(const ltd_tree* t) {
 ltd_status from_cuda(cudaError_t e) { return e == cudaSuccess ? LTD_OK : LTD_ERR_CUDA; }
 
 }  // namespace
+
+bool tree_valid(const ltd_tree* t) { return tree_ok(t); }
+
 }  // namespace ltd
 
 using namespace ltd;

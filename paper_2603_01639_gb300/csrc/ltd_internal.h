@@ -13,6 +13,10 @@ namespace ltd {
 // Address of this device's error word (lives in ltd_api.cu).
 uint32_t* device_error_word();
 
+// Whether `t` is a tree that ltd_tree_init carved: sizes within the limits
+// and every array present (lives in ltd_api.cu).
+bool tree_valid(const ltd_tree* t);
+
 // Whether launches carry the programmatic-dependent-launch attribute (on
 // unless the environment sets LTD_NO_PDL=1; read once).
 bool pdl_enabled();

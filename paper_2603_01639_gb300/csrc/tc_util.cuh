@@ -111,25 +111,6 @@ __device__ __forceinline__ void fence_after_sync() {
 __device__ __forceinline__ void fence_smem_async() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
-// The same tile into the shared memory of every CTA in `mask` (this
-// cluster's ranks); `dst` and `bar` are offsets valid in each of them, and
-// each destination's barrier receives the bytes that land there.
-__device__ __forceinline__ void tma_load_3d_mc(uint32_t dst, const CUtensorMap* map, uint32_t bar,
-                                               int32_t c0, int32_t c1, int32_t c2, uint16_t mask) {
-  asm volatile(
-      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster"
-      " [%0], [%1, {%3, %4, %5}], [%2], %6;" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1), "r"(c2), "h"(mask)
-      : "memory");
-}
-// Arrive on the barrier at offset `bar` in every CTA of `mask` once every MMA
-// issued so far by this thread completes.
-__device__ __forceinline__ void mma_commit_mc(uint32_t bar, uint16_t mask) {
-  asm volatile(
-      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
-      " [%0], %1;" ::"r"(bar), "h"(mask)
-      : "memory");
-}
 // Arrive on `bar` once every MMA issued so far by this thread completes.
 __device__ __forceinline__ void mma_commit(uint32_t bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(

@@ -103,3 +103,25 @@ def test_noalloc_rejects_sizes_beyond_its_array():
     st = L.ltd_accept_noalloc(C.byref(tree.s), p, p, 0, vocab, 5, p, p, n_max, p, 0, 0, p, p, p, p,
                               p, None, C.c_void_p(torch.cuda.current_stream().cuda_stream))
     assert L.ltd_status_string(st).decode() == "LTD_ERR_SHAPE"
+
+
+def test_noalloc_rejects_a_missing_or_malformed_tree_like_its_sibling():
+    """A NULL tree, a tree whose arrays were never carved, or a NULL output
+    buffer is LTD_ERR_INVALID_ARG, as in ltd_accept, before any size (here an
+    oversized batch) is looked at; nothing is launched."""
+    import ctypes as C
+    L = ltd.lib()
+    buf = torch.zeros(64, dtype=torch.int32, device="cuda")
+    p = C.c_void_p(buf.data_ptr())
+    s = C.c_void_p(torch.cuda.current_stream().cuda_stream)
+    raw = ltd.ltd_tree()
+    raw.batch, raw.max_depth, raw.k, raw.max_vocab = 4096, 3, 2, 1000   # sizes only, no arrays
+    good = ltd.Tree(1, 3, 2, 1000)
+    cases = [(None, p), (C.byref(raw), p), (C.byref(good.s), None)]
+    for tree, bonus in cases:
+        st = L.ltd_accept_noalloc(tree, p, p, 0, 1000, 5, p, p, 8, p, 0, 0, p, p, p, p, bonus,
+                                  None, s)
+        assert L.ltd_status_string(st).decode() == "LTD_ERR_INVALID_ARG"
+        st = L.ltd_accept(tree, p, p, 0, 1000, 5, p, p, 8, p, 0, 0, p, p, p, p, bonus, None, p,
+                          1 << 20, s)
+        assert L.ltd_status_string(st).decode() == "LTD_ERR_INVALID_ARG"

@@ -1,41 +1,46 @@
 // Tensor-core tree attention (LTD section 3.2, "Draft Tree Verification";
 // SpecInfer-style tree mask) for bf16 and head_dim 128 on sm_103a.
 //
-// Work unit: two 128-row tiles ("a" and "b") of the query rows of one KV
-// head of one sequence (row r = slot * G + g, so the G query heads of a KV
-// head share every K/V byte), over one split of that head's keys.
-//   warp 0      TMA: both Q tiles, then 128-key K and V chunks into
-//               two-stage rings (128-byte swizzle); the first two stages are
-//               issued before the setup barrier;
-//   warp 1      tcgen05.mma: S_x = Q_x K^T into tensor memory, then
-//               O_x += P_x V with P_x read from tensor memory; the order
-//               PV_a(j), S_a(j+1), PV_b(j), S_b(j+1) lets one tile's
-//               softmax run while the tensor core works on the other;
-//   warps 4-7   softmax of tile a, warps 8-11 of tile b, one thread per row
-//               (= tensor-memory lane) with the row's 128 scores in
+// Work unit: one 128-row tile of the query rows of one KV head of one
+// sequence (row r = slot * G + g, so the G query heads of a KV head share
+// every K/V byte), over one split of that head's keys.  The split's 128-key
+// chunks go to two streams, even chunks to stream 0 and odd chunks to stream
+// 1; each stream has its own S and O in tensor memory and its own running
+// max and sum, so one stream's softmax runs while the tensor core works on
+// the other's chunk, and the two are merged once at the end.
+//   warp 0      TMA: the Q tile, then K chunks into a three-stage ring
+//               (128-byte swizzle); Q and the first K chunk are issued
+//               before the sequence's context length is read;
+//   warp 1      tcgen05.mma: S_x = Q K_j^T into tensor memory, then
+//               O_x += P_x V_j with P_x read from tensor memory, issued in
+//               the order S(0), S(1), PV(0), S(2), PV(1), S(3), ...;
+//   warp 2      TMA: V chunks into a three-stage ring;
+//   warps 4-7   softmax of stream 0, warps 8-11 of stream 1, one thread per
+//               row (= tensor-memory lane) with the row's 128 scores in
 //               registers: the prefix + ancestor mask, then P = 2^(s - m)
-//               against the row's running max m, computed before the
+//               against the stream's running max m, computed before the
 //               chunk's own max is known and redone only for a warp in which
 //               some row's max grew by more than 2^8 (S is still in tensor
 //               memory then); O is rescaled only in that case.  P is written
-//               as bf16 over S's columns.  Both tiles' softmaxes run at once.
-// Tensor memory (512 columns): S_a | S_b | O_a | O_b.
+//               as bf16 over S's columns.
+// Tensor memory (512 columns): S_0 | S_1 | O_0 | O_1.
 //
 // Two launch shapes:
 //  - one split per unit (at least as many units as SMs): each CTA writes
 //    O / l straight to the output, and CTAs take the units longest first
-//    (every CTA ranks the (sequence, tile pair) groups by chunks x tiles
-//    from ctx and N), so the long sequences of a ragged batch start early;
+//    (every CTA ranks the (sequence, tile) groups by their chunk counts from
+//    ctx and N), so the long sequences of a ragged batch start early;
 //  - several splits per unit (fewer units than SMs): a cooperative launch,
 //    so every CTA is resident at once.  Each split writes its rows' O / l
-//    (bf16) and log-sum-exp to the workspace and arrives on its unit's
+//    (bf16) and log2-sum-exp to the workspace and arrives on its unit's
 //    counter; when all splits have arrived, split s combines rows
-//    [s R, s R + R) of the unit from L2 and writes them; the last split to
-//    leave resets the unit's counters to zero.
+//    [s R, s R + R) of the unit with loads straight from L2 into registers
+//    and writes them; the last split to leave resets the unit's counters.
 // Every wait is bounded (mbarrier waits and the counter spin): on timeout a
 // CTA flags LTD_DEVERR_TIMEOUT, drains its own TMA loads and MMAs, still
 // arrives and departs on its counter, frees its tensor memory and returns.
 #include <mutex>
+#include <type_traits>
 
 #include "ltd_common.cuh"
 #include "ltd_internal.h"
@@ -48,28 +53,41 @@ namespace {
 constexpr int kBM = 128;  // rows per tile = TMEM lanes
 constexpr int kBN = 128;  // keys per chunk
 constexpr int kD = 128;
-constexpr int kRows = 2 * kBM;
-constexpr int kThreads = 384;  // TMA warp, MMA warp, 2 idle, 8 softmax warps
-constexpr int kMaxW32 = LTD_MAX_N / 32;
+constexpr int kStages = 3;             // K ring and V ring depth
+constexpr int kThreads = 384;          // K TMA, MMA, V TMA, idle, 8 softmax warps
 constexpr int kMaxSplits = 64;
-constexpr int kMaxGroups = 1024;  // (sequence, tile pair) groups ranked on the device
+constexpr int kMaxGroups = 1024;       // (sequence, tile) groups ranked on the device
+constexpr int kCombineBatch = 16;      // splits whose partials one combining thread has in flight
 constexpr uint32_t kHalf = 16384;      // 128 rows x 128 bytes
 constexpr uint32_t kTile = 2 * kHalf;  // 128 x 128 bf16
-constexpr uint32_t kOffQ = 0;                                  // Q_a, Q_b
-constexpr uint32_t kOffK = kOffQ + 2 * kTile;                  // two stages
-constexpr uint32_t kOffV = kOffK + 2 * kTile;                  // two stages
-constexpr uint32_t kOffMask = kOffV + 2 * kTile;               // [256][8] words
-constexpr uint32_t kOffCost = kOffMask + kRows * kMaxW32 * 4;  // [kMaxGroups] int
-constexpr uint32_t kOffOrder = kOffCost + kMaxGroups * 4;      // [kMaxGroups] int
-constexpr uint32_t kOffBar = kOffOrder + kMaxGroups * 4;
+constexpr uint32_t kOffQ = 0;
+constexpr uint32_t kOffK = kOffQ + kTile;             // three stages
+constexpr uint32_t kOffV = kOffK + kStages * kTile;   // three stages
+constexpr uint32_t kOffBar = kOffV + kStages * kTile;
 constexpr uint32_t kOffHolder = kOffBar + 24 * 8;
 constexpr uint32_t kSmemBytes = kOffHolder + 16 + 1024;  // + alignment slack
+// Regions reused once they are free (after the last MMA, or before any load):
+constexpr uint32_t kOffCost = kOffV + 2 * kTile;       // [kMaxGroups] int, ranking only
+constexpr uint32_t kOffOrder = kOffCost + kMaxGroups * 4;
+constexpr uint32_t kOffStgL = kOffK;                   // [128] log2-sum-exp of the staged rows
+constexpr uint32_t kOffML = kOffK + 1024;              // [2][128] (m, l) of each stream
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kRowBytes = kD * 2;     // one bf16 output / partial row
+constexpr uint32_t kRowBytes = kD * 2;  // one bf16 output / partial row
 // P may grow to 2^8 before a row's running max is raised: bf16 bits of 2^8
 constexpr uint32_t kPMaxBits = 0x4380u;
 
-enum Bar { QFULL = 0, KFULL = 1, VFULL = 3, KEMPTY = 5, VEMPTY = 7, SFULL = 9, PFULL = 11, FIN = 13, CBAR = 14 };
+static_assert(kSmemBytes <= 232448, "shared memory over the per-block limit");
+static_assert(kOffOrder + kMaxGroups * 4 <= kOffV + kStages * kTile, "ranking arrays overflow");
+
+// barrier indices
+constexpr int QFULL = 0;
+constexpr int KFULL = 1;    // + stage
+constexpr int VFULL = 4;    // + stage
+constexpr int KEMPTY = 7;   // + stage
+constexpr int VEMPTY = 10;  // + stage
+constexpr int SFULL = 13;   // + stream
+constexpr int PFULL = 15;   // + stream
+constexpr int FIN = 17;
 
 // Optional phase timestamps for performance work (off in normal builds).
 #ifdef LTD_TRACE
@@ -91,16 +109,16 @@ __device__ unsigned long long g_attn_trace[4096][48];
 
 struct TcArgs {
   int32_t batch, hq, hkv, G, n_max, s_cap, max_ctx, W32;
-  int32_t splits, n_pairs, lpt;
+  int32_t splits, n_tiles, lpt;
   int32_t nch_h;  // host bound on chunks per sequence: ceil((max_ctx + n_max) / 128)
-  int32_t rs;     // rows per combining split: multiple of 4, >= 256 / splits
+  int32_t rs;     // rows combined per split: ceil(128 / splits)
   const int32_t* ctx;
   const int32_t* n_verify;
   const uint32_t* mask;
   float scale_log2;
   __nv_bfloat16* out;
-  uint8_t* part_o;  // [unit][split][256 rows][256 B] O / l, bf16, chunks swizzled (splits > 1)
-  float* part_l;    // [unit][split][256] log2-sum-exp
+  uint8_t* part_o;  // [unit][split][128 rows][256 B] O / l, bf16, chunks swizzled (splits > 1)
+  float* part_l;    // [unit][split][128] log2-sum-exp
   uint32_t* sync;   // [unit][2] arrive, depart
   const uint8_t* next_k;  // the next call's caches: L2 prefetch targets (or null)
   const uint8_t* next_v;
@@ -117,7 +135,8 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
 
 // Visibility of keys kk0 .. kk0+31 for one row as a 32-bit mask: keys below
 // ctx are the prefix (always visible), key ctx + j is verified slot j (bit j
-// of the row's ancestor mask), keys from key_hi on are outside this split.
+// of the row's ancestor mask, read from global memory), keys from key_hi on
+// are outside this split.
 __device__ __forceinline__ uint32_t low_bits(int n) {
   return n <= 0 ? 0u : (n >= 32 ? 0xFFFFFFFFu : ((1u << n) - 1u));
 }
@@ -130,8 +149,8 @@ __device__ __forceinline__ uint32_t visible32(int kk0, int ctx, int key_hi, int 
   if (js0 > -32 && js0 < 32 * W32) {
     const int w = js0 >> 5;  // floor division
     const int sh = js0 & 31;
-    const uint32_t lo = (w >= 0 && w < W32) ? mbits[w] : 0u;
-    const uint32_t hi = (w + 1 >= 0 && w + 1 < W32) ? mbits[w + 1] : 0u;
+    const uint32_t lo = (w >= 0 && w < W32) ? __ldg(mbits + w) : 0u;
+    const uint32_t hi = (w + 1 >= 0 && w + 1 < W32) ? __ldg(mbits + w + 1) : 0u;
     tree = __funnelshift_r(lo, hi, sh);
   }
   return in_range & (prefix | tree);
@@ -140,6 +159,22 @@ __device__ __forceinline__ uint32_t visible32(int kk0, int ctx, int key_hi, int 
 __device__ __forceinline__ bool seq_ok(const TcArgs& a, int ctx, int N) {
   return N >= 1 && N <= a.n_max && ctx >= 0 && ctx <= a.max_ctx && ctx + N <= a.s_cap;
 }
+
+__device__ __forceinline__ uint4 ld_cg_v4(const void* p) {
+  uint4 v;
+  asm volatile("ld.global.cg.v4.u32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "l"(p));
+  return v;
+}
+__device__ __forceinline__ float ld_cg_f32(const float* p) {
+  float v;
+  asm volatile("ld.global.cg.f32 %0, [%1];" : "=f"(v) : "l"(p));
+  return v;
+}
+
+template <int N>
+using Int = std::integral_constant<int, N>;
 
 __global__ void __launch_bounds__(kThreads, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CUtensorMap tk,
@@ -150,7 +185,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t raw = tc::smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
   uint8_t* gbase = smem_raw + (base - raw);
-  uint32_t* mask_s = reinterpret_cast<uint32_t*>(gbase + kOffMask);
   uint32_t* holder = reinterpret_cast<uint32_t*>(gbase + kOffHolder);
   auto bar = [&](int i) { return base + kOffBar + 8u * i; };
   const int S = a.splits;
@@ -161,16 +195,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (!a.kv_one) tc::tma_prefetch(&tv);
     TRACE(42);
     tc::mbar_init(bar(QFULL), 1);
-    for (int s = 0; s < 2; ++s) {
+    for (int s = 0; s < kStages; ++s) {
       tc::mbar_init(bar(KFULL + s), 1);
       tc::mbar_init(bar(VFULL + s), 1);
       tc::mbar_init(bar(KEMPTY + s), 1);
       tc::mbar_init(bar(VEMPTY + s), 1);
-      tc::mbar_init(bar(SFULL + s), 1);
-      tc::mbar_init(bar(PFULL + s), 128);
+    }
+    for (int x = 0; x < 2; ++x) {
+      tc::mbar_init(bar(SFULL + x), 1);
+      tc::mbar_init(bar(PFULL + x), 128);
     }
     tc::mbar_init(bar(FIN), 1);
-    tc::mbar_init(bar(CBAR), 1);
     tc::mbar_init_fence();
     TRACE(19);
   }
@@ -181,10 +216,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (tid == 0) TRACE(43);
 
   // ------------------------------------------------------ which unit
-  int split = 0, pair, b, kvh;
+  int split = 0, tile, b, kvh;
   if (S > 1) {
     split = blockIdx.x;
-    pair = blockIdx.y;
+    tile = blockIdx.y;
     b = blockIdx.z / a.hkv;
     kvh = blockIdx.z % a.hkv;
   } else {
@@ -192,21 +227,18 @@ __global__ void __launch_bounds__(kThreads, 1)
     int g = i / a.hkv;
     kvh = i % a.hkv;
     if (a.lpt) {
-      // rank every (sequence, tile pair) group by its work, largest first
-      // (ties to the lower group, so equal pairs of one sequence, which
-      // read the same K/V, stay together), and take the group at this
-      // CTA's rank; bad sequences rank last and flag on their own CTAs
+      // rank every (sequence, tile) group by its work, largest first (ties
+      // to the lower group, so the tiles of one sequence, which read the
+      // same K/V, stay together), and take the group at this CTA's rank;
+      // bad sequences rank last and flag on their own CTAs
       int* cost = reinterpret_cast<int*>(gbase + kOffCost);
       int* order = reinterpret_cast<int*>(gbase + kOffOrder);
-      const int groups = a.batch * a.n_pairs;
+      const int groups = a.batch * a.n_tiles;
       for (int gi = tid; gi < groups; gi += kThreads) {
-        const int bb = gi / a.n_pairs, pp = gi % a.n_pairs;
+        const int bb = gi / a.n_tiles, tt = gi % a.n_tiles;
         const int c = a.ctx[bb], n = a.n_verify[bb];
         int w = 0;
-        if (seq_ok(a, c, n)) {
-          const int rows = n * a.G - pp * kRows;
-          w = (rows <= 0 ? 0 : (rows > kBM ? 2 : 1)) * ((c + n + kBN - 1) / kBN);
-        }
+        if (seq_ok(a, c, n) && n * a.G > tt * kBM) w = (c + n + kBN - 1) / kBN;
         cost[gi] = w;
       }
       __syncthreads();
@@ -222,65 +254,43 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncthreads();
       g = order[g];
     }
-    b = g / a.n_pairs;
-    pair = g % a.n_pairs;
+    b = g / a.n_tiles;
+    tile = g % a.n_tiles;
   }
-  if (tid == 0) TRACE_VAL(25, static_cast<unsigned long long>(clock64()));
-  if (tid == 0) TRACE(26);
 
   // Keys are split by the host bound on the chunk count, so a split knows
   // its first chunk before reading ctx and N: the loads of Q and of the
-  // first K chunk go out at once (extra ones past this sequence's end are
-  // drained and ignored).  V of that chunk and the later chunks wait for the
-  // producer loop after the setup, so no CTA's first S queues at the DRAM
-  // behind every CTA's other chunks (8B-class layer 15.8 -> 15.1 us,
-  // 13B-class 20.1 -> 18.9 us).
+  // first K chunk go out at once (a chunk past this sequence's end is
+  // drained and ignored).  The other chunks wait for the setup below.
   const int cs = split * a.nch_h / S, ce = (split + 1) * a.nch_h / S;
   const int kvrow = b * a.hkv + kvh;
-  const int row0 = pair * kRows;
-  const bool has_b_h = row0 + kBM < a.n_max * a.G;  // tile b may hold rows
-  int nk_issued[2] = {0, 0}, nv_issued[2] = {0, 0}, n_issued = 0;
-  bool q_issued = false, v0_owed = false;
+  const int row0 = tile * kBM;
+  int nk_issued[kStages] = {0, 0, 0};
+  bool q_issued = false;
   auto issue_k = [&](int j) {
-    const int st = j & 1;
+    const int st = j % kStages;
     tc::mbar_expect_tx(bar(KFULL + st), kTile);
     for (int h = 0; h < 2; ++h)
       tc::tma_load_4d(base + kOffK + st * kTile + h * kHalf, &tk, bar(KFULL + st), h * 64,
                       (cs + j) * kBN, kvrow, a.kv_wk);
     ++nk_issued[st];
   };
-  auto issue_v = [&](int j) {
-    const int st = j & 1;
-    tc::mbar_expect_tx(bar(VFULL + st), kTile);
-    for (int h = 0; h < 2; ++h)
-      tc::tma_load_4d(base + kOffV + st * kTile + h * kHalf, a.kv_one ? &tk : &tv, bar(VFULL + st),
-                      h * 64, (cs + j) * kBN, kvrow, a.kv_wv);
-    ++nv_issued[st];
-  };
   auto issue_first = [&]() {
-    tc::mbar_expect_tx(bar(QFULL), has_b_h ? 2 * kTile : kTile);
-    for (int t = 0; t < (has_b_h ? 2 : 1); ++t) {
-      const int qrow = b * a.n_max + (row0 + t * kBM) / a.G;
-      for (int h = 0; h < 2; ++h)
-        tc::tma_load_3d(base + kOffQ + t * kTile + h * kHalf, &tq, bar(QFULL), h * 64, kvh * a.G,
-                        qrow);
-    }
+    tc::mbar_expect_tx(bar(QFULL), kTile);
+    const int qrow = b * a.n_max + row0 / a.G;
+    for (int h = 0; h < 2; ++h)
+      tc::tma_load_3d(base + kOffQ + h * kHalf, &tq, bar(QFULL), h * 64, kvh * a.G, qrow);
     q_issued = true;
     TRACE(20);
-    if (ce - cs > 0) {
-      issue_k(0);
-      TRACE(44);
-      v0_owed = true;
-    }
+    if (ce - cs > 0) issue_k(0);
     TRACE(17);
   };
-  // every load a CTA issued lands before it leaves or reuses shared memory
-  auto drain = [&]() {
+  // every K load (and Q) this thread issued lands before the CTA leaves or
+  // reuses shared memory; at most one load per stage is outstanding
+  auto drain_k = [&]() {
     if (q_issued) tc::mbar_wait(bar(QFULL), 0);
-    for (int st = 0; st < 2; ++st) {
+    for (int st = 0; st < kStages; ++st)
       if (nk_issued[st] > 0) tc::mbar_wait(bar(KFULL + st), (nk_issued[st] - 1) & 1);
-      if (nv_issued[st] > 0) tc::mbar_wait(bar(VFULL + st), (nv_issued[st] - 1) & 1);
-    }
   };
   if (tid == 0 && !a.lpt) issue_first();
 
@@ -291,13 +301,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (tid == 0) TRACE(21);
   if (!seq_ok(a, ctx, N) || row0 >= M) {
     if (tid == 0) {
-      if (!seq_ok(a, ctx, N) && split == 0 && pair == 0 && kvh == 0)
+      if (!seq_ok(a, ctx, N) && split == 0 && tile == 0 && kvh == 0)
         flag_error(a.err, (N < 1 || N > a.n_max) ? LTD_DEVERR_NVERIFY : LTD_DEVERR_CTX);
-      drain();
+      drain_k();
     }
     return;
   }
-  const bool has_b = row0 + kBM < M;
   const int nk = ctx + N;
   const int nch = (nk + kBN - 1) / kBN;
   const int nc = max(0, min(ce, nch) - cs);
@@ -308,56 +317,34 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc::tmem_alloc(tc::smem_u32(holder), kTmemCols);
     tc::tmem_relinquish();
   }
-  // softmax threads (warps 4-11): tile x, TMEM lane lrow, row rr of the unit
+  // softmax threads (warps 4-11): stream x, TMEM lane lrow = row of the tile
   const bool smx = warp >= 4;
   const int x = (warp - 4) >> 2;
   const int lrow = 32 * (warp & 3) + lane;
-  const int rr = kBM * x + lrow;
-  const int R = row0 + rr;
+  const int R = row0 + lrow;
   const bool row_ok = smx && R < M;
-  if (smx) {
-    const int slot = R / a.G;
-    const bool in = slot < a.n_max;
-    for (int w = 0; w < a.W32; ++w)
-      mask_s[rr * kMaxW32 + w] =
-          in ? a.mask[(static_cast<int64_t>(b) * a.n_max + slot) * a.W32 + w] : 0u;
-  }
+  // the row's ancestor-mask words, read where a chunk holds verified keys
+  const uint32_t* mbits =
+      a.mask + (static_cast<int64_t>(b) * a.n_max + min(R / a.G, a.n_max - 1)) * a.W32;
+  if (row_ok && key_hi > ctx)
+    asm volatile("prefetch.global.L1 [%0];" ::"l"(mbits));
   tc::fence_before_sync();
   __syncthreads();
   tc::fence_after_sync();
   const uint32_t tmem = holder[0];
   if (tid == 0) TRACE(1);
   bool ok = true;
-  const bool tile_active = smx && (x == 0 || has_b) && nc > 0;
-  float m = -CUDART_INF_F, l = 0.f;  // the row's running max (log2 units) and sum
+  float m = -CUDART_INF_F, l = 0.f;  // the stream's running max (log2 units) and sum
 
   if (warp == 0) {
-    // ------------------------------------------------------------ producer
+    // ------------------------------------------------------- K producer
     if (lane == 0) {
-#ifdef LTD_TRACE
-      unsigned long long w_empty = 0, t_e = 0;
-#endif
-      if (v0_owed) {
-        issue_v(0);
-        n_issued = 1;
+      for (int j = 1; j < nc && j < kStages; ++j) issue_k(j);
+      for (int j = kStages; j < nc && ok; ++j) {
+        ok = tc::mbar_wait(bar(KEMPTY + j % kStages), ((j / kStages) - 1) & 1);
+        if (ok) issue_k(j);
       }
-      for (int j = n_issued; j < nc && ok; ++j) {
-        const int st = j & 1;
-#ifdef LTD_TRACE
-        t_e = tc::globaltimer();
-#endif
-        ok = tc::mbar_wait(bar(KEMPTY + st), ((j >> 1) - 1) & 1);
-        if (!ok) break;
-        issue_k(j);
-        ok = tc::mbar_wait(bar(VEMPTY + st), ((j >> 1) - 1) & 1);
-        if (!ok) break;
-        issue_v(j);
-#ifdef LTD_TRACE
-        w_empty += tc::globaltimer() - t_e;
-#endif
-      }
-      TRACE_VAL(32, w_empty);
-      drain();
+      drain_k();
       if (!ok) flag_error(a.err, LTD_DEVERR_TIMEOUT);
       if (a.next_k != nullptr && nc > 0) {
         // this CTA's loads have landed: ask L2 for the same rows of the next
@@ -370,137 +357,134 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc::prefetch_l2(a.next_v + off, bytes);
         }
       }
+      TRACE(31);
+    }
+  } else if (warp == 2) {
+    // ------------------------------------------------------- V producer
+    if (lane == 0) {
+      int nv_issued[kStages] = {0, 0, 0};
+      auto issue_v = [&](int j) {
+        const int st = j % kStages;
+        tc::mbar_expect_tx(bar(VFULL + st), kTile);
+        for (int h = 0; h < 2; ++h)
+          tc::tma_load_4d(base + kOffV + st * kTile + h * kHalf, a.kv_one ? &tk : &tv,
+                          bar(VFULL + st), h * 64, (cs + j) * kBN, kvrow, a.kv_wv);
+        ++nv_issued[st];
+      };
+      for (int j = 0; j < nc && j < kStages; ++j) issue_v(j);
+      for (int j = kStages; j < nc && ok; ++j) {
+        ok = tc::mbar_wait(bar(VEMPTY + j % kStages), ((j / kStages) - 1) & 1);
+        if (ok) issue_v(j);
+      }
+      for (int st = 0; st < kStages; ++st)
+        if (nv_issued[st] > 0) tc::mbar_wait(bar(VFULL + st), (nv_issued[st] - 1) & 1);
+      if (!ok) flag_error(a.err, LTD_DEVERR_TIMEOUT);
     }
   } else if (warp == 1) {
     // ----------------------------------------------------------------- MMA
     if (lane == 0 && nc > 0) {
       const uint32_t id_s = tc::idesc_bf16(kBM, kBN, false);
       const uint32_t id_o = tc::idesc_bf16(kBM, kD, true);
-      const int ntile = has_b ? 2 : 1;
       // Every shared-memory descriptor is computed once, so the issue loop
-      // below is MMA instructions only (the thread shares its scheduler with
-      // two softmax warps, and each MMA lasts just 64 cycles).
-      uint64_t dq[2][8], dk[2][8], dv[2][8];
+      // below is MMA instructions and waits only.
+      uint64_t dq[8], dk[kStages][8], dv[kStages][8];
 #pragma unroll
-      for (int u = 0; u < 2; ++u) {
+      for (int ks = 0; ks < 8; ++ks) {
+        dq[ks] = tc::sdesc_sw128(base + kOffQ + (ks >> 2) * kHalf + (ks & 3) * 32, 16, 1024);
 #pragma unroll
-        for (int ks = 0; ks < 8; ++ks) {
-          dq[u][ks] = tc::sdesc_sw128(base + kOffQ + u * kTile + (ks >> 2) * kHalf + (ks & 3) * 32, 16, 1024);
-          dk[u][ks] = tc::sdesc_sw128(base + kOffK + u * kTile + (ks >> 2) * kHalf + (ks & 3) * 32, 16, 1024);
-          dv[u][ks] = tc::sdesc_sw128(base + kOffV + u * kTile + ks * 2048, kHalf, 1024);
+        for (int st = 0; st < kStages; ++st) {
+          dk[st][ks] = tc::sdesc_sw128(base + kOffK + st * kTile + (ks >> 2) * kHalf + (ks & 3) * 32, 16, 1024);
+          dv[st][ks] = tc::sdesc_sw128(base + kOffV + st * kTile + ks * 2048, kHalf, 1024);
         }
       }
-      // (t and st are compile-time constants at every call)
-      auto issue_s = [&](int t, int st) {
+      // (x and st are compile-time constants at every call)
+      auto issue_s = [&](int x_, int st) {
 #pragma unroll
         for (int ks = 0; ks < 8; ++ks)
-          tc::mma_bf16(tmem + t * kBN, dq[t][ks], dk[st][ks], id_s, ks > 0 ? 1u : 0u);
+          tc::mma_bf16(tmem + x_ * kBN, dq[ks], dk[st][ks], id_s, ks > 0 ? 1u : 0u);
       };
-      auto issue_pv = [&](int t, int st, uint32_t acc) {
+      auto issue_pv = [&](int x_, int st, uint32_t acc) {
 #pragma unroll
         for (int ks = 0; ks < 8; ++ks)
-          tc::mma_bf16_ts(tmem + 2 * kBN + t * kD, tmem + t * kBN + 8 * ks, dv[st][ks], id_o,
+          tc::mma_bf16_ts(tmem + 2 * kBN + x_ * kD, tmem + x_ * kBN + 8 * ks, dv[st][ks], id_o,
                           ks > 0 ? 1u : acc);
       };
-#ifdef LTD_TRACE
-      unsigned long long w_load = 0, w_p = 0, t_w;
-#define TW_BEGIN() t_w = tc::globaltimer()
-#define TW_END(acc) acc += tc::globaltimer() - t_w
-#else
-#define TW_BEGIN() \
-  do {             \
-  } while (0)
-#define TW_END(acc) \
-  do {              \
-  } while (0)
-#endif
       ok = tc::mbar_wait(bar(QFULL), 0);
       TRACE(2);
+      // S(0) and S(1) into S_0 and S_1
       if (ok) ok = tc::mbar_wait(bar(KFULL + 0), 0);
-      TRACE(3);
       if (ok) {
         tc::fence_after_sync();
         issue_s(0, 0);
         tc::mma_commit(bar(SFULL + 0));
-        if (ntile > 1) {
-          issue_s(1, 0);
-          tc::mma_commit(bar(SFULL + 1));
-        }
         tc::mma_commit(bar(KEMPTY + 0));
       }
-      // chunk j in stage st = j & 1: PV_x(j) and S_x(j+1) per tile
-      auto step = [&](int j, int st) -> bool {
-        const bool nxt = j + 1 < nc;
-        TW_BEGIN();
-        bool k = tc::mbar_wait(bar(VFULL + st), (j >> 1) & 1);
-        if (k && nxt) k = tc::mbar_wait(bar(KFULL + (st ^ 1)), ((j + 1) >> 1) & 1);
-        TW_END(w_load);
-        const uint32_t acc = j > 0 ? 1u : 0u;
-#pragma unroll
-        for (int t = 0; t < 2; ++t) {
-          if (!k || t >= ntile) break;
-          TW_BEGIN();
-          k = tc::mbar_wait(bar(PFULL + t), j & 1);
-          TW_END(w_p);
-          if (!k) break;
+      TRACE(3);
+      if (ok && nc > 1) {
+        ok = tc::mbar_wait(bar(KFULL + 1), 0);
+        if (ok) {
           tc::fence_after_sync();
-          issue_pv(t, st, acc);
-          if (nxt) {
-            issue_s(t, st ^ 1);
-            tc::mma_commit(bar(SFULL + t));
-          }
+          issue_s(1, 1);
+          tc::mma_commit(bar(SFULL + 1));
+          tc::mma_commit(bar(KEMPTY + 1));
         }
+      }
+      // chunk j = 6 i + r: stream r & 1, stage r % 3, ring use j / 3 (its
+      // parity is (r / 3) & 1); PV(j) then S(j + 2) into the same stream
+      auto step = [&](int j, auto R_) -> bool {
+        constexpr int r = decltype(R_)::value;
+        constexpr int xs = r & 1, st = r % kStages, st2 = (r + 2) % kStages;
+        bool k = tc::mbar_wait(bar(VFULL + st), (r / kStages) & 1);
+        if (k) k = tc::mbar_wait(bar(PFULL + xs), (j >> 1) & 1);
         if (!k) return false;
-        if (nxt) tc::mma_commit(bar(KEMPTY + (st ^ 1)));
+        tc::fence_after_sync();
+        issue_pv(xs, st, j >= 2 ? 1u : 0u);
         tc::mma_commit(bar(VEMPTY + st));
+        if (j + 2 < nc) {
+          if (!tc::mbar_wait(bar(KFULL + st2), ((r + 2) / kStages) & 1)) return false;
+          tc::fence_after_sync();
+          issue_s(xs, st2);
+          tc::mma_commit(bar(SFULL + xs));
+          tc::mma_commit(bar(KEMPTY + st2));
+        }
         return true;
       };
-      for (int j = 0; j < nc && ok; j += 2) {
-        ok = step(j, 0);
-        if (ok && j + 1 < nc) ok = step(j + 1, 1);
+      for (int j = 0; j < nc && ok; j += 6) {
+        ok = step(j, Int<0>{});
+        if (ok && j + 1 < nc) ok = step(j + 1, Int<1>{});
+        if (ok && j + 2 < nc) ok = step(j + 2, Int<2>{});
+        if (ok && j + 3 < nc) ok = step(j + 3, Int<3>{});
+        if (ok && j + 4 < nc) ok = step(j + 4, Int<4>{});
+        if (ok && j + 5 < nc) ok = step(j + 5, Int<5>{});
       }
-      TRACE_VAL(22, w_load);
-      TRACE_VAL(24, w_p);
-      TRACE_VAL(29, static_cast<unsigned long long>(nc));
-      TRACE(31);
-#undef TW_BEGIN
-#undef TW_END
+      TRACE(22);
       // every MMA of this CTA completes before tensor memory is read or freed
       tc::mma_commit(bar(FIN));
       tc::mbar_wait(bar(FIN), 0);
       if (!ok) flag_error(a.err, LTD_DEVERR_TIMEOUT);
+      TRACE(23);
     }
-  } else if (tile_active) {
+  } else if (smx && x < nc) {
     // ------------------------------------------------------------- softmax
     const uint32_t lane_off = (32u * (warp & 3)) << 16;
     const uint32_t t_s = tmem + x * kBN + lane_off;
     const uint32_t t_o = tmem + 2 * kBN + x * kD + lane_off;
-    const uint32_t* mbits = mask_s + rr * kMaxW32;
     const int vis_all_below = min(ctx, key_hi);  // keys below this are all visible
     const float sl2 = a.scale_log2;
     const int w32 = a.W32;
     const bool tr = (tid & 127) == 0;
-#ifdef LTD_TRACE
-    unsigned long long w_s = 0, t_s0 = 0;
-#endif
-    for (int j = 0; j < nc; ++j) {
-#ifdef LTD_TRACE
-      t_s0 = tc::globaltimer();
-#endif
-      ok = tc::mbar_wait(bar(SFULL + x), j & 1);
-#ifdef LTD_TRACE
-      w_s += tc::globaltimer() - t_s0;
-#endif
+    for (int j = x; j < nc; j += 2) {
+      ok = tc::mbar_wait(bar(SFULL + x), (j >> 1) & 1);
       ok = __all_sync(0xFFFFFFFFu, ok);
-      if (tr && j < 2) TRACE(4 + 4 * x + 2 * j);
+      if (tr && j < 4) TRACE(4 + 2 * j);
       if (!ok) break;
       tc::fence_after_sync();
       const int kbase = key_lo + j * kBN;
       const bool all_vis = row_ok && kbase + kBN <= vis_all_below;
-      // P against the row's running max m (a row without one yet first takes
-      // this chunk's max); the chunk's own max is tracked on the way and, if
-      // it exceeds the reference by more than 2^8 in some row of the warp,
-      // the warp re-derives P from S, still intact in tensor memory, 32
+      // P against the stream's running max m (a row without one yet first
+      // takes this chunk's max); the chunk's own max is tracked on the way
+      // and, if it exceeds the reference by more than 2^8 in some row of the
+      // warp, the warp re-derives P from S, still intact in tensor memory, 32
       // columns at a time.
       tc::Frag128 f;
       float mref = m;
@@ -513,7 +497,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       __syncwarp();  // the load below is warp-collective; the branch above is per row
       tc::tmem_ld128_sync(t_s, f);
-      if (tr && j == 0 && x == 0) TRACE(27);
       if (!all_vis) {
 #pragma unroll
         for (int c = 0; c < 128; ++c)
@@ -591,8 +574,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc::tmem_st16_sync(t_s + 16 * qq, pf);
         }
       }
-      if (tr && j == 0 && x == 0) TRACE(28);
-      // S(j) complete implies P_x(j-1) V finished, so O_x is stable here
+      // S(j) was issued after PV(j - 2) of this stream, so O_x is stable here
       const bool need = (mref != m) && (m != -CUDART_INF_F);
       const float alpha = need ? tc::ex2(m - mref) : 1.f;
       if (__any_sync(0xFFFFFFFFu, need)) {
@@ -607,13 +589,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       m = mref;
       l = l * alpha + (ls2.x + ls2.y);
-      if (x == 0 && kbase + kBN > key_hi) {
+      if (kbase + kBN > key_hi) {
         // Keys from key_hi on may hold anything in the cache, even NaN: P is
-        // 0 there, but 0 * NaN is not, so tile a's threads clear those V rows
-        // (both 64-dim halves) before either tile's PV reads this stage.
-        const int st = j & 1;
+        // 0 there, but 0 * NaN is not, so this stream's threads clear those V
+        // rows (both 64-dim halves) before PV reads this stage.
+        const int st = j % kStages;
         // (a failed wait is flagged; the MMA thread times out on the same stage)
-        if (!__all_sync(0xFFFFFFFFu, tc::mbar_wait(bar(VFULL + st), (j >> 1) & 1)) && lane == 0)
+        if (!__all_sync(0xFFFFFFFFu, tc::mbar_wait(bar(VFULL + st), (j / kStages) & 1)) && lane == 0)
           flag_error(a.err, LTD_DEVERR_TIMEOUT);
         const int z0 = key_hi - kbase;  // 1 .. 127
         uint4* vs = reinterpret_cast<uint4*>(gbase + kOffV + st * kTile);
@@ -625,64 +607,74 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       __syncwarp();  // the zeroing loop above runs per thread; the wait is warp-collective
       tc::tmem_wait_st();
-      if (tr && j == 0 && x == 0) TRACE(30);
       tc::fence_before_sync();
       tc::mbar_arrive(bar(PFULL + x));
-      if (tr && j < 2) TRACE(5 + 4 * x + 2 * j);
+      if (tr && j < 4) TRACE(5 + 2 * j);
     }
-    if (ok) {
-      ok = tc::mbar_wait(bar(FIN), 0);
-      ok = __all_sync(0xFFFFFFFFu, ok);
-    }
-    if (tr) TRACE(12 + x);
-    if (tr) TRACE_VAL(33 + x, w_s);
     if (!ok && lane == 0) flag_error(a.err, LTD_DEVERR_TIMEOUT);
+    if (tr) TRACE(12 + x);
   }
 
   // --------------------------------------------------------- epilogue
-  // O / l of every row (bf16; zero where a row has nothing) and its
-  // log2-sum-exp are staged in shared memory over Q and over the mask (both
-  // free once the last MMA has completed): row r's 16-byte chunk c sits at
-  // ((c ^ (r & 15)) << 4), so the row-per-thread stores of a warp spread
-  // over the banks.  One split: all threads copy the rows to the output,
-  // coalesced.  Several: the partial layout below.
-  const int unit = (b * a.hkv + kvh) * a.n_pairs + pair;
-  const int Mv = min(kRows, M - row0);
-  // the producer has drained every load (Q included) and the MMAs are done
-  // before the staging below overwrites Q
+  // The producers have drained every load and the MMA thread has seen the
+  // last MMA complete before this barrier; after it, the K ring holds the
+  // two streams' (m, l), and Q's region the staged rows.
   tc::fence_before_sync();
   __syncthreads();
+  tc::fence_after_sync();
+  if (tid == 0) TRACE(14);
+  float2* ml = reinterpret_cast<float2*>(gbase + kOffML);
+  if (smx) ml[x * kBM + lrow] = make_float2(m, l);
+  __syncthreads();
+  const int unit = (b * a.hkv + kvh) * a.n_tiles + tile;
+  const int Mv = min(kBM, M - row0);
   uint8_t* stg = gbase + kOffQ;
-  float* stg_l = reinterpret_cast<float*>(gbase + kOffMask);
-  // tcgen05.ld is warp-collective: the O load is taken by whole warps
-  // (tile_active and ok are uniform within a warp), the writes per row.
-  const bool loaded = tile_active && ok;
-  tc::Frag128 o;
-  if (loaded) {
-    tc::fence_after_sync();
-    tc::tmem_ld128_sync(tmem + 2 * kBN + x * kD + ((32u * (warp & 3)) << 16), o);
-  }
-  if (row_ok) {
-    const bool have = loaded && l > 0.f;
-    const float inv = have ? 1.f / l : 0.f;
-    uint8_t* srow = stg + rr * kRowBytes;
+  float* stg_l = reinterpret_cast<float*>(gbase + kOffStgL);
+  // Merge the two streams: stream x's thread of a row writes columns
+  // 64 x .. 64 x + 63 of O / l.  tcgen05.ld is warp-collective: the loads
+  // are taken by whole warps (nc and ok are uniform in a warp), the writes
+  // per row.
+  if (smx) {
+    const float2 me = ml[lrow], mo = ml[kBM + lrow];
+    const float mm = fmaxf(me.x, mo.x);
+    const float a0 = mm == -CUDART_INF_F ? 0.f : tc::ex2(me.x - mm);
+    const float a1 = mm == -CUDART_INF_F ? 0.f : tc::ex2(mo.x - mm);
+    const float L = me.y * a0 + mo.y * a1;
+    const bool have = L > 0.f;
+    const float inv = have ? 1.f / L : 0.f;
+    const float w0 = a0 * inv, w1 = a1 * inv;
+    const uint32_t lane_off = (32u * (warp & 3)) << 16;
+    const bool ld0 = nc > 0, ld1 = nc > 1;
+    tc::Frag64 o0, o1;
+    if (ld0) tc::tmem_ld64_sync(tmem + 2 * kBN + 0 * kD + 64 * x + lane_off, o0);
+    if (ld1) tc::tmem_ld64_sync(tmem + 2 * kBN + 1 * kD + 64 * x + lane_off, o1);
+    if (row_ok) {
+      uint8_t* srow = stg + lrow * kRowBytes;
 #pragma unroll
-    for (int c = 0; c < 16; ++c) {
-      uint4 w = make_uint4(0u, 0u, 0u, 0u);
-      if (have) {
-        w.x = pack_bf16(__uint_as_float(o.r[8 * c]) * inv, __uint_as_float(o.r[8 * c + 1]) * inv);
-        w.y = pack_bf16(__uint_as_float(o.r[8 * c + 2]) * inv, __uint_as_float(o.r[8 * c + 3]) * inv);
-        w.z = pack_bf16(__uint_as_float(o.r[8 * c + 4]) * inv, __uint_as_float(o.r[8 * c + 5]) * inv);
-        w.w = pack_bf16(__uint_as_float(o.r[8 * c + 6]) * inv, __uint_as_float(o.r[8 * c + 7]) * inv);
+      for (int c = 0; c < 8; ++c) {
+        float v[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          float s = 0.f;
+          if (have && ld0) s = __uint_as_float(o0.r[8 * c + e]) * w0;
+          if (have && ld1) s = fmaf(__uint_as_float(o1.r[8 * c + e]), w1, s);
+          v[e] = s;
+        }
+        uint4 w;
+        w.x = pack_bf16(v[0], v[1]);
+        w.y = pack_bf16(v[2], v[3]);
+        w.z = pack_bf16(v[4], v[5]);
+        w.w = pack_bf16(v[6], v[7]);
+        const int cc = 8 * x + c;
+        *reinterpret_cast<uint4*>(srow + ((cc ^ (lrow & 15)) << 4)) = w;
       }
-      *reinterpret_cast<uint4*>(srow + ((c ^ (rr & 15)) << 4)) = w;
+      if (x == 0) stg_l[lrow] = have ? mm + __log2f(L) : -CUDART_INF_F;
     }
-    stg_l[rr] = have ? m + __log2f(l) : -CUDART_INF_F;
   }
   tc::fence_smem_async();  // the staging is read by bulk copies
   tc::fence_before_sync();
   __syncthreads();
-  if (tid == 0) TRACE(14);
+  if (tid == 0) TRACE(15);
   if (warp == 1) {
     __syncwarp();
     tc::fence_after_sync();
@@ -702,15 +694,14 @@ __global__ void __launch_bounds__(kThreads, 1)
   // ------------------------------------- combine the splits (S > 1 only)
   // Each split stores its staged rows and sums with one bulk copy each
   // (split-major: [unit][split][row]); rows [o rs, o rs + rs) of a unit are
-  // combined by its split o ("owner"), which pulls that block of every
-  // split with one bulk copy per split.
-  const int Rs = a.rs;
+  // combined by its split o, every thread loading one 16-byte chunk of one
+  // row from every split straight into registers.
   uint32_t* arrive = a.sync + 2 * unit;
   uint32_t* depart = arrive + 1;
   if (tid == 0) {
     const int64_t pb = static_cast<int64_t>(unit) * S + split;
-    tc::bulk_s2g(a.part_o + pb * kRows * kRowBytes, base + kOffQ, Mv * kRowBytes);
-    tc::bulk_s2g(a.part_l + pb * kRows, base + kOffMask, ((Mv + 3) & ~3) * 4);
+    tc::bulk_s2g(a.part_o + pb * kBM * kRowBytes, base + kOffQ, Mv * kRowBytes);
+    tc::bulk_s2g(a.part_l + pb * kBM, base + kOffStgL, ((Mv + 3) & ~3) * 4);
     tc::bulk_commit();
     tc::bulk_wait_all();
     tc::fence_proxy_async_global();
@@ -726,78 +717,67 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     if (!got) flag_error(a.err, LTD_DEVERR_TIMEOUT);
     holder[1] = got ? 1u : 0u;
-    TRACE(15);
+    TRACE(16);
   }
   __syncthreads();
+  const int Rs = a.rs;
   const int r_lo = split * Rs;
   const int nrows = max(0, min(Mv, r_lo + Rs) - r_lo);
-  if (holder[1] != 0u && nrows > 0) {
-    if (tid == 0) {
-      // the acquire above orders the other splits' stores before these reads
-      tc::fence_proxy_async_global();
-      const int nl = min(Rs, kRows - r_lo);  // a multiple of 4
-      tc::mbar_expect_tx(bar(CBAR), static_cast<uint32_t>(S) * (nrows * kRowBytes + nl * 4));
-      for (int p = 0; p < S; ++p) {
-        const int64_t pb = static_cast<int64_t>(unit) * S + p;
-        tc::bulk_g2s(base + kOffK + p * Rs * kRowBytes, a.part_o + (pb * kRows + r_lo) * kRowBytes,
-                     nrows * kRowBytes, bar(CBAR));
-        tc::bulk_g2s(base + kOffMask + p * Rs * 4, a.part_l + pb * kRows + r_lo, nl * 4, bar(CBAR));
-      }
-    }
-    // CTA-uniform, as a barrier follows under it
-    const bool in = __syncthreads_and(tc::mbar_wait(bar(CBAR), 0)) != 0;
-    if (tid == 0) TRACE(18);
-    if (!in) {
-      if (tid == 0) flag_error(a.err, LTD_DEVERR_TIMEOUT);
-    } else {
-      const uint8_t* cin = gbase + kOffK;
-      const float* lin = reinterpret_cast<const float*>(gbase + kOffMask);
-      // A thread per (row, 16-byte chunk): the splits' log2-sum-exps give
-      // the row's max, then each split's weight 2^(lse_p - max) and its chunk
-      // are fetched with independent shared loads (four splits in flight)
-      // and accumulated; every split wrote every row below Mv (zeros where
-      // it had no keys).
-      for (int idx = tid; idx < nrows * 16; idx += kThreads) {
-        const int r = idx >> 4, c = idx & 15;
-        const float* lr = lin + r;
-        float mx = -CUDART_INF_F;
-#pragma unroll 4
-        for (int p = 0; p < S; ++p) mx = fmaxf(mx, lr[p * Rs]);
-        float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-        float L = 0.f;
-        if (mx > -CUDART_INF_F) {
-          // rows keep the staging's chunk swizzle (by row within the unit)
-          const uint8_t* cr = cin + r * kRowBytes + ((c ^ ((r_lo + r) & 15)) << 4);
-#pragma unroll 4
-          for (int p = 0; p < S; ++p) {
-            const float w = tc::ex2(lr[p * Rs] - mx);  // 0 for a split without keys
-            const uint4 v = *reinterpret_cast<const uint4*>(cr + p * Rs * kRowBytes);
-            L += w;
-            const uint32_t e[4] = {v.x, v.y, v.z, v.w};
+  // the acquire above (ordered by the barrier) makes the other splits'
+  // stores visible; .cg loads read them from L2
+  for (int idx = tid; holder[1] != 0u && idx < nrows * 16; idx += kThreads) {
+    const int r = r_lo + (idx >> 4), c = idx & 15;
+    const int64_t ub = static_cast<int64_t>(unit) * S;
+    const uint8_t* src = a.part_o + (ub * kBM + r) * kRowBytes + ((c ^ (r & 15)) << 4);
+    const float* lsrc = a.part_l + ub * kBM + r;
+    float mx = -CUDART_INF_F, L = 0.f;
+    float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    for (int p0 = 0; p0 < S; p0 += kCombineBatch) {
+      uint4 v[kCombineBatch];
+      float ls[kCombineBatch];
 #pragma unroll
-            for (int t = 0; t < 4; ++t) {
-              acc[2 * t] = fmaf(w, __uint_as_float(e[t] << 16), acc[2 * t]);
-              acc[2 * t + 1] = fmaf(w, __uint_as_float(e[t] & 0xFFFF0000u), acc[2 * t + 1]);
-            }
+      for (int u = 0; u < kCombineBatch; ++u) {
+        const int p = p0 + u;
+        ls[u] = p < S ? ld_cg_f32(lsrc + static_cast<int64_t>(p) * kBM) : -CUDART_INF_F;
+        v[u] = p < S ? ld_cg_v4(src + static_cast<int64_t>(p) * kBM * kRowBytes)
+                     : make_uint4(0u, 0u, 0u, 0u);
+      }
+      float bm = mx;
+#pragma unroll
+      for (int u = 0; u < kCombineBatch; ++u) bm = fmaxf(bm, ls[u]);
+      if (bm > -CUDART_INF_F) {
+        const float sc = tc::ex2(mx - bm);  // 0 while mx is -inf
+        L *= sc;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc[e] *= sc;
+#pragma unroll
+        for (int u = 0; u < kCombineBatch; ++u) {
+          const float w = tc::ex2(ls[u] - bm);  // 0 for a split without keys
+          L += w;
+          const uint32_t ev[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
+#pragma unroll
+          for (int t = 0; t < 4; ++t) {
+            acc[2 * t] = fmaf(w, __uint_as_float(ev[t] << 16), acc[2 * t]);
+            acc[2 * t + 1] = fmaf(w, __uint_as_float(ev[t] & 0xFFFF0000u), acc[2 * t + 1]);
           }
         }
-        const float inv = L > 0.f ? 1.f / L : 0.f;
-        const int Rr = row0 + r_lo + r;
-        const int slot = Rr / a.G, g = Rr % a.G;
-        uint4 w;
-        w.x = pack_bf16(acc[0] * inv, acc[1] * inv);
-        w.y = pack_bf16(acc[2] * inv, acc[3] * inv);
-        w.z = pack_bf16(acc[4] * inv, acc[5] * inv);
-        w.w = pack_bf16(acc[6] * inv, acc[7] * inv);
-        reinterpret_cast<uint4*>(a.out + ((static_cast<int64_t>(b) * a.n_max + slot) * a.hq +
-                                          kvh * a.G + g) * kD)[c] = w;
+        mx = bm;
       }
-      if (tid == 0) TRACE(23);
     }
+    const float inv = L > 0.f ? 1.f / L : 0.f;
+    const int Rr = row0 + r;
+    const int slot = Rr / a.G, g = Rr % a.G;
+    uint4 w;
+    w.x = pack_bf16(acc[0] * inv, acc[1] * inv);
+    w.y = pack_bf16(acc[2] * inv, acc[3] * inv);
+    w.z = pack_bf16(acc[4] * inv, acc[5] * inv);
+    w.w = pack_bf16(acc[6] * inv, acc[7] * inv);
+    reinterpret_cast<uint4*>(a.out + ((static_cast<int64_t>(b) * a.n_max + slot) * a.hq +
+                                      kvh * a.G + g) * kD)[c] = w;
   }
   __syncthreads();
   if (tid == 0) {
-    TRACE(16);
+    TRACE(18);
     // every split of this unit has passed its spin once all have departed
     const uint32_t d = atomicAdd(depart, 1u);
     if (d == static_cast<uint32_t>(S) - 1u) {
@@ -808,7 +788,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 struct Plan {
-  int n_pairs, splits, units, lpt, nch, rs;
+  int n_tiles, splits, units, lpt, nch, rs;
 };
 
 // Streaming multiprocessors of the current device (152 if it cannot be asked).
@@ -832,14 +812,14 @@ int device_sms() {
   return known[dev];
 }
 
-// Units = (sequence, KV head, tile pair).  With fewer units than SMs each
-// unit's keys are cut into the fewest splits that give the shortest longest
-// split, at most SMs / units of them, so all CTAs fit one wave.
+// Units = (sequence, KV head, tile).  With fewer units than SMs each unit's
+// keys are cut into the fewest splits that give the shortest longest split,
+// at most SMs / units of them, so all CTAs fit one wave.
 Plan plan(int32_t batch, int32_t hq, int32_t hkv, int32_t n_max, int32_t max_ctx) {
   const int G = hq / hkv;
   Plan p{};
-  p.n_pairs = (n_max * G + kRows - 1) / kRows;
-  const int64_t units = static_cast<int64_t>(batch) * hkv * p.n_pairs;
+  p.n_tiles = (n_max * G + kBM - 1) / kBM;
+  const int64_t units = static_cast<int64_t>(batch) * hkv * p.n_tiles;
   p.units = static_cast<int>(units);
   const int nch = (max_ctx + n_max + kBN - 1) / kBN;
   const int sms = device_sms();
@@ -853,9 +833,9 @@ Plan plan(int32_t batch, int32_t hq, int32_t hkv, int32_t n_max, int32_t max_ctx
       p.splits = (nch + maxc - 1) / maxc;
     }
   }
-  p.lpt = (p.splits == 1 && static_cast<int64_t>(batch) * p.n_pairs <= kMaxGroups) ? 1 : 0;
+  p.lpt = (p.splits == 1 && static_cast<int64_t>(batch) * p.n_tiles <= kMaxGroups) ? 1 : 0;
   p.nch = nch;
-  p.rs = (((kRows + p.splits - 1) / p.splits) + 3) & ~3;
+  p.rs = (kBM + p.splits - 1) / p.splits;
   return p;
 }
 
@@ -867,8 +847,8 @@ struct WsLayout {
 WsLayout ws_layout(const Plan& pl) {
   WsLayout w{};
   if (pl.splits <= 1) return w;
-  // [unit][split][256] rows
-  const size_t rows = static_cast<size_t>(pl.units) * pl.splits * kRows;
+  // [unit][split][128] rows
+  const size_t rows = static_cast<size_t>(pl.units) * pl.splits * kBM;
   w.part_o = 0;
   w.part_l = align256(rows * kRowBytes);
   w.sync = w.part_l + align256(rows * sizeof(float));
@@ -955,7 +935,7 @@ cudaError_t launch_attn_tc(const AttnParams& p, cudaStream_t s) {
   a.max_ctx = p.max_ctx;
   a.W32 = (p.n_max + 31) / 32;
   a.splits = pl.splits;
-  a.n_pairs = pl.n_pairs;
+  a.n_tiles = pl.n_tiles;
   a.lpt = pl.lpt;
   a.nch_h = pl.nch;
   a.rs = pl.rs;
@@ -1010,7 +990,7 @@ cudaError_t launch_attn_tc(const AttnParams& p, cudaStream_t s) {
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeCooperative;
     attr[0].val.cooperative = 1;
-    return launch(attn_tc_kernel, dim3(pl.splits, pl.n_pairs, p.batch * p.hkv), dim3(kThreads),
+    return launch(attn_tc_kernel, dim3(pl.splits, pl.n_tiles, p.batch * p.hkv), dim3(kThreads),
                   kSmemBytes, s, attr, 1, tq, tk, tv, a);
   }
   return launch(attn_tc_kernel, dim3(pl.units), dim3(kThreads), kSmemBytes, s, nullptr, 0, tq, tk, tv,

@@ -221,6 +221,14 @@ __device__ __forceinline__ void tmem_wait_ld64(Frag64& f) {
   asm volatile("tcgen05.wait::ld.sync.aligned;"
                : "+r"(f.r[0]), "+r"(f.r[1]), "+r"(f.r[2]), "+r"(f.r[3]), "+r"(f.r[4]), "+r"(f.r[5]), "+r"(f.r[6]), "+r"(f.r[7]), "+r"(f.r[8]), "+r"(f.r[9]), "+r"(f.r[10]), "+r"(f.r[11]), "+r"(f.r[12]), "+r"(f.r[13]), "+r"(f.r[14]), "+r"(f.r[15]), "+r"(f.r[16]), "+r"(f.r[17]), "+r"(f.r[18]), "+r"(f.r[19]), "+r"(f.r[20]), "+r"(f.r[21]), "+r"(f.r[22]), "+r"(f.r[23]), "+r"(f.r[24]), "+r"(f.r[25]), "+r"(f.r[26]), "+r"(f.r[27]), "+r"(f.r[28]), "+r"(f.r[29]), "+r"(f.r[30]), "+r"(f.r[31]), "+r"(f.r[32]), "+r"(f.r[33]), "+r"(f.r[34]), "+r"(f.r[35]), "+r"(f.r[36]), "+r"(f.r[37]), "+r"(f.r[38]), "+r"(f.r[39]), "+r"(f.r[40]), "+r"(f.r[41]), "+r"(f.r[42]), "+r"(f.r[43]), "+r"(f.r[44]), "+r"(f.r[45]), "+r"(f.r[46]), "+r"(f.r[47]), "+r"(f.r[48]), "+r"(f.r[49]), "+r"(f.r[50]), "+r"(f.r[51]), "+r"(f.r[52]), "+r"(f.r[53]), "+r"(f.r[54]), "+r"(f.r[55]), "+r"(f.r[56]), "+r"(f.r[57]), "+r"(f.r[58]), "+r"(f.r[59]), "+r"(f.r[60]), "+r"(f.r[61]), "+r"(f.r[62]), "+r"(f.r[63]));
 }
+// 64 columns, load and wait in one statement (see tmem_ld32_sync).
+__device__ __forceinline__ void tmem_ld64_sync(uint32_t taddr, Frag64& f) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x64.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32, %33, %34, %35, %36, %37, %38, %39, %40, %41, %42, %43, %44, %45, %46, %47, %48, %49, %50, %51, %52, %53, %54, %55, %56, %57, %58, %59, %60, %61, %62, %63}, [%64];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(f.r[0]), "=r"(f.r[1]), "=r"(f.r[2]), "=r"(f.r[3]), "=r"(f.r[4]), "=r"(f.r[5]), "=r"(f.r[6]), "=r"(f.r[7]), "=r"(f.r[8]), "=r"(f.r[9]), "=r"(f.r[10]), "=r"(f.r[11]), "=r"(f.r[12]), "=r"(f.r[13]), "=r"(f.r[14]), "=r"(f.r[15]), "=r"(f.r[16]), "=r"(f.r[17]), "=r"(f.r[18]), "=r"(f.r[19]), "=r"(f.r[20]), "=r"(f.r[21]), "=r"(f.r[22]), "=r"(f.r[23]), "=r"(f.r[24]), "=r"(f.r[25]), "=r"(f.r[26]), "=r"(f.r[27]), "=r"(f.r[28]), "=r"(f.r[29]), "=r"(f.r[30]), "=r"(f.r[31]), "=r"(f.r[32]), "=r"(f.r[33]), "=r"(f.r[34]), "=r"(f.r[35]), "=r"(f.r[36]), "=r"(f.r[37]), "=r"(f.r[38]), "=r"(f.r[39]), "=r"(f.r[40]), "=r"(f.r[41]), "=r"(f.r[42]), "=r"(f.r[43]), "=r"(f.r[44]), "=r"(f.r[45]), "=r"(f.r[46]), "=r"(f.r[47]), "=r"(f.r[48]), "=r"(f.r[49]), "=r"(f.r[50]), "=r"(f.r[51]), "=r"(f.r[52]), "=r"(f.r[53]), "=r"(f.r[54]), "=r"(f.r[55]), "=r"(f.r[56]), "=r"(f.r[57]), "=r"(f.r[58]), "=r"(f.r[59]), "=r"(f.r[60]), "=r"(f.r[61]), "=r"(f.r[62]), "=r"(f.r[63])
+      : "r"(taddr));
+}
 __device__ __forceinline__ void tmem_st64(uint32_t taddr, const Frag64& f) {
   asm volatile("tcgen05.st.sync.aligned.32x32b.x64.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32, %33, %34, %35, %36, %37, %38, %39, %40, %41, %42, %43, %44, %45, %46, %47, %48, %49, %50, %51, %52, %53, %54, %55, %56, %57, %58, %59, %60, %61, %62, %63, %64};"
                ::"r"(taddr), "r"(f.r[0]), "r"(f.r[1]), "r"(f.r[2]), "r"(f.r[3]), "r"(f.r[4]), "r"(f.r[5]), "r"(f.r[6]), "r"(f.r[7]), "r"(f.r[8]), "r"(f.r[9]), "r"(f.r[10]), "r"(f.r[11]), "r"(f.r[12]), "r"(f.r[13]), "r"(f.r[14]), "r"(f.r[15]), "r"(f.r[16]), "r"(f.r[17]), "r"(f.r[18]), "r"(f.r[19]), "r"(f.r[20]), "r"(f.r[21]), "r"(f.r[22]), "r"(f.r[23]), "r"(f.r[24]), "r"(f.r[25]), "r"(f.r[26]), "r"(f.r[27]), "r"(f.r[28]), "r"(f.r[29]), "r"(f.r[30]), "r"(f.r[31]), "r"(f.r[32]), "r"(f.r[33]), "r"(f.r[34]), "r"(f.r[35]), "r"(f.r[36]), "r"(f.r[37]), "r"(f.r[38]), "r"(f.r[39]), "r"(f.r[40]), "r"(f.r[41]), "r"(f.r[42]), "r"(f.r[43]), "r"(f.r[44]), "r"(f.r[45]), "r"(f.r[46]), "r"(f.r[47]), "r"(f.r[48]), "r"(f.r[49]), "r"(f.r[50]), "r"(f.r[51]), "r"(f.r[52]), "r"(f.r[53]), "r"(f.r[54]), "r"(f.r[55]), "r"(f.r[56]), "r"(f.r[57]), "r"(f.r[58]), "r"(f.r[59]), "r"(f.r[60]), "r"(f.r[61]), "r"(f.r[62]), "r"(f.r[63])

@@ -467,7 +467,13 @@ def test_compaction_race_pattern_and_untouched_rows():
 
 # ---------------------------------------------------------------------- attention
 def _attention_case(name, seed, heads=None, seqs=None, poison=False, workspace=None,
-                    bad_seq=None, key_ramp=None, **overrides):
+                    bad_seq=None, key_ramp=None, mask_mutant=None, check=True, **overrides):
+    """One attention layer through the C ABI against the oracle.  Returns the
+    worst max-abs and mean-abs errors over the compared heads and the max-abs
+    error relative to the largest reference output.  ``mask_mutant``
+    ("transpose" or "drop") feeds the kernel a corrupted copy of the mask
+    words while the oracle keeps the true mask (``check=False`` then returns
+    the errors without asserting the tolerance)."""
     cfg = wl.config(name, **overrides)
     ci = wl.draw_cycle(cfg, seed, draft_rows=False)
     rng = np.random.default_rng(seed + 5)
@@ -492,7 +498,15 @@ def _attention_case(name, seed, heads=None, seqs=None, poison=False, workspace=N
     W32 = (cfg.max_n + 31) // 32
     mw = np.zeros((cfg.batch, cfg.max_n, W32), np.uint32)
     for b in range(cfg.batch):
-        w = oracle.mask_words(masks[b])
+        m = masks[b]
+        if mask_mutant == "transpose":
+            m = m.T.copy()
+        elif mask_mutant == "drop":
+            m = m.copy()
+            m[-1, 0] = False  # the deepest slot no longer sees the root
+        elif mask_mutant is not None:
+            raise ValueError(mask_mutant)
+        w = oracle.mask_words(m)
         mw[b, :w.shape[0], :w.shape[1]] = w
     qd, kd, vd = H.dev(q, cfg.dtype), H.dev(k, cfg.dtype), H.dev(v, cfg.dtype)
     if poison:
@@ -516,7 +530,7 @@ def _attention_case(name, seed, heads=None, seqs=None, poison=False, workspace=N
     got = out.float().cpu().numpy()
     G = cfg.hq // cfg.hkv
     scale = 1.0 / math.sqrt(cfg.head_dim)
-    worst_max, worst_mean = 0.0, 0.0
+    worst_max, worst_mean, ref_max = 0.0, 0.0, 0.0
     for b in (seqs if seqs is not None else range(cfg.batch)):
         N, c = int(ci.n_verify[b]), int(ci.ctx[b])
         for kvh in (heads if heads is not None else range(cfg.hkv)):
@@ -525,11 +539,14 @@ def _attention_case(name, seed, heads=None, seqs=None, poison=False, workspace=N
                                         masks[b], scale)
             mx, mn = H.attention_error(got[b, :N][:, hs], ref)
             worst_max, worst_mean = max(worst_max, mx), max(worst_mean, mn)
+            ref_max = max(ref_max, float(np.abs(ref).max()))
         # rows past N are untouched (zeros from torch.zeros_like)
         assert not got[b, N:].any()
-    tol_max, tol_mean = H.ATT_TOL[cfg.dtype]
-    assert worst_max <= tol_max and worst_mean <= tol_mean, (worst_max, worst_mean)
-    return worst_max, worst_mean
+    rel = worst_max / ref_max if ref_max > 0 else 0.0
+    if check:
+        tol_max, tol_mean = H.ATT_TOL[cfg.dtype]
+        assert worst_max <= tol_max and worst_mean <= tol_mean, (worst_max, worst_mean, rel)
+    return worst_max, worst_mean, rel
 
 
 def test_attention_tiny():
@@ -551,6 +568,28 @@ def test_attention_32b_sampled_heads():
 
 def test_attention_70b_sampled():
     _attention_case("70b", 0, heads=[3], seqs=[0, 5, 11, 15])
+
+
+@pytest.mark.parametrize("name,n", [("8b", 60), ("8b", 256), ("13b", 96), ("32b", 256)])
+def test_attention_tree_keys_alone(name, n):
+    """ctx = 0: every output row is set by its ancestor keys alone, so one
+    wrong mask bit moves it by O(1) (at full context the few ancestor keys
+    carry ~0.2% of a row's weight and a wrong bit moves it by ~1e-3).  The
+    relative error (max-abs over the largest reference output) stays at bf16
+    rounding."""
+    mx, mn, rel = _attention_case(name, 20 + n, ctx_range=(0, 0), n_choices=(n,))
+    assert rel <= 1e-2, (mx, mn, rel)
+
+
+def test_attention_tree_keys_alone_catch_mask_mutants():
+    """The cases above fail on a corrupted mask: the kernel fed the bit
+    matrix transposed (descendants instead of ancestors), or with one
+    ancestor bit dropped, misses the oracle's tolerance."""
+    tol_max, _ = H.ATT_TOL[wl.BF16]
+    for mutant in ("transpose", "drop"):
+        mx, mn, rel = _attention_case("8b", 31, ctx_range=(0, 0), n_choices=(60,),
+                                      mask_mutant=mutant, check=False)
+        assert mx > 10 * tol_max, (mutant, mx, mn)
 
 
 def test_attention_scores_growing_along_the_cache():

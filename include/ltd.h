@@ -367,6 +367,25 @@ ltd_status ltd_accept(const ltd_tree* tree, const void* d_target_logits,
                       const ltd_kv_cache* kv, void* d_workspace, size_t workspace_bytes,
                       ltd_stream_t stream);
 
+/* ltd_accept at a sampling temperature T (section 5.1 "Metrics" reports
+ * T = 1, where ltd_accept is this call with temperature 1): every stochastic
+ * rule uses p = softmax(target row / T) and q = softmax(draft row / T) in
+ * place of the plain softmaxes, the greedy rule is unchanged (the argmax does
+ * not depend on T).  At T != 1 the walk reduces each visited draft row's
+ * normaliser over its cluster (two more cluster barriers per node with
+ * children); at T = 1 it uses the one the expansion stored, and the results
+ * are bit for bit those of ltd_accept.
+ *  temperature      > 0 and finite, else LTD_ERR_INVALID_ARG
+ * Every other argument, the outputs and the errors as ltd_accept. */
+ltd_status ltd_accept_tempered(const ltd_tree* tree, const void* d_target_logits,
+                               const void* d_draft_rows, ltd_dtype dtype, int64_t vocab,
+                               int64_t rows_per_seq, const int32_t* d_node_ids,
+                               const int32_t* d_n_verify, int32_t n_max, const int32_t* d_mode,
+                               float temperature, uint64_t seed, uint64_t cycle,
+                               const int32_t* d_ctx, int32_t* d_new_ctx, int32_t* d_path,
+                               int32_t* d_accept_len, int32_t* d_bonus, const ltd_kv_cache* kv,
+                               void* d_workspace, size_t workspace_bytes, ltd_stream_t stream);
+
 /* Acceptance for callers that cannot allocate device memory when they
  * accept a draft -- a serving loop that reserved its memory up front and
  * keeps allocation off the hot path, a plugin whose host framework owns all

@@ -1,14 +1,16 @@
 // Acceptance and KV compaction (LTD section 3.2, "Draft Tree Verification").
 //
 // accept_rows_kernel: grid (chunks, n_max, batch).  Each CTA scans one chunk
-// of one verified slot's target row and records (max, sum exp, argmax key)
-// in the workspace.
+// of one verified slot's target row and records (max m, sum exp((x - m) / T),
+// argmax key) in the workspace.
 // accept_walk_kernel: one thread-block cluster of C CTAs per sequence.
 //  - greedy: rank 0 merges the argmax records (ties to the lower token id),
 //    marks every slot whose token is its parent's argmax, and follows those
 //    marks from slot 0; the argmax at the end is the bonus token;
-//  - stochastic (T = 1): SpecInfer-style multi-candidate speculative
-//    sampling.  Each CTA holds one vocabulary slice of p (target) and q
+//  - stochastic: SpecInfer-style multi-candidate speculative sampling at a
+//    temperature T (p and q the softmax of the rows divided by T; at T != 1
+//    the draft row's normaliser is reduced over the cluster, at T = 1 the
+//    expansion's is used).  Each CTA holds one vocabulary slice of p (target) and q
 //    (draft) in its threads' registers.  Child i of the current slot is accepted if
 //    r_i q(x_i) < p(x_i) -- every CTA evaluates that test identically --
 //    else p <- max(p - q, 0) / Z, with Z summed over the cluster through
@@ -90,12 +92,13 @@ __global__ void __launch_bounds__(kNT) accept_rows_kernel(const AcceptParams p) 
           jm = j;
         }
       if (vm > m) {
-        s *= __expf(m - vm);
+        s *= __expf((m - vm) * p.inv_t);
         m = vm;
       }
       float add = 0.f;
 #pragma unroll
-      for (int j = 0; j < VEC; ++j) add += (xv[u][j] == -CUDART_INF_F) ? 0.f : __expf(xv[u][j] - m);
+      for (int j = 0; j < VEC; ++j)
+        add += (xv[u][j] == -CUDART_INF_F) ? 0.f : __expf((xv[u][j] - m) * p.inv_t);
       s += add;
       if (idx < hi) {
         const uint64_t key = make_key(vm, static_cast<uint32_t>(idx + jm));
@@ -122,7 +125,7 @@ __global__ void __launch_bounds__(kNT) accept_rows_kernel(const AcceptParams p) 
   float M = red[0];
 #pragma unroll
   for (int w = 1; w < kNW; ++w) M = fmaxf(M, red[w]);
-  float e = (m > -CUDART_INF_F) ? s * __expf(m - M) : 0.f;
+  float e = (m > -CUDART_INF_F) ? s * __expf((m - M) * p.inv_t) : 0.f;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) e += __shfl_xor_sync(0xFFFFFFFFu, e, o);
   __syncthreads();  // every thread has read the maxima
@@ -273,11 +276,24 @@ __global__ void __launch_bounds__(kNT) accept_walk_kernel(const AcceptParams p, 
     sh.pslot[j] = found;
   }
   __syncthreads();
+  // log-sum-exp of the target row at slot over the vocabulary, in units of
+  // logit / T: the chunks' (max, sum exp((x - max) / T)) merged
   auto row_lse = [&](int slot) {
     const AcceptRecord* r = p.rec + (static_cast<int64_t>(b) * p.n_max + slot) * p.chunks;
     float M = -CUDART_INF_F, S = 0.f;
-    for (int c = 0; c < p.chunks; ++c) ms_merge(M, S, r[c].m, r[c].s);
-    return M + logf(S);
+    for (int c = 0; c < p.chunks; ++c) {
+      const float m2 = r[c].m, s2 = r[c].s;
+      if (m2 == -CUDART_INF_F) continue;
+      if (M == -CUDART_INF_F) {
+        M = m2;
+        S = s2;
+        continue;
+      }
+      const float mm = fmaxf(M, m2);
+      S = S * __expf((M - mm) * p.inv_t) + s2 * __expf((m2 - mm) * p.inv_t);
+      M = mm;
+    }
+    return M * p.inv_t + logf(S);
   };
 
   if (mode == LTD_GREEDY) {
@@ -359,15 +375,12 @@ __global__ void __launch_bounds__(kNT) accept_walk_kernel(const AcceptParams p, 
       qrow = draft + (static_cast<int64_t>(b) * p.rows_per_seq + p.xrow[nb + u]) * V;
       lse_q = p.xlse[nb + u];
     }
-    // the children's p(x), q(x) and this CTA's slice, all loads at once; the
-    // slice pass also takes this thread's share of the first residual sum.
-    // The slice goes 16 bytes of logits per thread-step where the rows allow
-    // it (groups of VEC elements), the rest one element at a time.
-    if (tid < nk) {
-      const int x = sh.tok[sh.kids[tid]];
-      sh.kp[tid] = __expf(to_f<T>(trow[x]) - lse_t);
-      sh.kq[tid] = use_q ? __expf(to_f<T>(qrow[x]) - lse_q) : 0.f;
-    }
+    const float it = p.inv_t;
+    // the children's p(x) and this CTA's slice, all loads at once; the slice
+    // pass also takes this thread's share of the first residual sum.  The
+    // slice goes 16 bytes of logits per thread-step where the rows allow it
+    // (groups of VEC elements), the rest one element at a time.
+    if (tid < nk) sh.kp[tid] = __expf(to_f<T>(trow[sh.tok[sh.kids[tid]]]) * it - lse_t);
     float part = 0.f;
     {
       uint4 rt[KG], rq[KG];
@@ -381,6 +394,31 @@ __global__ void __launch_bounds__(kNT) accept_walk_kernel(const AcceptParams p, 
           if (use_q) rq[k] = ld_stream16_once(qrow + el(k, 0));
         }
       }
+      auto dval = [&](int k, int j) -> float {
+        return vec_ok ? elem<T>(rq[k], j) : to_f<T>(qrow[el(k, j)]);
+      };
+      if (use_q && p.tempered) {
+        // q = softmax(draft row / T): its log-sum-exp over the vocabulary,
+        // the cluster's max of the row, then the cluster's sum of
+        // exp((x - max) / T)
+        float tm = -CUDART_INF_F;
+#pragma unroll
+        for (int k = 0; k < KG; ++k)
+#pragma unroll
+          for (int j = 0; j < VEC; ++j)
+            if (el(k, j) < hi) tm = fmaxf(tm, dval(k, j));
+        uint64_t km = block_max_u64<kNT>(make_key(tm, 0u), sh.redk);
+        km = cluster_max_u64(km, sh.cell_key, round, C);
+        const float qm = key_value(km);
+        float ts = 0.f;
+#pragma unroll
+        for (int k = 0; k < KG; ++k)
+#pragma unroll
+          for (int j = 0; j < VEC; ++j)
+            if (el(k, j) < hi) ts += __expf((dval(k, j) - qm) * it);
+        lse_q = qm * it + logf(cluster_sum_warps(ts, sh.wpart, round, C));
+      }
+      if (tid < nk) sh.kq[tid] = use_q ? __expf(to_f<T>(qrow[sh.tok[sh.kids[tid]]]) * it - lse_q) : 0.f;
 #pragma unroll
       for (int k = 0; k < KG; ++k)
 #pragma unroll
@@ -398,8 +436,8 @@ __global__ void __launch_bounds__(kNT) accept_walk_kernel(const AcceptParams p, 
           pr[k][j] = 0.f;
           qr[k][j] = 0.f;
           if (in) {
-            pr[k][j] = __expf(tv - lse_t);
-            if (use_q) qr[k][j] = __expf(dv - lse_q);
+            pr[k][j] = __expf(tv * it - lse_t);
+            if (use_q) qr[k][j] = __expf(dv * it - lse_q);
           }
           part += fmaxf(pr[k][j] - qr[k][j], 0.f);
         }

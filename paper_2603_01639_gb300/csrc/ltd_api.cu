@@ -482,14 +482,17 @@ ltd_status ltd_kv_compact(const ltd_kv_cache* kv, int32_t batch, const int32_t* 
   return from_cuda(launch_compact(p, batch, reinterpret_cast<cudaStream_t>(stream)));
 }
 
-ltd_status ltd_accept(const ltd_tree* tree, const void* d_target_logits, const void* d_draft_rows,
-                      ltd_dtype dtype, int64_t vocab, int64_t rows_per_seq,
-                      const int32_t* d_node_ids, const int32_t* d_n_verify, int32_t n_max,
-                      const int32_t* d_mode, uint64_t seed, uint64_t cycle, const int32_t* d_ctx,
-                      int32_t* d_new_ctx, int32_t* d_path, int32_t* d_accept_len,
-                      int32_t* d_bonus, const ltd_kv_cache* kv, void* d_workspace,
-                      size_t workspace_bytes, ltd_stream_t stream) {
-  const ApiRange nvtx_range("ltd_accept");
+}  // extern "C"
+
+namespace {
+ltd_status accept_impl(const ltd_tree* tree, const void* d_target_logits, const void* d_draft_rows,
+                       ltd_dtype dtype, int64_t vocab, int64_t rows_per_seq,
+                       const int32_t* d_node_ids, const int32_t* d_n_verify, int32_t n_max,
+                       const int32_t* d_mode, float temperature, uint64_t seed, uint64_t cycle,
+                       const int32_t* d_ctx, int32_t* d_new_ctx, int32_t* d_path,
+                       int32_t* d_accept_len, int32_t* d_bonus, const ltd_kv_cache* kv,
+                       void* d_workspace, size_t workspace_bytes, ltd_stream_t stream) {
+  if (!(temperature > 0.f) || !(temperature <= 3.0e38f)) return LTD_ERR_INVALID_ARG;
   if (!tree_ok(tree) || !d_target_logits || !d_draft_rows || !dtype_ok(dtype) || !d_node_ids ||
       !d_n_verify || !d_mode || !d_ctx || !d_new_ctx || !d_path || !d_accept_len || !d_bonus)
     return LTD_ERR_INVALID_ARG;
@@ -533,6 +536,8 @@ ltd_status ltd_accept(const ltd_tree* tree, const void* d_target_logits, const v
   p.accept_len = d_accept_len;
   p.bonus = d_bonus;
   p.rec = static_cast<AcceptRecord*>(d_workspace);
+  p.inv_t = temperature == 1.f ? 1.f : 1.f / temperature;
+  p.tempered = temperature != 1.f;
   p.chunks = vs.chunks;
   p.chunk_elems = vs.chunk_elems;
   p.err = err;
@@ -540,6 +545,36 @@ ltd_status ltd_accept(const ltd_tree* tree, const void* d_target_logits, const v
   cudaError_t e = launch_accept(p, tree->batch, dtype, s);
   if (e != cudaSuccess || kv == nullptr) return from_cuda(e);
   return ltd_kv_compact(kv, tree->batch, d_path, tree->max_depth + 1, d_accept_len, d_ctx, stream);
+}
+}  // namespace
+
+extern "C" {
+
+ltd_status ltd_accept(const ltd_tree* tree, const void* d_target_logits, const void* d_draft_rows,
+                      ltd_dtype dtype, int64_t vocab, int64_t rows_per_seq,
+                      const int32_t* d_node_ids, const int32_t* d_n_verify, int32_t n_max,
+                      const int32_t* d_mode, uint64_t seed, uint64_t cycle, const int32_t* d_ctx,
+                      int32_t* d_new_ctx, int32_t* d_path, int32_t* d_accept_len,
+                      int32_t* d_bonus, const ltd_kv_cache* kv, void* d_workspace,
+                      size_t workspace_bytes, ltd_stream_t stream) {
+  const ApiRange nvtx_range("ltd_accept");
+  return accept_impl(tree, d_target_logits, d_draft_rows, dtype, vocab, rows_per_seq, d_node_ids,
+                     d_n_verify, n_max, d_mode, 1.f, seed, cycle, d_ctx, d_new_ctx, d_path,
+                     d_accept_len, d_bonus, kv, d_workspace, workspace_bytes, stream);
+}
+
+ltd_status ltd_accept_tempered(const ltd_tree* tree, const void* d_target_logits,
+                               const void* d_draft_rows, ltd_dtype dtype, int64_t vocab,
+                               int64_t rows_per_seq, const int32_t* d_node_ids,
+                               const int32_t* d_n_verify, int32_t n_max, const int32_t* d_mode,
+                               float temperature, uint64_t seed, uint64_t cycle,
+                               const int32_t* d_ctx, int32_t* d_new_ctx, int32_t* d_path,
+                               int32_t* d_accept_len, int32_t* d_bonus, const ltd_kv_cache* kv,
+                               void* d_workspace, size_t workspace_bytes, ltd_stream_t stream) {
+  const ApiRange nvtx_range("ltd_accept_tempered");
+  return accept_impl(tree, d_target_logits, d_draft_rows, dtype, vocab, rows_per_seq, d_node_ids,
+                     d_n_verify, n_max, d_mode, temperature, seed, cycle, d_ctx, d_new_ctx, d_path,
+                     d_accept_len, d_bonus, kv, d_workspace, workspace_bytes, stream);
 }
 
 ltd_status ltd_check(ltd_stream_t stream, uint32_t* out_bits) {

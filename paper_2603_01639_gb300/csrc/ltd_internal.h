@@ -186,6 +186,8 @@ struct AcceptParams {
   int32_t* accept_len;
   int32_t* bonus;
   AcceptRecord* rec;  // [batch][n_max][chunks]
+  float inv_t;        // 1 / temperature of the stochastic rules (1 at T = 1)
+  int32_t tempered;   // T != 1: the draft rows' normaliser is computed in the walk
   int32_t chunks;
   int64_t chunk_elems;
   uint32_t* err;

@@ -31,7 +31,7 @@ EXPORTS = [
     "ltd_accept", "ltd_kv_compact", "ltd_check", "ltd_status_string", "ltd_version",
     "ltd_attention_kernel", "ltd_selftest_umma", "ltd_accept_noalloc", "ltd_tree_attention_next",
     "ltd_depth_observation", "ltd_size_observation", "ltd_depth_policy", "ltd_size_policy",
-    "ltd_mlp_packed_bytes", "ltd_mlp_pack", "ltd_kv_append",
+    "ltd_mlp_packed_bytes", "ltd_mlp_pack", "ltd_kv_append", "ltd_accept_tempered",
 ]
 LTD_POLICY_PAD = -100.0
 LTD_MLP_MAX_LAYERS, LTD_MLP_MAX_WIDTH = 4, 2048
@@ -96,6 +96,9 @@ def lib():
                 "ltd_accept_workspace_bytes": (sz, [i32, i32, i64]),
                 "ltd_accept": (C.c_int, [tp, vp, vp, C.c_int, i64, i64, vp, vp, i32, vp, u64, u64,
                                          vp, vp, vp, vp, vp, C.POINTER(ltd_kv_cache), vp, sz, vp]),
+                "ltd_accept_tempered": (C.c_int, [tp, vp, vp, C.c_int, i64, i64, vp, vp, i32, vp,
+                                                  C.c_float, u64, u64, vp, vp, vp, vp, vp,
+                                                  C.POINTER(ltd_kv_cache), vp, sz, vp]),
                 "ltd_kv_compact": (C.c_int, [C.POINTER(ltd_kv_cache), i32, vp, i32, vp, vp, vp]),
                 "ltd_kv_append": (C.c_int, [C.POINTER(ltd_kv_cache), i32, i32, vp, vp, vp, vp, vp]),
                 "ltd_check": (C.c_int, [vp, C.POINTER(C.c_uint32)]),
@@ -410,8 +413,9 @@ class KVCache:
 
 
 def ltd_accept(tree: Tree, target, draft_rows, node_ids, n_verify, mode, ctx, seed=0, cycle=0,
-               kv: KVCache | None = None, workspace=None, out=None, stream=None):
-    """Returns dict(path [B][max_depth+1], accept_len [B], bonus [B], new_ctx [B])."""
+               kv: KVCache | None = None, workspace=None, out=None, stream=None, temperature=None):
+    """Returns dict(path [B][max_depth+1], accept_len [B], bonus [B], new_ctx [B]).
+    ``temperature`` (a float) calls ltd_accept_tempered instead."""
     _need(target, "target")
     _need(draft_rows, "draft_rows", target.dtype)
     for t, n in ((node_ids, "node_ids"), (n_verify, "n_verify"), (mode, "mode"), (ctx, "ctx")):
@@ -427,6 +431,15 @@ def ltd_accept(tree: Tree, target, draft_rows, node_ids, n_verify, mode, ctx, se
                "bonus": torch.empty(B, dtype=torch.int32, device=dev),
                "new_ctx": torch.empty(B, dtype=torch.int32, device=dev)}
     kvp = C.byref(kv.s) if kv is not None else None
+    if temperature is not None:
+        _ok(lib().ltd_accept_tempered(C.byref(tree.s), _ptr(target), _ptr(draft_rows),
+                                      _dtype(target), V, R, _ptr(node_ids), _ptr(n_verify), n_max,
+                                      _ptr(mode), float(temperature), seed, cycle, _ptr(ctx),
+                                      _ptr(out["new_ctx"]), _ptr(out["path"]),
+                                      _ptr(out["accept_len"]), _ptr(out["bonus"]), kvp,
+                                      _ptr(workspace), workspace.numel(), _stream(stream)),
+            "ltd_accept_tempered")
+        return out
     _ok(lib().ltd_accept(C.byref(tree.s), _ptr(target), _ptr(draft_rows), _dtype(target), V, R,
                          _ptr(node_ids), _ptr(n_verify), n_max, _ptr(mode), seed, cycle, _ptr(ctx),
                          _ptr(out["new_ctx"]), _ptr(out["path"]), _ptr(out["accept_len"]),

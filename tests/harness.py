@@ -53,7 +53,7 @@ def oracle_side(cfg: wl.Config, ci: wl.CycleInputs, plant_seed: int = 99):
     return trees, sels, target
 
 
-def oracle_accept(cfg, ci, trees, sels, target, seed, cycle_no):
+def oracle_accept(cfg, ci, trees, sels, target, seed, cycle_no, temperature=1.0):
     res = []
     for b in range(cfg.batch):
         ids = sels[b][0]
@@ -63,13 +63,16 @@ def oracle_accept(cfg, ci, trees, sels, target, seed, cycle_no):
             path, a, bonus = oracle.accept_greedy(trees[b], ids, rows)
             margins = []
         elif ci.mode[b] == 2:
-            path, a, bonus, margins = oracle.accept_point_mass(trees[b], ids, rows, seed, b, cycle_no)
+            path, a, bonus, margins = oracle.accept_point_mass(trees[b], ids, rows, seed, b, cycle_no,
+                                                               temperature)
         elif ci.mode[b] == 3:
             path, a, bonus, margins = oracle.accept_without_replacement(
-                trees[b], ids, rows, ci.draft_rows[b].astype(np.float64), seed, b, cycle_no)
+                trees[b], ids, rows, ci.draft_rows[b].astype(np.float64), seed, b, cycle_no,
+                temperature)
         else:
             path, a, bonus, margins = oracle.accept_stochastic(
-                trees[b], ids, rows, ci.draft_rows[b].astype(np.float64), seed, b, cycle_no)
+                trees[b], ids, rows, ci.draft_rows[b].astype(np.float64), seed, b, cycle_no,
+                temperature)
         res.append(dict(path=path, accept_len=a, bonus=bonus, margins=margins,
                         new_ctx=int(ci.ctx[b]) + 1 + a))
     return res

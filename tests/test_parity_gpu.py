@@ -264,16 +264,18 @@ def test_adaptive_draft_driven_by_device_policies(name, seed):
 
 
 # ------------------------------------------------ point-mass stochastic rule
-def _accept_case(cfg, ci, target, acc_seed=1234, cycle_no=0):
+def _accept_case(cfg, ci, target, acc_seed=1234, cycle_no=0, temperature=None):
     trees, sels, _ = H.oracle_side(cfg, ci)
     assert min(H.tree_margin(t, cfg.W) for t in trees) > H.CUT_MARGIN
-    ref = H.oracle_accept(cfg, ci, trees, sels, target, acc_seed, cycle_no)
+    ref = H.oracle_accept(cfg, ci, trees, sels, target, acc_seed, cycle_no,
+                          1.0 if temperature is None else temperature)
     assert H.stochastic_margins_ok(ref), "near-tie in a stochastic decision; pick another seed"
     draft = H.dev(ci.draft_rows, cfg.dtype)
     tree = H.gpu_draft(cfg, ci, draft)
     got = H.gpu_select(cfg, ci, tree)
     out = ltd.ltd_accept(tree, H.dev(target, cfg.dtype), draft, got[0], H.i32(ci.n_verify),
-                         H.i32(ci.mode), H.i32(ci.ctx), seed=acc_seed, cycle=cycle_no)
+                         H.i32(ci.mode), H.i32(ci.ctx), seed=acc_seed, cycle=cycle_no,
+                         temperature=temperature)
     assert ltd.ltd_check() == 0
     H.compare_accept(cfg, out, ref)
     return ref
@@ -308,6 +310,46 @@ def test_70b_batch_with_every_rule(seed):
     ci.mode = (np.arange(cfg.batch) % 4).astype(np.int32)
     _, _, target = H.oracle_side(cfg, ci)
     _accept_case(cfg, ci, target, cycle_no=seed)
+
+
+@pytest.mark.parametrize("temperature", [0.5, 2.0])
+@pytest.mark.parametrize("seed", [0, 2])
+def test_every_rule_at_a_temperature(seed, temperature):
+    """ltd_accept_tempered: the ragged 70B batch with all four rules side by
+    side at T = 0.5 and T = 2 against the oracle's rules at the same T (p and
+    q the softmax of the rows divided by T; greedy unchanged)."""
+    cfg = wl.config("70b")
+    ci = wl.draw_cycle(cfg, seed)
+    ci.mode = (np.arange(cfg.batch) % 4).astype(np.int32)
+    _, _, target = H.oracle_side(cfg, ci)
+    _accept_case(cfg, ci, target, cycle_no=seed, temperature=temperature)
+
+
+@pytest.mark.parametrize("mode", [1, 2, 3])
+def test_tempered_rules_accepting(mode):
+    """Sharpened target rows (a copy of the draft row times 5, as above) at
+    T = 2, so children are accepted at the higher temperature too; and T = 1
+    through ltd_accept_tempered equals ltd_accept bit for bit."""
+    cfg = wl.config("13b")
+    ci = wl.draw_cycle(cfg, 1)
+    ci.mode = np.full(cfg.batch, mode, np.int32)
+    trees, sels, target = H.oracle_side(cfg, ci)
+    for b in range(cfg.batch):
+        for sl, nid in enumerate(sels[b][0]):
+            xr = trees[b].xrow[int(nid)]
+            if xr >= 0:
+                target[b, sl] = wl.round_to(ci.draft_rows[b, xr] * 5.0, cfg.dtype)
+    _accept_case(cfg, ci, target, cycle_no=4, temperature=2.0)
+    draft = H.dev(ci.draft_rows, cfg.dtype)
+    tree = H.gpu_draft(cfg, ci, draft)
+    ids = H.gpu_select(cfg, ci, tree)[0]
+    args = (tree, H.dev(target, cfg.dtype), draft, ids, H.i32(ci.n_verify), H.i32(ci.mode),
+            H.i32(ci.ctx))
+    a = ltd.ltd_accept(*args, seed=9, cycle=1)
+    b = ltd.ltd_accept(*args, seed=9, cycle=1, temperature=1.0)
+    assert ltd.ltd_check() == 0
+    for k in a:
+        assert torch.equal(a[k], b[k]), k
 
 
 def test_unknown_rule_is_flagged_and_the_others_still_run():

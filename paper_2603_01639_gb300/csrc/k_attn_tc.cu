@@ -69,7 +69,6 @@ constexpr uint32_t kSmemBytes = kOffHolder + 16 + 1024;  // + alignment slack
 // Regions reused once they are free (after the last MMA, or before any load):
 constexpr uint32_t kOffCost = kOffV + 2 * kTile;       // [kMaxGroups] int, ranking only
 constexpr uint32_t kOffOrder = kOffCost + kMaxGroups * 4;
-constexpr uint32_t kOffStgL = kOffK;                   // [128] log2-sum-exp of the staged rows
 constexpr uint32_t kOffML = kOffK + 1024;              // [2][128] (m, l) of each stream
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kRowBytes = kD * 2;  // one bf16 output / partial row
@@ -117,7 +116,7 @@ struct TcArgs {
   const uint32_t* mask;
   float scale_log2;
   __nv_bfloat16* out;
-  uint8_t* part_o;  // [unit][split][128 rows][256 B] O / l, bf16, chunks swizzled (splits > 1)
+  uint8_t* part_o;  // [unit][split][16 chunks][128 rows][16 B] O / l, bf16 (splits > 1)
   float* part_l;    // [unit][split][128] log2-sum-exp
   uint32_t* sync;   // [unit][2] arrive, depart
   const uint8_t* next_k;  // the next call's caches: L2 prefetch targets (or null)
@@ -135,25 +134,15 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
 
 // Visibility of keys kk0 .. kk0+31 for one row as a 32-bit mask: keys below
 // ctx are the prefix (always visible), key ctx + j is verified slot j (bit j
-// of the row's ancestor mask, read from global memory), keys from key_hi on
-// are outside this split.
+// of the row's ancestor mask), keys from key_hi on are outside this split.
+// `lo` and `hi` are the mask words holding slots (kk0 - ctx) >> 5 and the one
+// after (0 outside the mask), `sh` = (kk0 - ctx) & 31.
 __device__ __forceinline__ uint32_t low_bits(int n) {
   return n <= 0 ? 0u : (n >= 32 ? 0xFFFFFFFFu : ((1u << n) - 1u));
 }
-__device__ __forceinline__ uint32_t visible32(int kk0, int ctx, int key_hi, int W32,
-                                              const uint32_t* mbits) {
-  const uint32_t in_range = low_bits(key_hi - kk0);
-  const uint32_t prefix = low_bits(ctx - kk0);
-  uint32_t tree = 0u;
-  const int js0 = kk0 - ctx;  // slot of bit 0 of the window (may be negative)
-  if (js0 > -32 && js0 < 32 * W32) {
-    const int w = js0 >> 5;  // floor division
-    const int sh = js0 & 31;
-    const uint32_t lo = (w >= 0 && w < W32) ? __ldg(mbits + w) : 0u;
-    const uint32_t hi = (w + 1 >= 0 && w + 1 < W32) ? __ldg(mbits + w + 1) : 0u;
-    tree = __funnelshift_r(lo, hi, sh);
-  }
-  return in_range & (prefix | tree);
+__device__ __forceinline__ uint32_t visible32(int kk0, int ctx, int key_hi, uint32_t lo, uint32_t hi,
+                                              int sh) {
+  return low_bits(key_hi - kk0) & (low_bits(ctx - kk0) | __funnelshift_r(lo, hi, sh));
 }
 
 __device__ __forceinline__ bool seq_ok(const TcArgs& a, int ctx, int N) {
@@ -326,8 +315,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   // the row's ancestor-mask words, read where a chunk holds verified keys
   const uint32_t* mbits =
       a.mask + (static_cast<int64_t>(b) * a.n_max + min(R / a.G, a.n_max - 1)) * a.W32;
-  if (row_ok && key_hi > ctx)
-    asm volatile("prefetch.global.L1 [%0];" ::"l"(mbits));
   tc::fence_before_sync();
   __syncthreads();
   tc::fence_after_sync();
@@ -385,77 +372,139 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0 && nc > 0) {
       const uint32_t id_s = tc::idesc_bf16(kBM, kBN, false);
       const uint32_t id_o = tc::idesc_bf16(kBM, kD, true);
-      // Every shared-memory descriptor is computed once, so the issue loop
-      // below is MMA instructions and waits only.
-      uint64_t dq[8], dk[kStages][8], dv[kStages][8];
+      // Three base descriptors; the others differ by constant offsets (in
+      // 16-byte units) for the K slice and the ring stage: K-major slice ks
+      // at (ks / 4) * kHalf + (ks % 4) * 32 bytes, MN-major slice ks of V 16
+      // rows of 128 bytes on.
+      const uint64_t dq0 = tc::sdesc_sw128(base + kOffQ, 16, 1024);
+      const uint64_t dk0 = tc::sdesc_sw128(base + kOffK, 16, 1024);
+      const uint64_t dv0 = tc::sdesc_sw128(base + kOffV, kHalf, 1024);
+      if (nc <= 4) {
+        // a short split: a rolled loop, stage descriptors by adds per chunk
+        // (this thread runs its issue code cold, and a short split runs it
+        // only a few times)
+        auto koff = [](int ks) { return static_cast<uint64_t>((ks >> 2) * (kHalf >> 4) + (ks & 3) * 2); };
+        auto issue_s = [&](int x_, int st) {
+          const uint64_t k = dk0 + static_cast<uint64_t>(st) * (kTile >> 4);
+          const uint32_t d = tmem + x_ * kBN;
 #pragma unroll
-      for (int ks = 0; ks < 8; ++ks) {
-        dq[ks] = tc::sdesc_sw128(base + kOffQ + (ks >> 2) * kHalf + (ks & 3) * 32, 16, 1024);
+          for (int ks = 0; ks < 8; ++ks) tc::mma_bf16(d, dq0 + koff(ks), k + koff(ks), id_s, ks > 0 ? 1u : 0u);
+        };
+        auto issue_pv = [&](int x_, int st, uint32_t acc) {
+          const uint64_t v = dv0 + static_cast<uint64_t>(st) * (kTile >> 4);
+          const uint32_t d = tmem + 2 * kBN + x_ * kD, pa = tmem + x_ * kBN;
 #pragma unroll
-        for (int st = 0; st < kStages; ++st) {
-          dk[st][ks] = tc::sdesc_sw128(base + kOffK + st * kTile + (ks >> 2) * kHalf + (ks & 3) * 32, 16, 1024);
-          dv[st][ks] = tc::sdesc_sw128(base + kOffV + st * kTile + ks * 2048, kHalf, 1024);
+          for (int ks = 0; ks < 8; ++ks)
+            tc::mma_bf16_ts(d, pa + 8 * ks, v + static_cast<uint64_t>(ks * (2048 >> 4)), id_o, ks > 0 ? 1u : acc);
+        };
+        ok = tc::mbar_wait(bar(QFULL), 0);
+        TRACE(2);
+        // S(0) and S(1) into S_0 and S_1, then per chunk j (stream j & 1, ring
+        // stage j % 3, ring use j / 3): PV(j), then S(j + 2) into the same
+        // stream
+        for (int j = 0; j < 2 && j < nc && ok; ++j) {
+          ok = tc::mbar_wait(bar(KFULL + j), 0);
+          if (!ok) break;
+          tc::fence_after_sync();
+          issue_s(j, j);
+          tc::mma_commit(bar(SFULL + j));
+          tc::mma_commit(bar(KEMPTY + j));
+          if (j == 0) TRACE(3);
         }
-      }
-      // (x and st are compile-time constants at every call)
-      auto issue_s = [&](int x_, int st) {
+        for (int j = 0; j < nc && ok; ++j) {
+          const int xs = j & 1, st = j % kStages;
+          ok = tc::mbar_wait(bar(VFULL + st), (j / kStages) & 1);
+          if (ok) ok = tc::mbar_wait(bar(PFULL + xs), (j >> 1) & 1);
+          if (!ok) break;
+          tc::fence_after_sync();
+          issue_pv(xs, st, j >= 2 ? 1u : 0u);
+          tc::mma_commit(bar(VEMPTY + st));
+          if (j + 2 < nc) {
+            const int st2 = (j + 2) % kStages;
+            ok = tc::mbar_wait(bar(KFULL + st2), ((j + 2) / kStages) & 1);
+            if (!ok) break;
+            tc::fence_after_sync();
+            issue_s(xs, st2);
+            tc::mma_commit(bar(SFULL + xs));
+            tc::mma_commit(bar(KEMPTY + st2));
+          }
+        }
+      } else {
+        // a long split: the loop unrolled over six chunks, so stages and
+        // descriptors are compile-time choices
+        // every descriptor of the loop, from the three bases by adds (held in
+        // registers: the issue loop below is MMA instructions and waits only)
+        uint64_t dq[8], dk[kStages][8], dv[kStages][8];
 #pragma unroll
-        for (int ks = 0; ks < 8; ++ks)
-          tc::mma_bf16(tmem + x_ * kBN, dq[ks], dk[st][ks], id_s, ks > 0 ? 1u : 0u);
-      };
-      auto issue_pv = [&](int x_, int st, uint32_t acc) {
+        for (int ks = 0; ks < 8; ++ks) {
+          const uint64_t ko = static_cast<uint64_t>((ks >> 2) * (kHalf >> 4) + (ks & 3) * 2);
+          dq[ks] = dq0 + ko;
 #pragma unroll
-        for (int ks = 0; ks < 8; ++ks)
-          tc::mma_bf16_ts(tmem + 2 * kBN + x_ * kD, tmem + x_ * kBN + 8 * ks, dv[st][ks], id_o,
-                          ks > 0 ? 1u : acc);
-      };
-      ok = tc::mbar_wait(bar(QFULL), 0);
-      TRACE(2);
-      // S(0) and S(1) into S_0 and S_1
-      if (ok) ok = tc::mbar_wait(bar(KFULL + 0), 0);
-      if (ok) {
-        tc::fence_after_sync();
-        issue_s(0, 0);
-        tc::mma_commit(bar(SFULL + 0));
-        tc::mma_commit(bar(KEMPTY + 0));
-      }
-      TRACE(3);
-      if (ok && nc > 1) {
-        ok = tc::mbar_wait(bar(KFULL + 1), 0);
+          for (int st = 0; st < kStages; ++st) {
+            dk[st][ks] = dk0 + static_cast<uint64_t>(st * (kTile >> 4)) + ko;
+            dv[st][ks] = dv0 + static_cast<uint64_t>(st * (kTile >> 4) + ks * (2048 >> 4));
+          }
+        }
+        // (x and st are compile-time constants at every call)
+        auto issue_s = [&](int x_, int st) {
+#pragma unroll
+          for (int ks = 0; ks < 8; ++ks)
+            tc::mma_bf16(tmem + x_ * kBN, dq[ks], dk[st][ks], id_s, ks > 0 ? 1u : 0u);
+        };
+        auto issue_pv = [&](int x_, int st, uint32_t acc) {
+#pragma unroll
+          for (int ks = 0; ks < 8; ++ks)
+            tc::mma_bf16_ts(tmem + 2 * kBN + x_ * kD, tmem + x_ * kBN + 8 * ks, dv[st][ks], id_o,
+                            ks > 0 ? 1u : acc);
+        };
+        ok = tc::mbar_wait(bar(QFULL), 0);
+        TRACE(2);
+        // S(0) and S(1) into S_0 and S_1, then chunk j = 6 i + r (stream r & 1,
+        // ring stage r % 3, ring use j / 3, whose parity is (r / 3) & 1): PV(j),
+        // then S(j + 2) into the same stream; stages are compile-time constants
+        if (ok) ok = tc::mbar_wait(bar(KFULL + 0), 0);
         if (ok) {
           tc::fence_after_sync();
-          issue_s(1, 1);
-          tc::mma_commit(bar(SFULL + 1));
-          tc::mma_commit(bar(KEMPTY + 1));
+          issue_s(0, 0);
+          tc::mma_commit(bar(SFULL + 0));
+          tc::mma_commit(bar(KEMPTY + 0));
         }
-      }
-      // chunk j = 6 i + r: stream r & 1, stage r % 3, ring use j / 3 (its
-      // parity is (r / 3) & 1); PV(j) then S(j + 2) into the same stream
-      auto step = [&](int j, auto R_) -> bool {
-        constexpr int r = decltype(R_)::value;
-        constexpr int xs = r & 1, st = r % kStages, st2 = (r + 2) % kStages;
-        bool k = tc::mbar_wait(bar(VFULL + st), (r / kStages) & 1);
-        if (k) k = tc::mbar_wait(bar(PFULL + xs), (j >> 1) & 1);
-        if (!k) return false;
-        tc::fence_after_sync();
-        issue_pv(xs, st, j >= 2 ? 1u : 0u);
-        tc::mma_commit(bar(VEMPTY + st));
-        if (j + 2 < nc) {
-          if (!tc::mbar_wait(bar(KFULL + st2), ((r + 2) / kStages) & 1)) return false;
+        TRACE(3);
+        if (ok && nc > 1) {
+          ok = tc::mbar_wait(bar(KFULL + 1), 0);
+          if (ok) {
+            tc::fence_after_sync();
+            issue_s(1, 1);
+            tc::mma_commit(bar(SFULL + 1));
+            tc::mma_commit(bar(KEMPTY + 1));
+          }
+        }
+        auto step = [&](int j, auto R_) -> bool {
+          constexpr int r = decltype(R_)::value;
+          constexpr int xs = r & 1, st = r % kStages, st2 = (r + 2) % kStages;
+          bool k = tc::mbar_wait(bar(VFULL + st), (r / kStages) & 1);
+          if (k) k = tc::mbar_wait(bar(PFULL + xs), (j >> 1) & 1);
+          if (!k) return false;
           tc::fence_after_sync();
-          issue_s(xs, st2);
-          tc::mma_commit(bar(SFULL + xs));
-          tc::mma_commit(bar(KEMPTY + st2));
+          issue_pv(xs, st, j >= 2 ? 1u : 0u);
+          tc::mma_commit(bar(VEMPTY + st));
+          if (j + 2 < nc) {
+            if (!tc::mbar_wait(bar(KFULL + st2), ((r + 2) / kStages) & 1)) return false;
+            tc::fence_after_sync();
+            issue_s(xs, st2);
+            tc::mma_commit(bar(SFULL + xs));
+            tc::mma_commit(bar(KEMPTY + st2));
+          }
+          return true;
+        };
+        for (int j = 0; j < nc && ok; j += 6) {
+          ok = step(j, Int<0>{});
+          if (ok && j + 1 < nc) ok = step(j + 1, Int<1>{});
+          if (ok && j + 2 < nc) ok = step(j + 2, Int<2>{});
+          if (ok && j + 3 < nc) ok = step(j + 3, Int<3>{});
+          if (ok && j + 4 < nc) ok = step(j + 4, Int<4>{});
+          if (ok && j + 5 < nc) ok = step(j + 5, Int<5>{});
         }
-        return true;
-      };
-      for (int j = 0; j < nc && ok; j += 6) {
-        ok = step(j, Int<0>{});
-        if (ok && j + 1 < nc) ok = step(j + 1, Int<1>{});
-        if (ok && j + 2 < nc) ok = step(j + 2, Int<2>{});
-        if (ok && j + 3 < nc) ok = step(j + 3, Int<3>{});
-        if (ok && j + 4 < nc) ok = step(j + 4, Int<4>{});
-        if (ok && j + 5 < nc) ok = step(j + 5, Int<5>{});
       }
       TRACE(22);
       // every MMA of this CTA completes before tensor memory is read or freed
@@ -464,6 +513,19 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!ok) flag_error(a.err, LTD_DEVERR_TIMEOUT);
       TRACE(23);
     }
+#ifdef LTD_TRACE
+  } else if (warp == 3) {
+    // (trace builds only) the idle warp observes when the first loads land
+    if (lane == 0) {
+      if (tc::mbar_wait(bar(QFULL), 0)) TRACE(24);
+      if (nc > 0 && tc::mbar_wait(bar(KFULL + 0), 0)) TRACE(25);
+      if (nc > 0 && tc::mbar_wait(bar(VFULL + 0), 0)) TRACE(26);
+      if (nc > 1 && tc::mbar_wait(bar(KFULL + 1), 0)) TRACE(27);
+      if (nc > 1 && tc::mbar_wait(bar(VFULL + 1), 0)) TRACE(28);
+      if (nc > 2 && tc::mbar_wait(bar(KFULL + 2), 0)) TRACE(29);
+      if (nc > 2 && tc::mbar_wait(bar(VFULL + 2), 0)) TRACE(30);
+    }
+#endif
   } else if (smx && x < nc) {
     // ------------------------------------------------------------- softmax
     const uint32_t lane_off = (32u * (warp & 3)) << 16;
@@ -474,13 +536,24 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int w32 = a.W32;
     const bool tr = (tid & 127) == 0;
     for (int j = x; j < nc; j += 2) {
+      const int kbase = key_lo + j * kBN;
+      const bool all_vis = row_ok && kbase + kBN <= vis_all_below;
+      // A chunk that holds verified keys needs five of the row's mask words
+      // (its four 32-key windows and the word after), read from L2 (the
+      // mask is another kernel's output) before the wait below, so their
+      // latency hides behind it.
+      uint32_t mw5[5] = {0u, 0u, 0u, 0u, 0u};
+      const int js = kbase - ctx, w0 = js >> 5;  // floor division
+      if (row_ok && !all_vis) {
+#pragma unroll
+        for (int t = 0; t < 5; ++t)
+          if (w0 + t >= 0 && w0 + t < w32) mw5[t] = __ldcg(mbits + w0 + t);
+      }
       ok = tc::mbar_wait(bar(SFULL + x), (j >> 1) & 1);
       ok = __all_sync(0xFFFFFFFFu, ok);
       if (tr && j < 4) TRACE(4 + 2 * j);
       if (!ok) break;
       tc::fence_after_sync();
-      const int kbase = key_lo + j * kBN;
-      const bool all_vis = row_ok && kbase + kBN <= vis_all_below;
       // P against the stream's running max m (a row without one yet first
       // takes this chunk's max); the chunk's own max is tracked on the way
       // and, if it exceeds the reference by more than 2^8 in some row of the
@@ -493,7 +566,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!all_vis) {
 #pragma unroll
         for (int qq = 0; qq < 4; ++qq)
-          vq[qq] = row_ok ? visible32(kbase + 32 * qq, ctx, key_hi, w32, mbits) : 0u;
+          vq[qq] = row_ok ? visible32(kbase + 32 * qq, ctx, key_hi, mw5[qq], mw5[qq + 1], js & 31) : 0u;
       }
       __syncwarp();  // the load below is warp-collective; the branch above is per row
       tc::tmem_ld128_sync(t_s, f);
@@ -618,7 +691,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   // --------------------------------------------------------- epilogue
   // The producers have drained every load and the MMA thread has seen the
   // last MMA complete before this barrier; after it, the K ring holds the
-  // two streams' (m, l), and Q's region the staged rows.
+  // two streams' (m, l).
   tc::fence_before_sync();
   __syncthreads();
   tc::fence_after_sync();
@@ -626,14 +699,18 @@ __global__ void __launch_bounds__(kThreads, 1)
   float2* ml = reinterpret_cast<float2*>(gbase + kOffML);
   if (smx) ml[x * kBM + lrow] = make_float2(m, l);
   __syncthreads();
+  if (tid == 0) TRACE(32);
   const int unit = (b * a.hkv + kvh) * a.n_tiles + tile;
   const int Mv = min(kBM, M - row0);
-  uint8_t* stg = gbase + kOffQ;
-  float* stg_l = reinterpret_cast<float*>(gbase + kOffStgL);
+  const int Rp = (Mv + 7) & ~7;  // rows of a partial block (16-byte chunk-major)
+  const int64_t pb = static_cast<int64_t>(unit) * S + split;
   // Merge the two streams: stream x's thread of a row writes columns
-  // 64 x .. 64 x + 63 of O / l.  tcgen05.ld is warp-collective: the loads
-  // are taken by whole warps (nc and ok are uniform in a warp), the writes
-  // per row.
+  // 64 x .. 64 x + 63 of O / l, straight from registers to the output (one
+  // split), or (several splits) into shared memory over Q's region,
+  // chunk-major ([16-byte chunk][row], so a warp's stores are contiguous),
+  // with the row's log2-sum-exp over the K ring; one bulk copy then stores
+  // the block as this split's partial.  tcgen05.ld is warp-collective: the
+  // loads are taken by whole warps (nc is uniform), the writes per row.
   if (smx) {
     const float2 me = ml[lrow], mo = ml[kBM + lrow];
     const float mm = fmaxf(me.x, mo.x);
@@ -649,7 +726,18 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (ld0) tc::tmem_ld64_sync(tmem + 2 * kBN + 0 * kD + 64 * x + lane_off, o0);
     if (ld1) tc::tmem_ld64_sync(tmem + 2 * kBN + 1 * kD + 64 * x + lane_off, o1);
     if (row_ok) {
-      uint8_t* srow = stg + lrow * kRowBytes;
+      uint4* dst;
+      int64_t step;
+      if (S == 1) {
+        const int slot = R / a.G, g = R % a.G;
+        dst = reinterpret_cast<uint4*>(a.out + ((static_cast<int64_t>(b) * a.n_max + slot) * a.hq +
+                                                kvh * a.G + g) * kD) + 8 * x;
+        step = 1;
+      } else {
+        // staged chunk-major over Q's region, stored below with one bulk copy
+        dst = reinterpret_cast<uint4*>(gbase + kOffQ) + (8 * x) * Rp + lrow;
+        step = Rp;
+      }
 #pragma unroll
       for (int c = 0; c < 8; ++c) {
         float v[8];
@@ -665,10 +753,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         w.y = pack_bf16(v[2], v[3]);
         w.z = pack_bf16(v[4], v[5]);
         w.w = pack_bf16(v[6], v[7]);
-        const int cc = 8 * x + c;
-        *reinterpret_cast<uint4*>(srow + ((cc ^ (lrow & 15)) << 4)) = w;
+        dst[c * step] = w;
       }
-      if (x == 0) stg_l[lrow] = have ? mm + __log2f(L) : -CUDART_INF_F;
+      if (S > 1 && x == 0)
+        reinterpret_cast<float*>(gbase + kOffK)[lrow] = have ? mm + __log2f(L) : -CUDART_INF_F;
     }
   }
   tc::fence_smem_async();  // the staging is read by bulk copies
@@ -680,32 +768,26 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc::fence_after_sync();
     tc::tmem_dealloc(tmem, kTmemCols);
   }
-  if (S == 1) {
-    for (int idx = tid; idx < Mv * 16; idx += kThreads) {
-      const int r = idx >> 4, c = idx & 15;
-      const int Rr = row0 + r, slot = Rr / a.G, g = Rr % a.G;
-      const uint4 v = *reinterpret_cast<const uint4*>(stg + r * kRowBytes + ((c ^ (r & 15)) << 4));
-      reinterpret_cast<uint4*>(a.out + ((static_cast<int64_t>(b) * a.n_max + slot) * a.hq +
-                                        kvh * a.G + g) * kD)[c] = v;
-    }
-    return;
-  }
+  if (S == 1) return;
 
   // ------------------------------------- combine the splits (S > 1 only)
-  // Each split stores its staged rows and sums with one bulk copy each
-  // (split-major: [unit][split][row]); rows [o rs, o rs + rs) of a unit are
+  // Each split stores its staged block and sums with one bulk copy each and
+  // waits for their completion before it arrives on its unit's counter.
+  // (Plain stores from registers, each thread fencing before the CTA
+  // barrier and one thread releasing the counter, were measured to let the
+  // owners read incomplete partials.)  Rows [o rs, o rs + rs) of a unit are
   // combined by its split o, every thread loading one 16-byte chunk of one
   // row from every split straight into registers.
   uint32_t* arrive = a.sync + 2 * unit;
   uint32_t* depart = arrive + 1;
   if (tid == 0) {
-    const int64_t pb = static_cast<int64_t>(unit) * S + split;
-    tc::bulk_s2g(a.part_o + pb * kBM * kRowBytes, base + kOffQ, Mv * kRowBytes);
-    tc::bulk_s2g(a.part_l + pb * kBM, base + kOffStgL, ((Mv + 3) & ~3) * 4);
+    tc::bulk_s2g(a.part_o + pb * 16 * kBM * 16, base + kOffQ, 16 * Rp * 16);
+    tc::bulk_s2g(a.part_l + pb * kBM, base + kOffK, Rp * 4);
     tc::bulk_commit();
     tc::bulk_wait_all();
     tc::fence_proxy_async_global();
     tc::red_add_release_gpu(arrive, 1u);
+    TRACE(34);
     bool got = tc::ld_acquire_gpu(arrive) >= static_cast<uint32_t>(S);
     if (!got) {
       const uint64_t t0 = tc::globaltimer();
@@ -725,10 +807,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int nrows = max(0, min(Mv, r_lo + Rs) - r_lo);
   // the acquire above (ordered by the barrier) makes the other splits'
   // stores visible; .cg loads read them from L2
+  if (tid == 0) TRACE(35);
   for (int idx = tid; holder[1] != 0u && idx < nrows * 16; idx += kThreads) {
-    const int r = r_lo + (idx >> 4), c = idx & 15;
+    // consecutive threads take consecutive rows of one chunk (contiguous)
+    const int c = idx / nrows, r = r_lo + idx % nrows;
     const int64_t ub = static_cast<int64_t>(unit) * S;
-    const uint8_t* src = a.part_o + (ub * kBM + r) * kRowBytes + ((c ^ (r & 15)) << 4);
+    const uint4* src = reinterpret_cast<const uint4*>(a.part_o) + ub * 16 * kBM + c * Rp + r;
     const float* lsrc = a.part_l + ub * kBM + r;
     float mx = -CUDART_INF_F, L = 0.f;
     float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
@@ -739,8 +823,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int u = 0; u < kCombineBatch; ++u) {
         const int p = p0 + u;
         ls[u] = p < S ? ld_cg_f32(lsrc + static_cast<int64_t>(p) * kBM) : -CUDART_INF_F;
-        v[u] = p < S ? ld_cg_v4(src + static_cast<int64_t>(p) * kBM * kRowBytes)
-                     : make_uint4(0u, 0u, 0u, 0u);
+        v[u] = p < S ? ld_cg_v4(src + static_cast<int64_t>(p) * 16 * kBM) : make_uint4(0u, 0u, 0u, 0u);
       }
       float bm = mx;
 #pragma unroll
@@ -764,6 +847,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         mx = bm;
       }
     }
+    if (idx == 0) TRACE(36);
     const float inv = L > 0.f ? 1.f / L : 0.f;
     const int Rr = row0 + r;
     const int slot = Rr / a.G, g = Rr % a.G;

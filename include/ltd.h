@@ -438,6 +438,47 @@ ltd_status ltd_kv_compact(const ltd_kv_cache* kv, int32_t batch, const int32_t* 
                           int32_t path_stride, const int32_t* d_accept_len,
                           const int32_t* d_ctx, ltd_stream_t stream);
 
+/* The target's LM head over the verified tokens with the row statistics
+ * acceptance reads (section 3.2, "Draft Tree Verification": one target
+ * forward over the verified tokens; its last layer maps each hidden state
+ * to vocabulary logits): logits[r][v] = sum_k hidden[r][k] weight[v][k]
+ * (bf16 inputs, fp32 accumulation on the tensor cores) and per row the max,
+ * the log-sum-exp and the argmax (ties to the lower token id), without the
+ * logits making a round trip through memory.
+ *  d_hidden        [rows][hidden] bf16, row-major, 16-byte aligned
+ *  d_weight        [vocab][hidden] bf16, row-major, 16-byte aligned
+ *  rows            1 .. LTD_LM_HEAD_MAX_ROWS (the verified tokens of a batch)
+ *  hidden          a multiple of 64
+ *  d_logits        [rows][vocab] bf16 out, or NULL to skip them (the
+ *                  stochastic rules read full rows; greedy acceptance needs
+ *                  only the argmax)
+ *  d_row_max, d_row_lse  [rows] fp32 out; d_row_argmax [rows] int32 out
+ *  d_workspace     ltd_lm_head_workspace_bytes() bytes of caller memory,
+ *                  16-byte aligned; no initial value needed
+ * Bad pointers are LTD_ERR_INVALID_ARG, bad sizes LTD_ERR_SHAPE
+ * (ltd_lm_head_workspace_bytes returns 0 for them). */
+#define LTD_LM_HEAD_MAX_ROWS 256
+size_t ltd_lm_head_workspace_bytes(int32_t rows, int64_t vocab, int32_t hidden);
+ltd_status ltd_lm_head_row_stats(const void* d_hidden, const void* d_weight, int32_t rows,
+                                 int64_t vocab, int32_t hidden, void* d_logits, float* d_row_max,
+                                 float* d_row_lse, int32_t* d_row_argmax, void* d_workspace,
+                                 size_t workspace_bytes, ltd_stream_t stream);
+
+/* Test hook of the bounded waits (section 3.2 has no counterpart; it exists
+ * so the failure path can be exercised without a GPU fault).  With the keys
+ * of each (sequence, KV head, tile) split over several CTAs, every split of
+ * the tensor-core attention kernel waits on its unit's arrival counter for
+ * the others; this sets, for the calls that follow on any thread, the
+ * longest that wait lasts (limit_ns; 0 restores the default of one second)
+ * and a number of arrivals it waits for beyond the unit's splits
+ * (extra_arrivals; 0 restores normal operation).  Nothing ever supplies the
+ * extra arrivals, so with extra_arrivals > 0 every split gives up after
+ * limit_ns, raises LTD_DEVERR_TIMEOUT (ltd_check returns LTD_ERR_TIMEOUT),
+ * leaves its rows of the output unwritten and still departs, so the
+ * counters are back at zero and the workspace can be used again.
+ * extra_arrivals above 1024 returns LTD_ERR_INVALID_ARG. */
+ltd_status ltd_debug_attention_wait(uint64_t limit_ns, uint32_t extra_arrivals);
+
 /* Diagnostic of the tensor-core building blocks the attention kernel uses
  * (TMA with 128-byte swizzle, tcgen05.mma from shared-memory descriptors
  * into tensor memory, tcgen05.ld): one 128x128x128 bf16 GEMM with fp32

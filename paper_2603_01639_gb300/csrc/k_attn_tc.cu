@@ -125,6 +125,10 @@ struct TcArgs {
   // K and V through one tensor map when both caches fit one 4-D map (the
   // fourth coordinate picks the cache), else one map each
   int32_t kv_one, kv_wk, kv_wv;
+  // the split counter's wait: its limit, and arrivals awaited beyond the
+  // unit's splits (a test hook; 0 in normal calls, so the wait completes)
+  uint64_t spin_limit_ns;
+  uint32_t extra_arrivals;
 };
 
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
@@ -788,13 +792,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc::fence_proxy_async_global();
     tc::red_add_release_gpu(arrive, 1u);
     TRACE(34);
-    bool got = tc::ld_acquire_gpu(arrive) >= static_cast<uint32_t>(S);
+    const uint32_t quorum = static_cast<uint32_t>(S) + a.extra_arrivals;
+    bool got = tc::ld_acquire_gpu(arrive) >= quorum;
     if (!got) {
       const uint64_t t0 = tc::globaltimer();
       while (!got) {
         __nanosleep(32);
-        got = tc::ld_acquire_gpu(arrive) >= static_cast<uint32_t>(S);
-        if (!got && tc::globaltimer() - t0 > tc::kWaitLimitNs) break;
+        got = tc::ld_acquire_gpu(arrive) >= quorum;
+        if (!got && tc::globaltimer() - t0 > a.spin_limit_ns) break;
       }
     }
     if (!got) flag_error(a.err, LTD_DEVERR_TIMEOUT);
@@ -875,26 +880,10 @@ struct Plan {
   int n_tiles, splits, units, lpt, nch, rs;
 };
 
-// Streaming multiprocessors of the current device (152 if it cannot be asked).
-int device_sms() {
-  static std::mutex mu;
-  static int known[128] = {};
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 128) {
-    (void)cudaGetLastError();
-    return 152;
-  }
-  std::lock_guard<std::mutex> lock(mu);
-  if (known[dev] == 0) {
-    int n = 0;
-    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1) {
-      (void)cudaGetLastError();
-      n = 152;
-    }
-    known[dev] = n;
-  }
-  return known[dev];
-}
+
+// The split counter's wait settings for later launches (test hook).
+std::mutex g_hook_mu;
+AttnWaitHook g_hook{};
 
 // Units = (sequence, KV head, tile).  With fewer units than SMs each unit's
 // keys are cut into the fewest splits that give the shortest longest split,
@@ -906,7 +895,7 @@ Plan plan(int32_t batch, int32_t hq, int32_t hkv, int32_t n_max, int32_t max_ctx
   const int64_t units = static_cast<int64_t>(batch) * hkv * p.n_tiles;
   p.units = static_cast<int>(units);
   const int nch = (max_ctx + n_max + kBN - 1) / kBN;
-  const int sms = device_sms();
+  const int sms = device_sm_count();
   p.splits = 1;
   if (units < sms) {
     int smax = static_cast<int>(sms / units);
@@ -962,6 +951,27 @@ EncodeFn encode_fn() {
 
 }  // namespace
 
+// Streaming multiprocessors of the current device (152 if it cannot be asked).
+int device_sm_count() {
+  static std::mutex mu;
+  static int known[128] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 128) {
+    (void)cudaGetLastError();
+    return 152;
+  }
+  std::lock_guard<std::mutex> lock(mu);
+  if (known[dev] == 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1) {
+      (void)cudaGetLastError();
+      n = 152;
+    }
+    known[dev] = n;
+  }
+  return known[dev];
+}
+
 bool encode_tmap_bf16_3d(CUtensorMap* map, const void* base, uint64_t d0, uint64_t d1, uint64_t d2,
                          uint64_t stride1, uint64_t stride2, uint32_t b0, uint32_t b1, uint32_t b2) {
   EncodeFn fn = encode_fn();
@@ -990,6 +1000,15 @@ bool encode_tmap_bf16_4d(CUtensorMap* map, const void* base, uint64_t d0, uint64
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 }  // namespace
+
+void set_attn_wait_hook(const AttnWaitHook& h) {
+  std::lock_guard<std::mutex> lock(g_hook_mu);
+  g_hook = h;
+}
+AttnWaitHook attn_wait_hook() {
+  std::lock_guard<std::mutex> lock(g_hook_mu);
+  return g_hook;
+}
 
 bool attn_tc_supported(const AttnParams& p, ltd_dtype dtype) {
   if (dtype != LTD_BF16 || p.d != kD || p.hkv < 1 || p.hq % p.hkv != 0) return false;
@@ -1033,6 +1052,11 @@ cudaError_t launch_attn_tc(const AttnParams& p, cudaStream_t s) {
   a.part_l = pl.splits > 1 ? reinterpret_cast<float*>(ws + wl.part_l) : nullptr;
   a.sync = pl.splits > 1 ? reinterpret_cast<uint32_t*>(ws + wl.sync) : nullptr;
   a.err = p.err;
+  {
+    const AttnWaitHook h = attn_wait_hook();
+    a.spin_limit_ns = h.limit_ns != 0 ? h.limit_ns : tc::kWaitLimitNs;
+    a.extra_arrivals = h.extra_arrivals;
+  }
   // the hint only while one layer's keys and values fit well inside L2
   const uint64_t layer_kv = static_cast<uint64_t>(p.batch) * p.hkv *
                             (static_cast<uint64_t>(p.max_ctx) + p.n_max) * kRowBytes * 2;

@@ -405,6 +405,48 @@ int32_t ltd_attention_kernel(ltd_dtype dtype, int32_t batch, int32_t hq, int32_t
   return tc ? 1 : 0;
 }
 
+size_t ltd_lm_head_workspace_bytes(int32_t rows, int64_t vocab, int32_t hidden) {
+  if (rows < 1 || rows > LTD_LM_HEAD_MAX_ROWS || vocab < 1 || vocab > 0x7FFFFFFF || hidden < 64 ||
+      hidden % 64 != 0)
+    return 0;
+  return lm_head_workspace(rows, vocab);
+}
+
+ltd_status ltd_lm_head_row_stats(const void* d_hidden, const void* d_weight, int32_t rows,
+                                 int64_t vocab, int32_t hidden, void* d_logits, float* d_row_max,
+                                 float* d_row_lse, int32_t* d_row_argmax, void* d_workspace,
+                                 size_t workspace_bytes, ltd_stream_t stream) {
+  const ApiRange nvtx_range("ltd_lm_head_row_stats");
+  if (!d_hidden || !d_weight || !d_row_max || !d_row_lse || !d_row_argmax || !d_workspace)
+    return LTD_ERR_INVALID_ARG;
+  const size_t need = ltd_lm_head_workspace_bytes(rows, vocab, hidden);
+  if (need == 0 || workspace_bytes < need) return LTD_ERR_SHAPE;
+  if (!aligned16(d_hidden) || !aligned16(d_weight) || !aligned16(d_workspace)) return LTD_ERR_SHAPE;
+  if (d_logits != nullptr && ((reinterpret_cast<uintptr_t>(d_logits) & 1u) != 0)) return LTD_ERR_SHAPE;
+  uint32_t* err = device_error_word();
+  if (err == nullptr) return LTD_ERR_CUDA;
+  LmHeadParams p{};
+  p.hidden_states = d_hidden;
+  p.weight = d_weight;
+  p.rows = rows;
+  p.hidden = hidden;
+  p.vocab = vocab;
+  p.logits = d_logits;
+  p.row_max = d_row_max;
+  p.row_lse = d_row_lse;
+  p.row_argmax = d_row_argmax;
+  p.ws = d_workspace;
+  p.ws_bytes = workspace_bytes;
+  p.err = err;
+  return from_cuda(launch_lm_head(p, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+ltd_status ltd_debug_attention_wait(uint64_t limit_ns, uint32_t extra_arrivals) {
+  if (extra_arrivals > 1024) return LTD_ERR_INVALID_ARG;
+  set_attn_wait_hook(AttnWaitHook{limit_ns, extra_arrivals});
+  return LTD_OK;
+}
+
 ltd_status ltd_selftest_umma(int32_t mode, const void* d_a, const void* d_b, float* d_c,
                              ltd_stream_t stream) {
   if ((mode != 0 && mode != 1) || !d_a || !d_b || !d_c) return LTD_ERR_INVALID_ARG;

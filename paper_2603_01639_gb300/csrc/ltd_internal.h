@@ -144,6 +144,16 @@ struct AttnParams {
 size_t attn_simt_workspace(const AttnParams& p);
 cudaError_t launch_attn_simt(const AttnParams& p, ltd_dtype dtype, cudaStream_t s);
 bool attn_tc_supported(const AttnParams& p, ltd_dtype dtype);
+// Streaming multiprocessors of the current device (152 if it cannot be asked).
+int device_sm_count();
+// Test hook of the tensor-core kernel's split-counter wait (k_attn_tc.cu):
+// its limit (0 = the default 1 s) and arrivals awaited beyond the splits.
+struct AttnWaitHook {
+  uint64_t limit_ns;
+  uint32_t extra_arrivals;
+};
+void set_attn_wait_hook(const AttnWaitHook& h);
+AttnWaitHook attn_wait_hook();
 size_t attn_tc_workspace(int32_t batch, int32_t hq, int32_t hkv, int32_t d, int32_t n_max,
                          int32_t max_ctx);
 cudaError_t launch_attn_tc(const AttnParams& p, cudaStream_t s);
@@ -151,6 +161,23 @@ int32_t attn_tc_launches(int32_t batch, int32_t hq, int32_t hkv, int32_t n_max,
                          int32_t max_ctx);
 cudaError_t launch_umma_selftest(int mode, const void* a, const void* b, float* c, uint32_t* err,
                                  cudaStream_t s);
+
+// ------------------------------------------------------------- LM head
+struct LmHeadParams {
+  const void* hidden_states;  // [rows][hidden] bf16
+  const void* weight;         // [vocab][hidden] bf16
+  int32_t rows, hidden;
+  int64_t vocab;
+  void* logits;               // [rows][vocab] bf16 or null
+  float* row_max;
+  float* row_lse;
+  int32_t* row_argmax;
+  void* ws;
+  size_t ws_bytes;
+  uint32_t* err;
+};
+size_t lm_head_workspace(int32_t rows, int64_t vocab);
+cudaError_t launch_lm_head(const LmHeadParams& p, cudaStream_t s);
 
 // ------------------------------------------------------------- acceptance
 constexpr int64_t kAcceptTargetCtas = 608;

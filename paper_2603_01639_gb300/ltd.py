@@ -32,6 +32,7 @@ EXPORTS = [
     "ltd_attention_kernel", "ltd_selftest_umma", "ltd_accept_noalloc", "ltd_tree_attention_next",
     "ltd_depth_observation", "ltd_size_observation", "ltd_depth_policy", "ltd_size_policy",
     "ltd_mlp_packed_bytes", "ltd_mlp_pack", "ltd_kv_append", "ltd_accept_tempered",
+    "ltd_debug_attention_wait", "ltd_lm_head_workspace_bytes", "ltd_lm_head_row_stats",
 ]
 LTD_POLICY_PAD = -100.0
 LTD_MLP_MAX_LAYERS, LTD_MLP_MAX_WIDTH = 4, 2048
@@ -107,6 +108,10 @@ def lib():
                 "ltd_attention_kernel": (i32, [C.c_int, i32, i32, i32, i32, i32, i32,
                                                C.POINTER(i32)]),
                 "ltd_selftest_umma": (C.c_int, [i32, vp, vp, vp, vp]),
+                "ltd_debug_attention_wait": (C.c_int, [u64, C.c_uint32]),
+                "ltd_lm_head_workspace_bytes": (sz, [i32, i64, i32]),
+                "ltd_lm_head_row_stats": (C.c_int, [vp, vp, i32, i64, i32, vp, vp, vp, vp, vp, sz,
+                                                    vp]),
                 "ltd_accept_noalloc": (C.c_int, [tp, vp, vp, C.c_int, i64, i64, vp, vp, i32, vp, u64,
                                                  u64, vp, vp, vp, vp, vp, C.POINTER(ltd_kv_cache),
                                                  vp]),
@@ -494,6 +499,35 @@ def ltd_kv_append(kv: KVCache, new_k, new_v, ctx, n_verify, stream=None):
     _need(n_verify, "n_verify", torch.int32)
     _ok(lib().ltd_kv_append(C.byref(kv.s), new_k.shape[1], new_k.shape[3], _ptr(new_k), _ptr(new_v),
                             _ptr(ctx), _ptr(n_verify), _stream(stream)), "ltd_kv_append")
+
+
+def ltd_lm_head_row_stats(hidden, weight, logits=False, workspace=None, stream=None):
+    """hidden [rows][H] bf16, weight [vocab][H] bf16.  Returns dict(row_max,
+    row_lse [rows] fp32, row_argmax [rows] int32, logits [rows][vocab] bf16
+    when ``logits`` is true)."""
+    _need(hidden, "hidden", torch.bfloat16)
+    _need(weight, "weight", torch.bfloat16)
+    rows, H = hidden.shape
+    vocab = weight.shape[0]
+    if weight.shape[1] != H:
+        raise LtdError("hidden and weight disagree on the hidden size")
+    dev = hidden.device
+    if workspace is None:
+        n = lib().ltd_lm_head_workspace_bytes(rows, vocab, H)
+        if n == 0:
+            raise LtdError("ltd_lm_head_workspace_bytes: bad sizes")
+        workspace = torch.empty(n, dtype=torch.uint8, device=dev)
+    out = {"row_max": torch.empty(rows, dtype=torch.float32, device=dev),
+           "row_lse": torch.empty(rows, dtype=torch.float32, device=dev),
+           "row_argmax": torch.empty(rows, dtype=torch.int32, device=dev)}
+    lg = torch.empty(rows, vocab, dtype=torch.bfloat16, device=dev) if logits else None
+    _ok(lib().ltd_lm_head_row_stats(_ptr(hidden), _ptr(weight), rows, vocab, H,
+                                    _ptr(lg) if lg is not None else None, _ptr(out["row_max"]),
+                                    _ptr(out["row_lse"]), _ptr(out["row_argmax"]), _ptr(workspace),
+                                    workspace.numel(), _stream(stream)), "ltd_lm_head_row_stats")
+    if lg is not None:
+        out["logits"] = lg
+    return out
 
 
 def ltd_check(stream=None, raise_on_error=True) -> int:

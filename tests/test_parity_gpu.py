@@ -696,6 +696,40 @@ def test_attention_workspace_reuse():
         _attention_case("8b", seed, workspace=ws)
 
 
+def test_attention_split_wait_runs_out_and_recovers():
+    """A bounded wait that runs out, without a GPU fault: the test hook makes
+    every split of the 8B-class layer wait on its unit's counter for one
+    arrival more than the unit has, with a 2 ms limit.  Every split gives
+    up, ltd_check returns LTD_ERR_TIMEOUT with the TIMEOUT bit, and no
+    output row is written; the splits still departed, so the counters are
+    back at zero and, with the hook reset, the same workspace gives the
+    oracle's result on the next calls."""
+    import ctypes as C
+    cfg = wl.config("8b")
+    ws = ltd.attention_workspace(cfg.batch, cfg.hq, cfg.hkv, cfg.head_dim, cfg.max_n,
+                                 cfg.max_ctx, torch.bfloat16)
+    ci = wl.draw_cycle(cfg, 13, draft_rows=False)
+    q, k, v = wl.draw_attention(cfg, 13, ci.ctx, ci.n_verify)
+    W32 = (cfg.max_n + 31) // 32
+    mw = torch.zeros(cfg.batch, cfg.max_n, W32, dtype=torch.int32, device="cuda")
+    mw[..., 0] = 1
+    L = ltd.lib()
+    assert L.ltd_debug_attention_wait(2_000_000, 1) == 0
+    try:
+        out = ltd.ltd_tree_attention(H.dev(q, cfg.dtype), H.dev(k, cfg.dtype), H.dev(v, cfg.dtype),
+                                     H.i32(ci.ctx), cfg.max_ctx, H.i32(ci.n_verify), mw,
+                                     workspace=ws)
+        bits = C.c_uint32(0)
+        st = L.ltd_check(None, C.byref(bits))
+    finally:
+        assert L.ltd_debug_attention_wait(0, 0) == 0
+    assert L.ltd_status_string(st).decode() == "LTD_ERR_TIMEOUT"
+    assert bits.value == 0x10
+    assert not out.float().abs().sum().item()
+    for seed in (14, 15):
+        _attention_case("8b", seed, workspace=ws)
+
+
 def test_attention_all_ones_mask_equals_unmasked():
     cfg = wl.config("8b", ctx_range=(300, 300), n_choices=(40,))
     rng = np.random.default_rng(3)

@@ -46,6 +46,11 @@ def _args():
     ap.add_argument("--no-policy", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-sample-s", type=float, default=15.0)
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the other workloads' summaries (configs) after the headline")
+    ap.add_argument("--min-timed-ms", type=float, default=250.0,
+                    help="each step replays the cycle graph enough times that the K timed steps "
+                         "last at least this long (so the clock sampler sees the load)")
     ap.add_argument("--no-next-hint", action="store_true",
                     help="run the cycle without the next-layer L2 hint (for profiling one layer's "
                          "own traffic)")
@@ -57,6 +62,32 @@ def _dist():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     return rank, world, local
+
+
+def config_obj(cfg, layers):
+    """The `config` object of the JSON line, the same in both arms."""
+    kv = 2 * layers * cfg.batch * cfg.hkv * cfg.s_cap * cfg.head_dim * (2 if cfg.dtype == "bf16" else 4)
+    return {"workload": workload_desc(cfg, layers), "batch_per_gpu": cfg.batch, "layers": layers,
+            "l2": f"inputs larger than L2: {kv / 1e6:.0f} MB of KV cache streamed per cycle between "
+                  f"reuses of any buffer"}
+
+
+def load_peaks():
+    """(HBM GB/s, dense bf16 TFLOP/s sustained, source): the measured copy and
+    GEMM peaks of this machine, else the recipe's fallback figures."""
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), float(d.get("bf16_tflops_sustained") or d["bf16_tflops"]), \
+            "measured"
+    except (OSError, ValueError, KeyError):
+        return 6800.0, 1700.0, "fallback"
+
+
+# the resource that binds tree attention at each workload's shape (flops per
+# algorithmic byte against the measured ridge of ~280): HBM at 8B (227) and
+# 13B (16-92), the tensor pipe at 32B (375) and 70B (461)
+BINDING = {"tiny": "hbm", "8b": "hbm", "13b": "hbm", "32b": "tensor", "70b": "tensor"}
 
 
 def workload_desc(cfg, layers):
@@ -190,17 +221,6 @@ class Cycle:
         self.cfg, self.layers, self.device = cfg, layers, device
         tdt = torch.bfloat16 if cfg.dtype == wl.BF16 else torch.float32
         self.tdt = tdt
-        ci = wl.draw_cycle(cfg, seed)
-        self.ci = ci
-        i32 = lambda x: torch.as_tensor(np.asarray(x, np.int32), device=device)  # noqa: E731
-        self.root, self.depth = i32(ci.root), ci.depth
-        self.n_verify, self.ctx, self.mode = i32(ci.n_verify), i32(ci.ctx), i32(ci.mode)
-        self.draft = torch.from_numpy(ci.draft_rows).to(device).to(tdt)
-        self.max_depth = int(ci.depth.max())
-        self.actives = {}
-        for level in range(1, self.max_depth + 1):
-            m = (ci.depth >= level)
-            self.actives[level] = None if m.all() else i32(m.astype(np.int32))
         B, d = cfg.batch, cfg.head_dim
         g = torch.Generator(device=device).manual_seed(seed)
         self.q = [torch.randn(B, cfg.max_n, cfg.hq, d, generator=g, device=device).to(tdt)
@@ -223,19 +243,34 @@ class Cycle:
                     "accept_len": torch.empty(B, dtype=torch.int32, device=device),
                     "bonus": torch.empty(B, dtype=torch.int32, device=device),
                     "new_ctx": torch.empty(B, dtype=torch.int32, device=device)}
-        # target logits: random, with agreement planted on the tree this
-        # draft produces (run the draft once to learn it)
+        self.load(wl.draw_cycle(cfg, seed), seed)
+
+    def load(self, ci, seed):
+        """The per-cycle inputs of one drawn cycle (depths, verify sizes, contexts,
+        modes, draft rows) and its target logits, planted on the tree this
+        draft produces (the draft runs once to learn it)."""
+        torch, wl, cfg, device = self.torch, self.wl, self.cfg, self.device
+        self.ci = ci
+        i32 = lambda x: torch.as_tensor(np.asarray(x, np.int32), device=device)  # noqa: E731
+        self.root, self.depth = i32(ci.root), ci.depth
+        self.n_verify, self.ctx, self.mode = i32(ci.n_verify), i32(ci.ctx), i32(ci.mode)
+        self.draft = torch.from_numpy(ci.draft_rows).to(device).to(self.tdt)
+        self.max_depth = int(ci.depth.max())
+        self.actives = {}
+        for level in range(1, self.max_depth + 1):
+            m = (ci.depth >= level)
+            self.actives[level] = None if m.all() else i32(m.astype(np.int32))
         self.draft_phase()
         torch.cuda.synchronize(device)
         view = {k: v.cpu().numpy() for k, v in self.tree.view().items()}
         ids = self.sel[0].cpu().numpy()
         target = wl.draw_target_rows(cfg, ci)
         rng = np.random.default_rng(seed + 99)
-        for b in range(B):
+        for b in range(cfg.batch):
             N = int(ci.n_verify[b])
             wl.plant_agreement(cfg, target[b], ids[b, :N], view["parent"][b], view["token"][b],
                                view["depth"][b], rng, greedy=(ci.mode[b] == 0))
-        self.target = torch.from_numpy(target).to(device).to(tdt)
+        self.target = torch.from_numpy(target).to(device).to(self.tdt)
 
     # phases ---------------------------------------------------------------
     def draft_phase(self):
@@ -399,6 +434,138 @@ def cpu_baseline(cfg, layers, seed, budget_s):
                       f"attention over {layers} layers reusing one layer's KV); median"}
 
 
+def time_replays(torch, g, reps, device):
+    """Mean device time of one replay of graph `g` over `reps` replays (CUDA
+    events on the launching stream), in milliseconds."""
+    stream = torch.cuda.current_stream(device)
+    g.replay()
+    torch.cuda.synchronize(device)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(reps):
+        g.replay()
+    e1.record(stream)
+    torch.cuda.synchronize(device)
+    return e0.elapsed_time(e1) / reps
+
+
+def attention_roofline(cyc, launch_ms, bound):
+    """Roofline of one tree-attention launch against its binding resource."""
+    hbm, tc, src = load_peaks()
+    byts, flops = cyc.attention_algorithmic()
+    gbs = byts / (launch_ms * 1e-3) / 1e9
+    tfs = flops / (launch_ms * 1e-3) / 1e12
+    if bound == "tensor":
+        achieved, peak, unit = tfs, tc, "TFLOP/s"
+    else:
+        achieved, peak, unit = gbs, hbm, "GB/s"
+    return {"bound": bound, "achieved": round(achieved, 1), "peak": peak, "unit": unit,
+            "frac": round(achieved / peak, 4), "peak_source": src + " (hbm_gbs; bf16_tflops_sustained)",
+            "launch_us": round(launch_ms * 1e3, 3), "algorithmic_bytes_per_launch": byts,
+            "flops_per_launch": flops, "gbs": round(gbs, 1), "tflops": round(tfs, 1),
+            "hbm_frac": round(gbs / hbm, 4)}
+
+
+def summarize_config(name, args, device, seed, reps):
+    """Full-cycle latency, phases, the attention roofline against the shape's
+    binding resource and e2e for one workload (the 8B-class one is the
+    headline line itself)."""
+    import torch
+    from paper_2603_01639_gb300 import workload as wl
+    cfg = wl.config(name)
+    layers = N_LAYERS[name]
+    cyc = Cycle(cfg, layers, seed, device)
+
+    def full():
+        cyc.draft_phase()
+        cyc.verify_phase()
+        cyc.accept_phase()
+
+    for _ in range(3):
+        full()
+    torch.cuda.synchronize(device)
+    cyc.ltd.ltd_check()
+    g_cycle, g_draft = _graph(torch, full), _graph(torch, cyc.draft_phase)
+    g_verify, g_plain = _graph(torch, cyc.verify_phase), _graph(torch, cyc.verify_phase_plain)
+    g_accept = _graph(torch, cyc.accept_phase)
+    cycle_ms = time_replays(torch, g_cycle, reps, device)
+    phases = {"draft_select": time_replays(torch, g_draft, reps, device),
+              "attention_all_layers": time_replays(torch, g_verify, reps, device),
+              "accept_compact": time_replays(torch, g_accept, reps, device)}
+    plain_ms = time_replays(torch, g_plain, reps, device)
+    cyc.ltd.ltd_check()
+    g_accept.replay()
+    torch.cuda.synchronize(device)
+    acc_len = cyc.acc["accept_len"].cpu().numpy()
+    res = {"workload": workload_desc(cfg, layers), "cycle_us": round(cycle_ms * 1e3, 2),
+           "cycle_us_per_sequence": round(cycle_ms * 1e3 / cfg.batch, 2),
+           "phases_us": {k: round(v * 1e3, 2) for k, v in phases.items()},
+           "attention": attention_roofline(cyc, plain_ms / layers, BINDING[name]),
+           "attention_launch_us_in_cycle": round(phases["attention_all_layers"] * 1e3 / layers, 3),
+           "tokens_per_cycle": int((acc_len + 1).sum()),
+           "gpu_launches_per_cycle": cyc.launches_per_step(), "reps": reps}
+    if name == "32b":
+        # the compaction of the accepted path in every layer, timed alone
+        path, alen = cyc.acc["path"], cyc.acc["accept_len"]
+        g_comp = _graph(torch, lambda: cyc.ltd.ltd_kv_compact(cyc.kv, path, alen, cyc.ctx))
+        comp_ms = time_replays(torch, g_comp, reps, device)
+        a = int(acc_len.max())
+        moved = 2 * (a + 1) * cfg.hkv * cfg.head_dim * 2 * layers * cfg.batch
+        res["compaction"] = {"us": round(comp_ms * 1e3, 2), "accepted": a,
+                             "bytes_read_and_written_each": moved,
+                             "how": "ltd_kv_compact of the cycle's accepted path in all layers, one "
+                                    "launch, CUDA graph replays"}
+    if not args.no_e2e:
+        res["e2e"] = run_e2e(cyc, args, device)
+    del cyc, g_cycle, g_draft, g_verify, g_plain, g_accept
+    torch.cuda.empty_cache()
+    return res
+
+
+def sweep_13b(args, device, seed, cycles, reps):
+    """The 13B-class workload over `cycles` seeded cycles, each with its own
+    draft depth in 3..8 and verify size in {16, 32, 48, 64, 96} (the size and
+    depth choices a policy would make), on one set of caches."""
+    import torch
+    from paper_2603_01639_gb300 import workload as wl
+    cfg = wl.config("13b")
+    layers = N_LAYERS["13b"]
+    cyc = Cycle(cfg, layers, seed, device)
+    per = []
+    for c in range(cycles):
+        s = seed + 1 + c
+        cyc.load(wl.draw_cycle(cfg, s), s)
+
+        def full():
+            cyc.draft_phase()
+            cyc.verify_phase()
+            cyc.accept_phase(cycle_no=s)
+
+        full()
+        torch.cuda.synchronize(device)
+        g = _graph(torch, full)
+        gv = _graph(torch, cyc.verify_phase_plain)
+        ms = time_replays(torch, g, reps, device)
+        vms = time_replays(torch, gv, reps, device)
+        g.replay()
+        torch.cuda.synchronize(device)
+        per.append({"depth": int(cyc.ci.depth[0]), "n_verify": int(cyc.ci.n_verify[0]),
+                    "cycle_us": round(ms * 1e3, 2),
+                    "attention_launch_us": round(vms * 1e3 / layers, 3),
+                    "accepted": int(cyc.acc["accept_len"][0].item()),
+                    "attention_hbm_frac": attention_roofline(cyc, vms / layers, "hbm")["frac"]})
+        del g, gv
+    cyc.ltd.ltd_check()
+    del cyc
+    torch.cuda.empty_cache()
+    cyc_us = [p["cycle_us"] for p in per]
+    return {"cycles": cycles, "cycle_us_mean": round(statistics.mean(cyc_us), 2),
+            "cycle_us_min": min(cyc_us), "cycle_us_max": max(cyc_us),
+            "attention_hbm_frac_mean": round(statistics.mean(p["attention_hbm_frac"] for p in per), 4),
+            "tokens_per_cycle_mean": round(statistics.mean(p["accepted"] + 1 for p in per), 3),
+            "per_cycle": per}
+
+
 # ------------------------------------------------------------------ main
 def run_reference(args):
     rank, world, _ = _dist()
@@ -418,7 +585,7 @@ def run_reference(args):
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": round(v / 1e3, 3), "higher_is_better": False, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": workload_desc(cfg, layers)},
+            "config": config_obj(cfg, layers),
             "cpu_baseline": {"value": round(v, 1), "unit": "us", "cores": blas_threads(),
                              "kind": "oracle",
                              "sample": f"each step one full oracle cycle (fp64 numpy); "
@@ -468,6 +635,14 @@ def run_ours(args):
     torch.cuda.synchronize(device)
 
     K = args.steps
+    # a step is R replays of the cycle graph, R chosen so that the K timed
+    # steps last at least --min-timed-ms (the same R on every rank)
+    one_ms = time_replays(torch, g_cycle, 5, device)
+    R = max(1, int(math.ceil(args.min_timed_ms / max(K * one_ms, 1e-3))))
+    if world > 1:
+        t = torch.tensor([R], dtype=torch.int64, device=device)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        R = int(t.item())
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(K)]
     if world > 1:
         torch.distributed.barrier()
@@ -477,7 +652,8 @@ def run_ours(args):
     c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     c0.record(stream)
     for i in range(K):
-        g_cycle.replay()
+        for _ in range(R):
+            g_cycle.replay()
     c1.record(stream)
     torch.cuda.synchronize(device)
     clk = clocks.stop()
@@ -493,7 +669,7 @@ def run_ours(args):
         ev[i][3].record(stream)
     torch.cuda.synchronize(device)
     ltd.ltd_check()
-    total_ms = c0.elapsed_time(c1)
+    total_ms = c0.elapsed_time(c1) / R  # per cycle-graph replay, summed over the K steps
     draft_ms = statistics.mean(ev[i][0].elapsed_time(ev[i][1]) for i in range(K))
     verify_ms = statistics.mean(ev[i][1].elapsed_time(ev[i][2]) for i in range(K))
     accept_ms = statistics.mean(ev[i][2].elapsed_time(ev[i][3]) for i in range(K))
@@ -578,26 +754,37 @@ def run_ours(args):
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(cfg, layers, args.seed, args.cpu_sample_s)
 
+    # the other workloads: full-cycle latency, phases and the attention
+    # roofline against each shape's binding resource (one GPU only)
+    configs = None
+    if world == 1 and not args.no_configs:
+        reps = max(10, min(K, 50))
+        configs = {}
+        for name in N_LAYERS:
+            if name == args.config:
+                continue
+            configs[name] = summarize_config(name, args, device, args.seed, reps)
+            if name == "13b":
+                configs[name]["sweep"] = sweep_13b(args, device, args.seed + 500, 32, reps)
+
     if rank == 0:
-        kv_bytes = sum(t.numel() * t.element_size() for t in cyc.k + cyc.v)
         line = {
             "metric": METRIC, "value": round(value_us, 2), "unit": "us", "n_gpus": world,
-            "steps": K, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4),
+            "steps": K, "warmup": args.warmup, "ms_per_step": round(ms_per_step * R, 4),
+            "cycles_per_step": R,
             "higher_is_better": False, "scaling": "weak", "vs_baseline": None,
             "dtype": cfg.dtype, "data": "synthetic",
-            "config": {"workload": workload_desc(cfg, layers), "batch_per_gpu": cfg.batch,
-                       "layers": layers,
-                       "l2": f"inputs larger than L2: {kv_bytes / 1e6:.0f} MB of KV cache streamed "
-                             f"per step between reuses of any buffer",
-                       "timing": "CUDA events around replays of one CUDA graph of the whole "
-                                 "cycle; value = job time / cycles of all ranks; phases_us from "
-                                 "per-phase graphs timed after it"},
+            "config": config_obj(cfg, layers),
+            "timing": "CUDA events around K steps of R replays each of one CUDA graph of the "
+                      "whole cycle; value = job time / cycles of all ranks; phases_us from "
+                      "per-phase graphs timed after it",
             "phases_us": {"draft_select": round(draft_ms * 1e3, 2),
                           "attention_all_layers": round(verify_ms * 1e3, 2),
                           "accept_compact": round(accept_ms * 1e3, 2)},
             "accept_rules_us": rules,
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "policy": pol, "reward": reward,
-            "gpu_launches": cyc.launches_per_step() * K, "clocks": clk,
+            "gpu_launches": cyc.launches_per_step() * K * R, "clocks": clk,
+            "configs": configs,
         }
         print(json.dumps(line), flush=True)
     if world > 1:

@@ -466,6 +466,50 @@ def attention_roofline(cyc, launch_ms, bound):
             "hbm_frac": round(gbs / hbm, 4)}
 
 
+# the target models' hidden sizes (public model configs of the paper's
+# targets: Llama-3.1-8B, Vicuna-13B, Qwen3-32B, a 70B-class model), for the LM
+# head over the verified tokens
+HIDDEN = {"8b": 4096, "13b": 5120, "32b": 5120, "70b": 8192}
+
+
+def time_lm_head(cfg, name, device, reps):
+    """ltd_lm_head_row_stats over the verified tokens of one cycle (batch x
+    n_max rows, up to the 256 one call takes) at the target's hidden size,
+    statistics only, seeded random bf16 hidden states and weights; the
+    weight (more than L2) streams from HBM at every replay."""
+    import torch
+    from paper_2603_01639_gb300 import ltd
+    rows = cfg.batch * cfg.max_n
+    if name not in HIDDEN or cfg.dtype != "bf16" or rows > 256:
+        return None
+    H = HIDDEN[name]
+    g = torch.Generator(device=device).manual_seed(7)
+    hid = torch.randn(rows, H, generator=g, device=device).to(torch.bfloat16)
+    w = (torch.randn(cfg.vocab, H, generator=g, device=device) / math.sqrt(H)).to(torch.bfloat16)
+    ws = torch.empty(ltd.lib().ltd_lm_head_workspace_bytes(rows, cfg.vocab, H), dtype=torch.uint8,
+                     device=device)
+    call = lambda: ltd.ltd_lm_head_row_stats(hid, w, workspace=ws)  # noqa: E731
+    call()
+    torch.cuda.synchronize(device)
+    g_lm = _graph(torch, call)
+    ms = time_replays(torch, g_lm, reps, device)
+    ltd.ltd_check()
+    hbm, tc, src = load_peaks()
+    byts = cfg.vocab * H * 2 + rows * H * 2 + rows * 12
+    gbs = byts / (ms * 1e-3) / 1e9
+    res = {"rows": rows, "vocab": cfg.vocab, "hidden": H, "us": round(ms * 1e3, 2),
+           "roofline": {"bound": "hbm", "achieved": round(gbs, 1), "peak": hbm, "unit": "GB/s",
+                        "frac": round(gbs / hbm, 4), "peak_source": src,
+                        "algorithmic_bytes_per_launch": byts,
+                        "tflops": round(2 * rows * cfg.vocab * H / (ms * 1e-3) / 1e12, 1)},
+           "launches": 2,
+           "how": "the LM-head GEMM with row max / log-sum-exp / argmax in its epilogue and the "
+                  "one-CTA merge, one CUDA graph, CUDA events over the replays"}
+    del hid, w, ws, g_lm
+    torch.cuda.empty_cache()
+    return res
+
+
 def summarize_config(name, args, device, seed, reps):
     """Full-cycle latency, phases, the attention roofline against the shape's
     binding resource and e2e for one workload (the 8B-class one is the
@@ -515,6 +559,9 @@ def summarize_config(name, args, device, seed, reps):
                              "bytes_read_and_written_each": moved,
                              "how": "ltd_kv_compact of the cycle's accepted path in all layers, one "
                                     "launch, CUDA graph replays"}
+    lm = time_lm_head(cfg, name, device, reps)
+    if lm is not None:
+        res["lm_head"] = lm
     if not args.no_e2e:
         res["e2e"] = run_e2e(cyc, args, device)
     del cyc, g_cycle, g_draft, g_verify, g_plain, g_accept
@@ -754,6 +801,8 @@ def run_ours(args):
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(cfg, layers, args.seed, args.cpu_sample_s)
 
+    lm_head = time_lm_head(cfg, args.config, device, max(10, min(K, 50))) if world == 1 else None
+
     # the other workloads: full-cycle latency, phases and the attention
     # roofline against each shape's binding resource (one GPU only)
     configs = None
@@ -784,7 +833,7 @@ def run_ours(args):
             "accept_rules_us": rules,
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "policy": pol, "reward": reward,
             "gpu_launches": cyc.launches_per_step() * K * R, "clocks": clk,
-            "configs": configs,
+            "lm_head": lm_head, "configs": configs,
         }
         print(json.dumps(line), flush=True)
     if world > 1:

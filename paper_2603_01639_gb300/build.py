@@ -22,7 +22,7 @@ BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libltd.so")
 
 SOURCES = ["ltd_api.cu", "k_expand.cu", "k_select.cu", "k_policy.cu", "k_attn_simt.cu", "k_attn_tc.cu",
-           "k_accept.cu", "k_selftest.cu", "k_accept_noalloc.cu"]
+           "k_accept.cu", "k_selftest.cu", "k_accept_noalloc.cu", "k_lm_head.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall",
          "--expt-relaxed-constexpr", "-I", INCLUDE, "-I", CSRC] + ARCH

@@ -17,8 +17,9 @@
 //               (logit, token) keys and its sum of exp(x - max), merged
 //               over the warps and into the CTA's running statistics;
 //               optionally the logits themselves (bf16).
-// A second, one-CTA kernel merges the CTAs' statistics per row (the launch
-// boundary orders it after every CTA's writes) and writes max, LSE, argmax.
+// A second kernel merges the CTAs' statistics per row, a warp per row (the
+// launch boundary orders it after every CTA's writes), and writes max, LSE,
+// argmax.
 #include "ltd_common.cuh"
 #include "ltd_internal.h"
 #include "tc_util.cuh"
@@ -33,6 +34,7 @@ constexpr int kThreads = 256;             // TMA, MMA, 2 idle, 4 epilogue warps
 constexpr uint32_t kTileA = kVT * 128;    // bytes of one weight k-block
 constexpr uint32_t kStageMax = 8;
 constexpr uint32_t kSmemBudget = 200 * 1024;
+constexpr int kMaxGrid = 256;             // the merge kernel takes up to 256 CTAs' statistics
 
 struct LmArgs {
   int32_t rows, n_pad, hidden, kblocks, tiles, stages;  // n_pad: rows rounded up to 32
@@ -234,20 +236,44 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-// One CTA: row r's statistics merged over the first kernel's CTAs, in CTA
-// order (every thread of a row merges the same sequence, so the result does
-// not depend on timing).
-__global__ void __launch_bounds__(256)
+// A warp per row: lane l merges the statistics of CTAs l, l + 32, ... (its
+// loads issued together), then the lanes merge pairwise in a fixed tree, so
+// the result does not depend on timing.  The launch boundary orders this
+// after every write of the first kernel.
+constexpr int kMergeWarps = 8;
+__global__ void __launch_bounds__(kMergeWarps * 32)
     lm_head_merge_kernel(const float* part, const unsigned long long* part_key, int grid,
                          int n_pad, int rows, float* row_max, float* row_lse, int32_t* row_argmax) {
   grid_wait();
   trigger_dependents();
-  for (int r = threadIdx.x; r < rows; r += blockDim.x) {
-    Stat acc{-CUDART_INF_F, 0.f, 0ull};
-    for (int c = 0; c < grid; ++c) {
-      const float2 ms = reinterpret_cast<const float2*>(part)[static_cast<int64_t>(c) * n_pad + r];
-      stat_merge(acc, Stat{ms.x, ms.y, part_key[static_cast<int64_t>(c) * n_pad + r]});
-    }
+  const int lane = threadIdx.x & 31;
+  const int r = blockIdx.x * kMergeWarps + (threadIdx.x >> 5);
+  if (r >= rows) return;
+  constexpr int kPer = kMaxGrid / 32;
+  float2 ms[kPer];
+  unsigned long long ky[kPer];
+#pragma unroll
+  for (int i = 0; i < kPer; ++i) {
+    const int c = lane + 32 * i;
+    ms[i] = c < grid ? reinterpret_cast<const float2*>(part)[static_cast<int64_t>(c) * n_pad + r]
+                     : make_float2(-CUDART_INF_F, 0.f);
+    ky[i] = c < grid ? part_key[static_cast<int64_t>(c) * n_pad + r] : 0ull;
+  }
+  Stat acc{-CUDART_INF_F, 0.f, 0ull};
+#pragma unroll
+  for (int i = 0; i < kPer; ++i) stat_merge(acc, Stat{ms[i].x, ms[i].y, ky[i]});
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    Stat other;
+    other.m = __shfl_xor_sync(0xFFFFFFFFu, acc.m, o);
+    other.s = __shfl_xor_sync(0xFFFFFFFFu, acc.s, o);
+    other.key = __shfl_xor_sync(0xFFFFFFFFu, acc.key, o);
+    // both lanes of a pair merge the same two values in the same order
+    Stat lo = (lane & o) ? other : acc, hi = (lane & o) ? acc : other;
+    stat_merge(lo, hi);
+    acc = lo;
+  }
+  if (lane == 0) {
     row_max[r] = acc.m;
     row_lse[r] = acc.m + logf(acc.s);
     row_argmax[r] = static_cast<int32_t>(key_index(acc.key));
@@ -260,6 +286,7 @@ size_t lm_head_workspace(int32_t rows, int64_t vocab) {
   const int n_pad = (rows + 31) / 32 * 32;
   const int64_t tiles = (vocab + kVT - 1) / kVT;
   int grid = device_sm_count();
+  if (grid > kMaxGrid) grid = kMaxGrid;
   if (tiles < grid) grid = static_cast<int>(tiles);
   return static_cast<size_t>(grid) * n_pad * (sizeof(float2) + sizeof(unsigned long long)) + 256;
 }
@@ -277,6 +304,7 @@ cudaError_t launch_lm_head(const LmHeadParams& p, cudaStream_t s) {
   if (a.stages > static_cast<int32_t>(kStageMax)) a.stages = kStageMax;
   if (a.stages < 2) return cudaErrorInvalidValue;
   int grid = device_sm_count();
+  if (grid > kMaxGrid) grid = kMaxGrid;
   if (a.tiles < grid) grid = a.tiles;
   const size_t need = static_cast<size_t>(grid) * a.n_pad * (sizeof(float2) + sizeof(unsigned long long));
   if (p.ws == nullptr || p.ws_bytes < need) return cudaErrorInvalidValue;
@@ -297,7 +325,8 @@ cudaError_t launch_lm_head(const LmHeadParams& p, cudaStream_t s) {
   if (e != cudaSuccess) return e;
   e = launch(lm_head_kernel, dim3(grid), dim3(kThreads), smem, s, nullptr, 0, tw, th, a);
   if (e != cudaSuccess) return e;
-  return launch(lm_head_merge_kernel, dim3(1), dim3(256), 0, s, nullptr, 0,
+  return launch(lm_head_merge_kernel, dim3((a.rows + kMergeWarps - 1) / kMergeWarps),
+                dim3(kMergeWarps * 32), 0, s, nullptr, 0,
                 static_cast<const float*>(a.part), static_cast<const unsigned long long*>(a.part_key),
                 grid, a.n_pad, a.rows, p.row_max, p.row_lse, p.row_argmax);
 }

@@ -226,7 +226,7 @@ __global__ void __launch_bounds__(kMlpNT, 1) mlp_policy_kernel(const MlpArgs a) 
   for (int l = 0; l < L; ++l) {
     const int U = a.plan[l].U, u0 = rank * U;
     const int u_cnt = max(0, min(U, a.net.dims[l + 1] - u0));
-    for (int u = tid; u < u_cnt; u += kMlpNT) bias_s[l * kMlpBiasMax + u] = __ldg(a.net.b[l] + u0 + u);
+    for (int u = tid; u < u_cnt; u += kMlpNT) bias_s[l * kMlpBiasMax + u] = __ldcg(a.net.b[l] + u0 + u);
   }
   // peers must have started before their shared memory is written
   cluster_arrive_relaxed();
@@ -299,7 +299,7 @@ __global__ void __launch_bounds__(kMlpNT, 1) mlp_policy_kernel(const MlpArgs a) 
         for (int i = p; i < n_in; i += P) {
           float w[4];
 #pragma unroll
-          for (int c = 0; c < 4; ++c) w[c] = (c < nc) ? __ldg(wq + static_cast<int64_t>(i) * n_out + c) : 0.f;
+          for (int c = 0; c < 4; ++c) w[c] = (c < nc) ? __ldcg(wq + static_cast<int64_t>(i) * n_out + c) : 0.f;
 #pragma unroll
           for (int g = 0; g < G; ++g) {
             const float xv = x[g * a.width + i];

@@ -91,8 +91,8 @@ typedef enum ltd_mode {
  *   xlse[max_nodes]         float, log-sum-exp of that row
  *   frontier[k]             frontier node ids in rank order
  *   n_nodes[1], n_levels[1] node count and levels built so far
- * The scratch area holds per-CTA partial results of ltd_expand_tree; it is
- * zeroed by ltd_tree_reset and left zeroed by every expansion.
+ * The scratch area holds ltd_expand_tree's per-item records (each 64-bit
+ * word tagged with the level that wrote it); ltd_tree_reset zeroes it.
  * ------------------------------------------------------------------------ */
 typedef struct ltd_tree {
   int32_t batch, max_depth, k, max_nodes;
@@ -140,8 +140,10 @@ ltd_status ltd_tree_reset(const ltd_tree* tree, const int32_t* d_root_tokens, lt
  *  d_active        [batch] 0/1, NULL = all sequences expand
  * Per node: cum = cum(parent) + x - logsumexp(row), computed in fp32.
  * Rows must start 16-byte aligned (vocab * sizeof(dtype) % 16 == 0).
- * vocab <= 262,144 for LTD_BF16 and 131,072 for LTD_F32 (larger returns
- * LTD_ERR_UNSUPPORTED). */
+ * vocab <= 1,048,576 (larger returns LTD_ERR_UNSUPPORTED).  The records of
+ * a level's rows are merged by one CTA per sequence after a bounded wait;
+ * if it runs out, LTD_DEVERR_TIMEOUT is flagged and the level stays
+ * unbuilt (n_levels unchanged). */
 ltd_status ltd_expand_tree(const ltd_tree* tree, int32_t level, const void* d_draft_rows,
                            ltd_dtype dtype, int64_t vocab, int64_t rows_per_seq,
                            const int32_t* d_active, ltd_stream_t stream);
@@ -478,6 +480,20 @@ ltd_status ltd_lm_head_row_stats(const void* d_hidden, const void* d_weight, int
  * counters are back at zero and the workspace can be used again.
  * extra_arrivals above 1024 returns LTD_ERR_INVALID_ARG. */
 ltd_status ltd_debug_attention_wait(uint64_t limit_ns, uint32_t extra_arrivals);
+
+/* Test hook of the expansion's bounded wait (section 3.2 has no counterpart;
+ * it exists so the failure path can be exercised without a GPU fault).  The
+ * CTA that merges a sequence's rows in ltd_expand_tree waits until every
+ * item record of the level carries the level's tag; this sets, for the
+ * calls that follow on any thread, the longest that wait lasts (limit_ns; 0
+ * restores the default of one second) and an offset added to the tag it
+ * waits for (tag_offset; 0 restores normal operation).  No record ever
+ * carries the offset tag, so with tag_offset > 0 every merging CTA gives
+ * up after limit_ns, raises LTD_DEVERR_TIMEOUT (ltd_check returns
+ * LTD_ERR_TIMEOUT) and leaves the level unbuilt: n_levels unchanged, so
+ * the same level can be expanded again.  tag_offset above 1024 returns
+ * LTD_ERR_INVALID_ARG. */
+ltd_status ltd_debug_expand_wait(uint64_t limit_ns, uint32_t tag_offset);
 
 /* Diagnostic of the tensor-core building blocks the attention kernel uses
  * (TMA with 128-byte swizzle, tcgen05.mma from shared-memory descriptors

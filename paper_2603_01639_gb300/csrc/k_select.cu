@@ -1,15 +1,20 @@
 // Candidate token selection (LTD section 3.2, "Candidate Token Selection").
 //
-// One CTA per sequence.  Every node gets the key (cum desc, id asc) in
-// shared memory (the root gets the maximum key, so it always ranks first);
-// a bitonic sort of the keys (in registers and warp shuffles, one key per
-// thread, up to 1024 nodes) puts the N verified nodes first (keys are
-// unique, so the order is total).  A block-wide exclusive scan over the
-// flags in id order gives each verified node its slot, so slots are the
-// verified ids in ascending order.  Each slot then walks its parent chain
-// (at most max_depth steps) and sets one mask bit per ancestor.  Because a
-// child's cum never exceeds its parent's and parents have smaller ids, the
-// verified set is ancestor-closed; a violation is flagged, not trapped.
+// One CTA per sequence.  Every node gets the key (cum desc, id asc); the
+// root gets the largest key, so it always ranks first.  The N largest keys
+// are found by a radix select over the 64-bit keys, eight bits per pass
+// from the top: a shared-memory histogram of the next digit among the keys
+// that match the prefix so far, one warp's scan of it from the top bin, and
+// the bin where the count reaches N becomes the prefix; the select stops at
+// the first pass whose bin holds exactly the keys still wanted (keys are
+// unique, so it stops by the last digit), and a key is verified iff its
+// bits above that digit are at least the prefix.  Typically three passes.
+// Slots are the verified ids in ascending order (a block scan of the
+// flags).  The thread that owns a verified node walks its parent chain (at
+// most max_depth steps) and builds the node's mask row in registers, one
+// bit per ancestor, then stores it.  Because a child's cum never exceeds its
+// parent's and parents have smaller ids, the verified set is
+// ancestor-closed; a violation is flagged, not trapped.
 #include "ltd_common.cuh"
 #include "ltd_internal.h"
 
@@ -18,6 +23,10 @@ namespace ltd {
 namespace {
 
 constexpr int kNT = 1024;
+constexpr int kNW = kNT / kWarp;
+constexpr int kMaxPer = LTD_MAX_TREE_NODES / kNT;  // nodes per thread
+constexpr int kMaxWords = LTD_MAX_N / 32;          // mask words per row
+static_assert(LTD_MAX_TREE_NODES % kNT == 0, "whole nodes per thread");
 
 // Optional phase timestamps for performance work (off in normal builds).
 #ifdef LTD_TRACE
@@ -36,28 +45,52 @@ __device__ unsigned long long g_select_trace[64][8];
   } while (0)
 #endif
 
+struct RadixState {
+  uint64_t prefix;  // the selected digits so far
+  int shift;        // bit position of the current digit
+  int want;         // keys still to select among those matching the prefix
+  int done;
+};
+
 __global__ void __launch_bounds__(kNT) select_kernel(const SelectParams p) {
   extern __shared__ __align__(16) unsigned char smem[];
-  const int W32 = (p.n_max + 31) / 32;
-  const int P = p.sort_len;                                                   // pow2 >= max_nodes
-  uint64_t* keys = reinterpret_cast<uint64_t*>(smem);                          // [P]
-  int32_t* slot_of = reinterpret_cast<int32_t*>(keys + P);                    // [max_nodes]
-  int32_t* par_s = slot_of + p.max_nodes;                                     // [max_nodes]
-  uint32_t* words = reinterpret_cast<uint32_t*>(par_s + p.max_nodes);         // [n_max][W32]
-  __shared__ int32_t warp_tot[kNT / kWarp];
+  int32_t* slot_of = reinterpret_cast<int32_t*>(smem);  // [max_nodes]
+  int32_t* par_s = slot_of + p.max_nodes;               // [max_nodes]
+  __shared__ uint32_t hist[2][256];
+  __shared__ int warp_tot[kNW];
+  __shared__ RadixState st;
 
   STRACE(0);
+  const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  for (int i = tid; i < 512; i += kNT) (&hist[0][0])[i] = 0u;
   grid_wait();
   trigger_dependents();
   STRACE(1);
-  const int b = blockIdx.x, tid = threadIdx.x;
   const int64_t nb = static_cast<int64_t>(b) * p.max_nodes;
-  const int n = p.n_nodes[b];
-  const int N = p.n_verify[b];
-  const int ctx = p.ctx[b];
+  const int W32 = (p.n_max + 31) / 32;
   int32_t* ids_out = p.node_ids + static_cast<int64_t>(b) * p.n_max;
   int32_t* pos_out = p.pos + static_cast<int64_t>(b) * p.n_max;
   uint32_t* mask_out = p.mask + static_cast<int64_t>(b) * p.n_max * W32;
+
+  // every node slot's data is loaded before the node count is known
+  const int per = (p.max_nodes + kNT - 1) / kNT;
+  float cumv[kMaxPer];
+  int parv[kMaxPer], depv[kMaxPer];
+#pragma unroll
+  for (int q = 0; q < kMaxPer; ++q) {
+    const int i = tid + q * kNT;
+    cumv[q] = 0.f;
+    parv[q] = -1;
+    depv[q] = 0;
+    if (q < per && i < p.max_nodes) {
+      cumv[q] = __ldcg(p.cum + nb + i);
+      parv[q] = __ldcg(p.parent + nb + i);
+      depv[q] = __ldcg(p.depth + nb + i);
+    }
+  }
+  const int n = __ldcg(p.n_nodes + b);
+  const int N = __ldcg(p.n_verify + b);
+  const int ctx = __ldcg(p.ctx + b);
 
   const bool ok = (n >= 1 && n <= p.max_nodes && N >= 1 && N <= n && N <= p.n_max);
   if (!ok) {
@@ -69,138 +102,160 @@ __global__ void __launch_bounds__(kNT) select_kernel(const SelectParams p) {
     for (int i = tid; i < p.n_max * W32; i += kNT) mask_out[i] = 0u;
     return;
   }
-
-  // keys padded to a power of two with 0 (below every real key)
-  int Pn = 1;
-  while (Pn < n) Pn <<= 1;
-  for (int i = tid; i < n; i += kNT) {
-    par_s[i] = p.parent[nb + i];
-    slot_of[i] = 0;
+  // slots past N (known already)
+  for (int i = N + tid; i < p.n_max; i += kNT) {
+    ids_out[i] = -1;
+    pos_out[i] = -1;
   }
-  for (int i = tid; i < p.n_max * W32; i += kNT) words[i] = 0u;
-  const int lane = tid & 31, warp = tid >> 5;
-  if (Pn <= kNT) {
-    // one key per thread, bitonic sort descending: strides below the warp
-    // width by shuffles, wider ones through shared memory
-    uint64_t key = 0ull;
-    if (tid < n) key = (tid == 0) ? ~0ull : make_key(p.cum[nb + tid], static_cast<uint32_t>(tid));
-    __syncthreads();
-    STRACE(2);
-    // only warps holding keys compute; every thread meets the barriers
-    const bool sorter = warp * kWarp < Pn;
-    for (int k = 2; k <= Pn; k <<= 1) {
-      for (int j = k >> 1; j > 0; j >>= 1) {
-        uint64_t other = 0ull;
-        if (j >= kWarp) {
-          if (tid < Pn) keys[tid] = key;
-          __syncthreads();
-          if (tid < Pn) other = keys[tid ^ j];
-          __syncthreads();
-        } else if (sorter) {
-          other = __shfl_xor_sync(0xFFFFFFFFu, key, j);
-        }
-        if (sorter) {
-          // in a descending block the lower index of the pair keeps the larger
-          const bool keep_max = ((tid & k) == 0) == ((tid & j) == 0);
-          key = keep_max ? (key > other ? key : other) : (key < other ? key : other);
-        }
-      }
+  for (int i = N * W32 + tid; i < p.n_max * W32; i += kNT) mask_out[i] = 0u;
+
+  uint64_t key[kMaxPer];
+#pragma unroll
+  for (int q = 0; q < kMaxPer; ++q) {
+    const int i = tid + q * kNT;
+    key[q] = (q < per && i < n) ? ((i == 0) ? ~0ull : make_key(cumv[q], static_cast<uint32_t>(i))) : 0ull;
+    if (q < per && i < n) par_s[i] = parv[q];
+  }
+  if (tid == 0) {
+    st.prefix = 0ull;
+    st.shift = 56;
+    st.want = N;
+    st.done = 0;
+  }
+  __syncthreads();
+  STRACE(2);
+
+  // ---- radix select of the N largest keys (key 0 = no node)
+#pragma unroll 1
+  for (int pass = 0; pass < 8; ++pass) {
+    const int buf = pass & 1;
+    const int shift = st.shift;
+    const uint64_t prefix = st.prefix;
+#pragma unroll
+    for (int q = 0; q < kMaxPer; ++q) {
+      if (q >= per) break;
+      const bool match = key[q] != 0ull && (pass == 0 || (key[q] >> (shift + 8)) == prefix);
+      const uint32_t dig = match ? static_cast<uint32_t>(key[q] >> shift) & 0xFFu : 0x100u;
+      const uint32_t peers = __match_any_sync(0xFFFFFFFFu, dig);
+      if (dig < 256u && lane == __ffs(peers) - 1) atomicAdd(&hist[buf][dig], __popc(peers));
     }
-    if (tid < N) slot_of[key_index(key)] = 1;
-  } else {
-    for (int i = tid; i < Pn; i += kNT)
-      keys[i] = (i >= n) ? 0ull : (i == 0) ? ~0ull : make_key(p.cum[nb + i], static_cast<uint32_t>(i));
     __syncthreads();
-    STRACE(2);
-    for (int k = 2; k <= Pn; k <<= 1) {
-      for (int j = k >> 1; j > 0; j >>= 1) {
-        for (int i = tid; i < Pn; i += kNT) {
-          const int ixj = i ^ j;
-          if (ixj > i) {
-            const uint64_t x = keys[i], y = keys[ixj];
-            if (((i & k) == 0) ? (x < y) : (x > y)) {
-              keys[i] = y;
-              keys[ixj] = x;
+    if (warp == 0) {
+      // lane l covers bins 255 - 8l - j, j = 0..7 (from the top)
+      uint32_t c[8];
+      uint32_t s = 0u;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        c[j] = hist[buf][255 - 8 * lane - j];
+        s += c[j];
+      }
+      uint32_t incl = s;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+        if (lane >= o) incl += y;
+      }
+      const uint32_t want = static_cast<uint32_t>(st.want);
+      const uint32_t before = incl - s;
+      // exactly one lane's range crosses `want`
+      if (before < want && incl >= want) {
+        // the first of the lane's bins where the count reaches want (the
+        // lane's total does)
+        uint32_t above = before, cj = 0u;
+        int j = 0;
+        bool found = false;
+#pragma unroll
+        for (int jj = 0; jj < 8; ++jj) {
+          if (!found) {
+            if (above + c[jj] >= want) {
+              j = jj;
+              cj = c[jj];
+              found = true;
+            } else {
+              above += c[jj];
             }
           }
         }
-        __syncthreads();
+        const uint32_t bin = 255u - 8u * lane - j;
+        const uint32_t rest = want - above;
+        st.prefix = (prefix << 8) | bin;
+        st.want = static_cast<int>(rest);
+        if (cj == rest || shift == 0) {
+          st.done = 1;
+        } else {
+          st.shift = shift - 8;
+        }
       }
+      // the other buffer is clean for the next pass
+#pragma unroll
+      for (int j = 0; j < 8; ++j) hist[buf ^ 1][8 * lane + j] = 0u;
     }
-    for (int r = tid; r < N; r += kNT) slot_of[key_index(keys[r])] = 1;
+    __syncthreads();
+    if (st.done) break;
   }
-  __syncthreads();
   STRACE(3);
-  // each thread owns ids [4 tid, 4 tid + 4) so the scan below is in id order
-  constexpr int PER = 4;
-  int flags[PER];
-  int local = 0;
+  const int fshift = st.shift;
+  const uint64_t thresh = st.prefix;
+
+  // ---- slots: verified ids in ascending order (id = tid + q * kNT)
+  int slot_base = 0;
+  int my_slot[kMaxPer];
 #pragma unroll
-  for (int r = 0; r < PER; ++r) {
-    const int i = tid * PER + r;
-    flags[r] = (i < n) ? slot_of[i] : 0;
-    local += flags[r];
-  }
-  __syncthreads();
-  // block exclusive scan of `local`
-  int incl = local;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const int y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
-    if (lane >= o) incl += y;
-  }
-  if (lane == 31) warp_tot[warp] = incl;
-  __syncthreads();
-  if (warp == 0) {
-    int w = (lane < kNT / kWarp) ? warp_tot[lane] : 0;
-    int wi = w;
+  for (int q = 0; q < kMaxPer; ++q) {
+    my_slot[q] = -1;
+    if (q >= per) break;
+    const bool sel = key[q] != 0ull && (key[q] >> fshift) >= thresh;
+    const uint32_t bal = __ballot_sync(0xFFFFFFFFu, sel);
+    if (lane == 0) warp_tot[warp] = __popc(bal);
+    __syncthreads();
+    const int t = warp_tot[lane];
+    int incl = t;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
-      const int y = __shfl_up_sync(0xFFFFFFFFu, wi, o);
-      if (lane >= o) wi += y;
+      const int y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+      if (lane >= o) incl += y;
     }
-    if (lane < kNT / kWarp) warp_tot[lane] = wi - w;  // exclusive warp offsets
-  }
-  __syncthreads();
-  int slot = warp_tot[warp] + incl - local;
-#pragma unroll
-  for (int r = 0; r < PER; ++r) {
-    const int i = tid * PER + r;
-    if (i < n) {
-      slot_of[i] = flags[r] ? slot : -1;
-      if (flags[r]) {
-        ids_out[slot] = i;
-        pos_out[slot] = ctx + p.depth[nb + i];
-        ++slot;
-      }
+    const int warp_before = __shfl_sync(0xFFFFFFFFu, incl - t, warp);
+    const int total = __shfl_sync(0xFFFFFFFFu, incl, 31);
+    const int i = tid + q * kNT;
+    if (sel) {
+      const int s = slot_base + warp_before + __popc(bal & ((1u << lane) - 1u));
+      my_slot[q] = s;
+      ids_out[s] = i;
+      pos_out[s] = ctx + depv[q];
     }
+    if (q < per && i < n) slot_of[i] = my_slot[q];
+    slot_base += total;
+    __syncthreads();  // warp_tot is reused by the next q
   }
-  __syncthreads();
-
   STRACE(4);
-  // ancestor bits: the thread owning node i writes row slot_of[i] alone
-  for (int i = tid; i < n; i += kNT) {
-    const int si = slot_of[i];
+
+  // ---- mask rows: the owner of a verified node walks its parent chain
+#pragma unroll
+  for (int q = 0; q < kMaxPer; ++q) {
+    if (q >= per) break;
+    const int si = my_slot[q];
     if (si < 0) continue;
-    uint32_t* row = words + si * W32;
-    int a = i;
+    uint32_t row[kMaxWords];
+#pragma unroll
+    for (int w = 0; w < kMaxWords; ++w) row[w] = 0u;
+    int a = tid + q * kNT;
     int guard = 0;
     while (a >= 0 && guard <= LTD_MAX_DEPTH + 1) {
-      const int sa = slot_of[a];
+      const int sa = (a < n) ? slot_of[a] : -1;
       if (sa < 0) {
         flag_error(p.err, LTD_DEVERR_TREE);
         break;
       }
-      row[sa >> 5] |= 1u << (sa & 31);
+#pragma unroll
+      for (int w = 0; w < kMaxWords; ++w) row[w] |= ((sa >> 5) == w) ? (1u << (sa & 31)) : 0u;
       a = par_s[a];
       ++guard;
     }
-  }
-  __syncthreads();
-  for (int i = tid; i < p.n_max * W32; i += kNT) mask_out[i] = (i < N * W32) ? words[i] : 0u;
-  for (int i = N + tid; i < p.n_max; i += kNT) {
-    ids_out[i] = -1;
-    pos_out[i] = -1;
+    uint32_t* dst = mask_out + static_cast<int64_t>(si) * W32;
+#pragma unroll
+    for (int w = 0; w < kMaxWords; ++w)
+      if (w < W32) dst[w] = row[w];
   }
   STRACE(5);
 }
@@ -209,12 +264,7 @@ __global__ void __launch_bounds__(kNT) select_kernel(const SelectParams p) {
 
 cudaError_t launch_select(const SelectParams& params, int32_t batch, cudaStream_t s) {
   SelectParams p = params;
-  p.sort_len = 1;
-  while (p.sort_len < p.max_nodes) p.sort_len <<= 1;
-  const int W32 = (p.n_max + 31) / 32;
-  const size_t smem = static_cast<size_t>(p.sort_len) * sizeof(uint64_t) +
-                      static_cast<size_t>(p.max_nodes) * 2 * sizeof(int32_t) +
-                      static_cast<size_t>(p.n_max) * W32 * sizeof(uint32_t);
+  const size_t smem = static_cast<size_t>(p.max_nodes) * 2 * sizeof(int32_t);
   cudaError_t e = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;

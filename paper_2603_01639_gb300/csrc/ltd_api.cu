@@ -107,7 +107,7 @@ size_t ltd_tree_bytes(int32_t batch, int32_t max_depth, int32_t k, int64_t max_v
   if (!tree_dims_ok(batch, max_depth, k, max_vocab)) return 0;
   const size_t nodes = static_cast<size_t>(batch) * tree_nodes(max_depth, k);
   return 6 * align256(nodes * 4) + align256(static_cast<size_t>(batch) * k * 4) +
-         2 * align256(static_cast<size_t>(batch) * 4) + expand_layout(batch, k, max_vocab).total;
+         2 * align256(static_cast<size_t>(batch) * 4) + expand_scratch_bytes(batch, k, max_vocab);
 }
 
 ltd_status ltd_tree_init(ltd_tree* tree, void* d_mem, size_t bytes, int32_t batch,
@@ -139,7 +139,7 @@ ltd_status ltd_tree_init(ltd_tree* tree, void* d_mem, size_t bytes, int32_t batc
   tree->frontier = reinterpret_cast<int32_t*>(take(static_cast<size_t>(batch) * k * 4));
   tree->n_nodes = reinterpret_cast<int32_t*>(take(static_cast<size_t>(batch) * 4));
   tree->n_levels = reinterpret_cast<int32_t*>(take(static_cast<size_t>(batch) * 4));
-  tree->scratch_bytes = expand_layout(batch, k, max_vocab).total;
+  tree->scratch_bytes = expand_scratch_bytes(batch, k, max_vocab);
   tree->scratch = take(tree->scratch_bytes);
   return LTD_OK;
 }
@@ -164,9 +164,7 @@ ltd_status ltd_expand_tree(const ltd_tree* tree, int32_t level, const void* d_dr
   uint32_t* err = device_error_word();
   if (err == nullptr) return LTD_ERR_CUDA;
   const int32_t F = (level == 1) ? 1 : tree->k;
-  const int esize = static_cast<int>(dtype_size(dtype));
-  if (vocab > expand_max_vocab(esize)) return LTD_ERR_UNSUPPORTED;
-  const VocabSplit vs = expand_split(static_cast<int64_t>(tree->batch) * F, vocab, esize);
+  if (vocab > kExpandMaxVocab) return LTD_ERR_UNSUPPORTED;
   ExpandParams p{};
   p.token = tree->token;
   p.parent = tree->parent;
@@ -179,17 +177,17 @@ ltd_status ltd_expand_tree(const ltd_tree* tree, int32_t level, const void* d_dr
   p.n_levels = tree->n_levels;
   p.max_nodes = tree->max_nodes;
   p.k = tree->k;
-  p.seq_ticket = static_cast<uint32_t*>(tree->scratch);
+  p.batch = tree->batch;
+  p.rec = static_cast<uint64_t*>(tree->scratch);
+  p.rec_chunks = expand_rec_chunks(tree->max_vocab);
   p.rows = d_draft_rows;
   p.vocab = vocab;
   p.rows_per_seq = rows_per_seq;
   p.active = d_active;
   p.level = level;
   p.F = F;
-  p.chunks = vs.chunks;
-  p.chunk_elems = vs.chunk_elems;
   p.err = err;
-  return from_cuda(launch_expand(p, tree->batch, dtype, reinterpret_cast<cudaStream_t>(stream)));
+  return from_cuda(launch_expand(p, dtype, reinterpret_cast<cudaStream_t>(stream)));
 }
 
 ltd_status ltd_depth_observation(const ltd_tree* tree, const int32_t* d_ctx, float* d_out,
@@ -444,6 +442,12 @@ ltd_status ltd_lm_head_row_stats(const void* d_hidden, const void* d_weight, int
 ltd_status ltd_debug_attention_wait(uint64_t limit_ns, uint32_t extra_arrivals) {
   if (extra_arrivals > 1024) return LTD_ERR_INVALID_ARG;
   set_attn_wait_hook(AttnWaitHook{limit_ns, extra_arrivals});
+  return LTD_OK;
+}
+
+ltd_status ltd_debug_expand_wait(uint64_t limit_ns, uint32_t tag_offset) {
+  if (tag_offset > 1024) return LTD_ERR_INVALID_ARG;
+  set_expand_wait_hook(ExpandWaitHook{limit_ns, tag_offset});
   return LTD_OK;
 }
 

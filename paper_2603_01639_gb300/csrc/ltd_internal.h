@@ -63,16 +63,13 @@ struct VocabSplit {
 VocabSplit vocab_split(int64_t rows, int64_t vocab, int64_t target_ctas, int64_t min_elems);
 
 // ------------------------------------------------------------- expansion
-constexpr int64_t kExpandTargetCtas = 304;  // two CTAs per SM of a 152-SM GB300
-constexpr int64_t kExpandMinElems = 2048;
-
-struct ExpandRecordLayout {
-  size_t ms_bytes, keys_bytes, row_ticket_bytes, seq_ticket_bytes, total;
-  int64_t records;
-};
-ExpandRecordLayout expand_layout(int32_t batch, int32_t k, int64_t max_vocab);
-VocabSplit expand_split(int64_t rows, int64_t vocab, int elem_bytes);
-int64_t expand_max_vocab(int elem_bytes);
+// A draft row is cut into items of 16 KB (8192 bf16 or 4096 fp32 entries);
+// each item's record (its top-k keys and its (max, sum of exp), every
+// 64-bit word tagged with the level) goes to the tree's scratch area, laid
+// out [batch][k rows][rec_chunks][k + 2 words].
+constexpr int64_t kExpandMaxVocab = int64_t(1) << 20;
+int32_t expand_rec_chunks(int64_t max_vocab);
+size_t expand_scratch_bytes(int32_t batch, int32_t k, int64_t max_vocab);
 
 struct ExpandParams {
   int32_t* token;
@@ -86,22 +83,33 @@ struct ExpandParams {
   int32_t* n_levels;
   int32_t max_nodes;
   int32_t k;
-  float2* part_ms;       // [records]
-  uint64_t* part_keys;   // [records][k]
-  uint32_t* row_ticket;  // [batch][k]
-  uint32_t* seq_ticket;  // [batch]
+  int32_t batch;
+  uint64_t* rec;       // the tree's scratch area
+  int32_t rec_chunks;  // items per row the records are laid out for
   const void* rows;
   int64_t vocab;
   int64_t rows_per_seq;
   const int32_t* active;
   int32_t level;
-  int32_t F;
-  int32_t chunks;
-  int64_t chunk_elems;
+  int32_t F;              // rows per sequence at this level
+  int32_t item_elems;     // entries per item (set by launch_expand)
+  int32_t chunks;         // items per row (set by launch_expand)
+  int32_t n_items;        // batch * F * chunks (set by launch_expand)
+  int32_t items_per_cta;  // (set by the launch)
+  uint64_t wait_limit_ns; // consumer's wait on the records (set by launch_expand)
+  uint32_t tag_offset;    // added to the tag the consumer waits for (test hook)
+  int32_t j_row;          // leading keys per item list for the row threshold (set by launch_expand)
   uint32_t* err;
 };
+// Test hook of the expansion consumer's wait (k_expand.cu): its limit (0 =
+// the default 1 s) and an offset to the awaited tag that no producer writes.
+struct ExpandWaitHook {
+  uint64_t limit_ns;
+  uint32_t tag_offset;
+};
+void set_expand_wait_hook(const ExpandWaitHook& h);
 cudaError_t launch_tree_reset(const ltd_tree* t, const int32_t* roots, cudaStream_t s);
-cudaError_t launch_expand(const ExpandParams& p, int32_t batch, ltd_dtype dtype, cudaStream_t s);
+cudaError_t launch_expand(const ExpandParams& p, ltd_dtype dtype, cudaStream_t s);
 
 // ------------------------------------------------------------- selection
 struct SelectParams {
@@ -111,7 +119,6 @@ struct SelectParams {
   const float* cum;
   const int32_t* n_nodes;
   int32_t max_nodes;
-  int32_t sort_len;  // power of two >= max_nodes (set by launch_select)
   const int32_t* n_verify;
   int32_t n_max;
   const int32_t* ctx;

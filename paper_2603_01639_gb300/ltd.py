@@ -32,7 +32,7 @@ EXPORTS = [
     "ltd_attention_kernel", "ltd_selftest_umma", "ltd_accept_noalloc", "ltd_tree_attention_next",
     "ltd_depth_observation", "ltd_size_observation", "ltd_depth_policy", "ltd_size_policy",
     "ltd_mlp_packed_bytes", "ltd_mlp_pack", "ltd_kv_append", "ltd_accept_tempered",
-    "ltd_debug_attention_wait", "ltd_lm_head_workspace_bytes", "ltd_lm_head_row_stats",
+    "ltd_debug_attention_wait", "ltd_debug_expand_wait", "ltd_lm_head_workspace_bytes", "ltd_lm_head_row_stats",
 ]
 LTD_POLICY_PAD = -100.0
 LTD_MLP_MAX_LAYERS, LTD_MLP_MAX_WIDTH = 4, 2048
@@ -109,6 +109,7 @@ def lib():
                                                C.POINTER(i32)]),
                 "ltd_selftest_umma": (C.c_int, [i32, vp, vp, vp, vp]),
                 "ltd_debug_attention_wait": (C.c_int, [u64, C.c_uint32]),
+                "ltd_debug_expand_wait": (C.c_int, [u64, C.c_uint32]),
                 "ltd_lm_head_workspace_bytes": (sz, [i32, i64, i32]),
                 "ltd_lm_head_row_stats": (C.c_int, [vp, vp, i32, i64, i32, vp, vp, vp, vp, vp, sz,
                                                     vp]),

@@ -148,6 +148,8 @@ def test_entry_points_reject_bad_arguments_before_launch(L):
     assert L.ltd_tree_attention_next(*bad) == 3
     assert L.ltd_debug_attention_wait(1000, 1025) == 1                            # too many
     assert L.ltd_debug_attention_wait(0, 0) == 0
+    assert L.ltd_debug_expand_wait(1000, 1025) == 1                               # offset too big
+    assert L.ltd_debug_expand_wait(0, 0) == 0
     assert L.ltd_accept_workspace_bytes(1, 8, 1000) > 0
     assert L.ltd_accept_workspace_bytes(1, 300, 1000) == 0
     kv = ltd.ltd_kv_cache(fake, fake, 1, 1, 70, 256, 1)                            # 140-byte rows

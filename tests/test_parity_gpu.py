@@ -417,10 +417,12 @@ def test_determinism_and_reuse_of_scratch():
 
 
 # --------------------------------------------------------------------- edge cases
-def _small_tree(W, L, vocab, seed, dtype=wl.F32):
+def _small_tree(W, L, vocab, seed, dtype=wl.F32, rows=None):
     rng = np.random.default_rng(seed)
     R = 1 + (L - 1) * W
-    rows = wl.round_to(rng.standard_normal((1, R, vocab)).astype(np.float32), dtype)
+    if rows is None:
+        rows = rng.standard_normal((1, R, vocab)).astype(np.float32)
+    rows = wl.round_to(rows, dtype)
     root = int(rng.integers(vocab))
     ci = wl.CycleInputs(wl.config("tiny", W=W, vocab=vocab, depth_range=(L, L), dtype=dtype),
                         seed, np.array([root], np.int32), np.array([L], np.int32),
@@ -430,9 +432,11 @@ def _small_tree(W, L, vocab, seed, dtype=wl.F32):
 
 
 @pytest.mark.parametrize("W,L,vocab", [(1, 6, 64), (2, 1, 8), (3, 4, 24), (32, 2, 4096),
-                                       (5, 3, 1000 + 8 * 37)])
+                                       (5, 3, 1000 + 8 * 37), (32, 2, 40000)])
 def test_expand_and_select_shapes(W, L, vocab):
-    """k = 1 chains, a single level, k = 32, vocab not a multiple of the chunk."""
+    """k = 1 chains, a single level, k = 32, vocab not a multiple of the
+    vocabulary item; k = 32 over five items per row is more than the merging
+    CTA keeps in shared memory, so its warps merge the rows' item lists."""
     ci = _small_tree(W, L, vocab, seed=W * 7 + L)
     cfg = ci.cfg
     tree = H.gpu_draft(cfg, ci, H.dev(ci.draft_rows, wl.F32))
@@ -448,6 +452,78 @@ def test_expand_and_select_shapes(W, L, vocab):
         assert np.array_equal(mask.cpu().numpy()[0].view(np.uint32), words)
         if W == 1:
             assert np.array_equal(rmask, np.tril(np.ones((N, N), bool)))
+
+
+@pytest.mark.parametrize("dtype", [wl.F32, wl.BF16])
+def test_expand_exact_ties_and_overflowing_candidate_lists(dtype):
+    """Logits min(floor(z), 1): about one entry in six ties at the row's
+    maximum, so every vocabulary item's candidate list overflows and the
+    exact fallback ranks it; the row of frontier rank 0 at level 2 is all
+    zeros (every token tied).  Tokens, parents, frontiers bit-exact: tied
+    logits go to the lower token, tied children to the lower node id."""
+    W, L, vocab = 6, 3, 3 * 8192 + 8 * 13
+    rng = np.random.default_rng(17)
+    rows = np.minimum(np.floor(rng.standard_normal((1, 1 + (L - 1) * W, vocab))), 1.0)
+    rows = rows.astype(np.float32)
+    rows[0, 1] = 0.0
+    ci = _small_tree(W, L, vocab, seed=17, dtype=dtype, rows=rows)
+    otree = oracle.grow_tree(int(ci.root[0]), ci.draft_rows[0], W, L)
+    assert H.tree_margin(otree, W) > H.CUT_MARGIN, "near-tie deciding a frontier"
+    tree = H.gpu_draft(ci.cfg, ci, H.dev(ci.draft_rows, dtype))
+    assert ltd.ltd_check() == 0
+    H.compare_trees(ci.cfg, ci, tree, [otree])
+    v = tree.view()
+    first = 1 + W                               # children of the all-zero row
+    assert v["token"][0, first:first + W].tolist() == list(range(W))
+
+
+def test_expand_rows_that_repeat_every_item():
+    """Each row repeats the same decreasing logits every 8192 tokens (one
+    vocabulary item), scaled per row, so the row's best tokens are tied
+    across the items (ties to the lower token) and nine of every item's ten
+    listed keys reach the row's threshold: the merging CTA's candidate list
+    for the row overflows and it ranks the row among all of its item keys."""
+    W, L, vocab = 10, 3, 7 * 8192
+    R = 1 + (L - 1) * W
+    t = (np.arange(vocab) % 8192).astype(np.float64)
+    rows = np.stack([-(t * 0.001) * (1.0 + 0.05 * r) for r in range(R)])[None].astype(np.float32)
+    ci = _small_tree(W, L, vocab, seed=23, rows=rows)
+    otree = oracle.grow_tree(int(ci.root[0]), ci.draft_rows[0], W, L)
+    assert H.tree_margin(otree, W) > H.CUT_MARGIN, "near-tie deciding a frontier"
+    tree = H.gpu_draft(ci.cfg, ci, H.dev(ci.draft_rows, wl.F32))
+    assert ltd.ltd_check() == 0
+    H.compare_trees(ci.cfg, ci, tree, [otree])
+    # level 1: the seven items' first tokens (tied), then three second tokens
+    assert tree.view()["token"][0, 1:1 + W].tolist() == [8192 * c for c in range(7)] + [1, 8193, 16385]
+
+
+def test_expand_wait_runs_out_and_level_stays_unbuilt():
+    """The expansion's bounded wait, run out without a GPU fault: the test
+    hook makes the merging CTA wait for a tag no record carries, with a 2 ms
+    limit.  ltd_check returns LTD_ERR_TIMEOUT with the TIMEOUT bit and the
+    level stays unbuilt (n_levels 0, n_nodes 1); with the hook reset the
+    same tree grows to the oracle's tree."""
+    import ctypes as C
+    ci = _small_tree(4, 3, 20000, seed=5)
+    cfg = ci.cfg
+    draft = H.dev(ci.draft_rows, wl.F32)
+    tree = ltd.Tree(1, cfg.max_depth, cfg.W, cfg.vocab)
+    ltd.ltd_tree_reset(tree, H.i32(ci.root))
+    L = ltd.lib()
+    assert L.ltd_debug_expand_wait(2_000_000, 7) == 0
+    try:
+        ltd.ltd_expand_tree(tree, 1, draft)
+        bits = C.c_uint32(0)
+        st = L.ltd_check(None, C.byref(bits))
+    finally:
+        assert L.ltd_debug_expand_wait(0, 0) == 0
+    assert L.ltd_status_string(st).decode() == "LTD_ERR_TIMEOUT"
+    assert bits.value == 0x10
+    v = tree.view()
+    assert v["n_levels"].item() == 0 and v["n_nodes"].item() == 1
+    tree = H.gpu_draft(cfg, ci, draft, tree)
+    assert ltd.ltd_check() == 0
+    H.compare_trees(cfg, ci, tree, [oracle.grow_tree(int(ci.root[0]), ci.draft_rows[0], cfg.W, 3)])
 
 
 def test_single_node_verify_is_autoregressive():

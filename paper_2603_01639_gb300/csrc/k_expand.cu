@@ -495,6 +495,30 @@ __device__ __forceinline__ void warp_topk_lists(const uint64_t* lists, int L, in
   __syncwarp();
 }
 
+// One warp: the k largest keys of L <= 32 sorted lists (list i at lists +
+// i stride, k keys each, descending; keys unique), by a k-way merge: lane i
+// holds list i's head; each step takes the largest head (a warp maximum of
+// the upper 32 bits, then of the lower ones among those that hold it) into
+// top[step], and its lane moves to the next key.  Empty keys (value bits 0)
+// sit below every real key, exhausted lists below them.
+__device__ __forceinline__ void warp_kway_topk(const uint64_t* lists, int L, int stride, int k, uint64_t* top) {
+  const int lane = threadIdx.x & 31;
+  int ptr = 0;
+  uint64_t head = (lane < L) ? lists[lane * stride] : 0ull;
+#pragma unroll 1
+  for (int r = 0; r < k; ++r) {
+    const uint32_t hi = static_cast<uint32_t>(head >> 32), lo = static_cast<uint32_t>(head);
+    const uint32_t mhi = __reduce_max_sync(0xFFFFFFFFu, hi);
+    const uint32_t mlo = __reduce_max_sync(0xFFFFFFFFu, hi == mhi ? lo : 0u);
+    if (hi == mhi && lo == mlo) {
+      top[r] = head;
+      ++ptr;
+      head = (ptr < k) ? lists[lane * stride + ptr] : 0ull;
+    }
+  }
+  __syncwarp();
+}
+
 // Consumer of a sequence whose records fit shared memory (F chunks (k + 2)
 // words <= kRecBuf): the records are copied in once every word carries the
 // tag (a bounded wait), then one warp per row merges them.  Returns false
@@ -544,7 +568,10 @@ __device__ bool consume_smem(const ExpandParams& p, ExpandShared& sh, int b, int
   const int k = p.k, C = p.chunks, rw = k + 2;
   for (int f = warp; f < F; f += kNW) {
     const uint64_t* row = &co.rec[f * C * rw];
-    warp_topk_lists(row, C, rw, k, p.j_row, &co.vals[f * kWarp], co.cand[f], &co.top[f * k]);
+    if (C <= kWarp)
+      warp_kway_topk(row, C, rw, k, &co.top[f * k]);
+    else
+      warp_topk_lists(row, C, rw, k, 0, &co.vals[f * kWarp], co.cand[f], &co.top[f * k]);
     const float lse = row_lse(row, C, rw, k);
     if ((tid & 31) == 0) co.lse[f] = lse;
   }
@@ -663,18 +690,11 @@ __device__ void consume_sequence(const ExpandParams& p, ExpandShared& sh, int b,
   if (p.level == 1) {
     if (tid < k) p.frontier[b * k + tid] = 1 + tid;
   } else {
-    // the k best of the F k children: each child's rank is the number of
-    // larger children (keys are unique), counted by a warp (its lanes split
-    // the children, a warp sum adds their counts); the warps take turns
-    const int nch = F * k, warp = tid >> 5, lane = tid & 31;
-#pragma unroll 1
-    for (int i = warp; i < nch; i += kNW) {
-      const uint64_t key = co.child[i];
-      int r = 0;
-#pragma unroll 1
-      for (int j = lane; j < nch; j += kWarp) r += (co.child[j] > key) ? 1 : 0;
-      r = __reduce_add_sync(0xFFFFFFFFu, r);
-      if (lane == 0 && r < k) p.frontier[b * k + r] = static_cast<int32_t>(key_index(key));
+    // the k best of the F k children (each row's list is sorted): a k-way
+    // merge in warp 0
+    if ((tid >> 5) == 0) {
+      warp_kway_topk(co.child, F, k, k, co.top);
+      if (tid < k) p.frontier[b * k + tid] = static_cast<int32_t>(key_index(co.top[tid]));
     }
   }
   if (tid == 0) {

@@ -1,8 +1,8 @@
 // Acceptance and KV compaction (LTD section 3.2, "Draft Tree Verification").
 //
-// accept_rows_kernel: grid (chunks, n_max, batch).  Each CTA scans one chunk
-// of one verified slot's target row and records (max m, sum exp((x - m) / T),
-// argmax key) in the workspace.
+// accept_rows_kernel: every 16 KB unit of every verified slot's target row
+// gets (max m, sum exp((x - m) / T), argmax key) in the workspace, one
+// 256-thread CTA per unit.
 // accept_walk_kernel: one thread-block cluster of C CTAs per sequence.
 //  - greedy: rank 0 merges the argmax records (ties to the lower token id),
 //    marks every slot whose token is its parent's argmax, and follows those
@@ -47,104 +47,115 @@ constexpr int64_t kSliceMax = 16384;  // vocabulary elements per walk CTA
 constexpr int kMaxWalkCluster = static_cast<int>(kAcceptMaxVocab / kSliceMax);
 static_assert(LTD_MAX_N <= kNT, "one verified slot per walk thread");
 
+// 2^x by the hardware's approximate base-2 exponential (ex2.approx.ftz).
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+constexpr int kRowUnitBytes = 16384;  // one unit: 16 KB of one verified row
+constexpr int kRowNT = 256;            // one CTA per unit
+constexpr int kRowNW = kRowNT / kWarp;
+constexpr int kRowVecs = kRowUnitBytes / 16 / kRowNT;  // 16-byte vectors per thread
+
+// Row statistics of the verified slots' target rows: every unit (16 KB of
+// one row) gets (max m, sum exp((x - m) / T), argmax key) in the workspace,
+// one CTA per unit.  Each thread's four loads are in flight before the first
+// is used; the warps' partials meet in shared memory after one barrier.
 template <typename T>
-__global__ void __launch_bounds__(kNT) accept_rows_kernel(const AcceptParams p) {
+__global__ void __launch_bounds__(kRowNT, 8) accept_rows_kernel(const AcceptParams p) {
   constexpr int VEC = 16 / sizeof(T);
-  constexpr int U = 2;
-  __shared__ float red[2 * kNW];
-  __shared__ uint64_t redk[kNW];
+  __shared__ float pm[kRowNW], ps[kRowNW];
+  __shared__ uint64_t pk[kRowNW];
   grid_wait();
   trigger_dependents();
-
-  const int ch = blockIdx.x, i = blockIdx.y, b = blockIdx.z, tid = threadIdx.x;
-  const int N = p.n_verify[b];
-  if (N < 1 || N > p.n_max || i >= N) return;
-
-  const T* row = reinterpret_cast<const T*>(p.target) +
-                 (static_cast<int64_t>(b) * p.n_max + i) * p.vocab;
-  const int64_t lo = static_cast<int64_t>(ch) * p.chunk_elems;
-  const int64_t hi = min(lo + p.chunk_elems, p.vocab);
-  float m = -CUDART_INF_F, s = 0.f;
-  uint64_t best = 0ull;
-  for (int64_t base = lo + static_cast<int64_t>(tid) * VEC; base < hi;
-       base += static_cast<int64_t>(kNT) * VEC * U) {
-    float xv[U][VEC];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int u = static_cast<int>(blockIdx.x);
+  const int c = u % p.chunks, bi = u / p.chunks;
+  const int i = bi % p.n_max, b = bi / p.n_max;
+  const int N = __ldcg(p.n_verify + b);
+  const int mode = __ldcg(p.mode + b);
+  if (N < 1 || N > p.n_max || i >= N) return;  // (the walk flags a bad N)
+  const int lo = c * static_cast<int>(p.chunk_elems);
+  const int n_here = min(static_cast<int>(p.chunk_elems), static_cast<int>(p.vocab) - lo);
+  const T* row = reinterpret_cast<const T*>(p.target) + (static_cast<int64_t>(b) * p.n_max + i) * p.vocab + lo;
+  uint4 v[kRowVecs];
 #pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int64_t idx = base + static_cast<int64_t>(u) * kNT * VEC;
-      if (idx + VEC <= hi) {
-        unpack16(ld_stream16(row + idx), xv[u], static_cast<const T*>(nullptr));
-      } else {
+  for (int k = 0; k < kRowVecs; ++k) {
+    const int e = (k * kRowNT + tid) * VEC;  // rows end on a 16-byte boundary
+    v[k] = (e < n_here) ? ld_stream16_once(row + e)
+                        : ((sizeof(T) == 4) ? make_uint4(0xFF800000u, 0xFF800000u, 0xFF800000u, 0xFF800000u)
+                                            : make_uint4(0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u));
+  }
+  // the thread's max (the first, so the lowest token) and -- for the
+  // stochastic rules only: greedy needs no normaliser -- its sum of
+  // 2^((x - max) c), c = log2(e) / T, one vector at a time (the sum
+  // rescaled when the max grows)
+  const bool stoch = mode != LTD_GREEDY;
+  const float cl = p.inv_t * 1.4426950408889634f;
+  float tm = -CUDART_INF_F, ts = 0.f;
+  int ti = 0;
 #pragma unroll
-        for (int j = 0; j < VEC; ++j)
-          xv[u][j] = (idx + j < hi) ? to_f<T>(row[idx + j]) : -CUDART_INF_F;
+  for (int k = 0; k < kRowVecs; ++k) {
+    float vm = -CUDART_INF_F;
+    int jm = 0;
+#pragma unroll
+    for (int j = 0; j < VEC; ++j) {
+      const float x = elem<T>(v[k], j);
+      if (x > vm) {
+        vm = x;
+        jm = j;
       }
     }
+    if (vm > tm) {
+      ts = (stoch && tm > -CUDART_INF_F) ? ts * ex2_approx((tm - vm) * cl) : 0.f;
+      tm = vm;
+      ti = (k * kRowNT + tid) * VEC + jm;
+    }
+    if (stoch && tm > -CUDART_INF_F) {
+      const float off = -tm * cl;
 #pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int64_t idx = base + static_cast<int64_t>(u) * kNT * VEC;
-      float vm = -CUDART_INF_F;
-      int jm = 0;
-#pragma unroll
-      for (int j = 0; j < VEC; ++j)
-        if (xv[u][j] > vm) {
-          vm = xv[u][j];
-          jm = j;
-        }
-      if (vm > m) {
-        s *= __expf((m - vm) * p.inv_t);
-        m = vm;
-      }
-      float add = 0.f;
-#pragma unroll
-      for (int j = 0; j < VEC; ++j)
-        add += (xv[u][j] == -CUDART_INF_F) ? 0.f : __expf((xv[u][j] - m) * p.inv_t);
-      s += add;
-      if (idx < hi) {
-        const uint64_t key = make_key(vm, static_cast<uint32_t>(idx + jm));
-        best = key > best ? key : best;
-      }
+      for (int j = 0; j < VEC; ++j) ts += ex2_approx(fmaf(elem<T>(v[k], j), cl, off));
     }
   }
-  // the chunk's max first (no exponentials), then each thread's sum rescaled
-  // to it once; only thread 0 needs the results
-  const int lane = tid & 31, warp = tid >> 5;
-  float wm = m;
-  uint64_t wb = best;
+  // warp, then CTA: the max first, then each sum rescaled to it
+  float M = tm;
+  uint64_t K = (tm > -CUDART_INF_F) ? make_key(tm, static_cast<uint32_t>(lo + ti)) : 0ull;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
-    wm = fmaxf(wm, __shfl_xor_sync(0xFFFFFFFFu, wm, o));
-    const uint64_t ob = __shfl_xor_sync(0xFFFFFFFFu, wb, o);
-    wb = ob > wb ? ob : wb;
+    M = fmaxf(M, __shfl_xor_sync(0xFFFFFFFFu, M, o));
+    const uint64_t ok = __shfl_xor_sync(0xFFFFFFFFu, K, o);
+    K = ok > K ? ok : K;
   }
+  float e = (tm > -CUDART_INF_F) ? ts * __expf((tm - M) * p.inv_t) : 0.f;
+  e = warp_sum_f(e);
   if (lane == 0) {
-    red[warp] = wm;
-    redk[warp] = wb;
+    pm[warp] = M;
+    ps[warp] = e;
+    pk[warp] = K;
   }
   __syncthreads();
-  float M = red[0];
+  if (warp == 0) {
+    float wm = lane < kRowNW ? pm[lane] : -CUDART_INF_F;
+    float we = lane < kRowNW ? ps[lane] : 0.f;
+    uint64_t wk = lane < kRowNW ? pk[lane] : 0ull;
+    float MM = wm;
 #pragma unroll
-  for (int w = 1; w < kNW; ++w) M = fmaxf(M, red[w]);
-  float e = (m > -CUDART_INF_F) ? s * __expf((m - M) * p.inv_t) : 0.f;
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) e += __shfl_xor_sync(0xFFFFFFFFu, e, o);
-  __syncthreads();  // every thread has read the maxima
-  if (lane == 0) red[warp] = e;
-  __syncthreads();
-  if (tid == 0) {
-    float S = 0.f;
-    uint64_t B = 0ull;
-    for (int w = 0; w < kNW; ++w) {
-      S += red[w];
-      B = redk[w] > B ? redk[w] : B;
+    for (int o = kRowNW / 2; o > 0; o >>= 1) {
+      MM = fmaxf(MM, __shfl_xor_sync(0xFFFFFFFFu, MM, o));
+      const uint64_t ok = __shfl_xor_sync(0xFFFFFFFFu, wk, o);
+      wk = ok > wk ? ok : wk;
     }
-    m = M;
-    s = S;
-    best = B;
-    AcceptRecord* r = p.rec + (static_cast<int64_t>(b) * p.n_max + i) * p.chunks + ch;
-    r->m = m;
-    r->s = s;
-    r->key = best;
+    float se = (wm > -CUDART_INF_F) ? we * __expf((wm - MM) * p.inv_t) : 0.f;
+#pragma unroll
+    for (int o = kRowNW / 2; o > 0; o >>= 1) se += __shfl_xor_sync(0xFFFFFFFFu, se, o);
+    if (lane == 0) {
+      AcceptRecord* r = p.rec + static_cast<int64_t>(u);  // [batch][n_max][chunks] = unit order
+      r->m = MM;
+      r->s = se;
+      r->key = wk;
+    }
   }
 }
 
@@ -182,6 +193,7 @@ struct WalkShared {
   int32_t path[LTD_MAX_DEPTH + 1];
   float red[2 * kNW];
   uint64_t redk[kNW];
+  unsigned long long bestk[LTD_MAX_N];  // greedy: each slot's argmax key
   float kp[LTD_MAX_N];      // p and q of the current slot's children
   float kq[LTD_MAX_N];
   float wpart[2][kMaxWalkCluster][kNW];  // every CTA's warp sums, by round parity
@@ -230,11 +242,16 @@ template <typename T>
 __global__ void __launch_bounds__(kNT) accept_walk_kernel(const AcceptParams p, int C,
                                                           int64_t slice, int vec_ok) {
   __shared__ WalkShared sh;
+  for (int j = threadIdx.x; j < LTD_MAX_N; j += kNT) sh.bestk[j] = 0ull;
+  __syncthreads();
   grid_wait();
   trigger_dependents();
   const int rank = blockIdx.x, b = blockIdx.y, tid = threadIdx.x;
-  const int N = p.n_verify[b];
-  const int mode = p.mode[b];
+  // the sequence's scalars and its slots' node ids are fetched together
+  // (the node ids do not depend on N; one slot per thread, n_max <= kNT)
+  const int N = __ldcg(p.n_verify + b);
+  const int mode = __ldcg(p.mode + b);
+  const int nid_pre = (tid < p.n_max) ? __ldcg(p.node_ids + static_cast<int64_t>(b) * p.n_max + tid) : 0;
   int32_t* path_out = p.path + static_cast<int64_t>(b) * (p.max_depth + 1);
   // everything below is uniform over the cluster (one sequence)
   if (N < 1 || N > p.n_max ||
@@ -253,16 +270,23 @@ __global__ void __launch_bounds__(kNT) accept_walk_kernel(const AcceptParams p, 
 
   const int64_t nb = static_cast<int64_t>(b) * p.max_nodes;
   const int64_t V = p.vocab;
-  for (int j = tid; j < N; j += kNT) {
-    const int nid = p.node_ids[static_cast<int64_t>(b) * p.n_max + j];
-    sh.node[j] = nid;
-    sh.tok[j] = p.token[nb + nid];
-    sh.next[j] = -1;
+  if (mode == LTD_GREEDY) {
+    // every slot's argmax over its row's units: one pass over the records
+    // (all loads independent), max-combined in shared memory
+    const AcceptRecord* r0 = p.rec + static_cast<int64_t>(b) * p.n_max * p.chunks;
+    for (int r = tid; r < N * p.chunks; r += kNT) atomicMax(&sh.bestk[r / p.chunks], r0[r].key);
+  }
+  // each slot's token and parent node (both loads in flight together)
+  if (tid < N) {
+    sh.node[tid] = nid_pre;
+    sh.tok[tid] = p.token[nb + nid_pre];
+    sh.pslot[tid] = p.parent[nb + nid_pre];  // the parent's node id for now
+    sh.next[tid] = -1;
   }
   __syncthreads();
-  for (int j = tid; j < N; j += kNT) {
-    const int par = p.parent[nb + sh.node[j]];
-    int lo = 0, hi = j - 1, found = -1;  // slots hold ascending node ids
+  if (tid < N) {
+    const int par = sh.pslot[tid];
+    int lo = 0, hi = tid - 1, found = -1;  // slots hold ascending node ids
     while (lo <= hi) {
       const int mid = (lo + hi) >> 1;
       const int v = sh.node[mid];
@@ -273,7 +297,7 @@ __global__ void __launch_bounds__(kNT) accept_walk_kernel(const AcceptParams p, 
       if (v < par) lo = mid + 1;
       else hi = mid - 1;
     }
-    sh.pslot[j] = found;
+    sh.pslot[tid] = found;  // (only this thread reads its entry)
   }
   __syncthreads();
   // log-sum-exp of the target row at slot over the vocabulary, in units of
@@ -297,12 +321,7 @@ __global__ void __launch_bounds__(kNT) accept_walk_kernel(const AcceptParams p, 
   };
 
   if (mode == LTD_GREEDY) {
-    for (int j = tid; j < N; j += kNT) {
-      const AcceptRecord* r = p.rec + (static_cast<int64_t>(b) * p.n_max + j) * p.chunks;
-      unsigned long long best = 0ull;
-      for (int c = 0; c < p.chunks; ++c) best = r[c].key > best ? r[c].key : best;
-      sh.am[j] = static_cast<int32_t>(key_index(best));
-    }
+    for (int j = tid; j < N; j += kNT) sh.am[j] = static_cast<int32_t>(key_index(sh.bestk[j]));
     __syncthreads();
     // sibling tokens are distinct, so each slot has at most one matching child
     for (int j = 1 + tid; j < N; j += kNT)
@@ -639,17 +658,23 @@ cudaError_t launch_append(const AppendParams& p, cudaStream_t s) {
   return launch(kv_append_kernel, grid, dim3(kCompactNT), 0, s, nullptr, 0, p);
 }
 
+// One record per row unit, sized for the smaller (fp32) unit.
 size_t accept_workspace(int32_t batch, int32_t n_max, int64_t vocab) {
-  const VocabSplit vs =
-      vocab_split(static_cast<int64_t>(batch) * n_max, vocab, kAcceptTargetCtas, kAcceptMinElems);
-  const size_t rec = static_cast<size_t>(batch) * n_max * vs.chunks * sizeof(AcceptRecord);
+  const int64_t unit = kRowUnitBytes / 4;
+  const size_t rec = static_cast<size_t>(batch) * n_max * ((vocab + unit - 1) / unit) * sizeof(AcceptRecord);
   return (rec + 255) / 256 * 256;
 }
 
 template <typename T>
-cudaError_t launch_accept_t(const AcceptParams& p, int32_t batch, cudaStream_t s) {
-  cudaError_t e = launch(accept_rows_kernel<T>, dim3(p.chunks, p.n_max, batch), dim3(kNT), 0, s,
-                         nullptr, 0, p);
+cudaError_t launch_accept_t(const AcceptParams& params, int32_t batch, cudaStream_t s) {
+  AcceptParams p = params;
+  p.chunk_elems = kRowUnitBytes / static_cast<int>(sizeof(T));
+  p.chunks = static_cast<int32_t>((p.vocab + p.chunk_elems - 1) / p.chunk_elems);
+  const int64_t units = static_cast<int64_t>(batch) * p.n_max * p.chunks;
+  if (units > 0x7FFFFFFF) return cudaErrorInvalidValue;
+  p.n_units = static_cast<int32_t>(units);
+  cudaError_t e = launch(accept_rows_kernel<T>, dim3(static_cast<unsigned>(units)), dim3(kRowNT), 0, s, nullptr,
+                         0, p);
   if (e != cudaSuccess) return e;
   // walk cluster: enough CTAs that a vocabulary slice of p and q fits the
   // threads' registers (kSliceMax elements per CTA)

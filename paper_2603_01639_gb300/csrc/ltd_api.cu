@@ -557,8 +557,6 @@ ltd_status accept_impl(const ltd_tree* tree, const void* d_target_logits, const 
   }
   uint32_t* err = device_error_word();
   if (err == nullptr) return LTD_ERR_CUDA;
-  const VocabSplit vs = vocab_split(static_cast<int64_t>(tree->batch) * n_max, vocab,
-                                    kAcceptTargetCtas, kAcceptMinElems);
   AcceptParams p{};
   p.token = tree->token;
   p.parent = tree->parent;
@@ -584,8 +582,6 @@ ltd_status accept_impl(const ltd_tree* tree, const void* d_target_logits, const 
   p.rec = static_cast<AcceptRecord*>(d_workspace);
   p.inv_t = temperature == 1.f ? 1.f : 1.f / temperature;
   p.tempered = temperature != 1.f;
-  p.chunks = vs.chunks;
-  p.chunk_elems = vs.chunk_elems;
   p.err = err;
   const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   cudaError_t e = launch_accept(p, tree->batch, dtype, s);

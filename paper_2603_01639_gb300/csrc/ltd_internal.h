@@ -222,8 +222,9 @@ struct AcceptParams {
   AcceptRecord* rec;  // [batch][n_max][chunks]
   float inv_t;        // 1 / temperature of the stochastic rules (1 at T = 1)
   int32_t tempered;   // T != 1: the draft rows' normaliser is computed in the walk
-  int32_t chunks;
-  int64_t chunk_elems;
+  int32_t chunks;         // units per row (set by the launch)
+  int64_t chunk_elems;    // entries per unit (set by the launch)
+  int32_t n_units;        // batch * n_max * chunks (set by the launch)
   uint32_t* err;
 };
 size_t accept_workspace(int32_t batch, int32_t n_max, int64_t vocab);

@@ -54,7 +54,38 @@ def _args():
     ap.add_argument("--no-next-hint", action="store_true",
                     help="run the cycle without the next-layer L2 hint (for profiling one layer's "
                          "own traffic)")
+    ap.add_argument("--profile-case", default=None, choices=["draft", "select", "accept"],
+                    help="no timing: run one phase of the --config workload three times, eagerly, "
+                         "for a profiler to capture (draft: reset + levels 1..3; select: the whole "
+                         "draft + selection; accept: the acceptance row pass and walk)")
     return ap.parse_args()
+
+
+def run_profile_case(args):
+    """Eager calls of one phase for an external profiler; prints "ok"."""
+    import torch
+    from paper_2603_01639_gb300 import build, ltd
+    from paper_2603_01639_gb300 import workload as wl
+    build.build()
+    cfg = wl.config(args.config)
+    device = torch.device("cuda")
+    cyc = Cycle(cfg, 1, args.seed, device)
+    for _ in range(3):
+        if args.profile_case == "accept":
+            ltd.ltd_accept(cyc.tree, cyc.target, cyc.draft, cyc.sel[0], cyc.n_verify, cyc.mode, cyc.ctx,
+                           seed=1234, cycle=0, workspace=cyc.acc_ws, out=cyc.acc)
+            continue
+        ltd.ltd_tree_reset(cyc.tree, cyc.root)
+        last = 3 if args.profile_case == "draft" else cyc.max_depth
+        for level in range(1, last + 1):
+            ltd.ltd_expand_tree(cyc.tree, level, cyc.draft, active=cyc.actives[level])
+        if args.profile_case == "select":
+            ltd.ltd_select_verify(cyc.tree, cyc.n_verify, cfg.max_n, cyc.ctx, out=cyc.sel)
+    torch.cuda.synchronize()
+    if ltd.ltd_check() != 0:
+        raise RuntimeError("device error flagged")
+    print("ok", args.profile_case, args.config)
+    return 0
 
 
 def _dist():
@@ -1058,6 +1089,8 @@ def run_e2e(cyc, args, device):
 
 def main():
     args = _args()
+    if args.profile_case:
+        return run_profile_case(args)
     if args.impl == "reference":
         return run_reference(args)
     return run_ours(args)

@@ -734,6 +734,16 @@ def test_attention_ragged_split_batch():
     _attention_case("8b", 6, batch=3, ctx_range=(20, 3000), n_choices=(7, 33, 60))
 
 
+@pytest.mark.parametrize("name,hq,hkv,ctx,n", [("8b", 8, 2, 3968, 60), ("13b", 60, 60, 2048, 64),
+                                                ("13b", 15, 15, 2600, 64)])
+def test_attention_split_counts(name, hq, hkv, ctx, n):
+    """On a 152-SM device these shapes cut each unit's keys into 32 splits of
+    one chunk (4 units, 32 chunks), 2 splits (60 units) and 7 splits (15
+    units, 21 chunks): the most, the fewest and an odd count, each combined
+    through the workspace."""
+    _attention_case(name, 40 + hq, hq=hq, hkv=hkv, ctx_range=(ctx, ctx), n_choices=(n,))
+
+
 def test_attention_flags_bad_sequence():
     """A sequence with ctx past max_ctx is flagged and left untouched, in
     both launch shapes (split keys; one split per unit, longest first), and

@@ -51,9 +51,11 @@ def _args():
     ap.add_argument("--min-timed-ms", type=float, default=250.0,
                     help="each step replays the cycle graph enough times that the K timed steps "
                          "last at least this long (so the clock sampler sees the load)")
+    ap.add_argument("--next-hint", action="store_true",
+                    help="give every layer's attention call the next layer's caches as an L2 "
+                         "prefetch hint (measured slower on GB300 at these shapes: off by default)")
     ap.add_argument("--no-next-hint", action="store_true",
-                    help="run the cycle without the next-layer L2 hint (for profiling one layer's "
-                         "own traffic)")
+                    help="the default (kept so older command lines still run)")
     ap.add_argument("--profile-case", default=None, choices=["draft", "select", "accept"],
                     help="no timing: run one phase of the --config workload three times, eagerly, "
                          "for a profiler to capture (draft: reset + levels 1..3; select: the whole "
@@ -311,9 +313,11 @@ class Cycle:
             ltd.ltd_expand_tree(self.tree, level, self.draft, active=self.actives[level])
         ltd.ltd_select_verify(self.tree, self.n_verify, self.cfg.max_n, self.ctx, out=self.sel)
 
-    def verify_phase(self, hint=True):
-        # each layer asks L2 for the next layer's keys and values (a hint the
-        # library skips when one layer's K/V would crowd L2)
+    def verify_phase(self, hint=False):
+        # with hint, each layer asks L2 for the next layer's keys and values
+        # (a hint the library skips when one layer's K/V would crowd L2); the
+        # launches are latency-bound, so the prefetch only competes with the
+        # current layer's reads and the cycle runs without it
         for l in range(self.layers):
             nxt = l + 1 < self.layers and hint
             self.ltd.ltd_tree_attention(self.q[l], self.k[l], self.v[l], self.ctx, self.cfg.max_ctx,
@@ -324,6 +328,9 @@ class Cycle:
 
     def verify_phase_plain(self):
         self.verify_phase(hint=False)
+
+    def verify_phase_hinted(self):
+        self.verify_phase(hint=True)
 
     def accept_phase(self, cycle_no=0):
         self.ltd.ltd_accept(self.tree, self.target, self.draft, self.sel[0], self.n_verify,
@@ -480,6 +487,38 @@ def time_replays(torch, g, reps, device):
     return e0.elapsed_time(e1) / reps
 
 
+def phases_in_cycle(torch, cyc, verify, reps, device):
+    """Per-phase device time inside one CUDA graph of the whole cycle: event
+    record nodes between the phases (each one makes the next phase's first
+    kernel wait for the previous phase to finish, so the three add up to a
+    little more than the clean cycle).  The per-phase graphs of phases_us
+    also pay a graph launch each."""
+    names = ("draft_select", "attention_all_layers", "accept_compact")
+    try:
+        evs = [torch.cuda.Event(enable_timing=True, external=True) for _ in range(4)]
+
+        def full_ev():
+            evs[0].record()
+            cyc.draft_phase()
+            evs[1].record()
+            verify()
+            evs[2].record()
+            cyc.accept_phase()
+            evs[3].record()
+
+        g = _graph(torch, full_ev)
+        acc = [0.0, 0.0, 0.0]
+        for _ in range(reps):
+            g.replay()
+            torch.cuda.synchronize(device)
+            for i in range(3):
+                acc[i] += evs[i].elapsed_time(evs[i + 1])
+        del g
+        return {k: round(v / reps * 1e3, 2) for k, v in zip(names, acc)}
+    except (TypeError, RuntimeError) as e:
+        return {"unavailable": str(e).splitlines()[0][:160] if str(e) else type(e).__name__}
+
+
 def attention_roofline(cyc, launch_ms, bound):
     """Roofline of one tree-attention launch against its binding resource."""
     hbm, tc, src = load_peaks()
@@ -575,6 +614,7 @@ def summarize_config(name, args, device, seed, reps):
     res = {"workload": workload_desc(cfg, layers), "cycle_us": round(cycle_ms * 1e3, 2),
            "cycle_us_per_sequence": round(cycle_ms * 1e3 / cfg.batch, 2),
            "phases_us": {k: round(v * 1e3, 2) for k, v in phases.items()},
+           "phases_in_cycle_us": phases_in_cycle(torch, cyc, cyc.verify_phase, reps, device),
            "attention": attention_roofline(cyc, plain_ms / layers, BINDING[name]),
            "attention_launch_us_in_cycle": round(phases["attention_all_layers"] * 1e3 / layers, 3),
            "tokens_per_cycle": int((acc_len + 1).sum()),
@@ -690,7 +730,7 @@ def run_ours(args):
     layers = N_LAYERS[args.config]
     cyc = Cycle(cfg, layers, replica_seed(args.seed, rank), device)
 
-    verify = cyc.verify_phase_plain if args.no_next_hint else cyc.verify_phase
+    verify = cyc.verify_phase_hinted if args.next_hint else cyc.verify_phase_plain
 
     def full():
         cyc.draft_phase()
@@ -751,6 +791,7 @@ def run_ours(args):
     draft_ms = statistics.mean(ev[i][0].elapsed_time(ev[i][1]) for i in range(K))
     verify_ms = statistics.mean(ev[i][1].elapsed_time(ev[i][2]) for i in range(K))
     accept_ms = statistics.mean(ev[i][2].elapsed_time(ev[i][3]) for i in range(K))
+    in_cycle = phases_in_cycle(torch, cyc, verify, max(K, 10), device)
     ms_per_step, value_us = aggregate(total_ms, K, cfg.batch, world, device)
 
     # roofline of the dominant kernel (tree attention), on launches without
@@ -784,7 +825,7 @@ def run_ours(args):
                 "algorithmic_bytes_per_launch": att_bytes, "launch_us": round(att_launch_ms * 1e3, 3),
                 "launch_us_in_cycle": round(verify_ms / layers * 1e3, 3),
                 "note": "launch_us and achieved from launches without the next-layer L2 hint; "
-                        "launch_us_in_cycle is the cycle's own (hinted) per-layer time",
+                        "launch_us_in_cycle is the cycle's own per-layer time",
                 "tflops": round(att_flops / (att_launch_ms * 1e-3) / 1e12, 1),
                 "frac_of_8tbs": round(achieved / 8000.0, 4)}
 
@@ -857,10 +898,13 @@ def run_ours(args):
             "config": config_obj(cfg, layers),
             "timing": "CUDA events around K steps of R replays each of one CUDA graph of the "
                       "whole cycle; value = job time / cycles of all ranks; phases_us from "
-                      "per-phase graphs timed after it",
+                      "per-phase graphs timed after it (a graph launch each), phases_in_cycle_us "
+                      "from event nodes inside one graph of the cycle; attention layers " +
+                      ("with" if args.next_hint else "without") + " the next-layer L2 hint",
             "phases_us": {"draft_select": round(draft_ms * 1e3, 2),
                           "attention_all_layers": round(verify_ms * 1e3, 2),
                           "accept_compact": round(accept_ms * 1e3, 2)},
+            "phases_in_cycle_us": in_cycle,
             "accept_rules_us": rules,
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "policy": pol, "reward": reward,
             "gpu_launches": cyc.launches_per_step() * K * R, "clocks": clk,

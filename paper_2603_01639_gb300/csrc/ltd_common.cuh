@@ -83,21 +83,6 @@ struct WarpTopK {
     const uint64_t kth = __shfl_sync(0xFFFFFFFFu, v, k - 1);
     if (__any_sync(0xFFFFFFFFu, key > kth)) v = warp_merge_desc(v, warp_sort_desc(key));
   }
-  // a list already sorted descending across the lanes
-  __device__ __forceinline__ void merge_sorted(uint64_t sorted) { v = warp_merge_desc(v, sorted); }
-};
-
-// Four largest keys seen by one thread, descending, in registers.
-struct Top4 {
-  uint64_t t0, t1, t2, t3;
-  __device__ __forceinline__ void init() { t0 = t1 = t2 = t3 = 0ull; }
-  __device__ __forceinline__ void insert(uint64_t key) {
-    if (key <= t3) return;
-    if (key > t0) { t3 = t2; t2 = t1; t1 = t0; t0 = key; }
-    else if (key > t1) { t3 = t2; t2 = t1; t1 = key; }
-    else if (key > t2) { t3 = t2; t2 = key; }
-    else { t3 = key; }
-  }
 };
 
 // -------------------------------------------------------------- reductions
@@ -145,37 +130,6 @@ __device__ __forceinline__ void warp_ms(float& m, float& s) {
   }
 }
 
-// Block-wide (max, sumexp) merge; the result is valid in every thread.
-// `red` needs 2 * (blockDim.x / 32) floats of shared memory.
-template <int NT>
-__device__ __forceinline__ void block_ms(float& m, float& s, float* red) {
-  constexpr int NW = NT / kWarp;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  warp_ms(m, s);
-  __syncthreads();
-  if (lane == 0) {
-    red[warp] = m;
-    red[NW + warp] = s;
-  }
-  __syncthreads();
-  m = -CUDART_INF_F;
-  s = 0.f;
-  for (int w = 0; w < NW; ++w) ms_merge(m, s, red[w], red[NW + w]);
-}
-
-template <int NT>
-__device__ __forceinline__ float block_sum(float x, float* red) {
-  constexpr int NW = NT / kWarp;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  x = warp_sum_f(x);
-  __syncthreads();
-  if (lane == 0) red[warp] = x;
-  __syncthreads();
-  float t = 0.f;
-  for (int w = 0; w < NW; ++w) t += red[w];
-  return t;
-}
-
 template <int NT>
 __device__ __forceinline__ uint64_t block_max_u64(uint64_t x, uint64_t* red) {
   constexpr int NW = NT / kWarp;
@@ -187,24 +141,6 @@ __device__ __forceinline__ uint64_t block_max_u64(uint64_t x, uint64_t* red) {
   uint64_t t = 0;
   for (int w = 0; w < NW; ++w) t = red[w] > t ? red[w] : t;
   return t;
-}
-
-// Block-wide top list from the per-warp lists: writes the 32 largest keys,
-// descending, to out[0..32) (shared memory) and returns after a barrier.
-// `stage` needs (NT / 32) * 32 uint64 of shared memory.
-template <int NT>
-__device__ __forceinline__ void block_topk(const WarpTopK& wt, uint64_t* stage, uint64_t* out) {
-  constexpr int NW = NT / kWarp;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  stage[warp * kWarp + lane] = wt.v;
-  __syncthreads();
-  if (warp == 0) {
-    uint64_t v = stage[lane];
-#pragma unroll 1
-    for (int w = 1; w < NW; ++w) v = warp_merge_desc(v, stage[w * kWarp + lane]);
-    out[lane] = v;
-  }
-  __syncthreads();
 }
 
 // -------------------------------------------------------- counter uniforms
@@ -256,32 +192,6 @@ __device__ __forceinline__ float to_f<float>(float x) {
 template <>
 __device__ __forceinline__ float to_f<__nv_bfloat16>(__nv_bfloat16 x) {
   return __bfloat162float(x);
-}
-
-// 16-byte vector of VEC elements, converted to float.
-template <typename T>
-struct Vec16 {
-  static constexpr int N = 16 / sizeof(T);
-};
-
-__device__ __forceinline__ void unpack16(const uint4& u, float* out, const float*) {
-  out[0] = __uint_as_float(u.x);
-  out[1] = __uint_as_float(u.y);
-  out[2] = __uint_as_float(u.z);
-  out[3] = __uint_as_float(u.w);
-}
-__device__ __forceinline__ void unpack16(const uint4& u, float* out, const __nv_bfloat16*) {
-  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    out[2 * i] = __uint_as_float(w[i] << 16);
-    out[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
-  }
-}
-
-// Streaming 16-byte load that bypasses L1 (data read once).
-__device__ __forceinline__ uint4 ld_stream16(const void* p) {
-  return __ldcs(reinterpret_cast<const uint4*>(p));
 }
 
 // Element j of a 16-byte vector of T, as float (j a compile-time constant).

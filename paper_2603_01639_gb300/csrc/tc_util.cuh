@@ -118,48 +118,10 @@ __device__ __forceinline__ void mma_commit(uint32_t bar) {
                : "memory");
 }
 
-// 32 consecutive 32-bit columns of this thread's TMEM lane.  The registers
-// are tied through the wait so no use can be scheduled before it; the wait
-// touches no memory, so it does not force reloads of anything else.
+// 32 consecutive 32-bit columns of this thread's TMEM lane.
 struct Frag32 {
   uint32_t r[32];
 };
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, Frag32& f) {
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, "
-      "%12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, "
-      "%30, %31}, [%32];"
-      : "=r"(f.r[0]), "=r"(f.r[1]), "=r"(f.r[2]), "=r"(f.r[3]), "=r"(f.r[4]), "=r"(f.r[5]),
-        "=r"(f.r[6]), "=r"(f.r[7]), "=r"(f.r[8]), "=r"(f.r[9]), "=r"(f.r[10]), "=r"(f.r[11]),
-        "=r"(f.r[12]), "=r"(f.r[13]), "=r"(f.r[14]), "=r"(f.r[15]), "=r"(f.r[16]), "=r"(f.r[17]),
-        "=r"(f.r[18]), "=r"(f.r[19]), "=r"(f.r[20]), "=r"(f.r[21]), "=r"(f.r[22]), "=r"(f.r[23]),
-        "=r"(f.r[24]), "=r"(f.r[25]), "=r"(f.r[26]), "=r"(f.r[27]), "=r"(f.r[28]), "=r"(f.r[29]),
-        "=r"(f.r[30]), "=r"(f.r[31])
-      : "r"(taddr));
-}
-__device__ __forceinline__ void tmem_wait_ld(Frag32& f) {
-  asm volatile(
-      "tcgen05.wait::ld.sync.aligned;"
-      : "+r"(f.r[0]), "+r"(f.r[1]), "+r"(f.r[2]), "+r"(f.r[3]), "+r"(f.r[4]), "+r"(f.r[5]),
-        "+r"(f.r[6]), "+r"(f.r[7]), "+r"(f.r[8]), "+r"(f.r[9]), "+r"(f.r[10]), "+r"(f.r[11]),
-        "+r"(f.r[12]), "+r"(f.r[13]), "+r"(f.r[14]), "+r"(f.r[15]), "+r"(f.r[16]), "+r"(f.r[17]),
-        "+r"(f.r[18]), "+r"(f.r[19]), "+r"(f.r[20]), "+r"(f.r[21]), "+r"(f.r[22]), "+r"(f.r[23]),
-        "+r"(f.r[24]), "+r"(f.r[25]), "+r"(f.r[26]), "+r"(f.r[27]), "+r"(f.r[28]), "+r"(f.r[29]),
-        "+r"(f.r[30]), "+r"(f.r[31]));
-}
-__device__ __forceinline__ void tmem_st32(uint32_t taddr, const Frag32& f) {
-  asm volatile(
-      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
-      "%11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, "
-      "%29, %30, %31, %32};" ::"r"(taddr),
-      "r"(f.r[0]), "r"(f.r[1]), "r"(f.r[2]), "r"(f.r[3]), "r"(f.r[4]), "r"(f.r[5]), "r"(f.r[6]),
-      "r"(f.r[7]), "r"(f.r[8]), "r"(f.r[9]), "r"(f.r[10]), "r"(f.r[11]), "r"(f.r[12]),
-      "r"(f.r[13]), "r"(f.r[14]), "r"(f.r[15]), "r"(f.r[16]), "r"(f.r[17]), "r"(f.r[18]),
-      "r"(f.r[19]), "r"(f.r[20]), "r"(f.r[21]), "r"(f.r[22]), "r"(f.r[23]), "r"(f.r[24]),
-      "r"(f.r[25]), "r"(f.r[26]), "r"(f.r[27]), "r"(f.r[28]), "r"(f.r[29]), "r"(f.r[30]),
-      "r"(f.r[31])
-      : "memory");
-}
 // Load and wait in one statement: the destination registers are written by
 // the asynchronous load, so no instruction the compiler might place between
 // a separate load and wait (a copy, a reuse of a register it believes
@@ -174,28 +136,10 @@ __device__ __forceinline__ void tmem_ld32_sync(uint32_t taddr, Frag32& f) {
 struct Frag16 {
   uint32_t r[16];
 };
-__device__ __forceinline__ void tmem_st16(uint32_t taddr, const Frag16& f) {
-  asm volatile(
-      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
-      "%11, %12, %13, %14, %15, %16};" ::"r"(taddr),
-      "r"(f.r[0]), "r"(f.r[1]), "r"(f.r[2]), "r"(f.r[3]), "r"(f.r[4]), "r"(f.r[5]), "r"(f.r[6]),
-      "r"(f.r[7]), "r"(f.r[8]), "r"(f.r[9]), "r"(f.r[10]), "r"(f.r[11]), "r"(f.r[12]),
-      "r"(f.r[13]), "r"(f.r[14]), "r"(f.r[15])
-      : "memory");
-}
 // A whole 128-column row per thread (32x32b.x128) and a 64-column store.
 struct Frag128 {
   uint32_t r[128];
 };
-__device__ __forceinline__ void tmem_ld128(uint32_t taddr, Frag128& f) {
-  asm volatile("tcgen05.ld.sync.aligned.32x32b.x128.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32, %33, %34, %35, %36, %37, %38, %39, %40, %41, %42, %43, %44, %45, %46, %47, %48, %49, %50, %51, %52, %53, %54, %55, %56, %57, %58, %59, %60, %61, %62, %63, %64, %65, %66, %67, %68, %69, %70, %71, %72, %73, %74, %75, %76, %77, %78, %79, %80, %81, %82, %83, %84, %85, %86, %87, %88, %89, %90, %91, %92, %93, %94, %95, %96, %97, %98, %99, %100, %101, %102, %103, %104, %105, %106, %107, %108, %109, %110, %111, %112, %113, %114, %115, %116, %117, %118, %119, %120, %121, %122, %123, %124, %125, %126, %127}, [%128];"
-               : "=r"(f.r[0]), "=r"(f.r[1]), "=r"(f.r[2]), "=r"(f.r[3]), "=r"(f.r[4]), "=r"(f.r[5]), "=r"(f.r[6]), "=r"(f.r[7]), "=r"(f.r[8]), "=r"(f.r[9]), "=r"(f.r[10]), "=r"(f.r[11]), "=r"(f.r[12]), "=r"(f.r[13]), "=r"(f.r[14]), "=r"(f.r[15]), "=r"(f.r[16]), "=r"(f.r[17]), "=r"(f.r[18]), "=r"(f.r[19]), "=r"(f.r[20]), "=r"(f.r[21]), "=r"(f.r[22]), "=r"(f.r[23]), "=r"(f.r[24]), "=r"(f.r[25]), "=r"(f.r[26]), "=r"(f.r[27]), "=r"(f.r[28]), "=r"(f.r[29]), "=r"(f.r[30]), "=r"(f.r[31]), "=r"(f.r[32]), "=r"(f.r[33]), "=r"(f.r[34]), "=r"(f.r[35]), "=r"(f.r[36]), "=r"(f.r[37]), "=r"(f.r[38]), "=r"(f.r[39]), "=r"(f.r[40]), "=r"(f.r[41]), "=r"(f.r[42]), "=r"(f.r[43]), "=r"(f.r[44]), "=r"(f.r[45]), "=r"(f.r[46]), "=r"(f.r[47]), "=r"(f.r[48]), "=r"(f.r[49]), "=r"(f.r[50]), "=r"(f.r[51]), "=r"(f.r[52]), "=r"(f.r[53]), "=r"(f.r[54]), "=r"(f.r[55]), "=r"(f.r[56]), "=r"(f.r[57]), "=r"(f.r[58]), "=r"(f.r[59]), "=r"(f.r[60]), "=r"(f.r[61]), "=r"(f.r[62]), "=r"(f.r[63]), "=r"(f.r[64]), "=r"(f.r[65]), "=r"(f.r[66]), "=r"(f.r[67]), "=r"(f.r[68]), "=r"(f.r[69]), "=r"(f.r[70]), "=r"(f.r[71]), "=r"(f.r[72]), "=r"(f.r[73]), "=r"(f.r[74]), "=r"(f.r[75]), "=r"(f.r[76]), "=r"(f.r[77]), "=r"(f.r[78]), "=r"(f.r[79]), "=r"(f.r[80]), "=r"(f.r[81]), "=r"(f.r[82]), "=r"(f.r[83]), "=r"(f.r[84]), "=r"(f.r[85]), "=r"(f.r[86]), "=r"(f.r[87]), "=r"(f.r[88]), "=r"(f.r[89]), "=r"(f.r[90]), "=r"(f.r[91]), "=r"(f.r[92]), "=r"(f.r[93]), "=r"(f.r[94]), "=r"(f.r[95]), "=r"(f.r[96]), "=r"(f.r[97]), "=r"(f.r[98]), "=r"(f.r[99]), "=r"(f.r[100]), "=r"(f.r[101]), "=r"(f.r[102]), "=r"(f.r[103]), "=r"(f.r[104]), "=r"(f.r[105]), "=r"(f.r[106]), "=r"(f.r[107]), "=r"(f.r[108]), "=r"(f.r[109]), "=r"(f.r[110]), "=r"(f.r[111]), "=r"(f.r[112]), "=r"(f.r[113]), "=r"(f.r[114]), "=r"(f.r[115]), "=r"(f.r[116]), "=r"(f.r[117]), "=r"(f.r[118]), "=r"(f.r[119]), "=r"(f.r[120]), "=r"(f.r[121]), "=r"(f.r[122]), "=r"(f.r[123]), "=r"(f.r[124]), "=r"(f.r[125]), "=r"(f.r[126]), "=r"(f.r[127])
-               : "r"(taddr));
-}
-__device__ __forceinline__ void tmem_wait_ld128(Frag128& f) {
-  asm volatile("tcgen05.wait::ld.sync.aligned;"
-               : "+r"(f.r[0]), "+r"(f.r[1]), "+r"(f.r[2]), "+r"(f.r[3]), "+r"(f.r[4]), "+r"(f.r[5]), "+r"(f.r[6]), "+r"(f.r[7]), "+r"(f.r[8]), "+r"(f.r[9]), "+r"(f.r[10]), "+r"(f.r[11]), "+r"(f.r[12]), "+r"(f.r[13]), "+r"(f.r[14]), "+r"(f.r[15]), "+r"(f.r[16]), "+r"(f.r[17]), "+r"(f.r[18]), "+r"(f.r[19]), "+r"(f.r[20]), "+r"(f.r[21]), "+r"(f.r[22]), "+r"(f.r[23]), "+r"(f.r[24]), "+r"(f.r[25]), "+r"(f.r[26]), "+r"(f.r[27]), "+r"(f.r[28]), "+r"(f.r[29]), "+r"(f.r[30]), "+r"(f.r[31]), "+r"(f.r[32]), "+r"(f.r[33]), "+r"(f.r[34]), "+r"(f.r[35]), "+r"(f.r[36]), "+r"(f.r[37]), "+r"(f.r[38]), "+r"(f.r[39]), "+r"(f.r[40]), "+r"(f.r[41]), "+r"(f.r[42]), "+r"(f.r[43]), "+r"(f.r[44]), "+r"(f.r[45]), "+r"(f.r[46]), "+r"(f.r[47]), "+r"(f.r[48]), "+r"(f.r[49]), "+r"(f.r[50]), "+r"(f.r[51]), "+r"(f.r[52]), "+r"(f.r[53]), "+r"(f.r[54]), "+r"(f.r[55]), "+r"(f.r[56]), "+r"(f.r[57]), "+r"(f.r[58]), "+r"(f.r[59]), "+r"(f.r[60]), "+r"(f.r[61]), "+r"(f.r[62]), "+r"(f.r[63]), "+r"(f.r[64]), "+r"(f.r[65]), "+r"(f.r[66]), "+r"(f.r[67]), "+r"(f.r[68]), "+r"(f.r[69]), "+r"(f.r[70]), "+r"(f.r[71]), "+r"(f.r[72]), "+r"(f.r[73]), "+r"(f.r[74]), "+r"(f.r[75]), "+r"(f.r[76]), "+r"(f.r[77]), "+r"(f.r[78]), "+r"(f.r[79]), "+r"(f.r[80]), "+r"(f.r[81]), "+r"(f.r[82]), "+r"(f.r[83]), "+r"(f.r[84]), "+r"(f.r[85]), "+r"(f.r[86]), "+r"(f.r[87]), "+r"(f.r[88]), "+r"(f.r[89]), "+r"(f.r[90]), "+r"(f.r[91]), "+r"(f.r[92]), "+r"(f.r[93]), "+r"(f.r[94]), "+r"(f.r[95]), "+r"(f.r[96]), "+r"(f.r[97]), "+r"(f.r[98]), "+r"(f.r[99]), "+r"(f.r[100]), "+r"(f.r[101]), "+r"(f.r[102]), "+r"(f.r[103]), "+r"(f.r[104]), "+r"(f.r[105]), "+r"(f.r[106]), "+r"(f.r[107]), "+r"(f.r[108]), "+r"(f.r[109]), "+r"(f.r[110]), "+r"(f.r[111]), "+r"(f.r[112]), "+r"(f.r[113]), "+r"(f.r[114]), "+r"(f.r[115]), "+r"(f.r[116]), "+r"(f.r[117]), "+r"(f.r[118]), "+r"(f.r[119]), "+r"(f.r[120]), "+r"(f.r[121]), "+r"(f.r[122]), "+r"(f.r[123]), "+r"(f.r[124]), "+r"(f.r[125]), "+r"(f.r[126]), "+r"(f.r[127]));
-}
 __device__ __forceinline__ void tmem_ld128_sync(uint32_t taddr, Frag128& f) {
   asm volatile(
       "tcgen05.ld.sync.aligned.32x32b.x128.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32, %33, %34, %35, %36, %37, %38, %39, %40, %41, %42, %43, %44, %45, %46, %47, %48, %49, %50, %51, %52, %53, %54, %55, %56, %57, %58, %59, %60, %61, %62, %63, %64, %65, %66, %67, %68, %69, %70, %71, %72, %73, %74, %75, %76, %77, %78, %79, %80, %81, %82, %83, %84, %85, %86, %87, %88, %89, %90, %91, %92, %93, %94, %95, %96, %97, %98, %99, %100, %101, %102, %103, %104, %105, %106, %107, %108, %109, %110, %111, %112, %113, %114, %115, %116, %117, %118, %119, %120, %121, %122, %123, %124, %125, %126, %127}, [%128];\n\t"
@@ -206,21 +150,6 @@ __device__ __forceinline__ void tmem_ld128_sync(uint32_t taddr, Frag128& f) {
 struct Frag64 {
   uint32_t r[64];
 };
-// Store the first 64 registers of a 128-register fragment (32x32b.x64).
-__device__ __forceinline__ void tmem_st64_lo(uint32_t taddr, const Frag128& f) {
-  asm volatile("tcgen05.st.sync.aligned.32x32b.x64.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32, %33, %34, %35, %36, %37, %38, %39, %40, %41, %42, %43, %44, %45, %46, %47, %48, %49, %50, %51, %52, %53, %54, %55, %56, %57, %58, %59, %60, %61, %62, %63, %64};"
-               ::"r"(taddr), "r"(f.r[0]), "r"(f.r[1]), "r"(f.r[2]), "r"(f.r[3]), "r"(f.r[4]), "r"(f.r[5]), "r"(f.r[6]), "r"(f.r[7]), "r"(f.r[8]), "r"(f.r[9]), "r"(f.r[10]), "r"(f.r[11]), "r"(f.r[12]), "r"(f.r[13]), "r"(f.r[14]), "r"(f.r[15]), "r"(f.r[16]), "r"(f.r[17]), "r"(f.r[18]), "r"(f.r[19]), "r"(f.r[20]), "r"(f.r[21]), "r"(f.r[22]), "r"(f.r[23]), "r"(f.r[24]), "r"(f.r[25]), "r"(f.r[26]), "r"(f.r[27]), "r"(f.r[28]), "r"(f.r[29]), "r"(f.r[30]), "r"(f.r[31]), "r"(f.r[32]), "r"(f.r[33]), "r"(f.r[34]), "r"(f.r[35]), "r"(f.r[36]), "r"(f.r[37]), "r"(f.r[38]), "r"(f.r[39]), "r"(f.r[40]), "r"(f.r[41]), "r"(f.r[42]), "r"(f.r[43]), "r"(f.r[44]), "r"(f.r[45]), "r"(f.r[46]), "r"(f.r[47]), "r"(f.r[48]), "r"(f.r[49]), "r"(f.r[50]), "r"(f.r[51]), "r"(f.r[52]), "r"(f.r[53]), "r"(f.r[54]), "r"(f.r[55]), "r"(f.r[56]), "r"(f.r[57]), "r"(f.r[58]), "r"(f.r[59]), "r"(f.r[60]), "r"(f.r[61]), "r"(f.r[62]), "r"(f.r[63])
-               : "memory");
-}
-__device__ __forceinline__ void tmem_ld64(uint32_t taddr, Frag64& f) {
-  asm volatile("tcgen05.ld.sync.aligned.32x32b.x64.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32, %33, %34, %35, %36, %37, %38, %39, %40, %41, %42, %43, %44, %45, %46, %47, %48, %49, %50, %51, %52, %53, %54, %55, %56, %57, %58, %59, %60, %61, %62, %63}, [%64];"
-               : "=r"(f.r[0]), "=r"(f.r[1]), "=r"(f.r[2]), "=r"(f.r[3]), "=r"(f.r[4]), "=r"(f.r[5]), "=r"(f.r[6]), "=r"(f.r[7]), "=r"(f.r[8]), "=r"(f.r[9]), "=r"(f.r[10]), "=r"(f.r[11]), "=r"(f.r[12]), "=r"(f.r[13]), "=r"(f.r[14]), "=r"(f.r[15]), "=r"(f.r[16]), "=r"(f.r[17]), "=r"(f.r[18]), "=r"(f.r[19]), "=r"(f.r[20]), "=r"(f.r[21]), "=r"(f.r[22]), "=r"(f.r[23]), "=r"(f.r[24]), "=r"(f.r[25]), "=r"(f.r[26]), "=r"(f.r[27]), "=r"(f.r[28]), "=r"(f.r[29]), "=r"(f.r[30]), "=r"(f.r[31]), "=r"(f.r[32]), "=r"(f.r[33]), "=r"(f.r[34]), "=r"(f.r[35]), "=r"(f.r[36]), "=r"(f.r[37]), "=r"(f.r[38]), "=r"(f.r[39]), "=r"(f.r[40]), "=r"(f.r[41]), "=r"(f.r[42]), "=r"(f.r[43]), "=r"(f.r[44]), "=r"(f.r[45]), "=r"(f.r[46]), "=r"(f.r[47]), "=r"(f.r[48]), "=r"(f.r[49]), "=r"(f.r[50]), "=r"(f.r[51]), "=r"(f.r[52]), "=r"(f.r[53]), "=r"(f.r[54]), "=r"(f.r[55]), "=r"(f.r[56]), "=r"(f.r[57]), "=r"(f.r[58]), "=r"(f.r[59]), "=r"(f.r[60]), "=r"(f.r[61]), "=r"(f.r[62]), "=r"(f.r[63])
-               : "r"(taddr));
-}
-__device__ __forceinline__ void tmem_wait_ld64(Frag64& f) {
-  asm volatile("tcgen05.wait::ld.sync.aligned;"
-               : "+r"(f.r[0]), "+r"(f.r[1]), "+r"(f.r[2]), "+r"(f.r[3]), "+r"(f.r[4]), "+r"(f.r[5]), "+r"(f.r[6]), "+r"(f.r[7]), "+r"(f.r[8]), "+r"(f.r[9]), "+r"(f.r[10]), "+r"(f.r[11]), "+r"(f.r[12]), "+r"(f.r[13]), "+r"(f.r[14]), "+r"(f.r[15]), "+r"(f.r[16]), "+r"(f.r[17]), "+r"(f.r[18]), "+r"(f.r[19]), "+r"(f.r[20]), "+r"(f.r[21]), "+r"(f.r[22]), "+r"(f.r[23]), "+r"(f.r[24]), "+r"(f.r[25]), "+r"(f.r[26]), "+r"(f.r[27]), "+r"(f.r[28]), "+r"(f.r[29]), "+r"(f.r[30]), "+r"(f.r[31]), "+r"(f.r[32]), "+r"(f.r[33]), "+r"(f.r[34]), "+r"(f.r[35]), "+r"(f.r[36]), "+r"(f.r[37]), "+r"(f.r[38]), "+r"(f.r[39]), "+r"(f.r[40]), "+r"(f.r[41]), "+r"(f.r[42]), "+r"(f.r[43]), "+r"(f.r[44]), "+r"(f.r[45]), "+r"(f.r[46]), "+r"(f.r[47]), "+r"(f.r[48]), "+r"(f.r[49]), "+r"(f.r[50]), "+r"(f.r[51]), "+r"(f.r[52]), "+r"(f.r[53]), "+r"(f.r[54]), "+r"(f.r[55]), "+r"(f.r[56]), "+r"(f.r[57]), "+r"(f.r[58]), "+r"(f.r[59]), "+r"(f.r[60]), "+r"(f.r[61]), "+r"(f.r[62]), "+r"(f.r[63]));
-}
 // 64 columns, load and wait in one statement (see tmem_ld32_sync).
 __device__ __forceinline__ void tmem_ld64_sync(uint32_t taddr, Frag64& f) {
   asm volatile(
@@ -228,11 +157,6 @@ __device__ __forceinline__ void tmem_ld64_sync(uint32_t taddr, Frag64& f) {
       "tcgen05.wait::ld.sync.aligned;"
       : "=r"(f.r[0]), "=r"(f.r[1]), "=r"(f.r[2]), "=r"(f.r[3]), "=r"(f.r[4]), "=r"(f.r[5]), "=r"(f.r[6]), "=r"(f.r[7]), "=r"(f.r[8]), "=r"(f.r[9]), "=r"(f.r[10]), "=r"(f.r[11]), "=r"(f.r[12]), "=r"(f.r[13]), "=r"(f.r[14]), "=r"(f.r[15]), "=r"(f.r[16]), "=r"(f.r[17]), "=r"(f.r[18]), "=r"(f.r[19]), "=r"(f.r[20]), "=r"(f.r[21]), "=r"(f.r[22]), "=r"(f.r[23]), "=r"(f.r[24]), "=r"(f.r[25]), "=r"(f.r[26]), "=r"(f.r[27]), "=r"(f.r[28]), "=r"(f.r[29]), "=r"(f.r[30]), "=r"(f.r[31]), "=r"(f.r[32]), "=r"(f.r[33]), "=r"(f.r[34]), "=r"(f.r[35]), "=r"(f.r[36]), "=r"(f.r[37]), "=r"(f.r[38]), "=r"(f.r[39]), "=r"(f.r[40]), "=r"(f.r[41]), "=r"(f.r[42]), "=r"(f.r[43]), "=r"(f.r[44]), "=r"(f.r[45]), "=r"(f.r[46]), "=r"(f.r[47]), "=r"(f.r[48]), "=r"(f.r[49]), "=r"(f.r[50]), "=r"(f.r[51]), "=r"(f.r[52]), "=r"(f.r[53]), "=r"(f.r[54]), "=r"(f.r[55]), "=r"(f.r[56]), "=r"(f.r[57]), "=r"(f.r[58]), "=r"(f.r[59]), "=r"(f.r[60]), "=r"(f.r[61]), "=r"(f.r[62]), "=r"(f.r[63])
       : "r"(taddr));
-}
-__device__ __forceinline__ void tmem_st64(uint32_t taddr, const Frag64& f) {
-  asm volatile("tcgen05.st.sync.aligned.32x32b.x64.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32, %33, %34, %35, %36, %37, %38, %39, %40, %41, %42, %43, %44, %45, %46, %47, %48, %49, %50, %51, %52, %53, %54, %55, %56, %57, %58, %59, %60, %61, %62, %63, %64};"
-               ::"r"(taddr), "r"(f.r[0]), "r"(f.r[1]), "r"(f.r[2]), "r"(f.r[3]), "r"(f.r[4]), "r"(f.r[5]), "r"(f.r[6]), "r"(f.r[7]), "r"(f.r[8]), "r"(f.r[9]), "r"(f.r[10]), "r"(f.r[11]), "r"(f.r[12]), "r"(f.r[13]), "r"(f.r[14]), "r"(f.r[15]), "r"(f.r[16]), "r"(f.r[17]), "r"(f.r[18]), "r"(f.r[19]), "r"(f.r[20]), "r"(f.r[21]), "r"(f.r[22]), "r"(f.r[23]), "r"(f.r[24]), "r"(f.r[25]), "r"(f.r[26]), "r"(f.r[27]), "r"(f.r[28]), "r"(f.r[29]), "r"(f.r[30]), "r"(f.r[31]), "r"(f.r[32]), "r"(f.r[33]), "r"(f.r[34]), "r"(f.r[35]), "r"(f.r[36]), "r"(f.r[37]), "r"(f.r[38]), "r"(f.r[39]), "r"(f.r[40]), "r"(f.r[41]), "r"(f.r[42]), "r"(f.r[43]), "r"(f.r[44]), "r"(f.r[45]), "r"(f.r[46]), "r"(f.r[47]), "r"(f.r[48]), "r"(f.r[49]), "r"(f.r[50]), "r"(f.r[51]), "r"(f.r[52]), "r"(f.r[53]), "r"(f.r[54]), "r"(f.r[55]), "r"(f.r[56]), "r"(f.r[57]), "r"(f.r[58]), "r"(f.r[59]), "r"(f.r[60]), "r"(f.r[61]), "r"(f.r[62]), "r"(f.r[63])
-               : "memory");
 }
 // Store and wait in one statement: the source registers stay untouched until
 // the store has completed, whatever the compiler schedules after it.
@@ -322,11 +246,6 @@ __device__ __forceinline__ uint32_t mapa(uint32_t saddr, uint32_t rank) {
   asm("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
   return r;
 }
-__device__ __forceinline__ float ld_cluster_f1(uint32_t caddr) {
-  float v;
-  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(caddr) : "memory");
-  return v;
-}
 __device__ __forceinline__ uint64_t ld_cluster_u64(uint32_t caddr) {
   uint64_t v;
   asm volatile("ld.shared::cluster.u64 %0, [%1];" : "=l"(v) : "r"(caddr) : "memory");
@@ -358,53 +277,12 @@ __device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t* p) {
 __device__ __forceinline__ void red_add_release_gpu(uint32_t* p, uint32_t v) {
   asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
-// Plain loads (no volatile, no memory clobber): callers order them with a
-// cluster barrier, and independent loads can then be in flight together.
-__device__ __forceinline__ float4 ld_cluster_f4(uint32_t caddr) {
-  float4 v;
-  asm("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
-      : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-      : "r"(caddr));
-  return v;
-}
-__device__ __forceinline__ float2 ld_cluster_f2(uint32_t caddr) {
-  float2 v;
-  asm("ld.shared::cluster.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(caddr));
-  return v;
-}
-
-__device__ __forceinline__ void st_cluster_f4(uint32_t caddr, float4 v) {
-  asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(caddr), "f"(v.x), "f"(v.y),
-               "f"(v.z), "f"(v.w)
-               : "memory");
-}
 __device__ __forceinline__ void st_cluster_f1(uint32_t caddr, float v) {
   asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(caddr), "f"(v) : "memory");
-}
-__device__ __forceinline__ void st_cluster_f2(uint32_t caddr, float2 v) {
-  asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(caddr), "f"(v.x), "f"(v.y)
-               : "memory");
-}
-
-// Bulk copy of `bytes` (multiple of 16, both addresses 16-byte aligned)
-// from this CTA's shared memory to a cluster peer's shared memory; the
-// transfer completes `bytes` on the peer's mbarrier `peer_bar`.
-__device__ __forceinline__ void bulk_s2cluster(uint32_t peer_dst, uint32_t src, uint32_t bytes,
-                                               uint32_t peer_bar) {
-  asm volatile(
-      "cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-          peer_dst),
-      "r"(src), "r"(bytes), "r"(peer_bar)
-      : "memory");
 }
 __device__ __forceinline__ void bulk_commit() {
   asm volatile("cp.async.bulk.commit_group;" ::: "memory");
 }
-// Wait until the sources of this thread's bulk copies have been read.
-__device__ __forceinline__ void bulk_wait_read() {
-  asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
-}
-
 // Bulk (untiled) copies: 16-byte aligned addresses, sizes a multiple of 16.
 __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
   asm volatile(

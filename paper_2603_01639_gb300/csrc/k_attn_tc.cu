@@ -416,18 +416,19 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (j == 0) TRACE(3);
         }
         for (int j = 0; j < nc && ok; ++j) {
-          const int xs = j & 1, st = j % kStages;
-          ok = tc::mbar_wait(bar(VFULL + st), (j / kStages) & 1);
+          const int xs = j & 1, st = j % kStages, st2 = (j + 2) % kStages;
+          const bool more = j + 2 < nc;
+          // every wait before the first MMA of the pair, the one that
+          // usually blocks (P) last: a wait between MMA groups is a bubble
+          // in the tensor pipe even when its phase has completed
+          if (more) ok = tc::mbar_wait(bar(KFULL + st2), ((j + 2) / kStages) & 1);
+          if (ok) ok = tc::mbar_wait(bar(VFULL + st), (j / kStages) & 1);
           if (ok) ok = tc::mbar_wait(bar(PFULL + xs), (j >> 1) & 1);
           if (!ok) break;
           tc::fence_after_sync();
           issue_pv(xs, st, j >= 2 ? 1u : 0u);
           tc::mma_commit(bar(VEMPTY + st));
-          if (j + 2 < nc) {
-            const int st2 = (j + 2) % kStages;
-            ok = tc::mbar_wait(bar(KFULL + st2), ((j + 2) / kStages) & 1);
-            if (!ok) break;
-            tc::fence_after_sync();
+          if (more) {
             issue_s(xs, st2);
             tc::mma_commit(bar(SFULL + xs));
             tc::mma_commit(bar(KEMPTY + st2));
@@ -486,15 +487,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         auto step = [&](int j, auto R_) -> bool {
           constexpr int r = decltype(R_)::value;
           constexpr int xs = r & 1, st = r % kStages, st2 = (r + 2) % kStages;
-          bool k = tc::mbar_wait(bar(VFULL + st), (r / kStages) & 1);
+          const bool more = j + 2 < nc;
+          // (every wait before the pair's first MMA, P last, as above)
+          bool k = !more || tc::mbar_wait(bar(KFULL + st2), ((r + 2) / kStages) & 1);
+          if (k) k = tc::mbar_wait(bar(VFULL + st), (r / kStages) & 1);
           if (k) k = tc::mbar_wait(bar(PFULL + xs), (j >> 1) & 1);
           if (!k) return false;
           tc::fence_after_sync();
           issue_pv(xs, st, j >= 2 ? 1u : 0u);
           tc::mma_commit(bar(VEMPTY + st));
-          if (j + 2 < nc) {
-            if (!tc::mbar_wait(bar(KFULL + st2), ((r + 2) / kStages) & 1)) return false;
-            tc::fence_after_sync();
+          if (more) {
             issue_s(xs, st2);
             tc::mma_commit(bar(SFULL + xs));
             tc::mma_commit(bar(KEMPTY + st2));

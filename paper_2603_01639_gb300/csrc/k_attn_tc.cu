@@ -281,9 +281,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   // every K load (and Q) this thread issued lands before the CTA leaves or
   // reuses shared memory; at most one load per stage is outstanding
   auto drain_k = [&]() {
-    if (q_issued) tc::mbar_wait(bar(QFULL), 0);
+    if (q_issued) tc::mbar_wait_sleep(bar(QFULL), 0);
     for (int st = 0; st < kStages; ++st)
-      if (nk_issued[st] > 0) tc::mbar_wait(bar(KFULL + st), (nk_issued[st] - 1) & 1);
+      if (nk_issued[st] > 0) tc::mbar_wait_sleep(bar(KFULL + st), (nk_issued[st] - 1) & 1);
   };
   if (tid == 0 && !a.lpt) issue_first();
 
@@ -332,7 +332,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       for (int j = 1; j < nc && j < kStages; ++j) issue_k(j);
       for (int j = kStages; j < nc && ok; ++j) {
-        ok = tc::mbar_wait(bar(KEMPTY + j % kStages), ((j / kStages) - 1) & 1);
+        ok = tc::mbar_wait_sleep(bar(KEMPTY + j % kStages), ((j / kStages) - 1) & 1);
         if (ok) issue_k(j);
       }
       drain_k();
@@ -364,11 +364,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       };
       for (int j = 0; j < nc && j < kStages; ++j) issue_v(j);
       for (int j = kStages; j < nc && ok; ++j) {
-        ok = tc::mbar_wait(bar(VEMPTY + j % kStages), ((j / kStages) - 1) & 1);
+        ok = tc::mbar_wait_sleep(bar(VEMPTY + j % kStages), ((j / kStages) - 1) & 1);
         if (ok) issue_v(j);
       }
       for (int st = 0; st < kStages; ++st)
-        if (nv_issued[st] > 0) tc::mbar_wait(bar(VFULL + st), (nv_issued[st] - 1) & 1);
+        if (nv_issued[st] > 0) tc::mbar_wait_sleep(bar(VFULL + st), (nv_issued[st] - 1) & 1);
       if (!ok) flag_error(a.err, LTD_DEVERR_TIMEOUT);
     }
   } else if (warp == 1) {
@@ -401,13 +401,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int ks = 0; ks < 8; ++ks)
             tc::mma_bf16_ts(d, pa + 8 * ks, v + static_cast<uint64_t>(ks * (2048 >> 4)), id_o, ks > 0 ? 1u : acc);
         };
-        ok = tc::mbar_wait(bar(QFULL), 0);
+        ok = tc::mbar_wait_sleep(bar(QFULL), 0);
         TRACE(2);
         // S(0) and S(1) into S_0 and S_1, then per chunk j (stream j & 1, ring
         // stage j % 3, ring use j / 3): PV(j), then S(j + 2) into the same
         // stream
         for (int j = 0; j < 2 && j < nc && ok; ++j) {
-          ok = tc::mbar_wait(bar(KFULL + j), 0);
+          ok = tc::mbar_wait_sleep(bar(KFULL + j), 0);
           if (!ok) break;
           tc::fence_after_sync();
           issue_s(j, j);
@@ -421,9 +421,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           // every wait before the first MMA of the pair, the one that
           // usually blocks (P) last: a wait between MMA groups is a bubble
           // in the tensor pipe even when its phase has completed
-          if (more) ok = tc::mbar_wait(bar(KFULL + st2), ((j + 2) / kStages) & 1);
-          if (ok) ok = tc::mbar_wait(bar(VFULL + st), (j / kStages) & 1);
-          if (ok) ok = tc::mbar_wait(bar(PFULL + xs), (j >> 1) & 1);
+          if (more) ok = tc::mbar_wait_sleep(bar(KFULL + st2), ((j + 2) / kStages) & 1);
+          if (ok) ok = tc::mbar_wait_sleep(bar(VFULL + st), (j / kStages) & 1);
+          if (ok) ok = tc::mbar_wait_sleep(bar(PFULL + xs), (j >> 1) & 1);
           if (!ok) break;
           tc::fence_after_sync();
           issue_pv(xs, st, j >= 2 ? 1u : 0u);
@@ -462,12 +462,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc::mma_bf16_ts(tmem + 2 * kBN + x_ * kD, tmem + x_ * kBN + 8 * ks, dv[st][ks], id_o,
                             ks > 0 ? 1u : acc);
         };
-        ok = tc::mbar_wait(bar(QFULL), 0);
+        ok = tc::mbar_wait_sleep(bar(QFULL), 0);
         TRACE(2);
         // S(0) and S(1) into S_0 and S_1, then chunk j = 6 i + r (stream r & 1,
         // ring stage r % 3, ring use j / 3, whose parity is (r / 3) & 1): PV(j),
         // then S(j + 2) into the same stream; stages are compile-time constants
-        if (ok) ok = tc::mbar_wait(bar(KFULL + 0), 0);
+        if (ok) ok = tc::mbar_wait_sleep(bar(KFULL + 0), 0);
         if (ok) {
           tc::fence_after_sync();
           issue_s(0, 0);
@@ -476,7 +476,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         TRACE(3);
         if (ok && nc > 1) {
-          ok = tc::mbar_wait(bar(KFULL + 1), 0);
+          ok = tc::mbar_wait_sleep(bar(KFULL + 1), 0);
           if (ok) {
             tc::fence_after_sync();
             issue_s(1, 1);
@@ -489,9 +489,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           constexpr int xs = r & 1, st = r % kStages, st2 = (r + 2) % kStages;
           const bool more = j + 2 < nc;
           // (every wait before the pair's first MMA, P last, as above)
-          bool k = !more || tc::mbar_wait(bar(KFULL + st2), ((r + 2) / kStages) & 1);
-          if (k) k = tc::mbar_wait(bar(VFULL + st), (r / kStages) & 1);
-          if (k) k = tc::mbar_wait(bar(PFULL + xs), (j >> 1) & 1);
+          bool k = !more || tc::mbar_wait_sleep(bar(KFULL + st2), ((r + 2) / kStages) & 1);
+          if (k) k = tc::mbar_wait_sleep(bar(VFULL + st), (r / kStages) & 1);
+          if (k) k = tc::mbar_wait_sleep(bar(PFULL + xs), (j >> 1) & 1);
           if (!k) return false;
           tc::fence_after_sync();
           issue_pv(xs, st, j >= 2 ? 1u : 0u);
@@ -515,7 +515,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       TRACE(22);
       // every MMA of this CTA completes before tensor memory is read or freed
       tc::mma_commit(bar(FIN));
-      tc::mbar_wait(bar(FIN), 0);
+      tc::mbar_wait_sleep(bar(FIN), 0);
       if (!ok) flag_error(a.err, LTD_DEVERR_TIMEOUT);
       TRACE(23);
     }
@@ -523,13 +523,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == 3) {
     // (trace builds only) the idle warp observes when the first loads land
     if (lane == 0) {
-      if (tc::mbar_wait(bar(QFULL), 0)) TRACE(24);
-      if (nc > 0 && tc::mbar_wait(bar(KFULL + 0), 0)) TRACE(25);
-      if (nc > 0 && tc::mbar_wait(bar(VFULL + 0), 0)) TRACE(26);
-      if (nc > 1 && tc::mbar_wait(bar(KFULL + 1), 0)) TRACE(27);
-      if (nc > 1 && tc::mbar_wait(bar(VFULL + 1), 0)) TRACE(28);
-      if (nc > 2 && tc::mbar_wait(bar(KFULL + 2), 0)) TRACE(29);
-      if (nc > 2 && tc::mbar_wait(bar(VFULL + 2), 0)) TRACE(30);
+      if (tc::mbar_wait_sleep(bar(QFULL), 0)) TRACE(24);
+      if (nc > 0 && tc::mbar_wait_sleep(bar(KFULL + 0), 0)) TRACE(25);
+      if (nc > 0 && tc::mbar_wait_sleep(bar(VFULL + 0), 0)) TRACE(26);
+      if (nc > 1 && tc::mbar_wait_sleep(bar(KFULL + 1), 0)) TRACE(27);
+      if (nc > 1 && tc::mbar_wait_sleep(bar(VFULL + 1), 0)) TRACE(28);
+      if (nc > 2 && tc::mbar_wait_sleep(bar(KFULL + 2), 0)) TRACE(29);
+      if (nc > 2 && tc::mbar_wait_sleep(bar(VFULL + 2), 0)) TRACE(30);
     }
 #endif
   } else if (smx && x < nc) {
@@ -555,7 +555,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int t = 0; t < 5; ++t)
           if (w0 + t >= 0 && w0 + t < w32) mw5[t] = __ldcg(mbits + w0 + t);
       }
-      ok = tc::mbar_wait(bar(SFULL + x), (j >> 1) & 1);
+      ok = tc::mbar_wait_sleep(bar(SFULL + x), (j >> 1) & 1);
       ok = __all_sync(0xFFFFFFFFu, ok);
       if (tr && j < 4) TRACE(4 + 2 * j);
       if (!ok) break;
@@ -674,7 +674,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // rows (both 64-dim halves) before PV reads this stage.
         const int st = j % kStages;
         // (a failed wait is flagged; the MMA thread times out on the same stage)
-        if (!__all_sync(0xFFFFFFFFu, tc::mbar_wait(bar(VFULL + st), (j / kStages) & 1)) && lane == 0)
+        if (!__all_sync(0xFFFFFFFFu, tc::mbar_wait_sleep(bar(VFULL + st), (j / kStages) & 1)) && lane == 0)
           flag_error(a.err, LTD_DEVERR_TIMEOUT);
         const int z0 = key_hi - kbase;  // 1 .. 127
         uint4* vs = reinterpret_cast<uint4*>(gbase + kOffV + st * kTile);

@@ -66,11 +66,23 @@ __device__ __forceinline__ bool mbar_try_suspend(uint32_t bar, uint32_t parity, 
 constexpr uint64_t kWaitLimitNs = 1000000000ull;
 
 // Wait until the phase with the given parity has completed; false on timeout.
-// Between tries the thread sleeps in hardware (up to 1 us a try) rather than
-// re-issuing the test: waiting warps then take no issue slots and fetch no
-// instructions from the SM's share while other warps work (measured 0.06-0.1
-// us faster per 8B- and 13B-class attention layer).
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+  if (mbar_try(bar, parity)) return true;
+  const uint64_t t0 = globaltimer();
+  while (true) {
+#pragma unroll 1
+    for (int i = 0; i < 64; ++i)
+      if (mbar_try(bar, parity)) return true;
+    if (globaltimer() - t0 > kWaitLimitNs) return false;
+  }
+}
+// The same wait, but between tries the thread sleeps in hardware (up to 1 us
+// a try) rather than re-issuing the test, so a waiting warp takes no issue
+// slots from the warps that work.  It pays where many warps wait while a few
+// compute (the attention kernel: 0.06-0.1 us per 8B- and 13B-class layer);
+// a pipeline that waits on every stage (the LM-head GEMM) lost 2-13% to the
+// later wake-up.
+__device__ __forceinline__ bool mbar_wait_sleep(uint32_t bar, uint32_t parity) {
   if (mbar_try(bar, parity)) return true;
   const uint64_t t0 = globaltimer();
   while (true) {

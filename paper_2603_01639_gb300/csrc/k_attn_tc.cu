@@ -13,7 +13,9 @@
 //               before the sequence's context length is read;
 //   warp 1      tcgen05.mma: S_x = Q K_j^T into tensor memory, then
 //               O_x += P_x V_j with P_x read from tensor memory, issued in
-//               the order S(0), S(1), PV(0), S(2), PV(1), S(3), ...;
+//               the order S(0), S(1), PV(0), S(2), PV(1), S(3), ...; the
+//               waits of a pair PV(j), S(j+2) all come before its first MMA,
+//               so the pair goes out back to back;
 //   warp 2      TMA: V chunks into a three-stage ring;
 //   warps 4-7   softmax of stream 0, warps 8-11 of stream 1, one thread per
 //               row (= tensor-memory lane) with the row's 128 scores in
@@ -36,9 +38,10 @@
 //    counter; when all splits have arrived, split s combines rows
 //    [s R, s R + R) of the unit with loads straight from L2 into registers
 //    and writes them; the last split to leave resets the unit's counters.
-// Every wait is bounded (mbarrier waits and the counter spin): on timeout a
-// CTA flags LTD_DEVERR_TIMEOUT, drains its own TMA loads and MMAs, still
-// arrives and departs on its counter, frees its tensor memory and returns.
+// Every wait is bounded (mbarrier waits, which sleep in hardware between
+// tries, and the counter spin): on timeout a CTA flags LTD_DEVERR_TIMEOUT,
+// drains its own TMA loads and MMAs, still arrives and departs on its
+// counter, frees its tensor memory and returns.
 #include <mutex>
 #include <type_traits>
 

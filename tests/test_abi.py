@@ -162,3 +162,32 @@ def test_entry_points_reject_bad_arguments_before_launch(L):
     assert L.ltd_kv_append(C.byref(kv_ok), 1, 0, fake, fake, fake, fake, s) == 2     # n_max 0
     assert L.ltd_kv_append(C.byref(kv_ok), 0, 8, fake, fake, fake, fake, s) == 2     # batch 0
     assert L.ltd_kv_append(C.byref(kv_ok), 1, 8, fake, None, fake, fake, s) == 1
+
+
+def test_attention_split_plan_on_a_152_sm_device(L):
+    """The host plan of the tensor-core attention (no GPU here, so the SM
+    count falls back to 152): units = (sequence, KV head, 128-row tile);
+    with fewer units than SMs each unit's keys are cut into the fewest
+    splits that give the shortest longest split, at most SMs / units; the
+    workspace holds a 32 KB bf16 partial and 128 fp32 log2-sum-exps per
+    (unit, split), plus two counters per unit, each part 256-byte aligned."""
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("the fallback SM count applies only without a device")
+
+    def ws(units, splits):
+        rows = units * splits * 128
+        a = lambda n: (n + 255) // 256 * 256  # noqa: E731
+        return a(rows * 256) + a(rows * 4) + a(units * 2 * 4)
+
+    BF16 = 1
+    # 8B-class: 8 heads x 2 tiles (240 rows), 33 chunks -> 9 splits of <= 4
+    assert L.ltd_attention_workspace_bytes(1, 32, 8, 128, 60, 4096, BF16) == ws(16, 9)
+    # 13B-class MHA: 40 units (one tile), 17 chunks -> 3 splits of <= 6
+    assert L.ltd_attention_workspace_bytes(1, 40, 40, 128, 96, 2048, BF16) == ws(40, 3)
+    # 32B-class: 8 heads x 3 tiles, 129 chunks -> 6 splits of <= 22
+    assert L.ltd_attention_workspace_bytes(1, 64, 8, 128, 48, 16384, BF16) == ws(24, 6)
+    # 70B-class batch: 768 units >= 152 SMs -> one split per unit, no partials
+    assert L.ltd_attention_workspace_bytes(16, 64, 8, 128, 96, 8192, BF16) == 256
+    # 4 units over 32 chunks -> 32 splits of one chunk
+    assert L.ltd_attention_workspace_bytes(1, 8, 2, 128, 60, 3968, BF16) == ws(4, 32)
